@@ -1,0 +1,498 @@
+#!/usr/bin/env python
+"""Benchmark of the SemPIC cache-hit path on GB300.
+
+A step is one cache-hit pass over the workload up to the first token --
+compose (layout + slot map), relocate (re-rotate + stitch, every layer), and
+for every layer the inline append and the prefill attention -- the timer
+boundary the paper defines for cache-hit TTFT, minus the Reader's linear and
+MLP layers (no weights here).  Decode steps lie outside that boundary; when
+the workload has decode tokens, one decode step over every layer is timed in
+the same run and reported under rows.a6_decode.
+
+Metric: cache-hit prefill query tokens per second (whole job), with the
+per-kernel rooflines (relocate GB/s vs HBM, prefill attention TF/s vs bf16
+tensor peak) in the same JSON line.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+       python bench.py --impl reference ...   (the CPU oracle, timed on the host)
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+GPU_GEN = {"tiny": "cpu", "llama8b_1layer": "cpu"}   # small inputs: CPU generator
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default="llama8b_1layer")
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--prefill-splits", type=int, default=0)
+    ap.add_argument("--decode-splits", type=int, default=0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--oracle-sample", default=None, help=argparse.SUPPRESS)
+    ap.add_argument("--oracle-seconds", type=float, default=10.0, help=argparse.SUPPRESS)
+    return ap.parse_args(argv)
+
+
+# ---------------------------------------------------------------- helpers
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def src_sha(name):
+    with open(os.path.join(ROOT, "paper_2607_28069_gb300", "csrc", name), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def ncu_traffic(kernel_key, src_file):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on
+    the current source of the kernel; else None."""
+    p = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(kernel_key)
+    if not e or e.get("src_sha") != src_sha(src_file):
+        return None
+    return e.get("bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        rows = []
+        for line in (self.out or "").splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i, v in enumerate(r)
+                          if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows),
+                "sm_max_mhz": max(r[1] for r in rows), "reasons": reasons,
+                "samples": len(rows)}
+
+
+# ---------------------------------------------------------- work accounting
+def work_of(wl):
+    """Algorithmic work of one TTFT pass (and one decode step), from the
+    request description: bytes for the HBM-bound rows, FLOPs for attention."""
+    spec = wl.spec
+    L, Hq, Hkv, d = spec.layers, spec.q_heads, spec.kv_heads, spec.head_dim
+    lens = wl.doc_len.cpu().tolist()
+    doc_tokens = sum(sum(lens[i] for i in docs) for docs in wl.meta["docs"])
+    pairs = 0
+    query_tokens = 0
+    ctx = []
+    for b, docs in enumerate(wl.meta["docs"]):
+        P = wl.meta["prefix"][b]
+        N = sum(lens[i] for i in docs)
+        Tq = spec.query_len
+        c = P + N + Tq
+        ctx.append(c)
+        pairs += P * (P + 1) // 2                       # prefix rows see the prefix
+        pairs += Tq * (P + N) + Tq * (Tq + 1) // 2      # query rows see all before them
+        query_tokens += Tq
+    inline_tokens = sum(wl.meta["prefix"]) + spec.batch * spec.query_len
+    row_bytes = Hkv * d * 2
+    return {
+        "query_tokens": query_tokens,
+        "relocate_bytes": 4 * row_bytes * doc_tokens * L,               # K,V read + write
+        "append_bytes": inline_tokens * (2 * Hq * d * 2 + 4 * row_bytes) * L,
+        "attend_flops": 4 * d * Hq * pairs * L,                         # QK^T and PV
+        "decode_bytes": sum(2 * row_bytes * (c + 1) for c in ctx) * L,  # K,V of step 0
+        "ctx": ctx,
+    }
+
+
+# ------------------------------------------------------------- oracle arms
+def oracle_sample(workload, seconds):
+    """Run the CPU oracle on a bounded sample of the workload (one request,
+    one layer per pass) until `seconds` elapse.  Returns the rate in query
+    tokens per second of the full workload (a request needs every layer)."""
+    import numpy as np  # noqa: F401
+
+    import oracle as O
+    from paper_2607_28069_gb300.workloads import WORKLOADS, generate
+    spec = WORKLOADS[workload]
+    small = workload in GPU_GEN
+    if not small:
+        import dataclasses
+        # same shapes per layer; one layer is enough for a per-layer sample
+        spec = dataclasses.replace(spec, layers=1, decode_steps=0)
+    wl = generate(spec, device="cpu", gen_device="cpu")
+    theta = O.rope_frequencies(spec.head_dim, spec.rope_base)
+    f64 = lambda t: t.float().numpy().astype("float64")  # noqa: E731
+    starts, lens = wl.doc_token_start.numpy(), wl.doc_len.numpy()
+    passes, t_total = 0, 0.0
+    b = 0
+    while t_total < seconds or passes == 0:
+        docs = wl.meta["docs"][b]
+        tin = int(wl.inline_len[b])
+        t0 = time.perf_counter()
+        lay = O.compose_layout(lens, wl.doc_base_pos.numpy(), docs, int(wl.prefix_len[b]),
+                               spec.query_len, wl.block_table[b].numpy(), spec.page_size)
+        k_docs = [f64(wl.k_pool[0, starts[x]:starts[x] + lens[x]]) for x in docs]
+        v_docs = [f64(wl.v_pool[0, starts[x]:starts[x] + lens[x]]) for x in docs]
+        O.cache_hit_prefill(lay, k_docs, v_docs, wl.doc_base_pos.numpy(),
+                            f64(wl.q_inline[0, b, :tin]), f64(wl.k_inline[0, b, :tin]),
+                            f64(wl.v_inline[0, b, :tin]), theta)
+        t_total += time.perf_counter() - t0
+        passes += 1
+        b = (b + 1) % spec.batch
+    full = WORKLOADS[workload]
+    # each pass = one request through one layer; a request needs `layers` of them
+    rate = passes * full.query_len / (t_total * full.layers)
+    return {"value": rate, "passes": passes, "seconds": t_total}
+
+
+def run_oracle_subprocess(workload, seconds):
+    cores = len(os.sched_getaffinity(0))
+    env = dict(os.environ)
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[k] = str(cores)
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--oracle-sample",
+                        workload, "--oracle-seconds", str(seconds)],
+                       capture_output=True, text=True, env=env, timeout=600)
+    if r.returncode != 0:
+        raise RuntimeError(f"oracle sample failed: {r.stderr[-2000:]}")
+    d = json.loads(r.stdout.strip().splitlines()[-1])
+    d["cores"] = cores
+    return d
+
+
+def sample_desc(workload):
+    from paper_2607_28069_gb300.workloads import WORKLOADS
+    s = WORKLOADS[workload]
+    return (f"fp64 numpy oracle, one request x one layer per pass ({s.query_len} query tokens "
+            f"over the full stitched context), repeated for >= the stated seconds; rate scaled to "
+            f"{s.layers} layer(s) per request")
+
+
+# --------------------------------------------------------------- GPU arm
+def main_gpu(args, rank, world):
+    import torch
+
+    import paper_2607_28069_gb300 as pic
+    from paper_2607_28069_gb300.pipeline import CacheHitPath
+    from paper_2607_28069_gb300.workloads import WORKLOADS, generate
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pic.load()
+    spec = WORKLOADS[args.workload]
+    import dataclasses
+    spec1 = spec if spec.decode_steps <= 1 else dataclasses.replace(spec, decode_steps=1)
+    wl = generate(spec1, device=dev, gen_device=GPU_GEN.get(args.workload, "cuda"))
+    path = CacheHitPath(wl, prefill_splits=args.prefill_splits, decode_splits=args.decode_splits)
+    work = work_of(wl)
+    L = spec.layers
+    geom = path.geom
+    psplits = pic.pic_prefill_num_splits(geom, spec.batch, path.max_inline, path.max_ctx,
+                                         args.prefill_splits)
+
+    # warm-up run and device-side status
+    path.ttft_pass()
+    if wl.q_dec is not None:
+        path.decode_pass(0)
+    torch.cuda.synchronize()
+    code, detail = pic.pic_device_status()
+    if code:
+        raise RuntimeError(f"device status {code} detail {detail}")
+
+    # one CUDA graph per call, so each call can be timed on its own
+    phases = [("compose", path.compose), ("relocate", path.relocate)]
+    for layer in range(L):
+        phases.append(("append", (lambda l=layer: path.append(l))))
+        phases.append(("attend", (lambda l=layer: path.attend(l))))
+    graphs = []
+    for name, fn in phases:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            fn()
+        graphs.append((name, g))
+    dec_graph = None
+    if wl.q_dec is not None:
+        dec_graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(dec_graph):
+            path.decode_pass(0)
+    torch.cuda.synchronize()
+
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    flush = torch.empty(max(2 * l2, 256 << 20), dtype=torch.uint8, device=dev)
+    sleep_cycles = int(2e9 * max(50e-6, 5e-6 * len(graphs)))
+    stream = torch.cuda.current_stream()
+
+    def one_step(evs):
+        flush.zero_()
+        torch.cuda._sleep(sleep_cycles)       # keep the GPU busy while the host enqueues
+        evs[0].record(stream)
+        for i, (_, g) in enumerate(graphs):
+            g.replay()
+            evs[i + 1].record(stream)
+
+    W, K = args.warmup, args.steps
+    for _ in range(W):
+        one_step([torch.cuda.Event(enable_timing=True) for _ in range(len(graphs) + 1)])
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(len(graphs) + 1)]
+              for _ in range(K)]
+    with ClockSampler(local) as clk:
+        for k in range(K):
+            one_step(events[k])
+        torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    step_ms = [ev[0].elapsed_time(ev[-1]) for ev in events]
+    phase_ms = {}
+    for ev in events:
+        for i, (name, _) in enumerate(graphs):
+            phase_ms.setdefault(name, []).append(ev[i].elapsed_time(ev[i + 1]))
+    total_ms = sum(step_ms)
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev, dtype=torch.float64)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / K
+    value = work["query_tokens"] * K * world / (total_ms / 1e3)
+
+    # per-row averages over the timed steps (ms per step)
+    per_step = {name: sum(v) / K for name, v in phase_ms.items()}
+    peaks, peak_src = load_peaks()
+    rows = {
+        "a1_compose": {"ms": per_step["compose"], "launches": 1},
+        "a2_a3_relocate": {
+            "ms": per_step["relocate"], "launches": 1,
+            "bytes": work["relocate_bytes"],
+            "gbs": work["relocate_bytes"] / (per_step["relocate"] * 1e6)},
+        "a4_append": {"ms": per_step["append"], "launches": L,
+                      "bytes": work["append_bytes"],
+                      "gbs": work["append_bytes"] / (per_step["append"] * 1e6)},
+        "a5_attend": {"ms": per_step["attend"], "launches": L * (2 if psplits > 1 else 1),
+                      "flops": work["attend_flops"], "splits": psplits,
+                      "tflops": work["attend_flops"] / (per_step["attend"] * 1e9)},
+    }
+    rows["a2_a3_relocate"]["frac_hbm"] = rows["a2_a3_relocate"]["gbs"] / peaks["hbm_gbs"]
+    rows["a5_attend"]["frac_bf16"] = rows["a5_attend"]["tflops"] / peaks["bf16_tflops"]
+    launches = 1 + 1 + L + rows["a5_attend"]["launches"]
+
+    # decode (outside the TTFT boundary), same run
+    if dec_graph is not None:
+        dsplits = pic.pic_decode_num_splits(geom, spec.batch, path.max_ctx, args.decode_splits)
+        dts = []
+        for k in range(max(3, K // 2) + 2):
+            flush.zero_()
+            torch.cuda._sleep(sleep_cycles)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            dec_graph.replay()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if k >= 2:
+                dts.append(e0.elapsed_time(e1))
+        dms = sum(dts) / len(dts)
+        rows["a6_decode"] = {
+            "ms": dms, "launches": L * (3 if dsplits > 1 else 2), "splits": dsplits,
+            "bytes": work["decode_bytes"], "gbs": work["decode_bytes"] / (dms * 1e6),
+            "tok_s": spec.batch / (dms / 1e3)}
+        rows["a6_decode"]["frac_hbm"] = rows["a6_decode"]["gbs"] / peaks["hbm_gbs"]
+
+    # dominant kernel of the step -> roofline object
+    if per_step["attend"] >= per_step["relocate"]:
+        per_launch_ms = per_step["attend"] / L
+        flops_launch = work["attend_flops"] / L
+        achieved = flops_launch / (per_launch_ms * 1e9)
+        traffic = ncu_traffic(f"attn_kernel|{args.workload}", "pic_prefill.cu")
+        roof = {"kernel": "attn_kernel (pic_attend_prefill)", "bound": "tensor",
+                "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                "frac": achieved / peaks["bf16_tflops"], "traffic": traffic,
+                "peak_source": f"{peak_src} bf16 burst"}
+    else:
+        achieved = rows["a2_a3_relocate"]["gbs"]
+        traffic = ncu_traffic(f"relocate_kernel|{args.workload}", "pic_relocate.cu")
+        roof = {"kernel": "relocate_kernel (pic_relocate)", "bound": "hbm",
+                "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / peaks["hbm_gbs"], "traffic": traffic,
+                "peak_source": f"{peak_src} copy"}
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        ins = [wl.req_doc_ids, wl.req_num_docs, wl.prefix_len, wl.query_len, wl.block_table,
+               wl.inline_len, wl.q_inline, wl.k_inline, wl.v_inline]
+        host_in = [t.cpu().pin_memory() for t in ins]
+        host_out = torch.empty(path.out.shape, dtype=path.out.dtype, pin_memory=True)
+        h2d = sum(t.numel() * t.element_size() for t in host_in)
+        d2h = host_out.numel() * host_out.element_size()
+        e_ms = []
+        for k in range(W + K):
+            flush.zero_()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for d_t, h_t in zip(ins, host_in):
+                d_t.copy_(h_t, non_blocking=True)
+            for _, g in graphs:
+                g.replay()
+            host_out.copy_(path.out, non_blocking=True)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if k >= W:
+                e_ms.append(e0.elapsed_time(e1))
+        e_total = sum(e_ms)
+        if world > 1:
+            t = torch.tensor([e_total], device=dev, dtype=torch.float64)
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            e_total = float(t.item())
+        e2e = {"value": work["query_tokens"] * K * world / (e_total / 1e3),
+               "unit": "query_tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    code, detail = pic.pic_device_status()
+    if code:
+        raise RuntimeError(f"device status {code} detail {detail} after the timed run")
+
+    out = {
+        "metric": "cache-hit prefill query tok/s (TTFT path: compose + relocate + append + "
+                  "prefill attention, all layers)",
+        "value": value, "unit": "query_tokens/s", "n_gpus": world, "steps": K, "warmup": W,
+        "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": args.workload, "description": spec.description,
+                   "batch": spec.batch, "layers": L, "q_heads": spec.q_heads,
+                   "kv_heads": spec.kv_heads, "head_dim": spec.head_dim,
+                   "query_len": spec.query_len, "ctx_tokens": work["ctx"],
+                   "l2_policy": f"L2 flushed before every step ({flush.numel() >> 20} MiB write)",
+                   "timing": "CUDA graph per call, CUDA events on the launching stream",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "gpu_launches": launches,
+        "rows": rows,
+        "roofline": roof,
+        "clocks": clk.summary(),
+        "e2e": e2e,
+    }
+    return out
+
+
+def main_reference(args):
+    from paper_2607_28069_gb300.workloads import WORKLOADS
+    spec = WORKLOADS[args.workload]
+    cores = len(os.sched_getaffinity(0))
+    rates = []
+    per = max(1.0, min(10.0, 150.0 / max(1, args.steps + args.warmup)))
+    for k in range(args.warmup + args.steps):
+        d = run_oracle_subprocess(args.workload, per)
+        if k >= args.warmup:
+            rates.append(d)
+    tot_tokens = sum(d["value"] * d["seconds"] for d in rates)
+    tot_s = sum(d["seconds"] for d in rates)
+    value = tot_tokens / tot_s
+    return {
+        "impl": "reference", "metric": "cache-hit prefill query tok/s (TTFT path: compose + "
+        "relocate + append + prefill attention, all layers)", "value": value,
+        "unit": "query_tokens/s", "n_gpus": args.gpus, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * spec.batch * spec.query_len / value,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": args.workload},
+        "cpu_baseline": {"value": value, "unit": "query_tokens/s", "cores": cores,
+                         "kind": "oracle", "sample": sample_desc(args.workload)},
+        "e2e": {"value": value, "unit": "query_tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    if args.oracle_sample:
+        print(json.dumps(oracle_sample(args.oracle_sample, args.oracle_seconds)))
+        return 0
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        print(json.dumps(main_reference(args)))
+        return 0
+    import torch
+    if world > 1:
+        torch.distributed.init_process_group("nccl")
+    # the oracle baseline runs before the GPU work so its subprocess starts clean
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        d = run_oracle_subprocess(args.workload, args.oracle_seconds)
+        cpu = {"value": d["value"], "unit": "query_tokens/s", "cores": d["cores"],
+               "kind": "oracle", "sample": sample_desc(args.workload) +
+               f"; {d['passes']} passes in {d['seconds']:.1f} s"}
+    out = main_gpu(args, rank, world)
+    out["cpu_baseline"] = cpu
+    if rank == 0:
+        print(json.dumps(out))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

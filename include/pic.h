@@ -1,0 +1,260 @@
+/*
+ * pic.h -- C ABI of the GB300 (sm_103a) cache-hit path of SemPIC-style
+ * position-independent KV caching.
+ *
+ * The path (SemPIC, "Cache-hit serving"; appendix "Position-Independent
+ * Linking"): cached document keys, compiled in isolation at a base position,
+ * are moved to their request-time logical positions with the key re-rotation
+ * of Eq. 3, stitched with the request's inline tokens into a paged KV cache in
+ * the canonical order P, D_1..D_m, Q (Eqs. 1-2), and read by the unchanged
+ * decoder's GQA softmax attention under the frontier causal mask, first for
+ * the inline tokens (prefill) and then for ordinary decoding.
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * - Every tensor pointer is DEVICE memory owned by the caller; the library
+ *   allocates nothing and keeps no pointer after a call returns.
+ * - Every call is asynchronous on `stream` (NULL = legacy default stream).
+ *   Outputs are valid once the stream has reached the call.
+ * - bf16 tensors are IEEE bfloat16, row-major, densely packed, in the layouts
+ *   given per argument.  Integer tensors are int32 unless noted.
+ * - Host-side argument checks return PIC_ERR_INVALID_ARG / PIC_ERR_UNSUPPORTED
+ *   before anything is launched.  Checks that need device data (document ids,
+ *   page ids, positions, lengths) run inside the kernels: a failing element is
+ *   skipped (never dereferenced) and the first failure is recorded in a
+ *   per-device status word read by pic_device_status().  Every wait inside a
+ *   kernel is bounded; expiry is recorded as PIC_DEV_TIMEOUT.
+ * - On a non-OK return, pic_last_error() gives a one-line reason (per thread).
+ * - No call throws; no call synchronises the stream except pic_device_status.
+ *
+ * Cache layout (all calls): k_cache / v_cache are
+ *     bf16 [num_layers][num_pages][num_kv_heads][page_size][head_dim]
+ * Logical position t of request b lives in page block_table[b][t / page_size]
+ * at row t % page_size ("slot" = page * page_size + row).
+ * Document pool layout: k_pool / v_pool are
+ *     bf16 [num_layers][pool_tokens][num_kv_heads][head_dim]
+ * document i occupying rows doc_token_start[i] .. + doc_len[i] - 1, its key
+ * at row j compiled at logical position doc_base_pos[i] + j.
+ */
+#ifndef PIC_H_
+#define PIC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define PIC_ABI_VERSION 1
+
+typedef struct CUstream_st *pic_stream_t; /* identical to cudaStream_t */
+
+typedef enum {
+  PIC_OK = 0,
+  PIC_ERR_INVALID_ARG = 1, /* a host-visible argument is out of range       */
+  PIC_ERR_UNSUPPORTED = 2, /* valid but not implemented (head_dim, page)    */
+  PIC_ERR_CUDA = 3,        /* a CUDA runtime/driver call failed             */
+  PIC_ERR_WORKSPACE = 4,   /* workspace missing, too small or misaligned    */
+  PIC_ERR_DEVICE = 5       /* pic_device_status found a device-side failure */
+} pic_status_t;
+
+/* Device-side failure codes reported by pic_device_status(). */
+#define PIC_DEV_OK 0
+#define PIC_DEV_BAD_DOC_ID 1        /* request names a doc outside the pool  */
+#define PIC_DEV_BAD_DOC_LEN 2       /* document length <= 0                  */
+#define PIC_DEV_BAD_REQUEST 3       /* negative prefix/query/doc count       */
+#define PIC_DEV_CTX_OVERFLOW 4      /* context exceeds max_ctx / max_inline  */
+#define PIC_DEV_BLOCK_TABLE_SHORT 5 /* block table has too few pages         */
+#define PIC_DEV_BAD_PAGE 6          /* page id outside [0, num_pages)        */
+#define PIC_DEV_BAD_POSITION 7      /* logical position out of range         */
+#define PIC_DEV_TIMEOUT 8           /* a bounded wait inside a kernel expired */
+
+/* RoPE pairing: element i with i + d/2 (half-split), or 2i with 2i+1. */
+#define PIC_ROPE_HALF 0
+#define PIC_ROPE_INTERLEAVED 1
+
+/* Model geometry shared by all calls. */
+typedef struct {
+  int32_t num_layers;
+  int32_t num_q_heads;   /* Hq; query head h reads kv head h / (Hq / Hkv)  */
+  int32_t num_kv_heads;  /* Hkv; must divide Hq                            */
+  int32_t head_dim;      /* d: 64 or 128                                   */
+  int32_t page_size;     /* tokens per page: 16                            */
+  int32_t rope_style;    /* PIC_ROPE_HALF or PIC_ROPE_INTERLEAVED          */
+  double rope_base;      /* theta_i = rope_base^(-2i/d)                    */
+  const double *inv_freq;/* nullable HOST pointer to d/2 frequencies that
+                            replace rope_base^(-2i/d) (scaled RoPE)        */
+} pic_geom_t;
+
+/* Library version (PIC_ABI_VERSION of the build). */
+int32_t pic_abi_version(void);
+
+/* One-line reason for the last non-OK status returned on this thread. */
+const char *pic_last_error(void);
+
+/*
+ * pic_device_status -- synchronise `stream`, then read and clear the status
+ * word of the current device.  *code receives a PIC_DEV_* value, *detail the
+ * request (or split) index of the first failure.  Returns PIC_ERR_DEVICE when
+ * *code != PIC_DEV_OK, PIC_ERR_CUDA when the synchronisation failed.
+ */
+pic_status_t pic_device_status(pic_stream_t stream, int32_t *code, int32_t *detail);
+
+/*
+ * pic_compose -- link operator R: logical layout of each request and its
+ * token-level slot map (Eqs. 1-2, "Background: Position-Independent
+ * Caching"; appendix "Logical Layout and Re-Rotation").
+ *
+ * Request b is laid out as prefix (positions 0..P_b-1), then its documents
+ * in the order req_doc_ids[b][0..m_b-1], then Tq_b query tokens.  For its
+ * k-th document (pool id i, length n_i):
+ *     doc_offset[b][k] = P_b + sum_{k'<k} n_{ids[b][k']}
+ *     doc_delta[b][k]  = doc_offset[b][k] - doc_base_pos[i]
+ * ctx_len[b] = P_b + sum_k n + Tq_b, and for 0 <= t < ctx_len[b]
+ *     slot_mapping[b][t] = block_table[b][t / page] * page + t % page.
+ * inline_pos[b][0..P_b+Tq_b-1] lists the inline tokens' logical positions:
+ * 0..P_b-1 then ctx_len[b]-Tq_b .. ctx_len[b]-1.
+ *
+ * Inputs (device, int32): doc_len, doc_base_pos [n_pool_docs];
+ *   req_doc_ids [batch][max_docs]; req_num_docs, prefix_len, query_len [batch];
+ *   block_table [batch][max_pages] (entries used must be in [0, num_pages)).
+ * Outputs (device): doc_offset, doc_delta int32 [batch][max_docs] (entries
+ *   k >= m_b are set to -1 / 0); slot_mapping int64 [batch][max_ctx];
+ *   inline_pos int32 [batch][max_inline] (unused tail -1);
+ *   ctx_len int32 [batch] (-1 for a request that failed a device check).
+ * Device checks: doc id range, doc length > 0, ctx <= max_ctx,
+ *   P + Tq <= max_inline, ceil(ctx / page) <= max_pages, page ids in range.
+ */
+pic_status_t pic_compose(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
+                         int32_t n_pool_docs, const int32_t *doc_len,
+                         const int32_t *doc_base_pos, const int32_t *req_doc_ids,
+                         const int32_t *req_num_docs, const int32_t *prefix_len,
+                         const int32_t *query_len, const int32_t *block_table,
+                         int32_t max_pages, int64_t num_pages, int32_t max_ctx,
+                         int32_t max_inline, int32_t *doc_offset, int32_t *doc_delta,
+                         int64_t *slot_mapping, int32_t *inline_pos, int32_t *ctx_len,
+                         pic_stream_t stream);
+
+/*
+ * pic_relocate -- key re-rotation and stitching of the cached documents
+ * (Eq. 3; only keys are rotated, values are copied as they are).
+ *
+ * For every layer l in [layer_begin, layer_end), request b, document k and
+ * token j < n of that document (pool id i):
+ *     k_cache[l][slot(offset_k + j)] = R(delta_k) * k_pool[l][start_i + j]
+ *     v_cache[l][slot(offset_k + j)] = v_pool[l][start_i + j]   (bit copy)
+ * where R(delta) rotates each RoPE pair by delta * theta_i (delta is the same
+ * for every token of a document, since base and target both advance by one
+ * per token, so R(b) R(a)^-1 = R(b - a)).  cos/sin come from the angle
+ * delta * theta_i formed and reduced in fp64; the rotation is fp32; K' is
+ * rounded to bf16 (round to nearest even).  delta == 0 reproduces k
+ * bit-exactly.  slot(t) = slot_mapping[b][t] as written by pic_compose.
+ *
+ * Inputs: pool tensors (layout above) with pool_tokens rows per layer;
+ *   doc_token_start int64 [n_pool_docs]; doc_len int32 [n_pool_docs];
+ *   req_doc_ids, doc_offset, doc_delta [batch][max_docs]; req_num_docs [batch];
+ *   slot_mapping int64 [batch][max_ctx].
+ * One launch; no workspace.  max_docs == 0 returns PIC_OK without launching.
+ */
+pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
+                          int32_t n_pool_docs, const void *k_pool, const void *v_pool,
+                          int64_t pool_tokens, const int64_t *doc_token_start,
+                          const int32_t *doc_len, const int32_t *req_doc_ids,
+                          const int32_t *req_num_docs, const int32_t *doc_offset,
+                          const int32_t *doc_delta, const int64_t *slot_mapping,
+                          int32_t max_ctx, int64_t num_pages, void *k_cache, void *v_cache,
+                          int32_t layer_begin, int32_t layer_end, pic_stream_t stream);
+
+/*
+ * Prefill of one layer's inline tokens ("Cache-hit serving": only the
+ * request-specific inline tokens are processed; appendix "Position-Independent
+ * Linking": their KVs are interleaved with the prepared document states, and
+ * a frontier causal mask stops an inline token from attending to any later
+ * logical position).  Two calls, made in this order on the same workspace:
+ *
+ * pic_append_inline -- each inline token t of request b (logical position
+ *   p = inline_pos[b][t], t < inline_len[b]) gets its key R(p) k_new and value
+ *   v_new written to slot(p) = slot_mapping[b][p] of `layer`, and its rotated
+ *   query R(p) q written into the workspace (GQA-packed: the query heads that
+ *   share a kv head are adjacent rows).  One launch.
+ *
+ * pic_attend_prefill -- for every inline token and query head h (kv head
+ *   g = h / G, G = Hq / Hkv):
+ *       out[b][t][h] = sum_{s <= p} softmax_s(q.k_s / sqrt(d)) v_s
+ *   over the keys of logical positions 0..p of the stitched cache of `layer`,
+ *   reading the rotated queries pic_append_inline left in the workspace.
+ *   lse[b][t][h] (nullable) = natural-log sum-exp of those scaled scores.
+ *   Runs on the tensor cores (tcgen05.mma, TMEM accumulators, TMA loads of
+ *   the paged K/V through block_table).  num_splits: key-range splits per
+ *   128-row query tile (0 = automatic); splits are merged by log-sum-exp.
+ *
+ * q: bf16 [batch][max_inline][Hq][d]; k_new, v_new: bf16 [batch][max_inline][Hkv][d]
+ *   (un-rotated projections); inline_pos: int32 [batch][max_inline], ascending
+ *   per request; inline_len: int32 [batch]; slot_mapping: int64 [batch][max_ctx];
+ *   block_table: int32 [batch][max_pages].  Every position must be < max_ctx.
+ * out: bf16 [batch][max_inline][Hq][d]; lse: float [batch][max_inline][Hq] or NULL.
+ * workspace: >= pic_prefill_workspace_size(... num_splits ...) bytes, 256-byte
+ *   aligned, the same buffer for both calls (pic_append_inline only uses its
+ *   leading pic_prefill_workspace_size(..., 1) bytes).
+ */
+size_t pic_prefill_workspace_size(const pic_geom_t *geom, int32_t batch, int32_t max_inline,
+                                  int32_t max_ctx, int32_t num_splits);
+
+/* Split count pic_attend_prefill uses for these sizes (num_splits 0 = its
+ * automatic choice); > 1 means a second (merge) launch.  0 on bad arguments. */
+int32_t pic_prefill_num_splits(const pic_geom_t *geom, int32_t batch, int32_t max_inline,
+                               int32_t max_ctx, int32_t num_splits);
+
+pic_status_t pic_append_inline(const pic_geom_t *geom, int32_t layer, int32_t batch,
+                               int32_t max_inline, const void *q, const void *k_new,
+                               const void *v_new, const int32_t *inline_pos,
+                               const int32_t *inline_len, const int64_t *slot_mapping,
+                               int32_t max_ctx, int64_t num_pages, void *k_cache, void *v_cache,
+                               void *workspace, size_t workspace_bytes, pic_stream_t stream);
+
+pic_status_t pic_attend_prefill(const pic_geom_t *geom, int32_t layer, int32_t batch,
+                                int32_t max_inline, const int32_t *inline_pos,
+                                const int32_t *inline_len, int32_t max_ctx,
+                                const int32_t *block_table, int32_t max_pages, int64_t num_pages,
+                                const void *k_cache, const void *v_cache, void *out, float *lse,
+                                int32_t num_splits, void *workspace, size_t workspace_bytes,
+                                pic_stream_t stream);
+
+/*
+ * pic_attend_decode -- one layer of one plain autoregressive decoding step over
+ * the completed cache (appendix "Position-Independent Linking": after the first
+ * token, generation proceeds as usual on the linked cache).
+ *
+ * For each request b with new-token position p = pos[b] + pos_offset:
+ *   k_cache/v_cache[layer][slot(p)] = R(p) k_new[b], v_new[b];
+ *   out[b][h] = sum_{s <= p} softmax_s(R(p) q[b][h] . k_s / sqrt(d)) v_s.
+ * slot(p) = block_table[b][p / page] * page + p % page.
+ * q: bf16 [batch][Hq][d]; k_new, v_new: bf16 [batch][Hkv][d]; pos: int32 [batch]
+ * (e.g. ctx_len from pic_compose) plus the scalar pos_offset (e.g. the step index);
+ * out: bf16 [batch][Hq][d]; lse: float [batch][Hq] or NULL.
+ * max_ctx: an upper bound on pos[b] + pos_offset + 1 (sizes the grid).
+ * num_splits: key-range splits per (request, kv head) (0 = automatic); the
+ * partial softmax states are merged by log-sum-exp.  Hq / Hkv <= 16.
+ * workspace: >= pic_decode_workspace_size(... same num_splits ...) bytes.
+ */
+size_t pic_decode_workspace_size(const pic_geom_t *geom, int32_t batch, int32_t max_ctx,
+                                 int32_t num_splits);
+
+/* Split count pic_attend_decode uses for these sizes (0 on bad arguments). */
+int32_t pic_decode_num_splits(const pic_geom_t *geom, int32_t batch, int32_t max_ctx,
+                              int32_t num_splits);
+
+pic_status_t pic_attend_decode(const pic_geom_t *geom, int32_t layer, int32_t batch,
+                               const void *q, const void *k_new, const void *v_new,
+                               const int32_t *pos, int32_t pos_offset, const int32_t *block_table,
+                               int32_t max_pages, int64_t num_pages, void *k_cache,
+                               void *v_cache, void *out, float *lse, int32_t max_ctx,
+                               int32_t num_splits, void *workspace, size_t workspace_bytes,
+                               pic_stream_t stream);
+
+#ifdef __cplusplus
+} /* extern "C" */
+#endif
+
+#endif /* PIC_H_ */

@@ -20,8 +20,8 @@ What the path computes (SemPIC, "Background: Position-Independent Caching" and
                          physical paged-cache slots (appendix, "Logical Layout
                          and Re-Rotation").
 2. ``rerotate_key``      moves a key created at position a to position b with
-                         k~_b = R(b) R(a)^-1 k_a (Eq. 3); values are reused
-                         unchanged.
+                         k~_b = R(b) R(a)^-1 k_a (Eq. 3); values are copied
+                         as they are.
 3. ``rotary``            the rotary transform R(p) itself (RoPE, cited by the
                          paper as the positional scheme of the evaluated
                          decoders) used for the inline tokens' own keys and
@@ -103,8 +103,7 @@ def rerotate_key(k: np.ndarray, a, b, theta: np.ndarray, style: str = HALF) -> n
     """Eq. 3: k~_b = R(b) R(a)^-1 k_a, written as the two rotations it names.
 
     R(a)^-1 is the rotation by -a (rotations are orthogonal), then R(b) is
-    applied.  Values are never passed through here: they are reused without
-    rotation.
+    applied.  Only keys go through here; values keep their cached numbers.
     """
     a = np.asarray(a, dtype=np.float64)
     b = np.asarray(b, dtype=np.float64)
@@ -178,7 +177,7 @@ def relocate_docs(layout: RequestLayout, k_docs, v_docs, doc_base_pos, theta, st
         a = doc_base_pos[d] + np.arange(n)
         b = layout.doc_offset[i] + np.arange(n)
         ks.append(rerotate_key(k_docs[i], a[:, None], b[:, None], theta, style))
-        vs.append(np.asarray(v_docs[i], dtype=np.float64))  # reused without rotation
+        vs.append(np.asarray(v_docs[i], dtype=np.float64))  # values are copied, not rotated
     if not ks:
         return None, None
     return np.concatenate(ks, 0), np.concatenate(vs, 0)

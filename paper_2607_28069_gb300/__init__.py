@@ -1,0 +1,272 @@
+"""SemPIC cache-hit path on GB300: thin Python binding of libpic.so.
+
+The functions below carry the names of the C entry points in include/pic.h
+and only marshal arguments (device pointers of torch tensors, sizes, the
+current CUDA stream).  Every step of the path runs in the CUDA kernels of
+libpic.so; if the library is missing, the calls raise -- there is no CPU
+fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import Optional
+
+import torch
+
+__all__ = [
+    "Geometry", "load", "lib_path", "pic_abi_version", "pic_compose", "pic_relocate",
+    "pic_append_inline", "pic_attend_prefill", "pic_prefill_workspace_size",
+    "pic_prefill_num_splits", "pic_decode_num_splits",
+    "pic_attend_decode", "pic_decode_workspace_size", "pic_device_status", "PicError",
+    "EXPORTED_SYMBOLS", "ROPE_HALF", "ROPE_INTERLEAVED",
+]
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(_PKG, "libpic.so")
+_lib = None
+
+ROPE_HALF = 0
+ROPE_INTERLEAVED = 1
+
+# Every symbol include/pic.h declares.
+EXPORTED_SYMBOLS = (
+    "pic_abi_version", "pic_last_error", "pic_device_status", "pic_compose", "pic_relocate",
+    "pic_prefill_workspace_size", "pic_prefill_num_splits", "pic_append_inline",
+    "pic_attend_prefill", "pic_decode_workspace_size", "pic_decode_num_splits",
+    "pic_attend_decode",
+)
+
+DEVICE_CODES = {
+    0: "ok", 1: "bad doc id", 2: "bad doc length", 3: "bad request", 4: "context overflow",
+    5: "block table short", 6: "bad page", 7: "bad position", 8: "timeout",
+}
+
+
+class PicError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"libpic status {status}: {msg}")
+        self.status = status
+
+
+class _Geom(ctypes.Structure):
+    _fields_ = [
+        ("num_layers", ctypes.c_int32), ("num_q_heads", ctypes.c_int32),
+        ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+        ("page_size", ctypes.c_int32), ("rope_style", ctypes.c_int32),
+        ("rope_base", ctypes.c_double), ("inv_freq", ctypes.POINTER(ctypes.c_double)),
+    ]
+
+
+@dataclass
+class Geometry:
+    num_layers: int
+    num_q_heads: int
+    num_kv_heads: int
+    head_dim: int
+    rope_base: float
+    page_size: int = 16
+    rope_style: int = ROPE_HALF
+    inv_freq: Optional[list] = None
+
+    def _c(self):
+        g = _Geom(self.num_layers, self.num_q_heads, self.num_kv_heads, self.head_dim,
+                  self.page_size, self.rope_style, float(self.rope_base), None)
+        if self.inv_freq is not None:
+            arr = (ctypes.c_double * len(self.inv_freq))(*[float(x) for x in self.inv_freq])
+            g.inv_freq = ctypes.cast(arr, ctypes.POINTER(ctypes.c_double))
+            g._keep = arr  # keep the array alive with the struct
+        return g
+
+
+def lib_path() -> str:
+    return _LIB_PATH
+
+
+def load():
+    """Load libpic.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(_LIB_PATH):
+        raise RuntimeError(f"{_LIB_PATH} is missing: run __graft_entry__.build() first")
+    lib = ctypes.CDLL(_LIB_PATH)
+    P, I32, I64, SZ, D = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t, ctypes.c_double
+    G = ctypes.POINTER(_Geom)
+    sig = {
+        "pic_abi_version": (I32, []),
+        "pic_last_error": (ctypes.c_char_p, []),
+        "pic_device_status": (I32, [P, P, P]),
+        "pic_compose": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, I32, I64, I32, I32,
+                              P, P, P, P, P, P]),
+        "pic_relocate": (I32, [G, I32, I32, I32, P, P, I64, P, P, P, P, P, P, P, I32, I64,
+                               P, P, I32, I32, P]),
+        "pic_prefill_workspace_size": (SZ, [G, I32, I32, I32, I32]),
+        "pic_append_inline": (I32, [G, I32, I32, I32, P, P, P, P, P, P, I32, I64, P, P, P, SZ,
+                                    P]),
+        "pic_attend_prefill": (I32, [G, I32, I32, I32, P, P, I32, P, I32, I64, P, P, P, P, I32,
+                                     P, SZ, P]),
+        "pic_decode_workspace_size": (SZ, [G, I32, I32, I32]),
+        "pic_prefill_num_splits": (I32, [G, I32, I32, I32, I32]),
+        "pic_decode_num_splits": (I32, [G, I32, I32, I32]),
+        "pic_attend_decode": (I32, [G, I32, I32, P, P, P, P, I32, P, I32, I64, P, P, P, P, I32, I32,
+                                    P, SZ, P]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    del D
+    _lib = lib
+    return lib
+
+
+def _check(status: int, what: str):
+    if status != 0:
+        msg = _lib.pic_last_error().decode(errors="replace")
+        raise PicError(status, f"{what}: {msg}")
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _ptr(t: Optional[torch.Tensor], dtype, name: str, allow_none=False):
+    if t is None:
+        if allow_none:
+            return None
+        raise ValueError(f"{name} is required")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+bf16, i32, i64, f32 = torch.bfloat16, torch.int32, torch.int64, torch.float32
+
+
+def pic_abi_version() -> int:
+    return load().pic_abi_version()
+
+
+def pic_device_status(stream=None):
+    """(code, detail) of the first device-side failure since the last read; clears it."""
+    lib = load()
+    code, detail = ctypes.c_int32(0), ctypes.c_int32(0)
+    st = lib.pic_device_status(_stream(stream), ctypes.byref(code), ctypes.byref(detail))
+    if st not in (0, 5):
+        _check(st, "pic_device_status")
+    return code.value, detail.value
+
+
+def pic_compose(geom: Geometry, doc_len, doc_base_pos, req_doc_ids, req_num_docs, prefix_len,
+                query_len, block_table, num_pages: int, max_ctx: int, max_inline: int,
+                doc_offset, doc_delta, slot_mapping, inline_pos, ctx_len, stream=None):
+    lib = load()
+    g = geom._c()
+    B, max_docs = req_doc_ids.shape
+    st = lib.pic_compose(
+        ctypes.byref(g), B, max_docs, doc_len.numel(), _ptr(doc_len, i32, "doc_len"),
+        _ptr(doc_base_pos, i32, "doc_base_pos"), _ptr(req_doc_ids, i32, "req_doc_ids"),
+        _ptr(req_num_docs, i32, "req_num_docs"), _ptr(prefix_len, i32, "prefix_len"),
+        _ptr(query_len, i32, "query_len"), _ptr(block_table, i32, "block_table"),
+        block_table.shape[1], num_pages, max_ctx, max_inline,
+        _ptr(doc_offset, i32, "doc_offset"), _ptr(doc_delta, i32, "doc_delta"),
+        _ptr(slot_mapping, i64, "slot_mapping"), _ptr(inline_pos, i32, "inline_pos"),
+        _ptr(ctx_len, i32, "ctx_len"), _stream(stream))
+    _check(st, "pic_compose")
+
+
+def pic_relocate(geom: Geometry, k_pool, v_pool, doc_token_start, doc_len, req_doc_ids,
+                 req_num_docs, doc_offset, doc_delta, slot_mapping, num_pages: int, k_cache,
+                 v_cache, layer_begin: int, layer_end: int, stream=None):
+    lib = load()
+    g = geom._c()
+    B, max_docs = req_doc_ids.shape
+    st = lib.pic_relocate(
+        ctypes.byref(g), B, max_docs, doc_len.numel(), _ptr(k_pool, bf16, "k_pool"),
+        _ptr(v_pool, bf16, "v_pool"), k_pool.shape[1],
+        _ptr(doc_token_start, i64, "doc_token_start"), _ptr(doc_len, i32, "doc_len"),
+        _ptr(req_doc_ids, i32, "req_doc_ids"), _ptr(req_num_docs, i32, "req_num_docs"),
+        _ptr(doc_offset, i32, "doc_offset"), _ptr(doc_delta, i32, "doc_delta"),
+        _ptr(slot_mapping, i64, "slot_mapping"), slot_mapping.shape[1], num_pages,
+        _ptr(k_cache, bf16, "k_cache"), _ptr(v_cache, bf16, "v_cache"), layer_begin, layer_end,
+        _stream(stream))
+    _check(st, "pic_relocate")
+
+
+def pic_prefill_workspace_size(geom: Geometry, batch: int, max_inline: int, max_ctx: int,
+                               num_splits: int = 0) -> int:
+    g = geom._c()
+    return load().pic_prefill_workspace_size(ctypes.byref(g), batch, max_inline, max_ctx,
+                                             num_splits)
+
+
+def pic_prefill_num_splits(geom: Geometry, batch: int, max_inline: int, max_ctx: int,
+                           num_splits: int = 0) -> int:
+    g = geom._c()
+    return load().pic_prefill_num_splits(ctypes.byref(g), batch, max_inline, max_ctx, num_splits)
+
+
+def pic_decode_num_splits(geom: Geometry, batch: int, max_ctx: int, num_splits: int = 0) -> int:
+    g = geom._c()
+    return load().pic_decode_num_splits(ctypes.byref(g), batch, max_ctx, num_splits)
+
+
+def pic_append_inline(geom: Geometry, layer: int, q, k_new, v_new, inline_pos, inline_len,
+                      slot_mapping, num_pages: int, k_cache, v_cache, workspace, stream=None):
+    lib = load()
+    g = geom._c()
+    B, max_inline = inline_pos.shape
+    st = lib.pic_append_inline(
+        ctypes.byref(g), layer, B, max_inline, _ptr(q, bf16, "q"), _ptr(k_new, bf16, "k_new"),
+        _ptr(v_new, bf16, "v_new"), _ptr(inline_pos, i32, "inline_pos"),
+        _ptr(inline_len, i32, "inline_len"), _ptr(slot_mapping, i64, "slot_mapping"),
+        slot_mapping.shape[1], num_pages, _ptr(k_cache, bf16, "k_cache"),
+        _ptr(v_cache, bf16, "v_cache"), _ptr(workspace, torch.uint8, "workspace"),
+        workspace.numel(), _stream(stream))
+    _check(st, "pic_append_inline")
+
+
+def pic_attend_prefill(geom: Geometry, layer: int, inline_pos, inline_len, max_ctx: int,
+                       block_table, num_pages: int, k_cache, v_cache, out, lse=None,
+                       num_splits: int = 0, workspace=None, stream=None):
+    lib = load()
+    g = geom._c()
+    B, max_inline = inline_pos.shape
+    st = lib.pic_attend_prefill(
+        ctypes.byref(g), layer, B, max_inline, _ptr(inline_pos, i32, "inline_pos"),
+        _ptr(inline_len, i32, "inline_len"), max_ctx, _ptr(block_table, i32, "block_table"),
+        block_table.shape[1], num_pages, _ptr(k_cache, bf16, "k_cache"),
+        _ptr(v_cache, bf16, "v_cache"), _ptr(out, bf16, "out"),
+        _ptr(lse, f32, "lse", allow_none=True), num_splits,
+        _ptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream))
+    _check(st, "pic_attend_prefill")
+
+
+def pic_decode_workspace_size(geom: Geometry, batch: int, max_ctx: int, num_splits: int = 0) -> int:
+    g = geom._c()
+    return load().pic_decode_workspace_size(ctypes.byref(g), batch, max_ctx, num_splits)
+
+
+def pic_attend_decode(geom: Geometry, layer: int, q, k_new, v_new, pos, block_table,
+                      num_pages: int, k_cache, v_cache, out, max_ctx: int, lse=None,
+                      num_splits: int = 0, workspace=None, pos_offset: int = 0, stream=None):
+    lib = load()
+    g = geom._c()
+    B = pos.numel()
+    st = lib.pic_attend_decode(
+        ctypes.byref(g), layer, B, _ptr(q, bf16, "q"), _ptr(k_new, bf16, "k_new"),
+        _ptr(v_new, bf16, "v_new"), _ptr(pos, i32, "pos"), pos_offset,
+        _ptr(block_table, i32, "block_table"),
+        block_table.shape[1], num_pages, _ptr(k_cache, bf16, "k_cache"),
+        _ptr(v_cache, bf16, "v_cache"), _ptr(out, bf16, "out"),
+        _ptr(lse, f32, "lse", allow_none=True), max_ctx, num_splits,
+        _ptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream))
+    _check(st, "pic_attend_decode")

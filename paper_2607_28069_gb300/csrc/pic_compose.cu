@@ -1,0 +1,192 @@
+// pic_compose: the link operator's logical layout and slot map.
+//
+// SemPIC, "Background: Position-Independent Caching" (Eqs. 1-2): a request is
+// P, D_1..D_m, Q in canonical order and the link operator R assigns each
+// prepared document its final logical positions; appendix "Logical Layout and
+// Re-Rotation": at link time each logical prompt position is tied to the
+// physical cache slot that holds it.
+//
+// One grid row per request.  Every CTA of a row re-derives the document
+// offsets with a block-wide prefix sum over the document lengths (loaded in
+// parallel), then fills its 4096-position slice of the slot map.  Only the
+// first CTA of a row writes the per-document outputs, the inline positions and
+// ctx_len, and records device-side check failures.
+#include "pic_internal.cuh"
+
+namespace pic {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kSlotsPerCta = 4096;
+
+struct ComposeArgs {
+  int batch, max_docs, n_pool, max_pages, max_ctx, max_inline, page;
+  long long num_pages;
+  const int32_t *doc_len, *doc_base, *ids, *num_docs, *prefix, *query, *block_table;
+  int32_t *doc_offset, *doc_delta, *inline_pos, *ctx_len;
+  int64_t *slot_mapping;
+  int32_t *status;
+};
+
+// Inclusive block scan of one value per thread (kThreads threads).
+__device__ long long block_inclusive_scan(long long v, long long *warp_tot) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    long long t = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v += t;
+  }
+  if (lane == 31) warp_tot[warp] = v;
+  __syncthreads();
+  long long add = 0;
+  for (int w = 0; w < warp; ++w) add += warp_tot[w];
+  __syncthreads();
+  return v + add;
+}
+
+__global__ void __launch_bounds__(kThreads) compose_kernel(ComposeArgs a) {
+  const int b = blockIdx.y;
+  const int tid = threadIdx.x;
+  const bool lead = blockIdx.x == 0;
+  __shared__ long long warp_tot[kThreads / 32];
+  __shared__ long long s_carry;
+  __shared__ int s_err, s_err_detail;
+  if (tid == 0) {
+    s_carry = 0;
+    s_err = 0;
+    s_err_detail = b;
+  }
+  __syncthreads();
+
+  const int P = a.prefix[b], Tq = a.query[b], m = a.num_docs[b];
+  if (P < 0 || Tq < 0 || m < 0 || m > a.max_docs) {
+    if (lead && tid == 0) {
+      dev_fail(a.status, PIC_DEV_BAD_REQUEST, b);
+      a.ctx_len[b] = -1;
+    }
+    return;
+  }
+
+  for (int k0 = 0; k0 < m; k0 += kThreads) {
+    const int k = k0 + tid;
+    long long n = 0, base = 0;
+    if (k < m) {
+      const int id = a.ids[(size_t)b * a.max_docs + k];
+      if (id < 0 || id >= a.n_pool) {
+        atomicCAS(&s_err, 0, PIC_DEV_BAD_DOC_ID);
+      } else {
+        n = a.doc_len[id];
+        base = a.doc_base[id];
+        if (n <= 0) {
+          atomicCAS(&s_err, 0, PIC_DEV_BAD_DOC_LEN);
+          n = 0;
+        }
+      }
+    }
+    const long long incl = block_inclusive_scan(n, warp_tot);
+    const long long off = P + s_carry + incl - n;
+    if (lead && k < m) {
+      a.doc_offset[(size_t)b * a.max_docs + k] = (int32_t)off;
+      a.doc_delta[(size_t)b * a.max_docs + k] = (int32_t)(off - base);
+    }
+    __syncthreads();
+    if (tid == kThreads - 1) s_carry += incl;
+    __syncthreads();
+  }
+  if (lead)
+    for (int k = m + tid; k < a.max_docs; k += kThreads) {
+      a.doc_offset[(size_t)b * a.max_docs + k] = -1;
+      a.doc_delta[(size_t)b * a.max_docs + k] = 0;
+    }
+
+  const long long ctx = (long long)P + s_carry + Tq;
+  if (tid == 0) {
+    if (ctx > a.max_ctx || P + Tq > a.max_inline) atomicCAS(&s_err, 0, PIC_DEV_CTX_OVERFLOW);
+    else if ((ctx + a.page - 1) / a.page > a.max_pages)
+      atomicCAS(&s_err, 0, PIC_DEV_BLOCK_TABLE_SHORT);
+  }
+  __syncthreads();
+  const int err = s_err;
+
+  // Slot map slice of this CTA (positions beyond ctx get -1).
+  const long long t_begin = (long long)blockIdx.x * kSlotsPerCta;
+  const long long t_end = min((long long)a.max_ctx, t_begin + kSlotsPerCta);
+  int64_t *slots = a.slot_mapping + (size_t)b * a.max_ctx;
+  const int32_t *bt = a.block_table + (size_t)b * a.max_pages;
+  for (long long t = t_begin + tid; t < t_end; t += kThreads) {
+    long long s = -1;
+    if (!err && t < ctx) {
+      const int page = bt[t / a.page];
+      if (page < 0 || page >= a.num_pages) atomicCAS(&s_err, 0, PIC_DEV_BAD_PAGE);
+      else s = (long long)page * a.page + t % a.page;
+    }
+    slots[t] = s;
+  }
+  if (lead) {
+    int32_t *ip = a.inline_pos + (size_t)b * a.max_inline;
+    for (int i = tid; i < a.max_inline; i += kThreads) {
+      int v = -1;
+      if (!err && i < P) v = i;
+      else if (!err && i < P + Tq) v = (int)(ctx - Tq + (i - P));
+      ip[i] = v;
+    }
+  }
+  __syncthreads();
+  if (tid == 0 && s_err) dev_fail(a.status, s_err, s_err_detail);
+  if (lead && tid == 0) a.ctx_len[b] = s_err ? -1 : (int32_t)ctx;
+}
+
+}  // namespace
+}  // namespace pic
+
+extern "C" pic_status_t pic_compose(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
+                                    int32_t n_pool_docs, const int32_t *doc_len,
+                                    const int32_t *doc_base_pos, const int32_t *req_doc_ids,
+                                    const int32_t *req_num_docs, const int32_t *prefix_len,
+                                    const int32_t *query_len, const int32_t *block_table,
+                                    int32_t max_pages, int64_t num_pages, int32_t max_ctx,
+                                    int32_t max_inline, int32_t *doc_offset, int32_t *doc_delta,
+                                    int64_t *slot_mapping, int32_t *inline_pos, int32_t *ctx_len,
+                                    pic_stream_t stream) {
+  using namespace pic;
+  double theta[kMaxHalfDim];
+  pic_status_t st = check_geom(geom, theta);
+  if (st != PIC_OK) return st;
+  if (batch <= 0 || max_docs < 0 || n_pool_docs < 0 || max_pages <= 0 || num_pages <= 0 ||
+      max_ctx <= 0 || max_inline <= 0)
+    return fail(PIC_ERR_INVALID_ARG, "pic_compose: sizes must be positive");
+  if (num_pages > (int64_t)INT32_MAX)
+    return fail(PIC_ERR_INVALID_ARG, "pic_compose: num_pages exceeds int32");
+  if (!doc_len || !doc_base_pos || !req_num_docs || !prefix_len || !query_len || !block_table ||
+      !slot_mapping || !inline_pos || !ctx_len || (max_docs > 0 && (!req_doc_ids || !doc_offset || !doc_delta)))
+    return fail(PIC_ERR_INVALID_ARG, "pic_compose: NULL tensor");
+  int32_t *status = device_status_ptr();
+  if (!status) return fail(PIC_ERR_CUDA, "pic_compose: no device status word");
+  ComposeArgs a;
+  a.batch = batch;
+  a.max_docs = max_docs;
+  a.n_pool = n_pool_docs;
+  a.max_pages = max_pages;
+  a.max_ctx = max_ctx;
+  a.max_inline = max_inline;
+  a.page = geom->page_size;
+  a.num_pages = num_pages;
+  a.doc_len = doc_len;
+  a.doc_base = doc_base_pos;
+  a.ids = req_doc_ids;
+  a.num_docs = req_num_docs;
+  a.prefix = prefix_len;
+  a.query = query_len;
+  a.block_table = block_table;
+  a.doc_offset = doc_offset;
+  a.doc_delta = doc_delta;
+  a.inline_pos = inline_pos;
+  a.ctx_len = ctx_len;
+  a.slot_mapping = slot_mapping;
+  a.status = status;
+  dim3 grid((max_ctx + kSlotsPerCta - 1) / kSlotsPerCta, batch);
+  compose_kernel<<<grid, kThreads, 0, stream>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "pic_compose launch");
+  return PIC_OK;
+}

@@ -1,0 +1,680 @@
+// pic_attend_prefill: inline-token prefill over the stitched cache.
+//
+// SemPIC, "Cache-hit serving": a cache hit processes only the request-specific
+// inline tokens through the unchanged decoder; appendix "Position-Independent
+// Linking": inline KVs are interleaved with the prepared document states and a
+// frontier causal mask keeps every inline token from seeing logical
+// successors.  The Reader is the frozen base model (Eq. 7), so its attention is
+// ordinary GQA softmax attention with scale 1/sqrt(d).
+//
+// pic_append_inline (one layer, one launch): append_kernel applies RoPE to
+//     each inline key at its logical position and writes it with its value
+//     to the paged cache, and writes the rotated queries into a GQA-packed
+//     workspace [B][Hkv][rows][d] whose row r of kv head g is query head
+//     g*G + r % G of inline token r / G.  One 128-row tile therefore holds
+//     every query head that shares a K/V tile.
+// pic_attend_prefill (one layer):
+//  1. attn_kernel: one CTA per (128-row query tile, key split, kv head,
+//     request).  Warp-specialised: warp 0 issues TMA loads (Q once, then
+//     128-key K and V tiles page by page from the paged cache through the
+//     block table, 3-stage ring), warp 1 issues tcgen05.mma (S = Q K^T into
+//     TMEM, then O += P V with P read from TMEM), warps 2-5 run the online
+//     softmax on S rows straight from TMEM (one thread per row), write P back
+//     to TMEM as bf16 over S, rescale O only when the running maximum grew by
+//     more than 2^8, and finally normalise O.  Scores are kept in the log2
+//     domain (scale folded with log2 e) and exponentiated with ex2.approx.
+//  2. combine_kernel (only when the key range is split): log-sum-exp merge of
+//     the per-split partial (O, m, l).
+#include "pic_internal.cuh"
+
+namespace pic {
+namespace prefill {
+
+constexpr int BM = 128;  // query rows per tile (TMEM lanes)
+constexpr int BN = 128;  // keys per KV tile
+constexpr int NST = 3;   // K/V ring stages
+constexpr int kThreads = 192;
+constexpr int kMaxSplits = 32;
+constexpr uint32_t kTmemCols = 512;
+
+template <int D>
+struct Layout {
+  static constexpr int kTile = BN * D * 2;  // bytes of one K or V tile
+  static constexpr int kQ = 0;
+  static constexpr int kK = kQ + BM * D * 2;
+  static constexpr int kV = kK + NST * kTile;
+  static constexpr int kBar = kV + NST * kTile;
+  static constexpr int kBytes = kBar + 256;
+  static constexpr int kAlloc = kBytes + 1024;  // slack for 1024-byte alignment
+};
+
+// mbarrier slots (8 bytes each) inside the barrier area
+enum {
+  B_Q = 0,
+  B_KFULL = 1,
+  B_VFULL = B_KFULL + NST,
+  B_KVEMPTY = B_VFULL + NST,
+  B_SFULL = B_KVEMPTY + NST,
+  B_PFULL = B_SFULL + 2,
+  B_PFREE = B_PFULL + 2,
+  B_OFINAL = B_PFREE + 2,
+  B_COUNT = B_OFINAL + 1
+};
+
+struct Params {
+  int Hq, Hkv, G, max_inline, R_pad, m_tiles, num_splits, max_pages, oob_row;
+  long long num_pages, layer_row0;
+  const int32_t *inline_pos, *inline_len, *block_table;
+  __nv_bfloat16 *out;
+  float *lse, *part_o, *part_ml;
+  int32_t *status;
+  float scale_log2;
+};
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                const __grid_constant__ CUtensorMap tm_v, Params p) {
+  using L = Layout<D>;
+  constexpr int PANELS = D / 64;
+  constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
+  constexpr uint32_t IDESC_PV = idesc_bf16(BM, D, false, true);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                              ~(uintptr_t)1023);
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t bar0 = sbase + L::kBar;
+  auto bar = [&](int i) { return bar0 + 8u * (uint32_t)i; };
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + L::kBar + 8 * B_COUNT);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::kBar + 8 * B_COUNT + 8);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int mt = blockIdx.x / p.num_splits, split = blockIdx.x % p.num_splits;
+  const int hk = blockIdx.y, b = blockIdx.z;
+  const int detail = b;
+
+  // ---- work of this CTA (uniform across threads)
+  const int tin = min(max(p.inline_len[b], 0), p.max_inline);
+  const int rows = tin * p.G;
+  const int r0 = mt * BM;
+  if (r0 >= rows) return;  // no query row in this tile
+  const int r_last = min(r0 + BM, rows) - 1;
+  const int32_t *ipos = p.inline_pos + (size_t)b * p.max_inline;
+  const int kmin = ipos[r0 / p.G];
+  const int kmax = ipos[r_last / p.G];
+  const int n_kv_all = kmax >= 0 ? kmax / BN + 1 : 0;
+  const int per = (n_kv_all + p.num_splits - 1) / p.num_splits;
+  const int kv_begin = split * per;
+  const int n = max(0, min(per, n_kv_all - kv_begin));
+  const size_t part_row0 =
+      ((((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * p.num_splits + split) * BM;
+
+  if (n == 0) {  // empty split: neutral partial state
+    if (p.num_splits > 1 && threadIdx.x < BM) {
+      p.part_ml[(part_row0 + threadIdx.x) * 2] = -INFINITY;
+      p.part_ml[(part_row0 + threadIdx.x) * 2 + 1] = 0.f;
+    }
+    return;
+  }
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < B_COUNT; ++i) mbar_init(bar(i), (i == B_PFULL || i == B_PFULL + 1) ? 128 : 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = *tmem_slot;
+
+  if (warp == 0) {
+    // ===================================================== TMA producer
+    if (lane == 0) {
+      prefetch_tmap(&tm_q);
+      prefetch_tmap(&tm_k);
+      prefetch_tmap(&tm_v);
+      mbar_expect_tx(bar(B_Q), BM * D * 2);
+      const int qrow = (b * p.Hkv + hk) * p.R_pad + r0;
+      for (int pn = 0; pn < PANELS; ++pn)
+        tma_load_2d(sbase + L::kQ + pn * BM * 128, &tm_q, pn * 64, qrow, bar(B_Q));
+      const int32_t *bt = p.block_table + (size_t)b * p.max_pages;
+      int issued = 0;
+      for (int j = 0; j < n; ++j) {
+        const int st = j % NST;
+        if (j >= NST && !mbar_wait(bar(B_KVEMPTY + st), ((j / NST) - 1) & 1, abort_flag, p.status, detail))
+          break;
+        const int kt = kv_begin + j;
+        int ys[8];
+#pragma unroll
+        for (int pg = 0; pg < 8; ++pg) {
+          const int pidx = kt * 8 + pg;
+          int y = p.oob_row;
+          if (pidx * 16 <= kmax && pidx < p.max_pages) {
+            const int page = bt[pidx];
+            if (page >= 0 && page < p.num_pages)
+              y = (int)(p.layer_row0 + ((long long)page * p.Hkv + hk) * 16);
+            else
+              dev_fail(p.status, PIC_DEV_BAD_PAGE, detail);
+          }
+          ys[pg] = y;
+        }
+        mbar_expect_tx(bar(B_KFULL + st), L::kTile);
+#pragma unroll
+        for (int pg = 0; pg < 8; ++pg)
+          for (int pn = 0; pn < PANELS; ++pn)
+            tma_load_2d(sbase + L::kK + st * L::kTile + pn * BN * 128 + pg * 16 * 128, &tm_k,
+                        pn * 64, ys[pg], bar(B_KFULL + st));
+        mbar_expect_tx(bar(B_VFULL + st), L::kTile);
+#pragma unroll
+        for (int pg = 0; pg < 8; ++pg)
+          for (int pn = 0; pn < PANELS; ++pn)
+            tma_load_2d(sbase + L::kV + st * L::kTile + pn * BN * 128 + pg * 16 * 128, &tm_v,
+                        pn * 64, ys[pg], bar(B_VFULL + st));
+        issued = j + 1;
+      }
+      if (*abort_flag) {
+        // Let the copies already issued land before the CTA exits.
+        for (int j = max(0, issued - NST); j < issued; ++j) {
+          mbar_wait(bar(B_KFULL + j % NST), (j / NST) & 1, abort_flag, p.status, detail);
+          mbar_wait(bar(B_VFULL + j % NST), (j / NST) & 1, abort_flag, p.status, detail);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ===================================================== MMA issuer
+    if (lane == 0) {
+      const uint32_t tS0 = tbase, tO = tbase + 256;
+      bool ok = mbar_wait(bar(B_Q), 0, abort_flag, p.status, detail);
+      tc_fence_after();
+      for (int j = 0; ok && j <= n; ++j) {
+        if (j < n) {
+          const int st = j % NST, sb = j & 1;
+          if (!mbar_wait(bar(B_KFULL + st), (j / NST) & 1, abort_flag, p.status, detail)) break;
+          tc_fence_after();
+          const uint32_t kb = sbase + L::kK + st * L::kTile;
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * (BM * 128) + (kk & 3) * 32;
+            mma_ss(tS0 + sb * 128, sdesc_sw128(sbase + L::kQ + off, 16, 1024),
+                   sdesc_sw128(kb + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024), IDESC_QK,
+                   kk > 0);
+          }
+          mma_commit(bar(B_SFULL + sb));
+        }
+        if (j >= 1) {
+          const int pj = j - 1, pst = pj % NST, pb = pj & 1;
+          if (!mbar_wait(bar(B_PFULL + pb), (pj >> 1) & 1, abort_flag, p.status, detail)) break;
+          if (!mbar_wait(bar(B_VFULL + pst), (pj / NST) & 1, abort_flag, p.status, detail)) break;
+          tc_fence_after();
+          const uint32_t vb = sbase + L::kV + pst * L::kTile;
+#pragma unroll
+          for (int kk = 0; kk < BN / 16; ++kk)
+            mma_ts(tO, tS0 + pb * 128 + kk * 8, sdesc_sw128(vb + kk * 16 * 128, BN * 128, 1024),
+                   IDESC_PV, (pj > 0 || kk > 0));
+          mma_commit(bar(B_KVEMPTY + pst));
+          mma_commit(bar(B_PFREE + pb));
+        }
+      }
+      mma_commit(bar(B_OFINAL));
+    }
+  } else {
+    // ===================================================== softmax warps
+    const int wq = warp & 3;
+    const int row = wq * 32 + lane;
+    const int rg = r0 + row;
+    const bool valid = rg < rows;
+    const int tok = rg / p.G, g = rg % p.G;
+    const int pos = valid ? ipos[tok] : -1;
+    const uint32_t tl = tbase + ((uint32_t)(wq * 32) << 16);
+    float m_used = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < n; ++j) {
+      const int sb = j & 1;
+      const int key0 = (kv_begin + j) * BN;
+      if (!__all_sync(0xffffffffu, mbar_wait(bar(B_SFULL + sb), (j >> 1) & 1, abort_flag, p.status, detail))) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      float s[BN];
+#pragma unroll
+      for (int c = 0; c < BN / 32; ++c) tmem_ld32(tl + sb * 128 + c * 32, reinterpret_cast<uint32_t *>(s + c * 32));
+      tmem_wait_ld();
+      if (key0 + BN - 1 > kmin) {  // some key of the tile lies beyond some row
+#pragma unroll
+        for (int c = 0; c < BN; ++c)
+          if (key0 + c > pos) s[c] = -INFINITY;
+      }
+      float mx = s[0];
+#pragma unroll
+      for (int c = 1; c < BN; ++c) mx = fmaxf(mx, s[c]);
+      const float m_new = fmaxf(m_used, mx * p.scale_log2);
+      float alpha = 1.f;
+      const bool resc = m_new > m_used + 8.f;
+      if (resc) {
+        alpha = ex2(m_used - m_new);
+        m_used = m_new;
+      }
+      const float mref = (m_used == -INFINITY) ? 0.f : m_used;
+      l *= alpha;
+      uint32_t pk[BN / 2];
+#pragma unroll
+      for (int c = 0; c < BN; c += 2) {
+        const float p0 = ex2(fmaf(s[c], p.scale_log2, -mref));
+        const float p1 = ex2(fmaf(s[c + 1], p.scale_log2, -mref));
+        l += p0 + p1;
+        pk[c / 2] = pack2(p0, p1);
+      }
+      // O correction, only when some row of this warp moved its maximum.
+      if (j > 0 && __any_sync(0xffffffffu, resc)) {
+        const int pj = j - 1;
+        if (!__all_sync(0xffffffffu, mbar_wait(bar(B_PFREE + (pj & 1)), (pj >> 1) & 1, abort_flag, p.status, detail))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+          float o[32];
+          tmem_ld32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o));
+          tmem_wait_ld();
+#pragma unroll
+          for (int q = 0; q < 32; ++q) o[q] *= alpha;
+          tmem_st32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o));
+        }
+      }
+      tmem_st32(tl + sb * 128, pk);
+      tmem_st32(tl + sb * 128 + 32, pk + 32);
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(bar(B_PFULL + sb));
+    }
+    // ---- epilogue
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_OFINAL), 0, abort_flag, p.status, detail));
+    tc_fence_after();
+    if (ok) {
+      if (p.num_splits == 1) {
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+        __nv_bfloat16 *dst = p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D;
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+          float o[32];
+          tmem_ld32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o));
+          tmem_wait_ld();
+          if (valid) {
+#pragma unroll
+            for (int q = 0; q < 32; ++q) o[q] *= inv;
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              st_global16(dst + c * 32 + q * 8, pack8(o + q * 8));
+          }
+        }
+        if (valid && p.lse)
+          p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
+              l > 0.f ? (m_used + __log2f(l)) * 0.69314718055994531f : -INFINITY;
+      } else {
+        float *dst = p.part_o + (part_row0 + row) * D;
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+          float o[32];
+          tmem_ld32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o));
+          tmem_wait_ld();
+          if (valid) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              reinterpret_cast<float4 *>(dst + c * 32)[q] =
+                  make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+          }
+        }
+        p.part_ml[(part_row0 + row) * 2] = (l > 0.f) ? m_used : -INFINITY;
+        p.part_ml[(part_row0 + row) * 2 + 1] = l;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    if (*abort_flag && lane == 0) {
+      // make sure no MMA is still running on the TMEM we are about to free
+      mbar_wait(bar(B_OFINAL), 0, abort_flag, p.status, detail);
+    }
+    __syncwarp();
+    tmem_dealloc(tbase, kTmemCols);
+  }
+}
+
+// Merge split partials (O unnormalised, m in log2 units, l) by log-sum-exp.
+template <int D>
+__global__ void combine_kernel(Params p) {
+  const int mt = blockIdx.x, hk = blockIdx.y, b = blockIdx.z;
+  const int tin = min(max(p.inline_len[b], 0), p.max_inline);
+  const int rows = tin * p.G;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int S = p.num_splits;
+  for (int row = warp; row < BM; row += blockDim.x >> 5) {
+    const int rg = mt * BM + row;
+    if (rg >= rows) break;
+    const size_t base = (((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * S;
+    float ms = -INFINITY, ls = 0.f;
+    if (lane < S) {
+      ms = p.part_ml[((base + lane) * BM + row) * 2];
+      ls = p.part_ml[((base + lane) * BM + row) * 2 + 1];
+    }
+    float M = ms;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    const float w = (ms == -INFINITY) ? 0.f : ex2(ms - M);
+    float Lsum = w * ls;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, o);
+    float acc[D / 32];
+#pragma unroll
+    for (int q = 0; q < D / 32; ++q) acc[q] = 0.f;
+    for (int s = 0; s < S; ++s) {
+      const float ws = __shfl_sync(0xffffffffu, w, s);
+      if (ws == 0.f) continue;
+      const float *src = p.part_o + ((base + s) * BM + row) * D;
+#pragma unroll
+      for (int q = 0; q < D / 32; ++q) acc[q] = fmaf(ws, src[q * 32 + lane], acc[q]);
+    }
+    const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
+    const int tok = rg / p.G, g = rg % p.G;
+    __nv_bfloat16 *dst = p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D;
+#pragma unroll
+    for (int q = 0; q < D / 32; ++q) dst[q * 32 + lane] = __float2bfloat16_rn(acc[q] * inv);
+    if (p.lse && lane == 0)
+      p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
+          Lsum > 0.f ? (M + __log2f(Lsum)) * 0.69314718055994531f : -INFINITY;
+  }
+}
+
+// RoPE the inline keys/queries at their logical positions; keys and values go
+// to their cache slots, queries to the GQA-packed workspace.
+struct AppendArgs {
+  int Hq, Hkv, G, max_inline, max_ctx, R_pad;
+  long long num_pages;
+  const __nv_bfloat16 *q, *k, *v;
+  const int32_t *inline_pos, *inline_len;
+  const int64_t *slots;
+  __nv_bfloat16 *k_cache, *v_cache, *qpack;  // cache pointers already at the layer
+  int32_t *status;
+};
+
+template <int D>
+__global__ void __launch_bounds__(128) append_kernel(AppendArgs a, RopeParams rp) {
+  constexpr int HALF = D / 2, KC = D / 16, VC = D / 8;
+  const int t = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
+  const int tin = min(max(a.inline_len[b], 0), a.max_inline);
+  __shared__ float2 cs[HALF];
+  if (t >= tin) {  // zero the packed query rows of this token slot
+    for (int e = tid; e < a.Hkv * a.G * VC; e += blockDim.x) {
+      const int hk = e / (a.G * VC), r = e % (a.G * VC), g = r / VC, c = r % VC;
+      const int row = t * a.G + g;
+      if (row < a.R_pad)
+        st_global16(a.qpack + (((size_t)b * a.Hkv + hk) * a.R_pad + row) * D + c * 8,
+                    make_uint4(0, 0, 0, 0));
+    }
+    return;
+  }
+  const int pos = a.inline_pos[(size_t)b * a.max_inline + t];
+  const bool pos_ok = pos >= 0 && pos < a.max_ctx;
+  long long slot = pos_ok ? a.slots[(size_t)b * a.max_ctx + pos] : -1;
+  if (!pos_ok) {
+    if (tid == 0) dev_fail(a.status, PIC_DEV_BAD_POSITION, b);
+  } else if (slot < 0 || slot >= a.num_pages * 16) {
+    if (tid == 0) dev_fail(a.status, PIC_DEV_BAD_PAGE, b);
+    slot = -1;
+  }
+  for (int i = tid; i < HALF; i += blockDim.x) cs[i] = rope_cos_sin(pos_ok ? pos : 0, rp.theta[i]);
+  __syncthreads();
+  const size_t tok = (size_t)b * a.max_inline + t;
+  if (slot >= 0) {
+    const long long page = slot >> 4, r = slot & 15;
+    for (int e = tid; e < a.Hkv * KC; e += blockDim.x) {
+      const int h = e / KC, c = e % KC;
+      rotate_chunk(a.k + (tok * a.Hkv + h) * D, a.k_cache + ((page * a.Hkv + h) * 16 + r) * D, c,
+                   HALF, rp.style, cs + 8 * c, true);
+    }
+    for (int e = tid; e < a.Hkv * VC; e += blockDim.x) {
+      const int h = e / VC, c = e % VC;
+      st_global16(a.v_cache + ((page * a.Hkv + h) * 16 + r) * D + c * 8,
+                  ld_stream(a.v + (tok * a.Hkv + h) * D + c * 8));
+    }
+  }
+  for (int e = tid; e < a.Hq * KC; e += blockDim.x) {
+    const int h = e / KC, c = e % KC;
+    const int hk = h / a.G, g = h % a.G;
+    const int row = t * a.G + g;
+    rotate_chunk(a.q + (tok * a.Hq + h) * D, a.qpack + (((size_t)b * a.Hkv + hk) * a.R_pad + row) * D,
+                 c, HALF, rp.style, cs + 8 * c, true);
+  }
+}
+
+struct Plan {
+  int G, m_tiles, R_pad, splits;
+  size_t q_bytes, po_bytes, pml_bytes, total;
+};
+
+inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+inline Plan plan(const pic_geom_t *g, int batch, int max_inline, int max_ctx, int num_splits) {
+  Plan pl;
+  pl.G = g->num_q_heads / g->num_kv_heads;
+  pl.m_tiles = (int)(((long long)max_inline * pl.G + BM - 1) / BM);
+  pl.R_pad = pl.m_tiles * BM;
+  const int kv_tiles = (max_ctx + BN - 1) / BN;
+  if (num_splits <= 0) {
+    // Wave-aware choice: minimise waves * (tiles per split + fixed cost).
+    const long long ctas = (long long)batch * g->num_kv_heads * pl.m_tiles;
+    double best_cost = 1e300;
+    num_splits = 1;
+    for (int s = 1; s <= std::min(kMaxSplits, std::max(1, kv_tiles)); ++s) {
+      const long long waves = (ctas * s + 151) / 152;
+      const double cost = (double)waves * ((kv_tiles + s - 1) / s + 2) + (s > 1 ? 2.0 : 0.0);
+      if (cost < best_cost - 1e-9) {
+        best_cost = cost;
+        num_splits = s;
+      }
+    }
+  }
+  pl.splits = num_splits;
+  pl.q_bytes = align256((size_t)batch * g->num_kv_heads * pl.R_pad * g->head_dim * 2);
+  if (pl.splits > 1) {
+    const size_t rows = (size_t)batch * g->num_kv_heads * pl.m_tiles * pl.splits * BM;
+    pl.po_bytes = align256(rows * g->head_dim * 4);
+    pl.pml_bytes = align256(rows * 2 * 4);
+  } else {
+    pl.po_bytes = pl.pml_bytes = 0;
+  }
+  pl.total = pl.q_bytes + pl.po_bytes + pl.pml_bytes;
+  return pl;
+}
+
+}  // namespace prefill
+}  // namespace pic
+
+extern "C" size_t pic_prefill_workspace_size(const pic_geom_t *geom, int32_t batch,
+                                             int32_t max_inline, int32_t max_ctx,
+                                             int32_t num_splits) {
+  if (!geom || batch <= 0 || max_inline <= 0 || max_ctx <= 0 || geom->num_kv_heads <= 0 ||
+      geom->num_q_heads % geom->num_kv_heads)
+    return 0;
+  return pic::prefill::plan(geom, batch, max_inline, max_ctx, num_splits).total;
+}
+
+namespace pic {
+namespace prefill {
+
+// Checks shared by pic_append_inline and pic_attend_prefill.
+static pic_status_t check_common(const char *who, const pic_geom_t *geom, int32_t layer,
+                                 int32_t batch, int32_t max_inline, int32_t max_ctx,
+                                 int64_t num_pages, int32_t num_splits, void *workspace,
+                                 size_t workspace_bytes, RopeParams *rp, Plan *pl) {
+  pic_status_t st = make_rope(geom, rp);
+  if (st != PIC_OK) return st;
+  if (layer < 0 || layer >= geom->num_layers)
+    return fail(PIC_ERR_INVALID_ARG, "%s: layer %d outside [0, %d)", who, layer, geom->num_layers);
+  if (batch <= 0 || max_inline <= 0 || max_ctx <= 0 || num_pages <= 0)
+    return fail(PIC_ERR_INVALID_ARG, "%s: sizes must be positive", who);
+  if (num_splits < 0 || num_splits > kMaxSplits)
+    return fail(PIC_ERR_INVALID_ARG, "%s: num_splits %d outside [0, %d]", who, num_splits,
+                kMaxSplits);
+  const long long rows_total = (long long)geom->num_layers * num_pages * geom->num_kv_heads * 16;
+  if (rows_total + 16 >= (long long)INT32_MAX)
+    return fail(PIC_ERR_UNSUPPORTED, "%s: cache has more than 2^31 rows", who);
+  *pl = plan(geom, batch, max_inline, max_ctx, num_splits);
+  if ((long long)batch * geom->num_kv_heads * pl->R_pad >= (long long)INT32_MAX ||
+      pl->m_tiles * pl->splits > 65535 || geom->num_kv_heads > 65535 || batch > 65535)
+    return fail(PIC_ERR_UNSUPPORTED, "%s: problem too large for one launch", who);
+  if (!workspace || workspace_bytes < pl->total || (reinterpret_cast<uintptr_t>(workspace) & 255))
+    return fail(PIC_ERR_WORKSPACE, "%s: workspace needs %zu bytes, 256-aligned", who, pl->total);
+  return PIC_OK;
+}
+
+}  // namespace prefill
+}  // namespace pic
+
+extern "C" int32_t pic_prefill_num_splits(const pic_geom_t *geom, int32_t batch,
+                                          int32_t max_inline, int32_t max_ctx,
+                                          int32_t num_splits) {
+  if (!geom || batch <= 0 || max_inline <= 0 || max_ctx <= 0 || geom->num_kv_heads <= 0 ||
+      geom->num_q_heads % geom->num_kv_heads || num_splits < 0 ||
+      num_splits > pic::prefill::kMaxSplits)
+    return 0;
+  return pic::prefill::plan(geom, batch, max_inline, max_ctx, num_splits).splits;
+}
+
+extern "C" pic_status_t pic_append_inline(
+    const pic_geom_t *geom, int32_t layer, int32_t batch, int32_t max_inline, const void *q,
+    const void *k_new, const void *v_new, const int32_t *inline_pos, const int32_t *inline_len,
+    const int64_t *slot_mapping, int32_t max_ctx, int64_t num_pages, void *k_cache,
+    void *v_cache, void *workspace, size_t workspace_bytes, pic_stream_t stream) {
+  using namespace pic;
+  using namespace pic::prefill;
+  RopeParams rp;
+  Plan pl;
+  // the packed queries are the leading part of the prefill workspace (size of num_splits = 1)
+  pic_status_t st = check_common("pic_append_inline", geom, layer, batch, max_inline, max_ctx,
+                                 num_pages, 1, workspace, workspace_bytes, &rp, &pl);
+  if (st != PIC_OK) return st;
+  if (!q || !k_new || !v_new || !inline_pos || !inline_len || !slot_mapping || !k_cache ||
+      !v_cache)
+    return fail(PIC_ERR_INVALID_ARG, "pic_append_inline: NULL tensor");
+  if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k_new) |
+       reinterpret_cast<uintptr_t>(v_new) | reinterpret_cast<uintptr_t>(k_cache) |
+       reinterpret_cast<uintptr_t>(v_cache)) & 15)
+    return fail(PIC_ERR_INVALID_ARG, "pic_append_inline: bf16 tensors must be 16-byte aligned");
+  int32_t *status = device_status_ptr();
+  if (!status) return fail(PIC_ERR_CUDA, "pic_append_inline: no device status word");
+  const int D = geom->head_dim, Hkv = geom->num_kv_heads;
+  const size_t layer_elems = (size_t)num_pages * Hkv * 16 * D;
+  AppendArgs aa;
+  aa.Hq = geom->num_q_heads;
+  aa.Hkv = Hkv;
+  aa.G = pl.G;
+  aa.max_inline = max_inline;
+  aa.max_ctx = max_ctx;
+  aa.R_pad = pl.R_pad;
+  aa.num_pages = num_pages;
+  aa.q = static_cast<const __nv_bfloat16 *>(q);
+  aa.k = static_cast<const __nv_bfloat16 *>(k_new);
+  aa.v = static_cast<const __nv_bfloat16 *>(v_new);
+  aa.inline_pos = inline_pos;
+  aa.inline_len = inline_len;
+  aa.slots = slot_mapping;
+  aa.k_cache = static_cast<__nv_bfloat16 *>(k_cache) + (size_t)layer * layer_elems;
+  aa.v_cache = static_cast<__nv_bfloat16 *>(v_cache) + (size_t)layer * layer_elems;
+  aa.qpack = static_cast<__nv_bfloat16 *>(workspace);
+  aa.status = status;
+  const int t_slots = std::max(max_inline, (pl.R_pad + pl.G - 1) / pl.G);
+  if (t_slots > INT32_MAX / 2 || batch > 65535)
+    return fail(PIC_ERR_UNSUPPORTED, "pic_append_inline: grid too large");
+  dim3 agrid(t_slots, batch);
+  if (D == 128) append_kernel<128><<<agrid, 128, 0, stream>>>(aa, rp);
+  else append_kernel<64><<<agrid, 128, 0, stream>>>(aa, rp);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "pic_append_inline launch");
+  return PIC_OK;
+}
+
+extern "C" pic_status_t pic_attend_prefill(
+    const pic_geom_t *geom, int32_t layer, int32_t batch, int32_t max_inline,
+    const int32_t *inline_pos, const int32_t *inline_len, int32_t max_ctx,
+    const int32_t *block_table, int32_t max_pages, int64_t num_pages, const void *k_cache,
+    const void *v_cache, void *out, float *lse, int32_t num_splits, void *workspace,
+    size_t workspace_bytes, pic_stream_t stream) {
+  using namespace pic;
+  using namespace pic::prefill;
+  RopeParams rp;
+  Plan pl;
+  pic_status_t st = check_common("pic_attend_prefill", geom, layer, batch, max_inline, max_ctx,
+                                 num_pages, num_splits, workspace, workspace_bytes, &rp, &pl);
+  if (st != PIC_OK) return st;
+  if (max_pages <= 0) return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill: max_pages <= 0");
+  if (!inline_pos || !inline_len || !block_table || !k_cache || !v_cache || !out)
+    return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill: NULL tensor");
+  if ((reinterpret_cast<uintptr_t>(k_cache) | reinterpret_cast<uintptr_t>(v_cache) |
+       reinterpret_cast<uintptr_t>(out)) & 15)
+    return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill: bf16 tensors must be 16-byte aligned");
+  int32_t *status = device_status_ptr();
+  if (!status) return fail(PIC_ERR_CUDA, "pic_attend_prefill: no device status word");
+  const int D = geom->head_dim, Hkv = geom->num_kv_heads;
+  const long long rows_total = (long long)geom->num_layers * num_pages * Hkv * 16;
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+
+  CUtensorMap tq, tk, tv;
+  st = encode_tmap_2d(&tq, ws, D, (uint64_t)batch * Hkv * pl.R_pad, (uint64_t)D * 2, 64, BM);
+  if (st == PIC_OK) st = encode_tmap_2d(&tk, k_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
+  if (st == PIC_OK) st = encode_tmap_2d(&tv, v_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
+  if (st != PIC_OK) return st;
+  Params pp;
+  pp.Hq = geom->num_q_heads;
+  pp.Hkv = Hkv;
+  pp.G = pl.G;
+  pp.max_inline = max_inline;
+  pp.R_pad = pl.R_pad;
+  pp.m_tiles = pl.m_tiles;
+  pp.num_splits = pl.splits;
+  pp.max_pages = max_pages;
+  pp.oob_row = (int)rows_total;
+  pp.num_pages = num_pages;
+  pp.layer_row0 = (long long)layer * num_pages * Hkv * 16;
+  pp.inline_pos = inline_pos;
+  pp.inline_len = inline_len;
+  pp.block_table = block_table;
+  pp.out = static_cast<__nv_bfloat16 *>(out);
+  pp.lse = lse;
+  pp.part_o = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes) : nullptr;
+  pp.part_ml = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes + pl.po_bytes) : nullptr;
+  pp.status = status;
+  pp.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
+
+  dim3 grid(pl.m_tiles * pl.splits, Hkv, batch);
+  cudaError_t e;
+  if (D == 128) {
+    const int smem = Layout<128>::kAlloc;
+    e = cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill smem attribute");
+    attn_kernel<128><<<grid, kThreads, smem, stream>>>(tq, tk, tv, pp);
+  } else {
+    const int smem = Layout<64>::kAlloc;
+    e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill smem attribute");
+    attn_kernel<64><<<grid, kThreads, smem, stream>>>(tq, tk, tv, pp);
+  }
+  if (pl.splits > 1) {
+    dim3 cgrid(pl.m_tiles, Hkv, batch);
+    if (D == 128) combine_kernel<128><<<cgrid, 256, 0, stream>>>(pp);
+    else combine_kernel<64><<<cgrid, 256, 0, stream>>>(pp);
+  }
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill launch");
+  return PIC_OK;
+}

@@ -1,0 +1,113 @@
+"""The cache-hit path over one workload: device buffers plus the call sequence.
+
+compose -> relocate (all layers) -> per layer: prefill (inline append +
+attention) -> decode steps.  PyTorch only allocates device memory and
+supplies the stream; every step is a libpic call.
+"""
+from __future__ import annotations
+
+import torch
+
+from . import (Geometry, pic_append_inline, pic_attend_decode, pic_attend_prefill,
+               pic_compose, pic_decode_workspace_size, pic_prefill_workspace_size, pic_relocate)
+from .workloads import Workload
+
+
+class CacheHitPath:
+    def __init__(self, wl: Workload, prefill_splits: int = 0, decode_splits: int = 0,
+                 with_lse: bool = False, rope_style: int = 0, inv_freq=None):
+        spec = wl.spec
+        dev = wl.k_pool.device
+        self.wl = wl
+        self.geom = Geometry(spec.layers, spec.q_heads, spec.kv_heads, spec.head_dim,
+                             spec.rope_base, page_size=spec.page_size, rope_style=rope_style,
+                             inv_freq=inv_freq)
+        B, md = wl.req_doc_ids.shape
+        L, Hq, Hkv, d = spec.layers, spec.q_heads, spec.kv_heads, spec.head_dim
+        self.B, self.max_docs = B, md
+        self.max_ctx = wl.max_ctx
+        self.max_inline = wl.tin_max
+        self.prefill_splits = prefill_splits
+        self.decode_splits = decode_splits
+        i32, i64, bf16 = torch.int32, torch.int64, torch.bfloat16
+        self.doc_offset = torch.empty((B, md), dtype=i32, device=dev)
+        self.doc_delta = torch.empty((B, md), dtype=i32, device=dev)
+        self.slot_mapping = torch.empty((B, self.max_ctx), dtype=i64, device=dev)
+        self.inline_pos = torch.empty((B, self.max_inline), dtype=i32, device=dev)
+        self.ctx_len = torch.empty((B,), dtype=i32, device=dev)
+        shape = (L, wl.num_pages, Hkv, spec.page_size, d)
+        self.k_cache = torch.zeros(shape, dtype=bf16, device=dev)
+        self.v_cache = torch.zeros(shape, dtype=bf16, device=dev)
+        u8 = torch.uint8
+        self.ws_prefill = torch.empty(
+            pic_prefill_workspace_size(self.geom, B, self.max_inline, self.max_ctx, prefill_splits),
+            dtype=u8, device=dev)
+        self.out = torch.empty((L, B, self.max_inline, Hq, d), dtype=bf16, device=dev)
+        self.lse = torch.empty((L, B, self.max_inline, Hq), dtype=torch.float32,
+                               device=dev) if with_lse else None
+        self.dec_out = self.dec_lse = self.ws_decode = None
+        if wl.q_dec is not None:
+            self.ws_decode = torch.empty(
+                pic_decode_workspace_size(self.geom, B, self.max_ctx, decode_splits),
+                dtype=u8, device=dev)
+            self.dec_out = torch.empty((L, B, Hq, d), dtype=bf16, device=dev)
+            self.dec_lse = torch.empty((L, B, Hq), dtype=torch.float32,
+                                       device=dev) if with_lse else None
+
+    # -- a1: layout and slot map
+    def compose(self):
+        wl = self.wl
+        pic_compose(self.geom, wl.doc_len, wl.doc_base_pos, wl.req_doc_ids, wl.req_num_docs,
+                    wl.prefix_len, wl.query_len, wl.block_table, wl.num_pages, self.max_ctx,
+                    self.max_inline, self.doc_offset, self.doc_delta, self.slot_mapping,
+                    self.inline_pos, self.ctx_len)
+
+    # -- a2 + a3: per-document rotation and stitching, all layers, one launch
+    def relocate(self, layer_begin: int = 0, layer_end: int | None = None):
+        wl = self.wl
+        if layer_end is None:
+            layer_end = wl.spec.layers
+        pic_relocate(self.geom, wl.k_pool, wl.v_pool, wl.doc_token_start, wl.doc_len,
+                     wl.req_doc_ids, wl.req_num_docs, self.doc_offset, self.doc_delta,
+                     self.slot_mapping, wl.num_pages, self.k_cache, self.v_cache, layer_begin,
+                     layer_end)
+
+    # -- a4: RoPE + append of the inline tokens of one layer
+    def append(self, layer: int):
+        wl = self.wl
+        pic_append_inline(self.geom, layer, wl.q_inline[layer], wl.k_inline[layer],
+                          wl.v_inline[layer], self.inline_pos, wl.inline_len, self.slot_mapping,
+                          wl.num_pages, self.k_cache, self.v_cache, self.ws_prefill)
+
+    # -- a5: prefill attention of one layer
+    def attend(self, layer: int):
+        wl = self.wl
+        pic_attend_prefill(self.geom, layer, self.inline_pos, wl.inline_len, self.max_ctx,
+                           wl.block_table, wl.num_pages, self.k_cache, self.v_cache,
+                           self.out[layer], None if self.lse is None else self.lse[layer],
+                           self.prefill_splits, self.ws_prefill)
+
+    def prefill(self, layer: int):
+        self.append(layer)
+        self.attend(layer)
+
+    # -- a6: one decode step of one layer (token position ctx_len + step)
+    def decode(self, step: int, layer: int):
+        wl = self.wl
+        pic_attend_decode(self.geom, layer, wl.q_dec[step, layer], wl.k_dec[step, layer],
+                          wl.v_dec[step, layer], self.ctx_len, wl.block_table, wl.num_pages,
+                          self.k_cache, self.v_cache, self.dec_out[layer], self.max_ctx,
+                          None if self.dec_lse is None else self.dec_lse[layer],
+                          self.decode_splits, self.ws_decode, pos_offset=step)
+
+    def ttft_pass(self):
+        """The cache-hit path up to the first token: layout, re-rotation and
+        stitching of every layer, then every layer's inline prefill."""
+        self.compose()
+        self.relocate()
+        for layer in range(self.wl.spec.layers):
+            self.prefill(layer)
+
+    def decode_pass(self, step: int):
+        for layer in range(self.wl.spec.layers):
+            self.decode(step, layer)

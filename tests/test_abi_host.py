@@ -1,0 +1,103 @@
+"""Host-side checks of the C ABI (no GPU needed): the library builds and loads,
+exports every function include/pic.h declares, and the calls that never reach
+the device (version, workspace sizes, argument validation) behave."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2607_28069_gb300 as pic
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "pic.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(pic.lib_path()):
+        from paper_2607_28069_gb300.build import build
+        build()
+    return pic.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(pic_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_header_declares_the_binding_symbols():
+    assert declared_functions() == sorted(pic.EXPORTED_SYMBOLS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    missing = [s for s in declared_functions() if not hasattr(lib, s)]
+    assert not missing, missing
+
+
+def test_version(lib):
+    assert pic.pic_abi_version() == 1
+
+
+def _geom(**kw):
+    g = dict(num_layers=2, num_q_heads=32, num_kv_heads=8, head_dim=128, rope_base=5e5)
+    g.update(kw)
+    return pic.Geometry(**g)
+
+
+def test_workspace_sizes_are_host_arithmetic(lib):
+    g = _geom()
+    # packed Q: B * Hkv * ceil(Tin*G/128)*128 rows of d bf16
+    ws1 = pic.pic_prefill_workspace_size(g, 1, 192, 4288, 1)
+    assert ws1 == 1 * 8 * 768 * 128 * 2
+    ws3 = pic.pic_prefill_workspace_size(g, 1, 192, 4288, 3)
+    assert ws3 > ws1
+    assert pic.pic_decode_workspace_size(g, 16, 33000, 1) == ((16 * 32 * 128 * 2 + 255) // 256) * 256
+    assert pic.pic_decode_workspace_size(_geom(num_kv_heads=0), 1, 10, 1) == 0
+    # one Llama-3-8B layer, 192 inline tokens over ~4.3k keys: 48 query tiles fill
+    # a third of the GPU, so the automatic choice splits the keys three ways
+    assert pic.pic_prefill_num_splits(g, 1, 192, 4288, 0) == 3
+    assert pic.pic_prefill_num_splits(g, 1, 192, 4288, 5) == 5
+    assert pic.pic_decode_num_splits(g, 16, 33000, 7) == 7
+    assert 1 <= pic.pic_decode_num_splits(g, 16, 33000, 0) <= 64
+
+
+def _call_compose_with(geom):
+    g = geom._c()
+    null = ctypes.c_void_p(0)
+    return pic.load().pic_compose(ctypes.byref(g), 1, 1, 1, null, null, null, null, null, null,
+                                  null, 1, 1, 16, 16, null, null, null, null, null, null)
+
+
+def test_invalid_geometry_rejected_before_launch(lib):
+    assert _call_compose_with(_geom(head_dim=96)) == 2          # PIC_ERR_UNSUPPORTED
+    assert b"head_dim" in pic.load().pic_last_error()
+    assert _call_compose_with(_geom(num_kv_heads=5)) == 1       # Hq % Hkv != 0
+    assert _call_compose_with(_geom(page_size=32)) == 2
+    assert _call_compose_with(_geom(rope_base=1.0)) == 1
+    assert _call_compose_with(_geom(rope_style=7)) == 1
+    # valid geometry but NULL tensors: still rejected on the host
+    assert _call_compose_with(_geom()) == 1
+    assert b"NULL" in pic.load().pic_last_error()
+
+
+def test_inv_freq_override_validated(lib):
+    bad = _geom(head_dim=64, inv_freq=[1.0] * 31 + [-1.0])
+    assert _call_compose_with(bad) == 1
+    assert b"inv_freq" in pic.load().pic_last_error()
+
+
+def test_binding_rejects_cpu_tensors():
+    import torch
+    with pytest.raises(ValueError):
+        pic._ptr(torch.zeros(4, dtype=torch.int32), torch.int32, "x")
+
+
+def test_product_path_does_not_import_the_oracle():
+    pkg = os.path.join(ROOT, "paper_2607_28069_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                src = open(os.path.join(dirpath, f)).read()
+                assert "import oracle" not in src and "from oracle" not in src, f
