@@ -58,6 +58,33 @@ INTERLEAVED = "interleaved"
 
 
 # --------------------------------------------------------------------------
+# bf16 storage (the paper executes in bfloat16: the stitched cache holds bf16
+# keys and values, and the Reader consumes bf16 queries)
+# --------------------------------------------------------------------------
+def round_bf16(x) -> np.ndarray:
+    """Round float64 values to the nearest bfloat16 value, ties to even.
+
+    bfloat16 keeps 8 significant bits and the float32 exponent range.  For a
+    normal value x = m * 2^e (0.5 <= |m| < 1), the kept significand is
+    rint(m * 2^8) (np.rint rounds half to even); below 2^-126 the spacing is
+    the fixed subnormal step 2^-133.  Results beyond the largest finite bf16
+    become infinities; NaN stays NaN.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    m, e = np.frexp(x)
+    out = np.ldexp(np.rint(m * 256.0), e - 8)
+    tiny = np.abs(x) < 2.0 ** -126
+    out = np.where(tiny, np.rint(x * 2.0 ** 133) * 2.0 ** -133, out)
+    bf16_max = (2.0 - 2.0 ** -7) * 2.0 ** 127
+    out = np.where(np.abs(out) > bf16_max, np.copysign(np.inf, x), out)
+    return np.where(np.isfinite(x), out, x)
+
+
+def _store(x, storage):
+    return round_bf16(x) if storage == "bf16" else x
+
+
+# --------------------------------------------------------------------------
 # Rotary transform R(p) and the re-rotation of Eq. 3
 # --------------------------------------------------------------------------
 def rope_frequencies(head_dim: int, base: float) -> np.ndarray:
@@ -184,12 +211,13 @@ def relocate_docs(layout: RequestLayout, k_docs, v_docs, doc_base_pos, theta, st
 
 
 def dense_context(layout: RequestLayout, k_docs, v_docs, doc_base_pos,
-                  k_inline, v_inline, theta, style=HALF):
+                  k_inline, v_inline, theta, style=HALF, storage=None):
     """Keys/values of the whole request indexed by logical position.
 
     Inline tokens (prefix then query, ``k_inline`` [P+Tq, Hkv, d] un-rotated)
     get RoPE at their own logical positions; documents are relocated with
-    Eq. 3.  Returns (K, V) of shape [ctx, Hkv, d].
+    Eq. 3.  Returns (K, V) of shape [ctx, Hkv, d].  storage="bf16" rounds the
+    rotated keys to bf16, as a bf16 cache holds them (values already are).
     """
     P = layout.prefix_len
     k_rot_inline = rotary(k_inline, layout.inline_pos[:, None], theta, style)
@@ -197,7 +225,7 @@ def dense_context(layout: RequestLayout, k_docs, v_docs, doc_base_pos,
     parts_k = [k_rot_inline[:P]] + ([kd] if kd is not None else []) + [k_rot_inline[P:]]
     parts_v = [np.asarray(v_inline[:P], np.float64)] + ([vd] if vd is not None else []) \
         + [np.asarray(v_inline[P:], np.float64)]
-    K = np.concatenate(parts_k, 0)
+    K = _store(np.concatenate(parts_k, 0), storage)
     V = np.concatenate(parts_v, 0)
     assert K.shape[0] == layout.ctx_len
     return K, V
@@ -266,21 +294,25 @@ def attention(q, q_pos, K, V, k_pos=None, scale=None, return_lse=False):
 # Whole path for one request and one layer
 # --------------------------------------------------------------------------
 def cache_hit_prefill(layout: RequestLayout, k_docs, v_docs, doc_base_pos,
-                      q_inline, k_inline, v_inline, theta, style=HALF, return_lse=False):
+                      q_inline, k_inline, v_inline, theta, style=HALF, return_lse=False,
+                      storage=None):
     """Cache hit: relocate the docs, RoPE the inline tokens, attend.
 
     ``q_inline`` [P+Tq, Hq, d], ``k_inline`` / ``v_inline`` [P+Tq, Hkv, d] are
     the un-rotated projections of the inline tokens (prefix then query).
     Returns the attention output of every inline token, plus the dense (K, V)
-    context the attention read.
+    context the attention read.  storage="bf16": rotated keys and queries are
+    rounded to bf16 before the (float64) attention.
     """
-    K, V = dense_context(layout, k_docs, v_docs, doc_base_pos, k_inline, v_inline, theta, style)
-    q_rot = rotary(q_inline, layout.inline_pos[:, None], theta, style)
+    K, V = dense_context(layout, k_docs, v_docs, doc_base_pos, k_inline, v_inline, theta, style,
+                         storage)
+    q_rot = _store(rotary(q_inline, layout.inline_pos[:, None], theta, style), storage)
     res = attention(q_rot, layout.inline_pos, K, V, return_lse=return_lse)
     return res, K, V
 
 
-def decode_step(K, V, q_new, k_new, v_new, pos, theta, style=HALF, return_lse=False):
+def decode_step(K, V, q_new, k_new, v_new, pos, theta, style=HALF, return_lse=False,
+                storage=None):
     """One autoregressive step over a completed cache (ordinary decoding).
 
     The new token at logical position ``pos`` (== len(K)) is appended with its
@@ -288,10 +320,10 @@ def decode_step(K, V, q_new, k_new, v_new, pos, theta, style=HALF, return_lse=Fa
     0..pos.  Returns (output [Hq, d], K', V').
     """
     assert pos == K.shape[0]
-    k_rot = rotary(k_new, pos, theta, style)
+    k_rot = _store(rotary(k_new, pos, theta, style), storage)
     K2 = np.concatenate([K, k_rot[None]], 0)
     V2 = np.concatenate([V, np.asarray(v_new, np.float64)[None]], 0)
-    q_rot = rotary(q_new, pos, theta, style)
+    q_rot = _store(rotary(q_new, pos, theta, style), storage)
     res = attention(q_rot[None], np.array([pos]), K2, V2, return_lse=return_lse)
     if return_lse:
         return (res[0][0], res[1][0]), K2, V2

@@ -52,9 +52,13 @@ def kv_tolerance_ok(gpu: np.ndarray, ref: np.ndarray, rel: float = 4e-3):
 
 
 def attn_close(gpu: np.ndarray, ref: np.ndarray, abs_tol=1e-2, row_rel=2e-2):
-    """Attention bar: max-abs <= 1e-2 and per-row relative L2 <= 2e-2."""
+    """Attention bar: |g - r| <= 1e-2 * max(1, max|r_row|) and per-row relative
+    L2 <= 2e-2.  The output is bf16, so rows with |o| > 1 (short contexts)
+    carry proportionally more rounding; for |o| <= 1 the bar is max-abs 1e-2.
+    Returns (ok, worst max-abs over rows scaled to the bar, worst row rel-L2)."""
     err = np.abs(gpu - ref)
-    max_abs = float(err.max(initial=0.0))
+    scale = np.maximum(1.0, np.abs(ref).max(axis=-1, keepdims=True))
+    max_abs = float((err / scale).max(initial=0.0))
     l2 = np.linalg.norm(gpu - ref, axis=-1) / np.maximum(np.linalg.norm(ref, axis=-1), 1e-6)
     worst = float(l2.max(initial=0.0))
     return (max_abs <= abs_tol and worst <= row_rel), max_abs, worst

@@ -5,7 +5,8 @@ Bars (written here, derived in the design doc):
 * layout, slot map, inline positions, ctx: bit-exact;
 * V and every copied value: bit-exact;
 * relocated / rotated K: |g - r| <= 4e-3 max(|r|, 2^-8 rowmax) and row rel-L2 <= 4e-3;
-* attention outputs: max-abs <= 1e-2 and per-row rel-L2 <= 2e-2.
+* attention outputs: |g - r| <= 1e-2 max(1, max|r_row|) and per-row rel-L2 <= 2e-2
+  against the exact fp64 oracle (peaked cases: against its bf16-storage mode).
 """
 import numpy as np
 import pytest
@@ -223,10 +224,11 @@ def test_needle_and_peaked_softmax(cuda_lib):
     path = CacheHitPath(wl, with_lse=True)
     path.ttft_pass()
     docs, k_docs, v_docs, q, k, v = request_inputs(wl, 0, 0)
+    # peaked scores: compare with the bf16-storage oracle (cache and queries in bf16)
     o_ref, _, _ = O.cache_hit_prefill(lay, k_docs, v_docs, wl.doc_base_pos.cpu().numpy(),
-                                      q, k, v, theta)
+                                      q, k, v, theta, storage="bf16")
     o_gpu = f64(path.out[0, 0, :q.shape[0]])
-    ok, max_abs, rowrel = attn_close(o_gpu, o_ref)
+    ok, max_abs, rowrel = attn_close(o_gpu, o_ref, abs_tol=1e-2, row_rel=1e-2)
     assert ok, (max_abs, rowrel)
     v_needle = f64(wl.v_pool[0, row, 0])
     assert np.linalg.norm(o_gpu[-1, 0] - v_needle) < 0.1 * np.linalg.norm(v_needle)

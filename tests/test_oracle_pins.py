@@ -420,3 +420,47 @@ def test_pins_catch_planted_rerotation_mistakes():
     assert np.allclose(O.rerotate_key(made_at_a, a, b, theta), good, atol=1e-9)
     assert not np.allclose(swapped, good, atol=1e-3)
     assert not np.allclose(absolute, good, atol=1e-3)
+
+
+# ---------------------------------------------------------- bf16 storage ---
+def test_round_bf16_matches_torch_on_float32_values():
+    """Library route: torch's float32 -> bfloat16 conversion rounds to nearest even."""
+    import torch
+    rng = np.random.default_rng(5)
+    x = np.concatenate([rng.standard_normal(20000) * 10.0 ** rng.integers(-30, 30, 20000),
+                        [0.0, -0.0, 1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, -(1.0 + 2 ** -8),
+                         2.0 ** -130, 3 * 2.0 ** -134, 3.3e38, -3.4e38, np.inf, -np.inf]])
+    x32 = x.astype(np.float32)
+    ref = torch.from_numpy(x32).to(torch.bfloat16).float().numpy().astype(np.float64)
+    got = O.round_bf16(x32.astype(np.float64))
+    assert np.array_equal(got, ref)
+
+
+def test_round_bf16_hand_values_and_brute_force():
+    from fractions import Fraction
+    assert O.round_bf16(1.0 + 2 ** -8) == 1.0                    # tie -> even (1.0)
+    assert O.round_bf16(1.0 + 3 * 2 ** -8) == 1.0 + 2 ** -6      # tie -> even (...10)
+    assert O.round_bf16(1.0 + 2 ** -8 + 2 ** -40) == 1.0 + 2 ** -7
+    assert np.isnan(O.round_bf16(np.nan))
+    rng = np.random.default_rng(11)
+    for v in rng.standard_normal(300) * 3:
+        # brute force: nearest of all bf16 values with the same exponent, ties even
+        e = int(np.floor(np.log2(abs(v))))
+        step = Fraction(2) ** (e - 7)
+        lo = (Fraction(v) // step) * step
+        cands = [lo, lo + step]
+        dist = [abs(Fraction(v) - c) for c in cands]
+        if dist[0] != dist[1]:
+            best = cands[int(dist[1] < dist[0])]
+        else:
+            best = cands[0] if (lo / step) % 2 == 0 else cands[1]
+        assert O.round_bf16(v) == float(best), v
+
+
+def test_bf16_storage_only_rounds_rotated_keys_and_queries():
+    theta, raw, k_docs, v_docs, lay, q, k, v = _tiny_request()
+    K, V = O.dense_context(lay, k_docs, v_docs, [0, 0], k, v, theta)
+    Kb, Vb = O.dense_context(lay, k_docs, v_docs, [0, 0], k, v, theta, storage="bf16")
+    assert np.array_equal(Kb, O.round_bf16(K)) and np.array_equal(Vb, V)
+    # unit roundoff of an 8-bit significand: |round(x) - x| <= 2^-8 |x|
+    assert (np.abs(Kb - K) <= 2.0 ** -8 * np.abs(K)).all()
