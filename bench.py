@@ -81,53 +81,87 @@ def ncu_traffic(kernel_key, src_file):
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
-              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    """SM clock and clock-event reasons sampled every ~1 ms during the timed
+    region through NVML (the driver's library, via ctypes); nvidia-smi every
+    200 ms when NVML is unavailable."""
+    REASONS = {0x8: "hw_slowdown", 0x40: "hw_thermal_slowdown", 0x20: "sw_thermal_slowdown",
+               0x4: "sw_power_cap", 0x80: "hw_power_brake_slowdown"}
 
-    def __init__(self, gpu_index):
-        self.gpu = gpu_index
-        self.proc = None
+    def __init__(self, torch_device):
+        self.dev = torch_device
+        self.samples = []
+        self.max_mhz = None
+        self.source = None
+        self._stop = None
+
+    def _nvml_open(self):
+        import ctypes
+        import torch
+        nvml = ctypes.CDLL("libnvidia-ml.so.1")
+        if nvml.nvmlInit_v2() != 0:
+            raise OSError("nvmlInit failed")
+        h = ctypes.c_void_p()
+        uuid = "GPU-" + str(torch.cuda.get_device_properties(self.dev).uuid)
+        if nvml.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(h)) != 0:
+            raise OSError("no NVML handle for " + uuid)
+        mx = ctypes.c_uint()
+        if nvml.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:
+            self.max_mhz = float(mx.value)
+        fn = getattr(nvml, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            getattr(nvml, "nvmlDeviceGetCurrentClocksThrottleReasons")
+        return nvml, h, fn
 
     def __enter__(self):
+        import threading
+        self._stop = threading.Event()
         try:
-            self.proc = subprocess.Popen(
-                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+            nvml, h, reasons_fn = self._nvml_open()
+            self.source = "nvml"
+
+            def loop():
+                import ctypes
+                clk, rs = ctypes.c_uint(), ctypes.c_ulonglong()
+                while not self._stop.is_set():
+                    if nvml.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0 and \
+                            reasons_fn(h, ctypes.byref(rs)) == 0:
+                        self.samples.append((float(clk.value), int(rs.value)))
+                    time.sleep(0.001)
+            self._t = threading.Thread(target=loop, daemon=True)
+            self._t.start()
+        except (OSError, AttributeError):
+            self.source = "nvidia-smi"
+            self._proc = subprocess.Popen(
+                ["nvidia-smi", "--query-gpu=clocks.sm,clocks.max.sm,clocks_event_reasons.active",
                  "--format=csv,noheader,nounits", "-lms", "200"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
-        except OSError:
-            self.proc = None
         return self
 
     def __exit__(self, *exc):
-        self.out = ""
-        if self.proc is not None:
-            self.proc.terminate()
-            try:
-                self.out, _ = self.proc.communicate(timeout=5)
-            except subprocess.TimeoutExpired:
-                self.proc.kill()
-                self.out, _ = self.proc.communicate()
+        self._stop.set()
+        if self.source == "nvml":
+            self._t.join(timeout=2)
+        elif self.source == "nvidia-smi":
+            self._proc.terminate()
+            out, _ = self._proc.communicate(timeout=5)
+            for line in out.splitlines():
+                parts = [x.strip() for x in line.split(",")]
+                try:
+                    self.samples.append((float(parts[0]), int(parts[2], 16)))
+                    self.max_mhz = float(parts[1])
+                except (ValueError, IndexError):
+                    pass
 
     def summary(self):
-        rows = []
-        for line in (self.out or "").splitlines():
-            parts = [x.strip() for x in line.split(",")]
-            if len(parts) < 9:
-                continue
-            try:
-                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
-            except ValueError:
-                continue
-        if not rows:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[i] for _, _, r in rows for i, v in enumerate(r)
-                          if v.lower() == "active"})
-        return {"sm_mhz": statistics.median(r[0] for r in rows),
-                "sm_max_mhz": max(r[1] for r in rows), "reasons": reasons,
-                "samples": len(rows)}
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": ["unsampled"],
+                    "source": self.source}
+        seen = 0
+        for _, r in self.samples:
+            seen |= r
+        return {"sm_mhz": statistics.median(c for c, _ in self.samples),
+                "sm_max_mhz": self.max_mhz,
+                "reasons": sorted(v for k, v in self.REASONS.items() if seen & k),
+                "samples": len(self.samples), "source": self.source}
 
 
 # ---------------------------------------------------------- work accounting
@@ -259,17 +293,33 @@ def main_gpu(args, rank, world):
     if code:
         raise RuntimeError(f"device status {code} detail {detail}")
 
-    # one CUDA graph per call, so each call can be timed on its own
-    phases = [("compose", path.compose), ("relocate", path.relocate)]
+    # The TTFT pass as CUDA graph(s) with timing events at every call boundary:
+    # one graph with external event nodes when torch supports them, else one
+    # graph per call with events between the replays.
+    calls = [("compose", path.compose), ("relocate", path.relocate)]
     for layer in range(L):
-        phases.append(("append", (lambda l=layer: path.append(l))))
-        phases.append(("attend", (lambda l=layer: path.attend(l))))
-    graphs = []
-    for name, fn in phases:
+        calls.append(("append", (lambda l=layer: path.append(l))))
+        calls.append(("attend", (lambda l=layer: path.attend(l))))
+    stream = torch.cuda.current_stream()
+    try:
+        bounds = [torch.cuda.Event(enable_timing=True, external=True)
+                  for _ in range(len(calls) + 1)]
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g):
-            fn()
-        graphs.append((name, g))
+            bounds[0].record()
+            for i, (_, fn) in enumerate(calls):
+                fn()
+                bounds[i + 1].record()
+        graphs = [g]
+        single = True
+    except (TypeError, RuntimeError):
+        graphs = []
+        for _, fn in calls:
+            gi = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gi):
+                fn()
+            graphs.append(gi)
+        single = False
     dec_graph = None
     if wl.q_dec is not None:
         dec_graph = torch.cuda.CUDAGraph()
@@ -280,37 +330,43 @@ def main_gpu(args, rank, world):
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
     flush = torch.empty(max(2 * l2, 256 << 20), dtype=torch.uint8, device=dev)
     sleep_cycles = int(2e9 * max(50e-6, 5e-6 * len(graphs)))
-    stream = torch.cuda.current_stream()
 
-    def one_step(evs):
+    def one_step():
+        """Flush L2, then one pass; returns per-call ms after synchronising."""
         flush.zero_()
-        torch.cuda._sleep(sleep_cycles)       # keep the GPU busy while the host enqueues
+        torch.cuda._sleep(sleep_cycles)   # GPU busy while the host enqueues
+        if single:
+            graphs[0].replay()
+            torch.cuda.synchronize()
+            return [bounds[i].elapsed_time(bounds[i + 1]) for i in range(len(calls))]
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(graphs) + 1)]
         evs[0].record(stream)
-        for i, (_, g) in enumerate(graphs):
-            g.replay()
+        for i, gi in enumerate(graphs):
+            gi.replay()
             evs[i + 1].record(stream)
+        torch.cuda.synchronize()
+        return [evs[i].elapsed_time(evs[i + 1]) for i in range(len(calls))]
 
     W, K = args.warmup, args.steps
+    torch.cuda._sleep(int(2e9 * 0.3))   # let the clocks ramp before warm-up
     for _ in range(W):
-        one_step([torch.cuda.Event(enable_timing=True) for _ in range(len(graphs) + 1)])
+        one_step()
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    events = [[torch.cuda.Event(enable_timing=True) for _ in range(len(graphs) + 1)]
-              for _ in range(K)]
-    with ClockSampler(local) as clk:
-        for k in range(K):
-            one_step(events[k])
-        torch.cuda.synchronize()
+    per_call = []
+    with ClockSampler(dev) as clk:
+        for _ in range(K):
+            per_call.append(one_step())
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    step_ms = [ev[0].elapsed_time(ev[-1]) for ev in events]
+    step_ms = [sum(x) for x in per_call]
     phase_ms = {}
-    for ev in events:
-        for i, (name, _) in enumerate(graphs):
-            phase_ms.setdefault(name, []).append(ev[i].elapsed_time(ev[i + 1]))
+    for x in per_call:
+        for (name, _), ms in zip(calls, x):
+            phase_ms.setdefault(name, []).append(ms)
     total_ms = sum(step_ms)
     if world > 1:
         t = torch.tensor([total_ms], device=dev, dtype=torch.float64)
@@ -395,8 +451,8 @@ def main_gpu(args, rank, world):
             e0.record(stream)
             for d_t, h_t in zip(ins, host_in):
                 d_t.copy_(h_t, non_blocking=True)
-            for _, g in graphs:
-                g.replay()
+            for gi in graphs:
+                gi.replay()
             host_out.copy_(path.out, non_blocking=True)
             e1.record(stream)
             torch.cuda.synchronize()
@@ -425,7 +481,8 @@ def main_gpu(args, rank, world):
                    "kv_heads": spec.kv_heads, "head_dim": spec.head_dim,
                    "query_len": spec.query_len, "ctx_tokens": work["ctx"],
                    "l2_policy": f"L2 flushed before every step ({flush.numel() >> 20} MiB write)",
-                   "timing": "CUDA graph per call, CUDA events on the launching stream",
+                   "timing": ("one CUDA graph per pass, timing-event nodes at call boundaries"
+                              if single else "one CUDA graph per call, events between replays"),
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
         "gpu_launches": launches,
         "rows": rows,

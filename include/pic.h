@@ -103,8 +103,8 @@ pic_status_t pic_device_status(pic_stream_t stream, int32_t *code, int32_t *deta
 
 /*
  * pic_compose -- link operator R: logical layout of each request and its
- * token-level slot map (Eqs. 1-2, "Background: Position-Independent
- * Caching"; appendix "Logical Layout and Re-Rotation").
+ * token-level maps (Eqs. 1-2, "Background: Position-Independent Caching";
+ * appendix "Logical Layout and Re-Rotation").
  *
  * Request b is laid out as prefix (positions 0..P_b-1), then its documents
  * in the order req_doc_ids[b][0..m_b-1], then Tq_b query tokens.  For its
@@ -112,59 +112,59 @@ pic_status_t pic_device_status(pic_stream_t stream, int32_t *code, int32_t *deta
  *     doc_offset[b][k] = P_b + sum_{k'<k} n_{ids[b][k']}
  *     doc_delta[b][k]  = doc_offset[b][k] - doc_base_pos[i]
  * ctx_len[b] = P_b + sum_k n + Tq_b, and for 0 <= t < ctx_len[b]
- *     slot_mapping[b][t] = block_table[b][t / page] * page + t % page.
+ *     slot_mapping[b][t] = block_table[b][t / page] * page + t % page
+ *     tok_map[b][t] = (k << 40) | (doc_token_start[i] + t - doc_offset[b][k])
+ *                     for a position t of the k-th document, -1 otherwise
+ * (the source row in the pool and the document index of every position).
  * inline_pos[b][0..P_b+Tq_b-1] lists the inline tokens' logical positions:
  * 0..P_b-1 then ctx_len[b]-Tq_b .. ctx_len[b]-1.
  *
- * Inputs (device, int32): doc_len, doc_base_pos [n_pool_docs];
- *   req_doc_ids [batch][max_docs]; req_num_docs, prefix_len, query_len [batch];
- *   block_table [batch][max_pages] (entries used must be in [0, num_pages)).
+ * Inputs (device): doc_len, doc_base_pos int32 [n_pool_docs]; doc_token_start
+ *   int64 [n_pool_docs]; req_doc_ids int32 [batch][max_docs]; req_num_docs,
+ *   prefix_len, query_len int32 [batch]; block_table int32 [batch][max_pages]
+ *   (entries used must be in [0, num_pages)).  max_docs <= 8192.
  * Outputs (device): doc_offset, doc_delta int32 [batch][max_docs] (entries
- *   k >= m_b are set to -1 / 0); slot_mapping int64 [batch][max_ctx];
- *   inline_pos int32 [batch][max_inline] (unused tail -1);
+ *   k >= m_b are set to -1 / 0); slot_mapping, tok_map int64 [batch][max_ctx]
+ *   (-1 beyond ctx_len); inline_pos int32 [batch][max_inline] (unused tail -1);
  *   ctx_len int32 [batch] (-1 for a request that failed a device check).
  * Device checks: doc id range, doc length > 0, ctx <= max_ctx,
  *   P + Tq <= max_inline, ceil(ctx / page) <= max_pages, page ids in range.
  */
 pic_status_t pic_compose(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
                          int32_t n_pool_docs, const int32_t *doc_len,
-                         const int32_t *doc_base_pos, const int32_t *req_doc_ids,
-                         const int32_t *req_num_docs, const int32_t *prefix_len,
-                         const int32_t *query_len, const int32_t *block_table,
-                         int32_t max_pages, int64_t num_pages, int32_t max_ctx,
-                         int32_t max_inline, int32_t *doc_offset, int32_t *doc_delta,
-                         int64_t *slot_mapping, int32_t *inline_pos, int32_t *ctx_len,
-                         pic_stream_t stream);
+                         const int32_t *doc_base_pos, const int64_t *doc_token_start,
+                         const int32_t *req_doc_ids, const int32_t *req_num_docs,
+                         const int32_t *prefix_len, const int32_t *query_len,
+                         const int32_t *block_table, int32_t max_pages, int64_t num_pages,
+                         int32_t max_ctx, int32_t max_inline, int32_t *doc_offset,
+                         int32_t *doc_delta, int64_t *slot_mapping, int64_t *tok_map,
+                         int32_t *inline_pos, int32_t *ctx_len, pic_stream_t stream);
 
 /*
  * pic_relocate -- key re-rotation and stitching of the cached documents
  * (Eq. 3; only keys are rotated, values are copied as they are).
  *
- * For every layer l in [layer_begin, layer_end), request b, document k and
- * token j < n of that document (pool id i):
- *     k_cache[l][slot(offset_k + j)] = R(delta_k) * k_pool[l][start_i + j]
- *     v_cache[l][slot(offset_k + j)] = v_pool[l][start_i + j]   (bit copy)
- * where R(delta) rotates each RoPE pair by delta * theta_i (delta is the same
- * for every token of a document, since base and target both advance by one
- * per token, so R(b) R(a)^-1 = R(b - a)).  cos/sin come from the angle
- * delta * theta_i formed and reduced in fp64; the rotation is fp32; K' is
- * rounded to bf16 (round to nearest even).  delta == 0 reproduces k
- * bit-exactly.  slot(t) = slot_mapping[b][t] as written by pic_compose.
+ * For every layer l in [layer_begin, layer_end), request b and position t
+ * with tok_map[b][t] = (k << 40) | row (written by pic_compose):
+ *     k_cache[l][slot(t)] = R(doc_delta[b][k]) * k_pool[l][row]
+ *     v_cache[l][slot(t)] = v_pool[l][row]                      (bit copy)
+ * with slot(t) = slot_mapping[b][t].  R(delta) rotates each RoPE pair by
+ * delta * theta_i (delta is the same for every token of a document, since
+ * base and target both advance by one per token, so R(b) R(a)^-1 = R(b - a)).
+ * cos/sin come from the angle delta * theta_i formed and reduced in fp64; the
+ * rotation is fp32; K' is rounded to bf16 (round to nearest even).
+ * delta == 0 reproduces k bit-exactly.
  *
- * Inputs: pool tensors (layout above) with pool_tokens rows per layer;
- *   doc_token_start int64 [n_pool_docs]; doc_len int32 [n_pool_docs];
- *   req_doc_ids, doc_offset, doc_delta [batch][max_docs]; req_num_docs [batch];
- *   slot_mapping int64 [batch][max_ctx].
- * One launch; no workspace.  max_docs == 0 returns PIC_OK without launching.
+ * Inputs: k_pool, v_pool (layout above) with pool_tokens rows per layer;
+ *   tok_map, slot_mapping int64 [batch][max_ctx]; doc_delta int32 [batch][max_docs].
+ * One launch, no workspace.  max_docs == 0 returns PIC_OK without launching.
  */
 pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
-                          int32_t n_pool_docs, const void *k_pool, const void *v_pool,
-                          int64_t pool_tokens, const int64_t *doc_token_start,
-                          const int32_t *doc_len, const int32_t *req_doc_ids,
-                          const int32_t *req_num_docs, const int32_t *doc_offset,
-                          const int32_t *doc_delta, const int64_t *slot_mapping,
-                          int32_t max_ctx, int64_t num_pages, void *k_cache, void *v_cache,
-                          int32_t layer_begin, int32_t layer_end, pic_stream_t stream);
+                          const void *k_pool, const void *v_pool, int64_t pool_tokens,
+                          const int64_t *tok_map, const int32_t *doc_delta,
+                          const int64_t *slot_mapping, int32_t max_ctx, int64_t num_pages,
+                          void *k_cache, void *v_cache, int32_t layer_begin, int32_t layer_end,
+                          pic_stream_t stream);
 
 /*
  * Prefill of one layer's inline tokens ("Cache-hit serving": only the

@@ -98,10 +98,9 @@ def load():
         "pic_abi_version": (I32, []),
         "pic_last_error": (ctypes.c_char_p, []),
         "pic_device_status": (I32, [P, P, P]),
-        "pic_compose": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, I32, I64, I32, I32,
-                              P, P, P, P, P, P]),
-        "pic_relocate": (I32, [G, I32, I32, I32, P, P, I64, P, P, P, P, P, P, P, I32, I64,
-                               P, P, I32, I32, P]),
+        "pic_compose": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, I32, I64, I32, I32,
+                              P, P, P, P, P, P, P]),
+        "pic_relocate": (I32, [G, I32, I32, P, P, I64, P, P, P, I32, I64, P, P, I32, I32, P]),
         "pic_prefill_workspace_size": (SZ, [G, I32, I32, I32, I32]),
         "pic_append_inline": (I32, [G, I32, I32, I32, P, P, P, P, P, P, I32, I64, P, P, P, SZ,
                                     P]),
@@ -165,36 +164,33 @@ def pic_device_status(stream=None):
     return code.value, detail.value
 
 
-def pic_compose(geom: Geometry, doc_len, doc_base_pos, req_doc_ids, req_num_docs, prefix_len,
-                query_len, block_table, num_pages: int, max_ctx: int, max_inline: int,
-                doc_offset, doc_delta, slot_mapping, inline_pos, ctx_len, stream=None):
+def pic_compose(geom: Geometry, doc_len, doc_base_pos, doc_token_start, req_doc_ids,
+                req_num_docs, prefix_len, query_len, block_table, num_pages: int, max_ctx: int,
+                max_inline: int, doc_offset, doc_delta, slot_mapping, tok_map, inline_pos,
+                ctx_len, stream=None):
     lib = load()
     g = geom._c()
     B, max_docs = req_doc_ids.shape
     st = lib.pic_compose(
         ctypes.byref(g), B, max_docs, doc_len.numel(), _ptr(doc_len, i32, "doc_len"),
-        _ptr(doc_base_pos, i32, "doc_base_pos"), _ptr(req_doc_ids, i32, "req_doc_ids"),
-        _ptr(req_num_docs, i32, "req_num_docs"), _ptr(prefix_len, i32, "prefix_len"),
-        _ptr(query_len, i32, "query_len"), _ptr(block_table, i32, "block_table"),
-        block_table.shape[1], num_pages, max_ctx, max_inline,
-        _ptr(doc_offset, i32, "doc_offset"), _ptr(doc_delta, i32, "doc_delta"),
-        _ptr(slot_mapping, i64, "slot_mapping"), _ptr(inline_pos, i32, "inline_pos"),
-        _ptr(ctx_len, i32, "ctx_len"), _stream(stream))
+        _ptr(doc_base_pos, i32, "doc_base_pos"), _ptr(doc_token_start, i64, "doc_token_start"),
+        _ptr(req_doc_ids, i32, "req_doc_ids"), _ptr(req_num_docs, i32, "req_num_docs"),
+        _ptr(prefix_len, i32, "prefix_len"), _ptr(query_len, i32, "query_len"),
+        _ptr(block_table, i32, "block_table"), block_table.shape[1], num_pages, max_ctx,
+        max_inline, _ptr(doc_offset, i32, "doc_offset"), _ptr(doc_delta, i32, "doc_delta"),
+        _ptr(slot_mapping, i64, "slot_mapping"), _ptr(tok_map, i64, "tok_map"),
+        _ptr(inline_pos, i32, "inline_pos"), _ptr(ctx_len, i32, "ctx_len"), _stream(stream))
     _check(st, "pic_compose")
 
 
-def pic_relocate(geom: Geometry, k_pool, v_pool, doc_token_start, doc_len, req_doc_ids,
-                 req_num_docs, doc_offset, doc_delta, slot_mapping, num_pages: int, k_cache,
-                 v_cache, layer_begin: int, layer_end: int, stream=None):
+def pic_relocate(geom: Geometry, k_pool, v_pool, tok_map, doc_delta, slot_mapping,
+                 num_pages: int, k_cache, v_cache, layer_begin: int, layer_end: int, stream=None):
     lib = load()
     g = geom._c()
-    B, max_docs = req_doc_ids.shape
+    B, max_docs = doc_delta.shape
     st = lib.pic_relocate(
-        ctypes.byref(g), B, max_docs, doc_len.numel(), _ptr(k_pool, bf16, "k_pool"),
-        _ptr(v_pool, bf16, "v_pool"), k_pool.shape[1],
-        _ptr(doc_token_start, i64, "doc_token_start"), _ptr(doc_len, i32, "doc_len"),
-        _ptr(req_doc_ids, i32, "req_doc_ids"), _ptr(req_num_docs, i32, "req_num_docs"),
-        _ptr(doc_offset, i32, "doc_offset"), _ptr(doc_delta, i32, "doc_delta"),
+        ctypes.byref(g), B, max_docs, _ptr(k_pool, bf16, "k_pool"), _ptr(v_pool, bf16, "v_pool"),
+        k_pool.shape[1], _ptr(tok_map, i64, "tok_map"), _ptr(doc_delta, i32, "doc_delta"),
         _ptr(slot_mapping, i64, "slot_mapping"), slot_mapping.shape[1], num_pages,
         _ptr(k_cache, bf16, "k_cache"), _ptr(v_cache, bf16, "v_cache"), layer_begin, layer_end,
         _stream(stream))

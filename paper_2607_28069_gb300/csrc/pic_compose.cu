@@ -8,8 +8,10 @@
 //
 // One grid row per request.  Every CTA of a row re-derives the document
 // offsets with a block-wide prefix sum over the document lengths (loaded in
-// parallel), then fills its 4096-position slice of the slot map.  Only the
-// first CTA of a row writes the per-document outputs, the inline positions and
+// parallel, kept in shared memory), then fills its 1024-position slice of the
+// slot map and of the token map (source pool row and document index of every
+// document position, found by binary search over the offsets).  Only the first
+// CTA of a row writes the per-document outputs, the inline positions and
 // ctx_len, and records device-side check failures.
 #include "pic_internal.cuh"
 
@@ -17,14 +19,17 @@ namespace pic {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kSlotsPerCta = 4096;
+constexpr int kPerThread = 4;
+constexpr int kSlotsPerCta = kThreads * kPerThread;
+constexpr int kMaxDocs = 8192;  // per request (shared-memory offsets)
 
 struct ComposeArgs {
   int batch, max_docs, n_pool, max_pages, max_ctx, max_inline, page;
   long long num_pages;
   const int32_t *doc_len, *doc_base, *ids, *num_docs, *prefix, *query, *block_table;
+  const int64_t *doc_start;
   int32_t *doc_offset, *doc_delta, *inline_pos, *ctx_len;
-  int64_t *slot_mapping;
+  int64_t *slot_mapping, *tok_map;
   int32_t *status;
 };
 
@@ -51,6 +56,9 @@ __global__ void __launch_bounds__(kThreads) compose_kernel(ComposeArgs a) {
   __shared__ long long warp_tot[kThreads / 32];
   __shared__ long long s_carry;
   __shared__ int s_err, s_err_detail;
+  extern __shared__ long long s_dyn[];
+  long long *s_start = s_dyn;                                             // [max_docs]
+  int32_t *s_off = reinterpret_cast<int32_t *>(s_dyn + a.max_docs);     // [max_docs]
   if (tid == 0) {
     s_carry = 0;
     s_err = 0;
@@ -69,7 +77,7 @@ __global__ void __launch_bounds__(kThreads) compose_kernel(ComposeArgs a) {
 
   for (int k0 = 0; k0 < m; k0 += kThreads) {
     const int k = k0 + tid;
-    long long n = 0, base = 0;
+    long long n = 0, base = 0, start = 0;
     if (k < m) {
       const int id = a.ids[(size_t)b * a.max_docs + k];
       if (id < 0 || id >= a.n_pool) {
@@ -77,6 +85,7 @@ __global__ void __launch_bounds__(kThreads) compose_kernel(ComposeArgs a) {
       } else {
         n = a.doc_len[id];
         base = a.doc_base[id];
+        start = a.doc_start[id];
         if (n <= 0) {
           atomicCAS(&s_err, 0, PIC_DEV_BAD_DOC_LEN);
           n = 0;
@@ -85,6 +94,10 @@ __global__ void __launch_bounds__(kThreads) compose_kernel(ComposeArgs a) {
     }
     const long long incl = block_inclusive_scan(n, warp_tot);
     const long long off = P + s_carry + incl - n;
+    if (k < m) {
+      s_off[k] = (int32_t)off;
+      s_start[k] = start;
+    }
     if (lead && k < m) {
       a.doc_offset[(size_t)b * a.max_docs + k] = (int32_t)off;
       a.doc_delta[(size_t)b * a.max_docs + k] = (int32_t)(off - base);
@@ -108,19 +121,38 @@ __global__ void __launch_bounds__(kThreads) compose_kernel(ComposeArgs a) {
   __syncthreads();
   const int err = s_err;
 
-  // Slot map slice of this CTA (positions beyond ctx get -1).
+  // Slot map and token map of this CTA's positions (beyond ctx: -1).
   const long long t_begin = (long long)blockIdx.x * kSlotsPerCta;
-  const long long t_end = min((long long)a.max_ctx, t_begin + kSlotsPerCta);
   int64_t *slots = a.slot_mapping + (size_t)b * a.max_ctx;
+  int64_t *tmap = a.tok_map + (size_t)b * a.max_ctx;
   const int32_t *bt = a.block_table + (size_t)b * a.max_pages;
-  for (long long t = t_begin + tid; t < t_end; t += kThreads) {
-    long long s = -1;
-    if (!err && t < ctx) {
-      const int page = bt[t / a.page];
-      if (page < 0 || page >= a.num_pages) atomicCAS(&s_err, 0, PIC_DEV_BAD_PAGE);
-      else s = (long long)page * a.page + t % a.page;
+  const long long span_end = ctx - Tq;  // documents occupy [P, span_end)
+  int page[kPerThread];
+#pragma unroll
+  for (int u = 0; u < kPerThread; ++u) {  // independent loads first
+    const long long t = t_begin + tid + u * kThreads;
+    page[u] = (!err && t < ctx) ? bt[t / a.page] : -2;
+  }
+#pragma unroll
+  for (int u = 0; u < kPerThread; ++u) {
+    const long long t = t_begin + tid + u * kThreads;
+    if (t >= a.max_ctx) continue;
+    long long sl = -1, tm = -1;
+    if (page[u] != -2) {
+      if (page[u] < 0 || page[u] >= a.num_pages) atomicCAS(&s_err, 0, PIC_DEV_BAD_PAGE);
+      else sl = (long long)page[u] * a.page + t % a.page;
+      if (t >= P && t < span_end) {  // document token: last doc whose offset <= t
+        int lo = 0, hi = m - 1;
+        while (lo < hi) {
+          const int mid = (lo + hi + 1) >> 1;
+          if (s_off[mid] <= t) lo = mid;
+          else hi = mid - 1;
+        }
+        tm = ((long long)lo << 40) | (s_start[lo] + (t - s_off[lo]));
+      }
     }
-    slots[t] = s;
+    slots[t] = sl;
+    tmap[t] = tm;
   }
   if (lead) {
     int32_t *ip = a.inline_pos + (size_t)b * a.max_inline;
@@ -141,13 +173,14 @@ __global__ void __launch_bounds__(kThreads) compose_kernel(ComposeArgs a) {
 
 extern "C" pic_status_t pic_compose(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
                                     int32_t n_pool_docs, const int32_t *doc_len,
-                                    const int32_t *doc_base_pos, const int32_t *req_doc_ids,
+                                    const int32_t *doc_base_pos, const int64_t *doc_token_start,
+                                    const int32_t *req_doc_ids,
                                     const int32_t *req_num_docs, const int32_t *prefix_len,
                                     const int32_t *query_len, const int32_t *block_table,
                                     int32_t max_pages, int64_t num_pages, int32_t max_ctx,
                                     int32_t max_inline, int32_t *doc_offset, int32_t *doc_delta,
-                                    int64_t *slot_mapping, int32_t *inline_pos, int32_t *ctx_len,
-                                    pic_stream_t stream) {
+                                    int64_t *slot_mapping, int64_t *tok_map,
+                                    int32_t *inline_pos, int32_t *ctx_len, pic_stream_t stream) {
   using namespace pic;
   double theta[kMaxHalfDim];
   pic_status_t st = check_geom(geom, theta);
@@ -157,9 +190,12 @@ extern "C" pic_status_t pic_compose(const pic_geom_t *geom, int32_t batch, int32
     return fail(PIC_ERR_INVALID_ARG, "pic_compose: sizes must be positive");
   if (num_pages > (int64_t)INT32_MAX)
     return fail(PIC_ERR_INVALID_ARG, "pic_compose: num_pages exceeds int32");
-  if (!doc_len || !doc_base_pos || !req_num_docs || !prefix_len || !query_len || !block_table ||
-      !slot_mapping || !inline_pos || !ctx_len || (max_docs > 0 && (!req_doc_ids || !doc_offset || !doc_delta)))
+  if (!doc_len || !doc_base_pos || !doc_token_start || !req_num_docs || !prefix_len ||
+      !query_len || !block_table || !slot_mapping || !tok_map || !inline_pos || !ctx_len ||
+      (max_docs > 0 && (!req_doc_ids || !doc_offset || !doc_delta)))
     return fail(PIC_ERR_INVALID_ARG, "pic_compose: NULL tensor");
+  if (max_docs > kMaxDocs)
+    return fail(PIC_ERR_UNSUPPORTED, "pic_compose: max_docs %d > %d", max_docs, kMaxDocs);
   int32_t *status = device_status_ptr();
   if (!status) return fail(PIC_ERR_CUDA, "pic_compose: no device status word");
   ComposeArgs a;
@@ -173,6 +209,7 @@ extern "C" pic_status_t pic_compose(const pic_geom_t *geom, int32_t batch, int32
   a.num_pages = num_pages;
   a.doc_len = doc_len;
   a.doc_base = doc_base_pos;
+  a.doc_start = doc_token_start;
   a.ids = req_doc_ids;
   a.num_docs = req_num_docs;
   a.prefix = prefix_len;
@@ -183,9 +220,16 @@ extern "C" pic_status_t pic_compose(const pic_geom_t *geom, int32_t batch, int32
   a.inline_pos = inline_pos;
   a.ctx_len = ctx_len;
   a.slot_mapping = slot_mapping;
+  a.tok_map = tok_map;
   a.status = status;
   dim3 grid((max_ctx + kSlotsPerCta - 1) / kSlotsPerCta, batch);
-  compose_kernel<<<grid, kThreads, 0, stream>>>(a);
+  const size_t smem = (size_t)max_docs * (sizeof(long long) + sizeof(int32_t)) + 16;
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(compose_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return cuda_fail(e, "pic_compose smem attribute");
+  }
+  compose_kernel<<<grid, kThreads, smem, stream>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_compose launch");
   return PIC_OK;

@@ -62,7 +62,7 @@ enum {
 };
 
 struct Params {
-  int Hq, Hkv, G, max_inline, R_pad, m_tiles, num_splits, max_pages, oob_row;
+  int batch, Hq, Hkv, G, max_inline, R_pad, m_tiles, num_splits, max_pages, oob_row;
   long long num_pages, layer_row0;
   const int32_t *inline_pos, *inline_len, *block_table;
   __nv_bfloat16 *out;
@@ -351,48 +351,51 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // Merge split partials (O unnormalised, m in log2 units, l) by log-sum-exp.
+// One warp per query row; lanes hold the splits' (m, l), then D/32 columns.
 template <int D>
-__global__ void combine_kernel(Params p) {
-  const int mt = blockIdx.x, hk = blockIdx.y, b = blockIdx.z;
-  const int tin = min(max(p.inline_len[b], 0), p.max_inline);
-  const int rows = tin * p.G;
+__global__ void __launch_bounds__(256) combine_kernel(Params p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long grow = (long long)blockIdx.x * (blockDim.x >> 5) + warp;
+  const long long per_b = (long long)p.Hkv * p.m_tiles * BM;
+  const int b = (int)(grow / per_b);
+  if (b >= p.batch) return;
+  const long long rem = grow % per_b;
+  const int hk = (int)(rem / ((long long)p.m_tiles * BM));
+  const int mt = (int)((rem / BM) % p.m_tiles), row = (int)(rem % BM);
+  const int tin = min(max(p.inline_len[b], 0), p.max_inline);
+  const int rg = mt * BM + row;
+  if (rg >= tin * p.G) return;
   const int S = p.num_splits;
-  for (int row = warp; row < BM; row += blockDim.x >> 5) {
-    const int rg = mt * BM + row;
-    if (rg >= rows) break;
-    const size_t base = (((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * S;
-    float ms = -INFINITY, ls = 0.f;
-    if (lane < S) {
-      ms = p.part_ml[((base + lane) * BM + row) * 2];
-      ls = p.part_ml[((base + lane) * BM + row) * 2 + 1];
-    }
-    float M = ms;
-#pragma unroll
-    for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    const float w = (ms == -INFINITY) ? 0.f : ex2(ms - M);
-    float Lsum = w * ls;
-#pragma unroll
-    for (int o = 16; o; o >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, o);
-    float acc[D / 32];
-#pragma unroll
-    for (int q = 0; q < D / 32; ++q) acc[q] = 0.f;
-    for (int s = 0; s < S; ++s) {
-      const float ws = __shfl_sync(0xffffffffu, w, s);
-      if (ws == 0.f) continue;
-      const float *src = p.part_o + ((base + s) * BM + row) * D;
-#pragma unroll
-      for (int q = 0; q < D / 32; ++q) acc[q] = fmaf(ws, src[q * 32 + lane], acc[q]);
-    }
-    const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
-    const int tok = rg / p.G, g = rg % p.G;
-    __nv_bfloat16 *dst = p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D;
-#pragma unroll
-    for (int q = 0; q < D / 32; ++q) dst[q * 32 + lane] = __float2bfloat16_rn(acc[q] * inv);
-    if (p.lse && lane == 0)
-      p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
-          Lsum > 0.f ? (M + __log2f(Lsum)) * 0.69314718055994531f : -INFINITY;
+  const size_t base = (((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * S;
+  float ms = -INFINITY, ls = 0.f;
+  if (lane < S) {
+    ms = p.part_ml[((base + lane) * BM + row) * 2];
+    ls = p.part_ml[((base + lane) * BM + row) * 2 + 1];
   }
+  float M = ms;
+#pragma unroll
+  for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  const float w = (ms == -INFINITY) ? 0.f : ex2(ms - M);
+  float Lsum = w * ls;
+#pragma unroll
+  for (int o = 16; o; o >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, o);
+  float acc[D / 32];
+#pragma unroll
+  for (int q = 0; q < D / 32; ++q) acc[q] = 0.f;
+  for (int s = 0; s < S; ++s) {
+    const float ws = __shfl_sync(0xffffffffu, w, s);
+    const float *src = p.part_o + ((base + s) * BM + row) * D;
+#pragma unroll
+    for (int q = 0; q < D / 32; ++q) acc[q] = fmaf(ws, ws == 0.f ? 0.f : src[q * 32 + lane], acc[q]);
+  }
+  const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
+  const int tok = rg / p.G, g = rg % p.G;
+  __nv_bfloat16 *dst = p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D;
+#pragma unroll
+  for (int q = 0; q < D / 32; ++q) dst[q * 32 + lane] = __float2bfloat16_rn(acc[q] * inv);
+  if (p.lse && lane == 0)
+    p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
+        Lsum > 0.f ? (M + __log2f(Lsum)) * 0.69314718055994531f : -INFINITY;
 }
 
 // RoPE the inline keys/queries at their logical positions; keys and values go
@@ -408,7 +411,7 @@ struct AppendArgs {
 };
 
 template <int D>
-__global__ void __launch_bounds__(128) append_kernel(AppendArgs a, RopeParams rp) {
+__global__ void __launch_bounds__(256) append_kernel(AppendArgs a, RopeParams rp) {
   constexpr int HALF = D / 2, KC = D / 16, VC = D / 8;
   const int t = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
   const int tin = min(max(a.inline_len[b], 0), a.max_inline);
@@ -423,7 +426,24 @@ __global__ void __launch_bounds__(128) append_kernel(AppendArgs a, RopeParams rp
     }
     return;
   }
-  const int pos = a.inline_pos[(size_t)b * a.max_inline + t];
+  const size_t tok = (size_t)b * a.max_inline + t;
+  const int nQ = a.Hq * KC, nK = a.Hkv * KC, nV = a.Hkv * VC;
+  // First round of loads goes out before the position is even known.
+  uint4 qa = make_uint4(0, 0, 0, 0), qb = qa, ka = qa, kb = qa, vv = qa;
+  const PairChunk pq = pair_chunk(tid % KC, HALF, rp.style);
+  if (tid < nQ) {
+    const __nv_bfloat16 *src = a.q + (tok * a.Hq + tid / KC) * D;
+    qa = ld_stream(src + pq.off_a);
+    qb = ld_stream(src + pq.off_b);
+  }
+  if (tid < nK) {
+    const __nv_bfloat16 *src = a.k + (tok * a.Hkv + tid / KC) * D;
+    ka = ld_stream(src + pq.off_a);
+    kb = ld_stream(src + pq.off_b);
+  }
+  if (tid < nV) vv = ld_stream(a.v + (tok * a.Hkv + tid / VC) * D + (tid % VC) * 8);
+
+  const int pos = a.inline_pos[tok];
   const bool pos_ok = pos >= 0 && pos < a.max_ctx;
   long long slot = pos_ok ? a.slots[(size_t)b * a.max_ctx + pos] : -1;
   if (!pos_ok) {
@@ -434,26 +454,64 @@ __global__ void __launch_bounds__(128) append_kernel(AppendArgs a, RopeParams rp
   }
   for (int i = tid; i < HALF; i += blockDim.x) cs[i] = rope_cos_sin(pos_ok ? pos : 0, rp.theta[i]);
   __syncthreads();
-  const size_t tok = (size_t)b * a.max_inline + t;
+  const long long page = slot >> 4, r = slot & 15;
+
+  auto rot_store = [&](uint4 xa, uint4 xb, int c, __nv_bfloat16 *dst) {
+    float x[8], y[8], u[8], w[8];
+    unpack8(xa, x);
+    unpack8(xb, y);
+    if (rp.style == PIC_ROPE_HALF) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) { u[i] = x[i]; w[i] = y[i]; }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        u[i] = x[2 * i]; w[i] = x[2 * i + 1];
+        u[4 + i] = y[2 * i]; w[4 + i] = y[2 * i + 1];
+      }
+    }
+    rotate8(u, w, cs + 8 * c);
+    if (rp.style == PIC_ROPE_HALF) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) { x[i] = u[i]; y[i] = w[i]; }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        x[2 * i] = u[i]; x[2 * i + 1] = w[i];
+        y[2 * i] = u[4 + i]; y[2 * i + 1] = w[4 + i];
+      }
+    }
+    const PairChunk pc = pair_chunk(c, HALF, rp.style);
+    st_global16(dst + pc.off_a, pack8(x));
+    st_global16(dst + pc.off_b, pack8(y));
+  };
+  auto q_dst = [&](int h) {
+    const int hk = h / a.G, g = h % a.G;
+    return a.qpack + (((size_t)b * a.Hkv + hk) * a.R_pad + (size_t)t * a.G + g) * D;
+  };
+  if (tid < nQ) rot_store(qa, qb, tid % KC, q_dst(tid / KC));
   if (slot >= 0) {
-    const long long page = slot >> 4, r = slot & 15;
-    for (int e = tid; e < a.Hkv * KC; e += blockDim.x) {
+    if (tid < nK)
+      rot_store(ka, kb, tid % KC, a.k_cache + ((page * a.Hkv + tid / KC) * 16 + r) * D);
+    if (tid < nV)
+      st_global16(a.v_cache + ((page * a.Hkv + tid / VC) * 16 + r) * D + (tid % VC) * 8, vv);
+  }
+  // remaining rounds (more than 256 tasks of a kind: very wide models)
+  for (int e = tid + blockDim.x; e < nQ; e += blockDim.x) {
+    const int h = e / KC, c = e % KC;
+    rotate_chunk(a.q + (tok * a.Hq + h) * D, q_dst(h), c, HALF, rp.style, cs + 8 * c, true);
+  }
+  if (slot >= 0) {
+    for (int e = tid + blockDim.x; e < nK; e += blockDim.x) {
       const int h = e / KC, c = e % KC;
       rotate_chunk(a.k + (tok * a.Hkv + h) * D, a.k_cache + ((page * a.Hkv + h) * 16 + r) * D, c,
                    HALF, rp.style, cs + 8 * c, true);
     }
-    for (int e = tid; e < a.Hkv * VC; e += blockDim.x) {
+    for (int e = tid + blockDim.x; e < nV; e += blockDim.x) {
       const int h = e / VC, c = e % VC;
       st_global16(a.v_cache + ((page * a.Hkv + h) * 16 + r) * D + c * 8,
                   ld_stream(a.v + (tok * a.Hkv + h) * D + c * 8));
     }
-  }
-  for (int e = tid; e < a.Hq * KC; e += blockDim.x) {
-    const int h = e / KC, c = e % KC;
-    const int hk = h / a.G, g = h % a.G;
-    const int row = t * a.G + g;
-    rotate_chunk(a.q + (tok * a.Hq + h) * D, a.qpack + (((size_t)b * a.Hkv + hk) * a.R_pad + row) * D,
-                 c, HALF, rp.style, cs + 8 * c, true);
   }
 }
 
@@ -597,8 +655,8 @@ extern "C" pic_status_t pic_append_inline(
   if (t_slots > INT32_MAX / 2 || batch > 65535)
     return fail(PIC_ERR_UNSUPPORTED, "pic_append_inline: grid too large");
   dim3 agrid(t_slots, batch);
-  if (D == 128) append_kernel<128><<<agrid, 128, 0, stream>>>(aa, rp);
-  else append_kernel<64><<<agrid, 128, 0, stream>>>(aa, rp);
+  if (D == 128) append_kernel<128><<<agrid, 256, 0, stream>>>(aa, rp);
+  else append_kernel<64><<<agrid, 256, 0, stream>>>(aa, rp);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_append_inline launch");
   return PIC_OK;
@@ -635,6 +693,7 @@ extern "C" pic_status_t pic_attend_prefill(
   if (st == PIC_OK) st = encode_tmap_2d(&tv, v_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
   if (st != PIC_OK) return st;
   Params pp;
+  pp.batch = batch;
   pp.Hq = geom->num_q_heads;
   pp.Hkv = Hkv;
   pp.G = pl.G;
@@ -670,7 +729,8 @@ extern "C" pic_status_t pic_attend_prefill(
     attn_kernel<64><<<grid, kThreads, smem, stream>>>(tq, tk, tv, pp);
   }
   if (pl.splits > 1) {
-    dim3 cgrid(pl.m_tiles, Hkv, batch);
+    const long long rows = (long long)batch * Hkv * pl.m_tiles * BM;
+    const unsigned cgrid = (unsigned)((rows + 7) / 8);
     if (D == 128) combine_kernel<128><<<cgrid, 256, 0, stream>>>(pp);
     else combine_kernel<64><<<cgrid, 256, 0, stream>>>(pp);
   }

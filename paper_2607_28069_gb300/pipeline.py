@@ -33,6 +33,7 @@ class CacheHitPath:
         self.doc_offset = torch.empty((B, md), dtype=i32, device=dev)
         self.doc_delta = torch.empty((B, md), dtype=i32, device=dev)
         self.slot_mapping = torch.empty((B, self.max_ctx), dtype=i64, device=dev)
+        self.tok_map = torch.empty((B, self.max_ctx), dtype=i64, device=dev)
         self.inline_pos = torch.empty((B, self.max_inline), dtype=i32, device=dev)
         self.ctx_len = torch.empty((B,), dtype=i32, device=dev)
         shape = (L, wl.num_pages, Hkv, spec.page_size, d)
@@ -57,18 +58,17 @@ class CacheHitPath:
     # -- a1: layout and slot map
     def compose(self):
         wl = self.wl
-        pic_compose(self.geom, wl.doc_len, wl.doc_base_pos, wl.req_doc_ids, wl.req_num_docs,
-                    wl.prefix_len, wl.query_len, wl.block_table, wl.num_pages, self.max_ctx,
-                    self.max_inline, self.doc_offset, self.doc_delta, self.slot_mapping,
-                    self.inline_pos, self.ctx_len)
+        pic_compose(self.geom, wl.doc_len, wl.doc_base_pos, wl.doc_token_start, wl.req_doc_ids,
+                    wl.req_num_docs, wl.prefix_len, wl.query_len, wl.block_table, wl.num_pages,
+                    self.max_ctx, self.max_inline, self.doc_offset, self.doc_delta,
+                    self.slot_mapping, self.tok_map, self.inline_pos, self.ctx_len)
 
     # -- a2 + a3: per-document rotation and stitching, all layers, one launch
     def relocate(self, layer_begin: int = 0, layer_end: int | None = None):
         wl = self.wl
         if layer_end is None:
             layer_end = wl.spec.layers
-        pic_relocate(self.geom, wl.k_pool, wl.v_pool, wl.doc_token_start, wl.doc_len,
-                     wl.req_doc_ids, wl.req_num_docs, self.doc_offset, self.doc_delta,
+        pic_relocate(self.geom, wl.k_pool, wl.v_pool, self.tok_map, self.doc_delta,
                      self.slot_mapping, wl.num_pages, self.k_cache, self.v_cache, layer_begin,
                      layer_end)
 
