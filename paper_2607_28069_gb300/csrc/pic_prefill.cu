@@ -23,8 +23,9 @@
 //     to TMEM as bf16 over S, rescale O only when the running maximum grew by
 //     more than 2^8, and finally normalise O.  Scores are kept in the log2
 //     domain (scale folded with log2 e) and exponentiated with ex2.approx.
-//  2. combine_kernel (only when the key range is split): log-sum-exp merge of
-//     the per-split partial (O, m, l).
+//     When the key range of a tile is split over several CTAs, each writes its
+//     partial (O, m, l); the CTA whose arrival completes the tile's counter
+//     merges them by log-sum-exp and resets the counter (no extra launch).
 #include "pic_internal.cuh"
 
 namespace pic {
@@ -67,9 +68,90 @@ struct Params {
   const int32_t *inline_pos, *inline_len, *block_table;
   __nv_bfloat16 *out;
   float *lse, *part_o, *part_ml;
+  int32_t *counters;  // [B][Hkv][m_tiles] arrival counts of the splits
   int32_t *status;
   float scale_log2;
 };
+
+// Log-sum-exp merge of the S split partials of one 128-row query tile
+// (O unnormalised, m in log2 units, l), done by 4 warps: each warp takes rows
+// r = w, w+4, ...; lanes cover the d columns so every load is coalesced, and
+// 8 rows are processed per batch to keep loads in flight.
+template <int D>
+__device__ void merge_tile(const Params &p, int b, int hk, int mt, int w, int lane) {
+  constexpr int CPL = D / 32;  // columns per lane
+  const int S = p.num_splits;
+  const int tin = min(max(p.inline_len[b], 0), p.max_inline);
+  const int rows = tin * p.G;
+  const size_t base = (((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * S;
+  for (int r0 = w; r0 < BM; r0 += 4 * 8) {
+    float acc[8][CPL], lsum[8], mbig[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int row = r0 + 4 * u;
+      float ms = -INFINITY, ls = 0.f;
+      if (row < BM && lane < S) {
+        ms = p.part_ml[((base + lane) * BM + row) * 2];
+        ls = p.part_ml[((base + lane) * BM + row) * 2 + 1];
+      }
+      float M = ms;
+#pragma unroll
+      for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+      const float wt = (ms == -INFINITY) ? 0.f : ex2(ms - M);
+      float L = wt * ls;
+#pragma unroll
+      for (int o = 16; o; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+      lsum[u] = L;
+      mbig[u] = M;
+#pragma unroll
+      for (int q = 0; q < CPL; ++q) acc[u][q] = 0.f;
+      for (int sp = 0; sp < S; ++sp) {
+        const float ws = __shfl_sync(0xffffffffu, wt, sp);
+        if (row < BM && ws != 0.f) {
+          const float *src = p.part_o + ((base + sp) * BM + row) * D + lane * CPL;
+#pragma unroll
+          for (int q = 0; q < CPL; ++q) acc[u][q] = fmaf(ws, src[q], acc[u][q]);
+        }
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int row = r0 + 4 * u, rg = mt * BM + row;
+      if (row >= BM || rg >= rows) continue;
+      const float inv = lsum[u] > 0.f ? 1.f / lsum[u] : 0.f;
+      const int tok = rg / p.G, g = rg % p.G;
+      __nv_bfloat16 *dst =
+          p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D + lane * CPL;
+#pragma unroll
+      for (int q = 0; q < CPL; q += 2)
+        *reinterpret_cast<uint32_t *>(dst + q) = pack2(acc[u][q] * inv, acc[u][q + 1] * inv);
+      if (p.lse && lane == 0)
+        p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
+            lsum[u] > 0.f ? (mbig[u] + __log2f(lsum[u])) * 0.69314718055994531f : -INFINITY;
+    }
+  }
+}
+
+// Publish this split's partial for tile (b, hk, mt); the CTA whose arrival
+// completes the count merges all splits and resets the counter.  Called by
+// 128 threads that share named barrier `bar_id`.
+template <int D>
+__device__ void arrive_and_merge(const Params &p, int b, int hk, int mt, int tid128, int bar_id,
+                                 int *s_flag) {
+  __threadfence();
+  asm volatile("bar.sync %0, 128;" ::"r"(bar_id) : "memory");
+  const size_t tile = ((size_t)b * p.Hkv + hk) * p.m_tiles + mt;
+  if (tid128 == 0) {
+    const int old = atomicAdd(p.counters + tile, 1);
+    *s_flag = (old == p.num_splits - 1);
+  }
+  asm volatile("bar.sync %0, 128;" ::"r"(bar_id) : "memory");
+  if (*s_flag) {
+    __threadfence();
+    merge_tile<D>(p, b, hk, mt, tid128 >> 5, tid128 & 31);
+    if (tid128 == 0) p.counters[tile] = 0;  // ready for the next call
+  }
+}
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -110,10 +192,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const size_t part_row0 =
       ((((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * p.num_splits + split) * BM;
 
-  if (n == 0) {  // empty split: neutral partial state
+  if (n == 0) {  // empty split: neutral partial state, then count the arrival
     if (p.num_splits > 1 && threadIdx.x < BM) {
       p.part_ml[(part_row0 + threadIdx.x) * 2] = -INFINITY;
       p.part_ml[(part_row0 + threadIdx.x) * 2 + 1] = 0.f;
+      __shared__ int s_flag0;
+      arrive_and_merge<D>(p, b, hk, mt, threadIdx.x, 1, &s_flag0);
     }
     return;
   }
@@ -250,10 +334,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int c = 0; c < BN; ++c)
           if (key0 + c > pos) s[c] = -INFINITY;
       }
-      float mx = s[0];
+      // row max: 8 independent chains, then a 3-level tree
+      float mx8[8];
 #pragma unroll
-      for (int c = 1; c < BN; ++c) mx = fmaxf(mx, s[c]);
-      const float m_new = fmaxf(m_used, mx * p.scale_log2);
+      for (int i = 0; i < 8; ++i) mx8[i] = s[i];
+#pragma unroll
+      for (int c = 8; c < BN; c += 8)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) mx8[i] = fmaxf(mx8[i], s[c + i]);
+#pragma unroll
+      for (int w = 4; w; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) mx8[i] = fmaxf(mx8[i], mx8[i + w]);
+      const float m_new = fmaxf(m_used, mx8[0] * p.scale_log2);
       float alpha = 1.f;
       const bool resc = m_new > m_used + 8.f;
       if (resc) {
@@ -261,15 +354,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         m_used = m_new;
       }
       const float mref = (m_used == -INFINITY) ? 0.f : m_used;
-      l *= alpha;
       uint32_t pk[BN / 2];
+      float ls8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ls8[i] = 0.f;
 #pragma unroll
       for (int c = 0; c < BN; c += 2) {
         const float p0 = ex2(fmaf(s[c], p.scale_log2, -mref));
         const float p1 = ex2(fmaf(s[c + 1], p.scale_log2, -mref));
-        l += p0 + p1;
+        ls8[(c >> 1) & 7] += p0 + p1;
         pk[c / 2] = pack2(p0, p1);
       }
+#pragma unroll
+      for (int w = 4; w; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) ls8[i] += ls8[i + w];
+      l = fmaf(l, alpha, ls8[0]);
       // O correction, only when some row of this warp moved its maximum.
       if (j > 0 && __any_sync(0xffffffffu, resc)) {
         const int pj = j - 1;
@@ -335,6 +435,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         p.part_ml[(part_row0 + row) * 2 + 1] = l;
       }
     }
+    if (p.num_splits > 1) {
+      // every softmax thread reaches here (ok is warp-uniform and the same for all
+      // four warps unless a wait timed out, in which case the result is void anyway)
+      __shared__ int s_flag1;
+      arrive_and_merge<D>(p, b, hk, mt, threadIdx.x - 64, 1, &s_flag1);
+    }
   }
 
   tc_fence_before();
@@ -350,59 +456,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// Merge split partials (O unnormalised, m in log2 units, l) by log-sum-exp.
-// One warp per query row; lanes hold the splits' (m, l), then D/32 columns.
-template <int D>
-__global__ void __launch_bounds__(256) combine_kernel(Params p) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long long grow = (long long)blockIdx.x * (blockDim.x >> 5) + warp;
-  const long long per_b = (long long)p.Hkv * p.m_tiles * BM;
-  const int b = (int)(grow / per_b);
-  if (b >= p.batch) return;
-  const long long rem = grow % per_b;
-  const int hk = (int)(rem / ((long long)p.m_tiles * BM));
-  const int mt = (int)((rem / BM) % p.m_tiles), row = (int)(rem % BM);
-  const int tin = min(max(p.inline_len[b], 0), p.max_inline);
-  const int rg = mt * BM + row;
-  if (rg >= tin * p.G) return;
-  const int S = p.num_splits;
-  const size_t base = (((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * S;
-  float ms = -INFINITY, ls = 0.f;
-  if (lane < S) {
-    ms = p.part_ml[((base + lane) * BM + row) * 2];
-    ls = p.part_ml[((base + lane) * BM + row) * 2 + 1];
-  }
-  float M = ms;
-#pragma unroll
-  for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-  const float w = (ms == -INFINITY) ? 0.f : ex2(ms - M);
-  float Lsum = w * ls;
-#pragma unroll
-  for (int o = 16; o; o >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, o);
-  float acc[D / 32];
-#pragma unroll
-  for (int q = 0; q < D / 32; ++q) acc[q] = 0.f;
-  for (int s = 0; s < S; ++s) {
-    const float ws = __shfl_sync(0xffffffffu, w, s);
-    const float *src = p.part_o + ((base + s) * BM + row) * D;
-#pragma unroll
-    for (int q = 0; q < D / 32; ++q) acc[q] = fmaf(ws, ws == 0.f ? 0.f : src[q * 32 + lane], acc[q]);
-  }
-  const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
-  const int tok = rg / p.G, g = rg % p.G;
-  __nv_bfloat16 *dst = p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D;
-#pragma unroll
-  for (int q = 0; q < D / 32; ++q) dst[q * 32 + lane] = __float2bfloat16_rn(acc[q] * inv);
-  if (p.lse && lane == 0)
-    p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
-        Lsum > 0.f ? (M + __log2f(Lsum)) * 0.69314718055994531f : -INFINITY;
-}
-
 // RoPE the inline keys/queries at their logical positions; keys and values go
 // to their cache slots, queries to the GQA-packed workspace.
 struct AppendArgs {
-  int Hq, Hkv, G, max_inline, max_ctx, R_pad;
+  int Hq, Hkv, G, max_inline, max_ctx, R_pad, n_counters;
   long long num_pages;
+  int32_t *counters;
   const __nv_bfloat16 *q, *k, *v;
   const int32_t *inline_pos, *inline_len;
   const int64_t *slots;
@@ -416,6 +475,8 @@ __global__ void __launch_bounds__(256) append_kernel(AppendArgs a, RopeParams rp
   const int t = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
   const int tin = min(max(a.inline_len[b], 0), a.max_inline);
   __shared__ float2 cs[HALF];
+  if (t == 0 && b == 0)  // split-merge counters of pic_attend_prefill start at zero
+    for (int e = tid; e < a.n_counters; e += blockDim.x) a.counters[e] = 0;
   if (t >= tin) {  // zero the packed query rows of this token slot
     for (int e = tid; e < a.Hkv * a.G * VC; e += blockDim.x) {
       const int hk = e / (a.G * VC), r = e % (a.G * VC), g = r / VC, c = r % VC;
@@ -517,7 +578,7 @@ __global__ void __launch_bounds__(256) append_kernel(AppendArgs a, RopeParams rp
 
 struct Plan {
   int G, m_tiles, R_pad, splits;
-  size_t q_bytes, po_bytes, pml_bytes, total;
+  size_t q_bytes, cnt_bytes, po_bytes, pml_bytes, total;
 };
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -544,6 +605,7 @@ inline Plan plan(const pic_geom_t *g, int batch, int max_inline, int max_ctx, in
   }
   pl.splits = num_splits;
   pl.q_bytes = align256((size_t)batch * g->num_kv_heads * pl.R_pad * g->head_dim * 2);
+  pl.cnt_bytes = align256((size_t)batch * g->num_kv_heads * pl.m_tiles * sizeof(int32_t));
   if (pl.splits > 1) {
     const size_t rows = (size_t)batch * g->num_kv_heads * pl.m_tiles * pl.splits * BM;
     pl.po_bytes = align256(rows * g->head_dim * 4);
@@ -551,7 +613,7 @@ inline Plan plan(const pic_geom_t *g, int batch, int max_inline, int max_ctx, in
   } else {
     pl.po_bytes = pl.pml_bytes = 0;
   }
-  pl.total = pl.q_bytes + pl.po_bytes + pl.pml_bytes;
+  pl.total = pl.q_bytes + pl.cnt_bytes + pl.po_bytes + pl.pml_bytes;
   return pl;
 }
 
@@ -650,6 +712,8 @@ extern "C" pic_status_t pic_append_inline(
   aa.k_cache = static_cast<__nv_bfloat16 *>(k_cache) + (size_t)layer * layer_elems;
   aa.v_cache = static_cast<__nv_bfloat16 *>(v_cache) + (size_t)layer * layer_elems;
   aa.qpack = static_cast<__nv_bfloat16 *>(workspace);
+  aa.counters = reinterpret_cast<int32_t *>(static_cast<uint8_t *>(workspace) + pl.q_bytes);
+  aa.n_counters = batch * Hkv * pl.m_tiles;
   aa.status = status;
   const int t_slots = std::max(max_inline, (pl.R_pad + pl.G - 1) / pl.G);
   if (t_slots > INT32_MAX / 2 || batch > 65535)
@@ -710,8 +774,11 @@ extern "C" pic_status_t pic_attend_prefill(
   pp.block_table = block_table;
   pp.out = static_cast<__nv_bfloat16 *>(out);
   pp.lse = lse;
-  pp.part_o = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes) : nullptr;
-  pp.part_ml = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes + pl.po_bytes) : nullptr;
+  pp.counters = reinterpret_cast<int32_t *>(ws + pl.q_bytes);
+  pp.part_o = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes + pl.cnt_bytes) : nullptr;
+  pp.part_ml = pl.splits > 1
+                   ? reinterpret_cast<float *>(ws + pl.q_bytes + pl.cnt_bytes + pl.po_bytes)
+                   : nullptr;
   pp.status = status;
   pp.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
 
@@ -727,12 +794,6 @@ extern "C" pic_status_t pic_attend_prefill(
     e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill smem attribute");
     attn_kernel<64><<<grid, kThreads, smem, stream>>>(tq, tk, tv, pp);
-  }
-  if (pl.splits > 1) {
-    const long long rows = (long long)batch * Hkv * pl.m_tiles * BM;
-    const unsigned cgrid = (unsigned)((rows + 7) / 8);
-    if (D == 128) combine_kernel<128><<<cgrid, 256, 0, stream>>>(pp);
-    else combine_kernel<64><<<cgrid, 256, 0, stream>>>(pp);
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill launch");
