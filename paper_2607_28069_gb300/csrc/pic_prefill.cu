@@ -17,15 +17,16 @@
 //  1. attn_kernel: one CTA per (128-row query tile, key split, kv head,
 //     request).  Warp-specialised: warp 0 issues TMA loads (Q once, then
 //     128-key K and V tiles page by page from the paged cache through the
-//     block table, 3-stage ring), warp 1 issues tcgen05.mma (S = Q K^T into
+//     block table, 3-stage ring; its 32 lanes issue the 32 page boxes of a
+//     tile at once and fetch the next tile's block-table entries ahead), warp 1 issues tcgen05.mma (S = Q K^T into
 //     TMEM, then O += P V with P read from TMEM), warps 2-5 run the online
 //     softmax on S rows straight from TMEM (one thread per row), write P back
 //     to TMEM as bf16 over S, rescale O only when the running maximum grew by
 //     more than 2^8, and finally normalise O.  Scores are kept in the log2
 //     domain (scale folded with log2 e) and exponentiated with ex2.approx.
-//     When the key range of a tile is split over several CTAs, each writes its
-//     partial (O, m, l); the CTA whose arrival completes the tile's counter
-//     merges them by log-sum-exp and resets the counter (no extra launch).
+//  2. combine_kernel (only when the key range of a tile is split over several
+//     CTAs): log-sum-exp merge of the per-split partials (O, m, l), one warp
+//     per query row.
 #include "pic_internal.cuh"
 
 namespace pic {
@@ -68,90 +69,9 @@ struct Params {
   const int32_t *inline_pos, *inline_len, *block_table;
   __nv_bfloat16 *out;
   float *lse, *part_o, *part_ml;
-  int32_t *counters;  // [B][Hkv][m_tiles] arrival counts of the splits
   int32_t *status;
   float scale_log2;
 };
-
-// Log-sum-exp merge of the S split partials of one 128-row query tile
-// (O unnormalised, m in log2 units, l), done by 4 warps: each warp takes rows
-// r = w, w+4, ...; lanes cover the d columns so every load is coalesced, and
-// 8 rows are processed per batch to keep loads in flight.
-template <int D>
-__device__ void merge_tile(const Params &p, int b, int hk, int mt, int w, int lane) {
-  constexpr int CPL = D / 32;  // columns per lane
-  const int S = p.num_splits;
-  const int tin = min(max(p.inline_len[b], 0), p.max_inline);
-  const int rows = tin * p.G;
-  const size_t base = (((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * S;
-  for (int r0 = w; r0 < BM; r0 += 4 * 8) {
-    float acc[8][CPL], lsum[8], mbig[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      const int row = r0 + 4 * u;
-      float ms = -INFINITY, ls = 0.f;
-      if (row < BM && lane < S) {
-        ms = p.part_ml[((base + lane) * BM + row) * 2];
-        ls = p.part_ml[((base + lane) * BM + row) * 2 + 1];
-      }
-      float M = ms;
-#pragma unroll
-      for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-      const float wt = (ms == -INFINITY) ? 0.f : ex2(ms - M);
-      float L = wt * ls;
-#pragma unroll
-      for (int o = 16; o; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-      lsum[u] = L;
-      mbig[u] = M;
-#pragma unroll
-      for (int q = 0; q < CPL; ++q) acc[u][q] = 0.f;
-      for (int sp = 0; sp < S; ++sp) {
-        const float ws = __shfl_sync(0xffffffffu, wt, sp);
-        if (row < BM && ws != 0.f) {
-          const float *src = p.part_o + ((base + sp) * BM + row) * D + lane * CPL;
-#pragma unroll
-          for (int q = 0; q < CPL; ++q) acc[u][q] = fmaf(ws, src[q], acc[u][q]);
-        }
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      const int row = r0 + 4 * u, rg = mt * BM + row;
-      if (row >= BM || rg >= rows) continue;
-      const float inv = lsum[u] > 0.f ? 1.f / lsum[u] : 0.f;
-      const int tok = rg / p.G, g = rg % p.G;
-      __nv_bfloat16 *dst =
-          p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D + lane * CPL;
-#pragma unroll
-      for (int q = 0; q < CPL; q += 2)
-        *reinterpret_cast<uint32_t *>(dst + q) = pack2(acc[u][q] * inv, acc[u][q + 1] * inv);
-      if (p.lse && lane == 0)
-        p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
-            lsum[u] > 0.f ? (mbig[u] + __log2f(lsum[u])) * 0.69314718055994531f : -INFINITY;
-    }
-  }
-}
-
-// Publish this split's partial for tile (b, hk, mt); the CTA whose arrival
-// completes the count merges all splits and resets the counter.  Called by
-// 128 threads that share named barrier `bar_id`.
-template <int D>
-__device__ void arrive_and_merge(const Params &p, int b, int hk, int mt, int tid128, int bar_id,
-                                 int *s_flag) {
-  __threadfence();
-  asm volatile("bar.sync %0, 128;" ::"r"(bar_id) : "memory");
-  const size_t tile = ((size_t)b * p.Hkv + hk) * p.m_tiles + mt;
-  if (tid128 == 0) {
-    const int old = atomicAdd(p.counters + tile, 1);
-    *s_flag = (old == p.num_splits - 1);
-  }
-  asm volatile("bar.sync %0, 128;" ::"r"(bar_id) : "memory");
-  if (*s_flag) {
-    __threadfence();
-    merge_tile<D>(p, b, hk, mt, tid128 >> 5, tid128 & 31);
-    if (tid128 == 0) p.counters[tile] = 0;  // ready for the next call
-  }
-}
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -192,12 +112,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const size_t part_row0 =
       ((((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * p.num_splits + split) * BM;
 
-  if (n == 0) {  // empty split: neutral partial state, then count the arrival
+  if (n == 0) {  // empty split: neutral partial state
     if (p.num_splits > 1 && threadIdx.x < BM) {
       p.part_ml[(part_row0 + threadIdx.x) * 2] = -INFINITY;
       p.part_ml[(part_row0 + threadIdx.x) * 2 + 1] = 0.f;
-      __shared__ int s_flag0;
-      arrive_and_merge<D>(p, b, hk, mt, threadIdx.x, 1, &s_flag0);
     }
     return;
   }
@@ -218,6 +136,23 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ===================================================== TMA producer
+    // All 32 lanes issue: lane l < 16 loads K box (page l / PANELS, panel
+    // l % PANELS), lane 16 + l the matching V box, so a tile's 2 * 8 * PANELS
+    // boxes go out in one instruction.  Lanes 0..7 fetch the block-table
+    // entries of the next tile one iteration ahead.
+    const int32_t *bt = p.block_table + (size_t)b * p.max_pages;
+    auto page_row = [&](int kt) -> int {  // lanes 0..7: TMA row of page `lane` of tile kt
+      int y = p.oob_row;
+      const int pidx = kt * 8 + lane;
+      if (lane < 8 && pidx * 16 <= kmax && pidx < p.max_pages) {
+        const int page = bt[pidx];
+        if (page >= 0 && page < p.num_pages)
+          y = (int)(p.layer_row0 + ((long long)page * p.Hkv + hk) * 16);
+        else
+          dev_fail(p.status, PIC_DEV_BAD_PAGE, detail);
+      }
+      return y;
+    };
     if (lane == 0) {
       prefetch_tmap(&tm_q);
       prefetch_tmap(&tm_k);
@@ -226,47 +161,38 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int qrow = (b * p.Hkv + hk) * p.R_pad + r0;
       for (int pn = 0; pn < PANELS; ++pn)
         tma_load_2d(sbase + L::kQ + pn * BM * 128, &tm_q, pn * 64, qrow, bar(B_Q));
-      const int32_t *bt = p.block_table + (size_t)b * p.max_pages;
-      int issued = 0;
-      for (int j = 0; j < n; ++j) {
-        const int st = j % NST;
-        if (j >= NST && !mbar_wait(bar(B_KVEMPTY + st), ((j / NST) - 1) & 1, abort_flag, p.status, detail))
-          break;
-        const int kt = kv_begin + j;
-        int ys[8];
-#pragma unroll
-        for (int pg = 0; pg < 8; ++pg) {
-          const int pidx = kt * 8 + pg;
-          int y = p.oob_row;
-          if (pidx * 16 <= kmax && pidx < p.max_pages) {
-            const int page = bt[pidx];
-            if (page >= 0 && page < p.num_pages)
-              y = (int)(p.layer_row0 + ((long long)page * p.Hkv + hk) * 16);
-            else
-              dev_fail(p.status, PIC_DEV_BAD_PAGE, detail);
-          }
-          ys[pg] = y;
-        }
-        mbar_expect_tx(bar(B_KFULL + st), L::kTile);
-#pragma unroll
-        for (int pg = 0; pg < 8; ++pg)
-          for (int pn = 0; pn < PANELS; ++pn)
-            tma_load_2d(sbase + L::kK + st * L::kTile + pn * BN * 128 + pg * 16 * 128, &tm_k,
-                        pn * 64, ys[pg], bar(B_KFULL + st));
-        mbar_expect_tx(bar(B_VFULL + st), L::kTile);
-#pragma unroll
-        for (int pg = 0; pg < 8; ++pg)
-          for (int pn = 0; pn < PANELS; ++pn)
-            tma_load_2d(sbase + L::kV + st * L::kTile + pn * BN * 128 + pg * 16 * 128, &tm_v,
-                        pn * 64, ys[pg], bar(B_VFULL + st));
-        issued = j + 1;
+    }
+    const int box = lane & 15;              // box index within K (or V)
+    const int bpage = box / PANELS, bpanel = box % PANELS;
+    const bool issues = box < 8 * PANELS;
+    int y_next = page_row(kv_begin);
+    int issued = 0;
+    for (int j = 0; j < n; ++j) {
+      const int st = j % NST;
+      const int y_mine = y_next;
+      if (j + 1 < n) y_next = page_row(kv_begin + j + 1);
+      if (j >= NST) {
+        const bool ok = mbar_wait(bar(B_KVEMPTY + st), ((j / NST) - 1) & 1, abort_flag, p.status, detail);
+        if (!__all_sync(0xffffffffu, ok)) break;
       }
-      if (*abort_flag) {
-        // Let the copies already issued land before the CTA exits.
-        for (int j = max(0, issued - NST); j < issued; ++j) {
-          mbar_wait(bar(B_KFULL + j % NST), (j / NST) & 1, abort_flag, p.status, detail);
-          mbar_wait(bar(B_VFULL + j % NST), (j / NST) & 1, abort_flag, p.status, detail);
-        }
+      const int y = __shfl_sync(0xffffffffu, y_mine, bpage);
+      if (lane == 0) mbar_expect_tx(bar(B_KFULL + st), L::kTile);
+      if (lane == 16) mbar_expect_tx(bar(B_VFULL + st), L::kTile);
+      __syncwarp();
+      if (issues) {
+        const uint32_t off = st * L::kTile + bpanel * BN * 128 + bpage * 16 * 128;
+        if (lane < 16)
+          tma_load_2d(sbase + L::kK + off, &tm_k, bpanel * 64, y, bar(B_KFULL + st));
+        else
+          tma_load_2d(sbase + L::kV + off, &tm_v, bpanel * 64, y, bar(B_VFULL + st));
+      }
+      issued = j + 1;
+    }
+    if (lane == 0 && *abort_flag) {
+      // Let the copies already issued land before the CTA exits.
+      for (int j = max(0, issued - NST); j < issued; ++j) {
+        mbar_wait(bar(B_KFULL + j % NST), (j / NST) & 1, abort_flag, p.status, detail);
+        mbar_wait(bar(B_VFULL + j % NST), (j / NST) & 1, abort_flag, p.status, detail);
       }
     }
   } else if (warp == 1) {
@@ -398,48 +324,33 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_OFINAL), 0, abort_flag, p.status, detail));
     tc_fence_after();
     if (ok) {
+      float o[D];
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) tmem_ld32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o + c * 32));
+      tmem_wait_ld();
       if (p.num_splits == 1) {
         const float inv = l > 0.f ? 1.f / l : 0.f;
         __nv_bfloat16 *dst = p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D;
+        if (valid) {
 #pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
-          float o[32];
-          tmem_ld32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o));
-          tmem_wait_ld();
-          if (valid) {
+          for (int q = 0; q < D; ++q) o[q] *= inv;
 #pragma unroll
-            for (int q = 0; q < 32; ++q) o[q] *= inv;
-#pragma unroll
-            for (int q = 0; q < 4; ++q)
-              st_global16(dst + c * 32 + q * 8, pack8(o + q * 8));
-          }
+          for (int q = 0; q < D / 8; ++q) st_global16(dst + q * 8, pack8(o + q * 8));
         }
         if (valid && p.lse)
           p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
               l > 0.f ? (m_used + __log2f(l)) * 0.69314718055994531f : -INFINITY;
       } else {
         float *dst = p.part_o + (part_row0 + row) * D;
+        if (valid) {
 #pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
-          float o[32];
-          tmem_ld32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o));
-          tmem_wait_ld();
-          if (valid) {
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-              reinterpret_cast<float4 *>(dst + c * 32)[q] =
-                  make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
-          }
+          for (int q = 0; q < D / 4; ++q)
+            reinterpret_cast<float4 *>(dst)[q] =
+                make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
         }
         p.part_ml[(part_row0 + row) * 2] = (l > 0.f) ? m_used : -INFINITY;
         p.part_ml[(part_row0 + row) * 2 + 1] = l;
       }
-    }
-    if (p.num_splits > 1) {
-      // every softmax thread reaches here (ok is warp-uniform and the same for all
-      // four warps unless a wait timed out, in which case the result is void anyway)
-      __shared__ int s_flag1;
-      arrive_and_merge<D>(p, b, hk, mt, threadIdx.x - 64, 1, &s_flag1);
     }
   }
 
@@ -456,12 +367,67 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// Merge the split partials (O unnormalised, m in log2 units, l) of every
+// query row by log-sum-exp: one warp per row, lanes over the d columns.  All
+// loads are issued unconditionally (an empty split's weight is zero and its
+// data is discarded by a select), so a row costs two dependent L2 round trips.
+template <int D>
+__global__ void __launch_bounds__(256) combine_kernel(Params p) {
+  constexpr int CPL = D / 32;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long grow = (long long)blockIdx.x * (blockDim.x >> 5) + warp;
+  const long long per_b = (long long)p.Hkv * p.m_tiles * BM;
+  const int b = (int)(grow / per_b);
+  if (b >= p.batch) return;
+  const long long rem = grow % per_b;
+  const int hk = (int)(rem / ((long long)p.m_tiles * BM));
+  const int mt = (int)((rem / BM) % p.m_tiles), row = (int)(rem % BM);
+  const int tin = min(max(p.inline_len[b], 0), p.max_inline);
+  const int rg = mt * BM + row;
+  if (rg >= tin * p.G) return;
+  const int S = p.num_splits;
+  const size_t base = (((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * S;
+  float ms = -INFINITY, ls = 0.f;
+  if (lane < S) {
+    ms = p.part_ml[((base + lane) * BM + row) * 2];
+    ls = p.part_ml[((base + lane) * BM + row) * 2 + 1];
+  }
+  float M = ms;
+#pragma unroll
+  for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  const float w = (ms == -INFINITY) ? 0.f : ex2(ms - M);
+  float Lsum = w * ls;
+#pragma unroll
+  for (int o = 16; o; o >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, o);
+  float acc[CPL];
+#pragma unroll
+  for (int q = 0; q < CPL; ++q) acc[q] = 0.f;
+  for (int sp = 0; sp < S; ++sp) {
+    const float ws = __shfl_sync(0xffffffffu, w, sp);
+    const float *src = p.part_o + ((base + sp) * BM + row) * D + lane * CPL;
+    float v[CPL];
+#pragma unroll
+    for (int q = 0; q < CPL; ++q) v[q] = src[q];
+#pragma unroll
+    for (int q = 0; q < CPL; ++q) acc[q] = fmaf(ws, ws == 0.f ? 0.f : v[q], acc[q]);
+  }
+  const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
+  const int tok = rg / p.G, g = rg % p.G;
+  __nv_bfloat16 *dst =
+      p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D + lane * CPL;
+#pragma unroll
+  for (int q = 0; q < CPL; q += 2)
+    *reinterpret_cast<uint32_t *>(dst + q) = pack2(acc[q] * inv, acc[q + 1] * inv);
+  if (p.lse && lane == 0)
+    p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
+        Lsum > 0.f ? (M + __log2f(Lsum)) * 0.69314718055994531f : -INFINITY;
+}
+
 // RoPE the inline keys/queries at their logical positions; keys and values go
 // to their cache slots, queries to the GQA-packed workspace.
 struct AppendArgs {
-  int Hq, Hkv, G, max_inline, max_ctx, R_pad, n_counters;
+  int Hq, Hkv, G, max_inline, max_ctx, R_pad;
   long long num_pages;
-  int32_t *counters;
   const __nv_bfloat16 *q, *k, *v;
   const int32_t *inline_pos, *inline_len;
   const int64_t *slots;
@@ -475,8 +441,6 @@ __global__ void __launch_bounds__(256) append_kernel(AppendArgs a, RopeParams rp
   const int t = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
   const int tin = min(max(a.inline_len[b], 0), a.max_inline);
   __shared__ float2 cs[HALF];
-  if (t == 0 && b == 0)  // split-merge counters of pic_attend_prefill start at zero
-    for (int e = tid; e < a.n_counters; e += blockDim.x) a.counters[e] = 0;
   if (t >= tin) {  // zero the packed query rows of this token slot
     for (int e = tid; e < a.Hkv * a.G * VC; e += blockDim.x) {
       const int hk = e / (a.G * VC), r = e % (a.G * VC), g = r / VC, c = r % VC;
@@ -578,7 +542,7 @@ __global__ void __launch_bounds__(256) append_kernel(AppendArgs a, RopeParams rp
 
 struct Plan {
   int G, m_tiles, R_pad, splits;
-  size_t q_bytes, cnt_bytes, po_bytes, pml_bytes, total;
+  size_t q_bytes, po_bytes, pml_bytes, total;
 };
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -605,7 +569,6 @@ inline Plan plan(const pic_geom_t *g, int batch, int max_inline, int max_ctx, in
   }
   pl.splits = num_splits;
   pl.q_bytes = align256((size_t)batch * g->num_kv_heads * pl.R_pad * g->head_dim * 2);
-  pl.cnt_bytes = align256((size_t)batch * g->num_kv_heads * pl.m_tiles * sizeof(int32_t));
   if (pl.splits > 1) {
     const size_t rows = (size_t)batch * g->num_kv_heads * pl.m_tiles * pl.splits * BM;
     pl.po_bytes = align256(rows * g->head_dim * 4);
@@ -613,7 +576,7 @@ inline Plan plan(const pic_geom_t *g, int batch, int max_inline, int max_ctx, in
   } else {
     pl.po_bytes = pl.pml_bytes = 0;
   }
-  pl.total = pl.q_bytes + pl.cnt_bytes + pl.po_bytes + pl.pml_bytes;
+  pl.total = pl.q_bytes + pl.po_bytes + pl.pml_bytes;
   return pl;
 }
 
@@ -712,8 +675,6 @@ extern "C" pic_status_t pic_append_inline(
   aa.k_cache = static_cast<__nv_bfloat16 *>(k_cache) + (size_t)layer * layer_elems;
   aa.v_cache = static_cast<__nv_bfloat16 *>(v_cache) + (size_t)layer * layer_elems;
   aa.qpack = static_cast<__nv_bfloat16 *>(workspace);
-  aa.counters = reinterpret_cast<int32_t *>(static_cast<uint8_t *>(workspace) + pl.q_bytes);
-  aa.n_counters = batch * Hkv * pl.m_tiles;
   aa.status = status;
   const int t_slots = std::max(max_inline, (pl.R_pad + pl.G - 1) / pl.G);
   if (t_slots > INT32_MAX / 2 || batch > 65535)
@@ -774,11 +735,8 @@ extern "C" pic_status_t pic_attend_prefill(
   pp.block_table = block_table;
   pp.out = static_cast<__nv_bfloat16 *>(out);
   pp.lse = lse;
-  pp.counters = reinterpret_cast<int32_t *>(ws + pl.q_bytes);
-  pp.part_o = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes + pl.cnt_bytes) : nullptr;
-  pp.part_ml = pl.splits > 1
-                   ? reinterpret_cast<float *>(ws + pl.q_bytes + pl.cnt_bytes + pl.po_bytes)
-                   : nullptr;
+  pp.part_o = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes) : nullptr;
+  pp.part_ml = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes + pl.po_bytes) : nullptr;
   pp.status = status;
   pp.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
 
@@ -794,6 +752,12 @@ extern "C" pic_status_t pic_attend_prefill(
     e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill smem attribute");
     attn_kernel<64><<<grid, kThreads, smem, stream>>>(tq, tk, tv, pp);
+  }
+  if (pl.splits > 1) {
+    const long long rows = (long long)batch * Hkv * pl.m_tiles * BM;
+    const unsigned cgrid = (unsigned)((rows + 7) / 8);
+    if (D == 128) combine_kernel<128><<<cgrid, 256, 0, stream>>>(pp);
+    else combine_kernel<64><<<cgrid, 256, 0, stream>>>(pp);
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill launch");

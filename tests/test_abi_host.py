@@ -48,10 +48,9 @@ def _geom(**kw):
 
 def test_workspace_sizes_are_host_arithmetic(lib):
     g = _geom()
-    # packed Q: B * Hkv * ceil(Tin*G/128)*128 rows of d bf16, then one int32
-    # split counter per query tile (rounded up to 256 bytes)
+    # packed Q: B * Hkv * ceil(Tin*G/128)*128 rows of d bf16
     ws1 = pic.pic_prefill_workspace_size(g, 1, 192, 4288, 1)
-    assert ws1 == 1 * 8 * 768 * 128 * 2 + 256
+    assert ws1 == 1 * 8 * 768 * 128 * 2
     ws3 = pic.pic_prefill_workspace_size(g, 1, 192, 4288, 3)
     assert ws3 > ws1
     assert pic.pic_decode_workspace_size(g, 16, 33000, 1) == ((16 * 32 * 128 * 2 + 255) // 256) * 256
