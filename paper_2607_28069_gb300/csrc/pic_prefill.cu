@@ -33,17 +33,19 @@ namespace pic {
 namespace prefill {
 
 constexpr int BM = 128;  // query rows per tile (TMEM lanes)
+constexpr int NQ = 2;    // query tiles per CTA, sharing every K/V tile
 constexpr int BN = 128;  // keys per KV tile
-constexpr int NST = 3;   // K/V ring stages
-constexpr int kThreads = 192;
+constexpr int NST = 2;   // K/V ring stages
+constexpr int kThreads = 64 + NQ * 128;  // producer warp, MMA warp, NQ softmax warpgroups
 constexpr int kMaxSplits = 32;
 constexpr uint32_t kTmemCols = 512;
 
 template <int D>
 struct Layout {
   static constexpr int kTile = BN * D * 2;  // bytes of one K or V tile
+  static constexpr int kQTile = BM * D * 2;
   static constexpr int kQ = 0;
-  static constexpr int kK = kQ + BM * D * 2;
+  static constexpr int kK = kQ + NQ * kQTile;
   static constexpr int kV = kK + NST * kTile;
   static constexpr int kBar = kV + NST * kTile;
   static constexpr int kBytes = kBar + 256;
@@ -56,10 +58,9 @@ enum {
   B_KFULL = 1,
   B_VFULL = B_KFULL + NST,
   B_KVEMPTY = B_VFULL + NST,
-  B_SFULL = B_KVEMPTY + NST,
-  B_PFULL = B_SFULL + 2,
-  B_PFREE = B_PFULL + 2,
-  B_OFINAL = B_PFREE + 2,
+  B_SFULL = B_KVEMPTY + NST,  // one per query tile
+  B_PFULL = B_SFULL + NQ,     // one per query tile (128 arrivals)
+  B_OFINAL = B_PFULL + NQ,
   B_COUNT = B_OFINAL + 1
 };
 
@@ -73,6 +74,12 @@ struct Params {
   float scale_log2;
 };
 
+// One CTA = (pair of 128-row query tiles, key split, kv head, request).
+// TMEM: S_t at columns 128 t (P_t written over it as bf16), O_t at 256 + 128 t.
+// MMA order per KV tile j: PV_0(j-1), QK_0(j), PV_1(j-1), QK_1(j).  Because
+// tcgen05 MMAs of one thread complete in order, "S_t(j) is ready" implies
+// PV_t(j-1) has finished, so softmax t may rescale O_t right away, and
+// softmax 0 runs while the tensor core works on tile 1 and vice versa.
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
@@ -92,36 +99,53 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::kBar + 8 * B_COUNT + 8);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int mt = blockIdx.x / p.num_splits, split = blockIdx.x % p.num_splits;
+  const int pair = blockIdx.x / p.num_splits, split = blockIdx.x % p.num_splits;
   const int hk = blockIdx.y, b = blockIdx.z;
   const int detail = b;
 
   // ---- work of this CTA (uniform across threads)
   const int tin = min(max(p.inline_len[b], 0), p.max_inline);
   const int rows = tin * p.G;
-  const int r0 = mt * BM;
-  if (r0 >= rows) return;  // no query row in this tile
-  const int r_last = min(r0 + BM, rows) - 1;
   const int32_t *ipos = p.inline_pos + (size_t)b * p.max_inline;
-  const int kmin = ipos[r0 / p.G];
-  const int kmax = ipos[r_last / p.G];
-  const int n_kv_all = kmax >= 0 ? kmax / BN + 1 : 0;
+  int r0[NQ], kmin[NQ], kmax[NQ], ntile = 0;
+#pragma unroll
+  for (int t = 0; t < NQ; ++t) {
+    r0[t] = (pair * NQ + t) * BM;
+    kmin[t] = kmax[t] = -1;
+    if (r0[t] < rows && t < p.m_tiles - pair * NQ) {
+      kmin[t] = ipos[r0[t] / p.G];
+      kmax[t] = ipos[(min(r0[t] + BM, rows) - 1) / p.G];
+      ntile = t + 1;
+    }
+  }
+  if (ntile == 0) return;  // no query row in this pair
+  const int kmax_all = ntile == 2 ? kmax[1] : kmax[0];
+  const int n_kv_all = kmax_all >= 0 ? kmax_all / BN + 1 : 0;
   const int per = (n_kv_all + p.num_splits - 1) / p.num_splits;
   const int kv_begin = split * per;
   const int n = max(0, min(per, n_kv_all - kv_begin));
-  const size_t part_row0 =
-      ((((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * p.num_splits + split) * BM;
+  int nt[NQ];  // KV tiles of this split that query tile t needs
+#pragma unroll
+  for (int t = 0; t < NQ; ++t)
+    nt[t] = (t < ntile && kmax[t] >= 0) ? max(0, min(n, kmax[t] / BN + 1 - kv_begin)) : 0;
+  auto part_row0 = [&](int t) {
+    return ((((size_t)b * p.Hkv + hk) * p.m_tiles + pair * NQ + t) * p.num_splits + split) * BM;
+  };
 
-  if (n == 0) {  // empty split: neutral partial state
-    if (p.num_splits > 1 && threadIdx.x < BM) {
-      p.part_ml[(part_row0 + threadIdx.x) * 2] = -INFINITY;
-      p.part_ml[(part_row0 + threadIdx.x) * 2 + 1] = 0.f;
-    }
+  if (n == 0) {  // empty split: neutral partial state for every tile
+    if (p.num_splits > 1 && threadIdx.x < BM)
+#pragma unroll
+      for (int t = 0; t < NQ; ++t) {
+        if (t >= ntile) break;
+        p.part_ml[(part_row0(t) + threadIdx.x) * 2] = -INFINITY;
+        p.part_ml[(part_row0(t) + threadIdx.x) * 2 + 1] = 0.f;
+      }
     return;
   }
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < B_COUNT; ++i) mbar_init(bar(i), (i == B_PFULL || i == B_PFULL + 1) ? 128 : 1);
+    for (int i = 0; i < B_COUNT; ++i)
+      mbar_init(bar(i), (i >= B_PFULL && i < B_PFULL + NQ) ? 128 : 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -144,7 +168,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto page_row = [&](int kt) -> int {  // lanes 0..7: TMA row of page `lane` of tile kt
       int y = p.oob_row;
       const int pidx = kt * 8 + lane;
-      if (lane < 8 && pidx * 16 <= kmax && pidx < p.max_pages) {
+      if (lane < 8 && pidx * 16 <= kmax_all && pidx < p.max_pages) {
         const int page = bt[pidx];
         if (page >= 0 && page < p.num_pages)
           y = (int)(p.layer_row0 + ((long long)page * p.Hkv + hk) * 16);
@@ -157,12 +181,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tmap(&tm_q);
       prefetch_tmap(&tm_k);
       prefetch_tmap(&tm_v);
-      mbar_expect_tx(bar(B_Q), BM * D * 2);
-      const int qrow = (b * p.Hkv + hk) * p.R_pad + r0;
-      for (int pn = 0; pn < PANELS; ++pn)
-        tma_load_2d(sbase + L::kQ + pn * BM * 128, &tm_q, pn * 64, qrow, bar(B_Q));
+      mbar_expect_tx(bar(B_Q), ntile * L::kQTile);
+#pragma unroll
+      for (int t = 0; t < NQ; ++t) {
+        if (t >= ntile) break;
+        const int qrow = (b * p.Hkv + hk) * p.R_pad + r0[t];
+#pragma unroll
+        for (int pn = 0; pn < PANELS; ++pn)
+          tma_load_2d(sbase + L::kQ + t * L::kQTile + pn * BM * 128, &tm_q, pn * 64, qrow, bar(B_Q));
+      }
     }
-    const int box = lane & 15;              // box index within K (or V)
+    const int box = lane & 15;  // box index within K (or V)
     const int bpage = box / PANELS, bpanel = box % PANELS;
     const bool issues = box < 8 * PANELS;
     int y_next = page_row(kv_begin);
@@ -198,64 +227,87 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     // ===================================================== MMA issuer
     if (lane == 0) {
-      const uint32_t tS0 = tbase, tO = tbase + 256;
       bool ok = mbar_wait(bar(B_Q), 0, abort_flag, p.status, detail);
       tc_fence_after();
       for (int j = 0; ok && j <= n; ++j) {
-        if (j < n) {
-          const int st = j % NST, sb = j & 1;
-          if (!mbar_wait(bar(B_KFULL + st), (j / NST) & 1, abort_flag, p.status, detail)) break;
-          tc_fence_after();
-          const uint32_t kb = sbase + L::kK + st * L::kTile;
+        bool k_ready = false;
 #pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * (BM * 128) + (kk & 3) * 32;
-            mma_ss(tS0 + sb * 128, sdesc_sw128(sbase + L::kQ + off, 16, 1024),
-                   sdesc_sw128(kb + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024), IDESC_QK,
-                   kk > 0);
+        for (int t = 0; t < NQ; ++t) {
+          if (t >= ntile) break;
+          const uint32_t tS = tbase + t * 128, tO = tbase + 256 + t * 128;
+          // O_t += P_t(j-1) V(j-1)
+          if (j >= 1 && j - 1 < nt[t]) {
+            const int pj = j - 1, pst = pj % NST;
+            if (!mbar_wait(bar(B_PFULL + t), pj & 1, abort_flag, p.status, detail) ||
+                !mbar_wait(bar(B_VFULL + pst), (pj / NST) & 1, abort_flag, p.status, detail)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t vb = sbase + L::kV + pst * L::kTile;
+#pragma unroll
+            for (int kk = 0; kk < BN / 16; ++kk)
+              mma_ts(tO, tS + kk * 8, sdesc_sw128(vb + kk * 16 * 128, BN * 128, 1024), IDESC_PV,
+                     (pj > 0 || kk > 0));
+            if (t == ntile - 1) mma_commit(bar(B_KVEMPTY + pst));  // last reader of V(j-1)
           }
-          mma_commit(bar(B_SFULL + sb));
-        }
-        if (j >= 1) {
-          const int pj = j - 1, pst = pj % NST, pb = pj & 1;
-          if (!mbar_wait(bar(B_PFULL + pb), (pj >> 1) & 1, abort_flag, p.status, detail)) break;
-          if (!mbar_wait(bar(B_VFULL + pst), (pj / NST) & 1, abort_flag, p.status, detail)) break;
-          tc_fence_after();
-          const uint32_t vb = sbase + L::kV + pst * L::kTile;
+          // S_t = Q_t K(j)^T
+          if (j < nt[t]) {
+            const int st = j % NST;
+            if (!k_ready) {
+              if (!mbar_wait(bar(B_KFULL + st), (j / NST) & 1, abort_flag, p.status, detail)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              k_ready = true;
+            }
+            const uint32_t kb = sbase + L::kK + st * L::kTile;
+            const uint32_t qb = sbase + L::kQ + t * L::kQTile;
 #pragma unroll
-          for (int kk = 0; kk < BN / 16; ++kk)
-            mma_ts(tO, tS0 + pb * 128 + kk * 8, sdesc_sw128(vb + kk * 16 * 128, BN * 128, 1024),
-                   IDESC_PV, (pj > 0 || kk > 0));
-          mma_commit(bar(B_KVEMPTY + pst));
-          mma_commit(bar(B_PFREE + pb));
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * (BM * 128) + (kk & 3) * 32;
+              mma_ss(tS, sdesc_sw128(qb + off, 16, 1024),
+                     sdesc_sw128(kb + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024), IDESC_QK,
+                     kk > 0);
+            }
+            mma_commit(bar(B_SFULL + t));
+          }
         }
       }
       mma_commit(bar(B_OFINAL));
     }
   } else {
-    // ===================================================== softmax warps
-    const int wq = warp & 3;
+    // ===================================================== softmax warpgroups
+    static_assert(NQ == 2, "softmax warpgroup selection assumes two query tiles");
+    const int t = (warp - 2) >> 2;  // query tile of this warpgroup
+    const int wq = warp & 3;        // TMEM lane quarter
     const int row = wq * 32 + lane;
-    const int rg = r0 + row;
-    const bool valid = rg < rows;
+    // constant-index selects keep the per-tile values in registers
+    const int my_r0 = t == 0 ? r0[0] : r0[1];
+    const int my_kmin = t == 0 ? kmin[0] : kmin[1];
+    const int my_n = t < ntile ? (t == 0 ? nt[0] : nt[1]) : 0;
+    const size_t my_part0 = part_row0(t);
+    const int rg = my_r0 + row;
+    const bool valid = t < ntile && rg < rows;
     const int tok = rg / p.G, g = rg % p.G;
     const int pos = valid ? ipos[tok] : -1;
     const uint32_t tl = tbase + ((uint32_t)(wq * 32) << 16);
+    const uint32_t tS = tl + t * 128, tO = tl + 256 + t * 128;
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
-    for (int j = 0; j < n; ++j) {
-      const int sb = j & 1;
+    for (int j = 0; j < my_n; ++j) {
       const int key0 = (kv_begin + j) * BN;
-      if (!__all_sync(0xffffffffu, mbar_wait(bar(B_SFULL + sb), (j >> 1) & 1, abort_flag, p.status, detail))) {
+      if (!__all_sync(0xffffffffu, mbar_wait(bar(B_SFULL + t), j & 1, abort_flag, p.status, detail))) {
         ok = false;
         break;
       }
       tc_fence_after();
       float s[BN];
 #pragma unroll
-      for (int c = 0; c < BN / 32; ++c) tmem_ld32(tl + sb * 128 + c * 32, reinterpret_cast<uint32_t *>(s + c * 32));
+      for (int c = 0; c < BN / 32; ++c) tmem_ld32(tS + c * 32, reinterpret_cast<uint32_t *>(s + c * 32));
       tmem_wait_ld();
-      if (key0 + BN - 1 > kmin) {  // some key of the tile lies beyond some row
+      if (key0 + BN - 1 > my_kmin) {  // some key of the tile lies beyond some row
 #pragma unroll
         for (int c = 0; c < BN; ++c)
           if (key0 + c > pos) s[c] = -INFINITY;
@@ -280,76 +332,82 @@ __global__ void __launch_bounds__(kThreads, 1)
         m_used = m_new;
       }
       const float mref = (m_used == -INFINITY) ? 0.f : m_used;
-      uint32_t pk[BN / 2];
+      // P = exp2(s * scale - m) as bf16, written over S in 16-column chunks as
+      // soon as each 32-key chunk is done (S was read completely above, so the
+      // overlap is harmless and the packed values never pile up in registers)
       float ls8[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) ls8[i] = 0.f;
 #pragma unroll
-      for (int c = 0; c < BN; c += 2) {
-        const float p0 = ex2(fmaf(s[c], p.scale_log2, -mref));
-        const float p1 = ex2(fmaf(s[c + 1], p.scale_log2, -mref));
-        ls8[(c >> 1) & 7] += p0 + p1;
-        pk[c / 2] = pack2(p0, p1);
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int c = 0; c < 32; c += 2) {
+          const float p0 = ex2(fmaf(s[c0 + c], p.scale_log2, -mref));
+          const float p1 = ex2(fmaf(s[c0 + c + 1], p.scale_log2, -mref));
+          ls8[(c >> 1) & 7] += p0 + p1;
+          pk[c / 2] = pack2(p0, p1);
+        }
+        tmem_st16(tS + c0 / 2, pk);
       }
 #pragma unroll
       for (int w = 4; w; w >>= 1)
 #pragma unroll
         for (int i = 0; i < w; ++i) ls8[i] += ls8[i + w];
       l = fmaf(l, alpha, ls8[0]);
-      // O correction, only when some row of this warp moved its maximum.
+      // O correction: PV_t(j-1) has completed (it precedes QK_t(j) in the MMA order)
       if (j > 0 && __any_sync(0xffffffffu, resc)) {
-        const int pj = j - 1;
-        if (!__all_sync(0xffffffffu, mbar_wait(bar(B_PFREE + (pj & 1)), (pj >> 1) & 1, abort_flag, p.status, detail))) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
 #pragma unroll
         for (int c = 0; c < D / 32; ++c) {
           float o[32];
-          tmem_ld32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o));
+          tmem_ld32(tO + c * 32, reinterpret_cast<uint32_t *>(o));
           tmem_wait_ld();
 #pragma unroll
           for (int q = 0; q < 32; ++q) o[q] *= alpha;
-          tmem_st32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o));
+          tmem_st32(tO + c * 32, reinterpret_cast<uint32_t *>(o));
         }
       }
-      tmem_st32(tl + sb * 128, pk);
-      tmem_st32(tl + sb * 128 + 32, pk + 32);
       tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(bar(B_PFULL + sb));
+      mbar_arrive(bar(B_PFULL + t));
     }
     // ---- epilogue
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_OFINAL), 0, abort_flag, p.status, detail));
     tc_fence_after();
-    if (ok) {
-      float o[D];
-#pragma unroll
-      for (int c = 0; c < D / 32; ++c) tmem_ld32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o + c * 32));
-      tmem_wait_ld();
-      if (p.num_splits == 1) {
-        const float inv = l > 0.f ? 1.f / l : 0.f;
-        __nv_bfloat16 *dst = p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D;
-        if (valid) {
-#pragma unroll
-          for (int q = 0; q < D; ++q) o[q] *= inv;
-#pragma unroll
-          for (int q = 0; q < D / 8; ++q) st_global16(dst + q * 8, pack8(o + q * 8));
+    if (ok && t < ntile) {
+      if (my_n == 0) {  // this tile needs none of the split's keys
+        if (p.num_splits > 1) {
+          p.part_ml[(my_part0 + row) * 2] = -INFINITY;
+          p.part_ml[(my_part0 + row) * 2 + 1] = 0.f;
         }
-        if (valid && p.lse)
-          p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
-              l > 0.f ? (m_used + __log2f(l)) * 0.69314718055994531f : -INFINITY;
       } else {
-        float *dst = p.part_o + (part_row0 + row) * D;
-        if (valid) {
+        float o[D];
 #pragma unroll
-          for (int q = 0; q < D / 4; ++q)
-            reinterpret_cast<float4 *>(dst)[q] =
-                make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+        for (int c = 0; c < D / 32; ++c) tmem_ld32(tO + c * 32, reinterpret_cast<uint32_t *>(o + c * 32));
+        tmem_wait_ld();
+        if (p.num_splits == 1) {
+          const float inv = l > 0.f ? 1.f / l : 0.f;
+          __nv_bfloat16 *dst = p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D;
+          if (valid) {
+#pragma unroll
+            for (int q = 0; q < D; ++q) o[q] *= inv;
+#pragma unroll
+            for (int q = 0; q < D / 8; ++q) st_global16(dst + q * 8, pack8(o + q * 8));
+          }
+          if (valid && p.lse)
+            p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
+                l > 0.f ? (m_used + __log2f(l)) * 0.69314718055994531f : -INFINITY;
+        } else {
+          float *dst = p.part_o + (my_part0 + row) * D;
+          if (valid) {
+#pragma unroll
+            for (int q = 0; q < D / 4; ++q)
+              reinterpret_cast<float4 *>(dst)[q] =
+                  make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+          }
+          p.part_ml[(my_part0 + row) * 2] = (l > 0.f) ? m_used : -INFINITY;
+          p.part_ml[(my_part0 + row) * 2 + 1] = l;
         }
-        p.part_ml[(part_row0 + row) * 2] = (l > 0.f) ? m_used : -INFINITY;
-        p.part_ml[(part_row0 + row) * 2 + 1] = l;
       }
     }
   }
@@ -555,7 +613,7 @@ inline Plan plan(const pic_geom_t *g, int batch, int max_inline, int max_ctx, in
   const int kv_tiles = (max_ctx + BN - 1) / BN;
   if (num_splits <= 0) {
     // Wave-aware choice: minimise waves * (tiles per split + fixed cost).
-    const long long ctas = (long long)batch * g->num_kv_heads * pl.m_tiles;
+    const long long ctas = (long long)batch * g->num_kv_heads * ((pl.m_tiles + NQ - 1) / NQ);
     double best_cost = 1e300;
     num_splits = 1;
     for (int s = 1; s <= std::min(kMaxSplits, std::max(1, kv_tiles)); ++s) {
@@ -740,7 +798,7 @@ extern "C" pic_status_t pic_attend_prefill(
   pp.status = status;
   pp.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
 
-  dim3 grid(pl.m_tiles * pl.splits, Hkv, batch);
+  dim3 grid(((pl.m_tiles + NQ - 1) / NQ) * pl.splits, Hkv, batch);
   cudaError_t e;
   if (D == 128) {
     const int smem = Layout<128>::kAlloc;
