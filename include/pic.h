@@ -253,6 +253,34 @@ pic_status_t pic_attend_decode(const pic_geom_t *geom, int32_t layer, int32_t ba
                                int32_t num_splits, void *workspace, size_t workspace_bytes,
                                pic_stream_t stream);
 
+/*
+ * pic_attend_decode_noalloc -- pic_attend_decode for callers that cannot
+ * allocate device memory while they decode (an engine that gave its whole
+ * memory budget to the KV cache, a runtime that forbids allocation after
+ * start-up, a plugin that only owns the tensors it is handed).  The paper has
+ * no counterpart: this is a deployment convenience of this library.
+ *
+ * Same arguments and results as pic_attend_decode, without the workspace:
+ * the scratch (rotated queries, per-split partial softmax states) lives in an
+ * 8 MiB array inside the library that every GPU which loads it holds until
+ * the process exits.  The call allocates nothing.
+ *  - The first call on a device (with that device current) looks the array
+ *    up with cudaGetSymbolAddress; make that first call before any stream
+ *    capture.
+ *  - Every call on a device shares the array: calls that overlap on the GPU
+ *    (e.g. on two streams) race.  No scratch value needs to start at zero.
+ *  - num_splits 0 picks the automatic split count, lowered until the scratch
+ *    fits; an explicit num_splits whose scratch exceeds 8 MiB, or a problem
+ *    too large even with one split, returns PIC_ERR_WORKSPACE.
+ */
+pic_status_t pic_attend_decode_noalloc(const pic_geom_t *geom, int32_t layer, int32_t batch,
+                                       const void *q, const void *k_new, const void *v_new,
+                                       const int32_t *pos, int32_t pos_offset,
+                                       const int32_t *block_table, int32_t max_pages,
+                                       int64_t num_pages, void *k_cache, void *v_cache, void *out,
+                                       float *lse, int32_t max_ctx, int32_t num_splits,
+                                       pic_stream_t stream);
+
 #ifdef __cplusplus
 } /* extern "C" */
 #endif

@@ -18,7 +18,7 @@ import torch
 __all__ = [
     "Geometry", "load", "lib_path", "pic_abi_version", "pic_compose", "pic_relocate",
     "pic_append_inline", "pic_attend_prefill", "pic_prefill_workspace_size",
-    "pic_prefill_num_splits", "pic_decode_num_splits",
+    "pic_prefill_num_splits", "pic_decode_num_splits", "pic_attend_decode_noalloc",
     "pic_attend_decode", "pic_decode_workspace_size", "pic_device_status", "PicError",
     "EXPORTED_SYMBOLS", "ROPE_HALF", "ROPE_INTERLEAVED",
 ]
@@ -35,7 +35,7 @@ EXPORTED_SYMBOLS = (
     "pic_abi_version", "pic_last_error", "pic_device_status", "pic_compose", "pic_relocate",
     "pic_prefill_workspace_size", "pic_prefill_num_splits", "pic_append_inline",
     "pic_attend_prefill", "pic_decode_workspace_size", "pic_decode_num_splits",
-    "pic_attend_decode",
+    "pic_attend_decode", "pic_attend_decode_noalloc",
 )
 
 DEVICE_CODES = {
@@ -107,6 +107,8 @@ def load():
         "pic_attend_prefill": (I32, [G, I32, I32, I32, P, P, I32, P, I32, I64, P, P, P, P, I32,
                                      P, SZ, P]),
         "pic_decode_workspace_size": (SZ, [G, I32, I32, I32]),
+        "pic_attend_decode_noalloc": (I32, [G, I32, I32, P, P, P, P, I32, P, I32, I64, P, P, P, P,
+                                            I32, I32, P]),
         "pic_prefill_num_splits": (I32, [G, I32, I32, I32, I32]),
         "pic_decode_num_splits": (I32, [G, I32, I32, I32]),
         "pic_attend_decode": (I32, [G, I32, I32, P, P, P, P, I32, P, I32, I64, P, P, P, P, I32, I32,
@@ -266,3 +268,20 @@ def pic_attend_decode(geom: Geometry, layer: int, q, k_new, v_new, pos, block_ta
         _ptr(lse, f32, "lse", allow_none=True), max_ctx, num_splits,
         _ptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream))
     _check(st, "pic_attend_decode")
+
+
+def pic_attend_decode_noalloc(geom: Geometry, layer: int, q, k_new, v_new, pos, block_table,
+                              num_pages: int, k_cache, v_cache, out, max_ctx: int, lse=None,
+                              num_splits: int = 0, pos_offset: int = 0, stream=None):
+    """pic_attend_decode without a workspace, for callers that cannot allocate
+    while decoding; the scratch is an array inside the library (see pic.h)."""
+    lib = load()
+    g = geom._c()
+    B = pos.numel()
+    st = lib.pic_attend_decode_noalloc(
+        ctypes.byref(g), layer, B, _ptr(q, bf16, "q"), _ptr(k_new, bf16, "k_new"),
+        _ptr(v_new, bf16, "v_new"), _ptr(pos, i32, "pos"), pos_offset,
+        _ptr(block_table, i32, "block_table"), block_table.shape[1], num_pages,
+        _ptr(k_cache, bf16, "k_cache"), _ptr(v_cache, bf16, "v_cache"), _ptr(out, bf16, "out"),
+        _ptr(lse, f32, "lse", allow_none=True), max_ctx, num_splits, _stream(stream))
+    _check(st, "pic_attend_decode_noalloc")

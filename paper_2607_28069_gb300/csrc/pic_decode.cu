@@ -17,6 +17,7 @@
 //     are merged through shared memory at the end.
 //  3. decode_combine_kernel (only with several splits): log-sum-exp merge.
 #include <algorithm>
+#include <mutex>
 
 #include "pic_internal.cuh"
 
@@ -503,5 +504,171 @@ extern "C" pic_status_t pic_attend_decode(const pic_geom_t *geom, int32_t layer,
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_attend_decode launch");
+  return PIC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// pic_attend_decode_noalloc: the same decoding step for callers that cannot
+// allocate device memory on the step path.
+//
+// Some callers cannot call cudaMalloc (or any allocator) while they decode: an
+// engine that has handed its whole memory budget to the KV cache, a runtime
+// that forbids allocation after start-up, or an embedding that only owns the
+// tensors it passes in.  For them this entry point takes no workspace: its
+// scratch (the rotated queries and the per-split partial softmax states) lives
+// in the file-scope device array below, which every GPU that loads the library
+// holds until the process exits.
+//
+// Set-up: the first call on each device (with that device current) looks up
+// the array's device address with cudaGetSymbolAddress and caches it; make
+// that first call before any stream capture.  The array is shared by every
+// call on the device and keeps the last call's contents: calls that overlap on
+// the GPU (for example on two streams) race on it.  Nothing in it needs to
+// start at zero: each call writes every scratch value before reading it.
+namespace pic {
+namespace decode {
+
+constexpr size_t kNoAllocScratchBytes = 8u << 20;  // 8 MiB per device
+static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocScratchBytes];
+
+static uint8_t *noalloc_scratch_ptr(pic_status_t *st) {
+  constexpr int kMaxDev = 64;
+  static uint8_t *ptrs[kMaxDev] = {nullptr};
+  static std::mutex mu;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess || dev < 0 || dev >= kMaxDev) {
+    *st = e != cudaSuccess ? cuda_fail(e, "pic_attend_decode_noalloc: cudaGetDevice")
+                           : fail(PIC_ERR_CUDA, "pic_attend_decode_noalloc: device %d", dev);
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lk(mu);
+  if (!ptrs[dev]) {
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) {
+      *st = cuda_fail(e, "pic_attend_decode_noalloc: cudaGetSymbolAddress");
+      return nullptr;
+    }
+    ptrs[dev] = static_cast<uint8_t *>(p);
+  }
+  *st = PIC_OK;
+  return ptrs[dev];
+}
+
+}  // namespace decode
+}  // namespace pic
+
+extern "C" pic_status_t pic_attend_decode_noalloc(const pic_geom_t *geom, int32_t layer,
+                                                  int32_t batch, const void *q, const void *k_new,
+                                                  const void *v_new, const int32_t *pos,
+                                                  int32_t pos_offset, const int32_t *block_table,
+                                                  int32_t max_pages, int64_t num_pages,
+                                                  void *k_cache, void *v_cache, void *out,
+                                                  float *lse, int32_t max_ctx, int32_t num_splits,
+                                                  pic_stream_t stream) {
+  using namespace pic;
+  using namespace pic::decode;
+  RopeParams rp;
+  pic_status_t st = make_rope(geom, &rp);
+  if (st != PIC_OK) return st;
+  if (layer < 0 || layer >= geom->num_layers)
+    return fail(PIC_ERR_INVALID_ARG, "pic_attend_decode_noalloc: layer %d outside [0, %d)", layer,
+                geom->num_layers);
+  if (batch <= 0 || max_pages <= 0 || num_pages <= 0 || max_ctx <= 0)
+    return fail(PIC_ERR_INVALID_ARG, "pic_attend_decode_noalloc: sizes must be positive");
+  if (num_splits < 0 || num_splits > kMaxSplits)
+    return fail(PIC_ERR_INVALID_ARG, "pic_attend_decode_noalloc: num_splits %d outside [0, %d]",
+                num_splits, kMaxSplits);
+  const int G = geom->num_q_heads / geom->num_kv_heads;
+  if (G > 16)
+    return fail(PIC_ERR_UNSUPPORTED,
+                "pic_attend_decode_noalloc: more than 16 query heads per kv head");
+  if (!q || !k_new || !v_new || !pos || !block_table || !k_cache || !v_cache || !out)
+    return fail(PIC_ERR_INVALID_ARG, "pic_attend_decode_noalloc: NULL tensor");
+  if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k_new) |
+       reinterpret_cast<uintptr_t>(v_new) | reinterpret_cast<uintptr_t>(k_cache) |
+       reinterpret_cast<uintptr_t>(v_cache)) & 15)
+    return fail(PIC_ERR_INVALID_ARG,
+                "pic_attend_decode_noalloc: bf16 tensors must be 16-byte aligned");
+  const int D = geom->head_dim, Hkv = geom->num_kv_heads;
+  const long long rows_total = (long long)geom->num_layers * num_pages * Hkv * 16;
+  if (rows_total + 16 >= 0x7fffff00LL)
+    return fail(PIC_ERR_UNSUPPORTED, "pic_attend_decode_noalloc: cache has more than 2^31 rows");
+  if (batch > 65535 || Hkv > 65535)
+    return fail(PIC_ERR_UNSUPPORTED, "pic_attend_decode_noalloc: grid too large");
+  // Scratch must fit the built-in array: the automatic split count is lowered
+  // until it does; an explicit split count that does not fit is rejected.
+  Plan pl = plan(geom, batch, max_ctx, num_splits);
+  if (num_splits == 0)
+    while (pl.total > kNoAllocScratchBytes && pl.splits > 1)
+      pl = plan(geom, batch, max_ctx, pl.splits - 1);
+  if (pl.total > kNoAllocScratchBytes)
+    return fail(PIC_ERR_WORKSPACE,
+                "pic_attend_decode_noalloc: needs %zu bytes of scratch, the built-in array holds "
+                "%zu (fewer splits or a smaller batch may fit; pic_attend_decode takes a "
+                "caller workspace instead)",
+                pl.total, kNoAllocScratchBytes);
+  uint8_t *ws = noalloc_scratch_ptr(&st);
+  if (!ws) return st;
+  int32_t *status = device_status_ptr();
+  if (!status) return fail(PIC_ERR_CUDA, "pic_attend_decode_noalloc: no device status word");
+  const size_t layer_elems = (size_t)num_pages * Hkv * 16 * D;
+
+  AppendArgs aa;
+  aa.Hq = geom->num_q_heads;
+  aa.Hkv = Hkv;
+  aa.max_pages = max_pages;
+  aa.pos_offset = pos_offset;
+  aa.num_pages = num_pages;
+  aa.q = static_cast<const __nv_bfloat16 *>(q);
+  aa.k = static_cast<const __nv_bfloat16 *>(k_new);
+  aa.v = static_cast<const __nv_bfloat16 *>(v_new);
+  aa.pos = pos;
+  aa.block_table = block_table;
+  aa.k_cache = static_cast<__nv_bfloat16 *>(k_cache) + (size_t)layer * layer_elems;
+  aa.v_cache = static_cast<__nv_bfloat16 *>(v_cache) + (size_t)layer * layer_elems;
+  aa.qrot = reinterpret_cast<__nv_bfloat16 *>(ws);
+  aa.status = status;
+  if (D == 128) decode_append_kernel<128><<<batch, 128, 0, stream>>>(aa, rp);
+  else decode_append_kernel<64><<<batch, 128, 0, stream>>>(aa, rp);
+
+  CUtensorMap tk, tv;
+  st = encode_tmap_2d(&tk, k_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
+  if (st == PIC_OK) st = encode_tmap_2d(&tv, v_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
+  if (st != PIC_OK) return st;
+
+  Params pp;
+  pp.Hq = geom->num_q_heads;
+  pp.Hkv = Hkv;
+  pp.G = G;
+  pp.max_pages = max_pages;
+  pp.splits = pl.splits;
+  pp.pages_per_split = pl.pages_per_split;
+  pp.pos_offset = pos_offset;
+  pp.num_pages = num_pages;
+  pp.layer_row0 = (long long)layer * num_pages * Hkv * 16;
+  pp.pos = pos;
+  pp.block_table = block_table;
+  pp.qrot = aa.qrot;
+  pp.out = static_cast<__nv_bfloat16 *>(out);
+  pp.lse = lse;
+  pp.part_o = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes) : nullptr;
+  pp.part_ml = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes + pl.po_bytes) : nullptr;
+  pp.status = status;
+  pp.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
+
+  dim3 grid(pl.splits, Hkv, batch);
+  cudaError_t e;
+  if (D == 128) e = G <= 8 ? launch_attn<128, 1>(grid, stream, tk, tv, pp) : launch_attn<128, 2>(grid, stream, tk, tv, pp);
+  else e = G <= 8 ? launch_attn<64, 1>(grid, stream, tk, tv, pp) : launch_attn<64, 2>(grid, stream, tk, tv, pp);
+  if (e != cudaSuccess) return cuda_fail(e, "pic_attend_decode_noalloc attention launch");
+  if (pl.splits > 1) {
+    dim3 cgrid(geom->num_q_heads, batch);
+    if (D == 128) decode_combine_kernel<128><<<cgrid, 32, 0, stream>>>(pp);
+    else decode_combine_kernel<64><<<cgrid, 32, 0, stream>>>(pp);
+  }
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "pic_attend_decode_noalloc launch");
   return PIC_OK;
 }

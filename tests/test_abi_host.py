@@ -55,9 +55,9 @@ def test_workspace_sizes_are_host_arithmetic(lib):
     assert ws3 > ws1
     assert pic.pic_decode_workspace_size(g, 16, 33000, 1) == ((16 * 32 * 128 * 2 + 255) // 256) * 256
     assert pic.pic_decode_workspace_size(_geom(num_kv_heads=0), 1, 10, 1) == 0
-    # one Llama-3-8B layer, 192 inline tokens over ~4.3k keys: 48 query tiles fill
-    # a third of the GPU, so the automatic choice splits the keys three ways
-    assert pic.pic_prefill_num_splits(g, 1, 192, 4288, 0) == 3
+    # one Llama-3-8B layer, 192 inline tokens over ~4.3k keys: 48 query tiles in
+    # 24 two-tile CTAs; six key splits fill the GPU in a single wave
+    assert pic.pic_prefill_num_splits(g, 1, 192, 4288, 0) == 6
     assert pic.pic_prefill_num_splits(g, 1, 192, 4288, 5) == 5
     assert pic.pic_decode_num_splits(g, 16, 33000, 7) == 7
     assert 1 <= pic.pic_decode_num_splits(g, 16, 33000, 0) <= 64
