@@ -222,6 +222,35 @@ pic_status_t pic_attend_prefill(const pic_geom_t *geom, int32_t layer, int32_t b
                                 pic_stream_t stream);
 
 /*
+ * pic_attend_prefill_fused -- pic_attend_prefill without the relocated cache:
+ * the same outputs, with every document key and value read straight from the
+ * pool as it was compiled (the benchmark spec's fused rotate-on-load variant of the
+ * re-rotation of Eq. 3).  Because rotations are orthogonal,
+ *     (R(p) q) . (R(delta_k) k) = (R(-delta_k) R(p) q) . k,
+ * so per document k the 128-row query tile is rotated by -delta_k (in TMEM)
+ * instead of rotating the document's keys; values are used as they are.
+ * Prefix and query keys come from the paged cache, so pic_compose and
+ * pic_append_inline must have run for this layer; pic_relocate is not needed.
+ * Extra inputs: k_pool, v_pool, pool_tokens (layout above), doc_token_start
+ *   int64 [n_pool_docs], doc_len int32 [n_pool_docs], and, from the request,
+ *   req_doc_ids, doc_offset, doc_delta [batch][max_docs] (max_docs <= 1024),
+ *   req_num_docs [batch].  Other arguments as pic_attend_prefill; the
+ *   workspace is the one pic_append_inline filled.
+ */
+pic_status_t pic_attend_prefill_fused(const pic_geom_t *geom, int32_t layer, int32_t batch,
+                                      int32_t max_inline, const int32_t *inline_pos,
+                                      const int32_t *inline_len, int32_t max_ctx,
+                                      const int32_t *block_table, int32_t max_pages,
+                                      int64_t num_pages, const void *k_cache, const void *v_cache,
+                                      const void *k_pool, const void *v_pool, int64_t pool_tokens,
+                                      int32_t max_docs, const int64_t *doc_token_start,
+                                      const int32_t *doc_len, const int32_t *req_doc_ids,
+                                      const int32_t *req_num_docs, const int32_t *doc_offset,
+                                      const int32_t *doc_delta, void *out, float *lse,
+                                      int32_t num_splits, void *workspace, size_t workspace_bytes,
+                                      pic_stream_t stream);
+
+/*
  * pic_attend_decode -- one layer of one plain autoregressive decoding step over
  * the completed cache (appendix "Position-Independent Linking": after the first
  * token, generation proceeds as usual on the linked cache).

@@ -17,7 +17,8 @@ import torch
 
 __all__ = [
     "Geometry", "load", "lib_path", "pic_abi_version", "pic_compose", "pic_relocate",
-    "pic_append_inline", "pic_attend_prefill", "pic_prefill_workspace_size",
+    "pic_append_inline", "pic_attend_prefill", "pic_attend_prefill_fused",
+    "pic_prefill_workspace_size",
     "pic_prefill_num_splits", "pic_decode_num_splits", "pic_attend_decode_noalloc",
     "pic_attend_decode", "pic_decode_workspace_size", "pic_device_status", "PicError",
     "EXPORTED_SYMBOLS", "ROPE_HALF", "ROPE_INTERLEAVED",
@@ -34,7 +35,7 @@ ROPE_INTERLEAVED = 1
 EXPORTED_SYMBOLS = (
     "pic_abi_version", "pic_last_error", "pic_device_status", "pic_compose", "pic_relocate",
     "pic_prefill_workspace_size", "pic_prefill_num_splits", "pic_append_inline",
-    "pic_attend_prefill", "pic_decode_workspace_size", "pic_decode_num_splits",
+    "pic_attend_prefill", "pic_attend_prefill_fused", "pic_decode_workspace_size", "pic_decode_num_splits",
     "pic_attend_decode", "pic_attend_decode_noalloc",
 )
 
@@ -106,6 +107,8 @@ def load():
                                     P]),
         "pic_attend_prefill": (I32, [G, I32, I32, I32, P, P, I32, P, I32, I64, P, P, P, P, I32,
                                      P, SZ, P]),
+        "pic_attend_prefill_fused": (I32, [G, I32, I32, I32, P, P, I32, P, I32, I64, P, P, P, P,
+                                           I64, I32, P, P, P, P, P, P, P, P, I32, P, SZ, P]),
         "pic_decode_workspace_size": (SZ, [G, I32, I32, I32]),
         "pic_attend_decode_noalloc": (I32, [G, I32, I32, P, P, P, P, I32, P, I32, I64, P, P, P, P,
                                             I32, I32, P]),
@@ -246,6 +249,29 @@ def pic_attend_prefill(geom: Geometry, layer: int, inline_pos, inline_len, max_c
         _ptr(lse, f32, "lse", allow_none=True), num_splits,
         _ptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream))
     _check(st, "pic_attend_prefill")
+
+
+def pic_attend_prefill_fused(geom: Geometry, layer: int, inline_pos, inline_len, max_ctx: int,
+                             block_table, num_pages: int, k_cache, v_cache, k_pool, v_pool,
+                             doc_token_start, doc_len, req_doc_ids, req_num_docs, doc_offset,
+                             doc_delta, out, lse=None, num_splits: int = 0, workspace=None,
+                             stream=None):
+    lib = load()
+    g = geom._c()
+    B, max_inline = inline_pos.shape
+    max_docs = req_doc_ids.shape[1]
+    st = lib.pic_attend_prefill_fused(
+        ctypes.byref(g), layer, B, max_inline, _ptr(inline_pos, i32, "inline_pos"),
+        _ptr(inline_len, i32, "inline_len"), max_ctx, _ptr(block_table, i32, "block_table"),
+        block_table.shape[1], num_pages, _ptr(k_cache, bf16, "k_cache"),
+        _ptr(v_cache, bf16, "v_cache"), _ptr(k_pool, bf16, "k_pool"), _ptr(v_pool, bf16, "v_pool"),
+        k_pool.shape[1], max_docs, _ptr(doc_token_start, i64, "doc_token_start"),
+        _ptr(doc_len, i32, "doc_len"), _ptr(req_doc_ids, i32, "req_doc_ids", allow_none=True),
+        _ptr(req_num_docs, i32, "req_num_docs"), _ptr(doc_offset, i32, "doc_offset", allow_none=True),
+        _ptr(doc_delta, i32, "doc_delta", allow_none=True), _ptr(out, bf16, "out"),
+        _ptr(lse, f32, "lse", allow_none=True), num_splits,
+        _ptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream))
+    _check(st, "pic_attend_prefill_fused")
 
 
 def pic_decode_workspace_size(geom: Geometry, batch: int, max_ctx: int, num_splits: int = 0) -> int:

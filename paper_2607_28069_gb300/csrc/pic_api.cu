@@ -106,6 +106,24 @@ pic_status_t encode_tmap_2d(CUtensorMap *map, const void *base, uint64_t inner, 
   return PIC_OK;
 }
 
+pic_status_t encode_tmap_3d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t mid,
+                            uint64_t outer, uint64_t mid_stride_bytes, uint64_t outer_stride_bytes,
+                            uint32_t box_inner, uint32_t box_mid, uint32_t box_outer) {
+  EncodeFn enc = get_encode();
+  if (!enc) return fail(PIC_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+  if ((reinterpret_cast<uintptr_t>(base) & 15) || (mid_stride_bytes & 15) || (outer_stride_bytes & 15))
+    return fail(PIC_ERR_INVALID_ARG, "tensor base/strides not 16-byte aligned");
+  cuuint64_t dims[3] = {inner, mid, outer};
+  cuuint64_t strides[2] = {mid_stride_bytes, outer_stride_bytes};
+  cuuint32_t box[3] = {box_inner, box_mid, box_outer};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims,
+                   strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(PIC_ERR_CUDA, "cuTensorMapEncodeTiled (3d) failed (%d)", (int)r);
+  return PIC_OK;
+}
+
 }  // namespace pic
 
 extern "C" {

@@ -44,6 +44,11 @@ inline pic_status_t make_rope(const pic_geom_t *g, RopeParams *rp) {
 pic_status_t encode_tmap_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t rows,
                             uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows);
 
+// Rows of `inner` elements with two strides: dims {inner, mid, outer}.
+pic_status_t encode_tmap_3d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t mid,
+                            uint64_t outer, uint64_t mid_stride_bytes, uint64_t outer_stride_bytes,
+                            uint32_t box_inner, uint32_t box_mid, uint32_t box_outer);
+
 constexpr int kMaxHalfDim = 64;
 
 // ---------------------------------------------------------- device helpers
@@ -233,6 +238,13 @@ PIC_DEV void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uin
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+PIC_DEV void tma_load_3d(uint32_t dst, const CUtensorMap *map, int x, int y, int z, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
       : "memory");
 }
 PIC_DEV void prefetch_tmap(const CUtensorMap *map) {

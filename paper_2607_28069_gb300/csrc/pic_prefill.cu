@@ -425,6 +425,556 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// ===========================================================================
+// Fused rotate-on-load prefill attention (documents read from the pool).
+//
+// Instead of reading relocated keys R(delta_k) k from the stitched cache, the
+// kernel reads the documents' keys and values straight from the pool (as they
+// were compiled) and rotates the *queries* the other way:
+//     (R(p) q) . (R(delta_k) k) = (R(-delta_k) R(p) q) . k,
+// since rotations are orthogonal.  Per document the query tile is turned into
+// Q'_k = R(-delta_k) Q in TMEM by the softmax threads (each owns one TMEM lane,
+// i.e. one query row) and the QK^T MMA takes its A operand from TMEM.  Prefix
+// and query keys (written by pic_append_inline) still come from the paged
+// cache.  A pool tile is 128 consecutive rows of one document: two 16 KB TMA
+// boxes per operand instead of 16 page boxes.
+//
+// Key tiles are segment aligned: the prefix [0, P) and the query span [Q0, Q1)
+// in 128-key tiles of the absolute position grid (keys outside the segment
+// masked), each document in 128-key tiles from its first token (keys past its
+// end masked).  Everything else (splits, pipeline, epilogue) is as in
+// attn_kernel's single-tile form.
+// TMEM: S_0 [0,128), S_1 [128,256), O [256,256+D), Q'_0 [384,384+D/2),
+// Q'_1 [448,448+D/2) (bf16 pairs).
+namespace fused {
+
+constexpr int BN = 128, NST = 2, kThreads = 192, kMaxDocs = 1024;
+
+template <int D>
+struct Layout {
+  static constexpr int kTile = BN * D * 2;
+  static constexpr int kQ = 0;
+  static constexpr int kK = kQ + BM * D * 2;
+  static constexpr int kV = kK + NST * kTile;
+  static constexpr int kMeta = kV + NST * kTile;
+  // seg_first[kMaxDocs + 3] int32, off/len/delta [kMaxDocs] int32, start [kMaxDocs] int64
+  static constexpr int kSegFirst = kMeta;
+  static constexpr int kOff = kSegFirst + (kMaxDocs + 4) * 4;
+  static constexpr int kLen = kOff + kMaxDocs * 4;
+  static constexpr int kDelta = kLen + kMaxDocs * 4;
+  static constexpr int kStart = kDelta + kMaxDocs * 4;
+  static constexpr int kCS = kStart + kMaxDocs * 8;  // 64 float2
+  static constexpr int kBar = kCS + 64 * 8;
+  static constexpr int kBytes = kBar + 256;
+  static constexpr int kAlloc = kBytes + 1024;
+};
+
+enum {
+  F_Q = 0,
+  F_KFULL = 1,
+  F_VFULL = F_KFULL + NST,
+  F_KVEMPTY = F_VFULL + NST,
+  F_SFULL = F_KVEMPTY + NST,
+  F_PFULL = F_SFULL + 2,
+  F_PFREE = F_PFULL + 2,
+  F_QREADY = F_PFREE + 2,
+  F_OFINAL = F_QREADY + 2,
+  F_COUNT = F_OFINAL + 1
+};
+
+struct FParams {
+  Params base;
+  RopeParams rp;
+  long long pool_tokens;
+  int max_docs, layer;
+  const int32_t *num_docs, *doc_offset, *doc_delta, *ids, *doc_len;
+  const int64_t *doc_start;
+};
+
+// The tile sequence seen by every role.  Segment s: 0 = prefix, 1..m = doc
+// s-1, m+1 = query.  seg_first[s] = index of the segment's first tile.
+struct TileInfo {
+  int doc;         // document index, -1 for a cache tile
+  int key_base;    // logical position of smem row 0
+  int vlo, vhi;    // valid logical key range of this tile
+  int cache_kt;    // absolute 128-key tile index (cache tiles)
+  long long prow;  // pool row of smem row 0 (document tiles)
+  bool doc_first;  // first tile of its document
+};
+
+struct Seq {
+  const int32_t *seg_first, *off, *len, *delta;
+  const long long *start;
+  int m, P, q_lo, q_hi;  // prefix end, query span [q_lo, q_hi)
+  __device__ TileInfo at(int t) const {
+    // segment containing global tile t (binary search over seg_first[0..m+2))
+    int lo = 0, hi = m + 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (seg_first[mid] <= t) lo = mid;
+      else hi = mid - 1;
+    }
+    const int j = t - seg_first[lo];
+    TileInfo ti;
+    if (lo == 0 || lo == m + 1) {
+      const int a = lo == 0 ? 0 : q_lo, e = lo == 0 ? P : q_hi;
+      ti.doc = -1;
+      ti.cache_kt = a / BN + j;
+      ti.key_base = ti.cache_kt * BN;
+      ti.vlo = max(a, ti.key_base);
+      ti.vhi = min(e, ti.key_base + BN);
+      ti.prow = 0;
+      ti.doc_first = false;
+    } else {
+      const int k = lo - 1;
+      ti.doc = k;
+      ti.cache_kt = -1;
+      ti.key_base = off[k] + j * BN;
+      ti.vlo = ti.key_base;
+      ti.vhi = min(off[k] + len[k], ti.key_base + BN);
+      ti.prow = start[k] + (long long)j * BN;
+      ti.doc_first = j == 0;
+    }
+    return ti;
+  }
+};
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_fused_kernel(const __grid_constant__ CUtensorMap tm_q,
+                      const __grid_constant__ CUtensorMap tm_k,
+                      const __grid_constant__ CUtensorMap tm_v,
+                      const __grid_constant__ CUtensorMap tm_kp,
+                      const __grid_constant__ CUtensorMap tm_vp, FParams fp) {
+  using L = Layout<D>;
+  const Params &p = fp.base;
+  constexpr int PANELS = D / 64;
+  constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
+  constexpr uint32_t IDESC_PV = idesc_bf16(BM, D, false, true);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                              ~(uintptr_t)1023);
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t bar0 = sbase + L::kBar;
+  auto bar = [&](int i) { return bar0 + 8u * (uint32_t)i; };
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + L::kBar + 8 * F_COUNT);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::kBar + 8 * F_COUNT + 8);
+  int32_t *s_seg = reinterpret_cast<int32_t *>(smem + L::kSegFirst);
+  int32_t *s_off = reinterpret_cast<int32_t *>(smem + L::kOff);
+  int32_t *s_len = reinterpret_cast<int32_t *>(smem + L::kLen);
+  int32_t *s_delta = reinterpret_cast<int32_t *>(smem + L::kDelta);
+  long long *s_start = reinterpret_cast<long long *>(smem + L::kStart);
+  float2 *s_cs = reinterpret_cast<float2 *>(smem + L::kCS);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int mt = blockIdx.x / p.num_splits, split = blockIdx.x % p.num_splits;
+  const int hk = blockIdx.y, b = blockIdx.z;
+  const int detail = b;
+
+  const int tin = min(max(p.inline_len[b], 0), p.max_inline);
+  const int rows = tin * p.G;
+  const int r0 = mt * BM;
+  if (r0 >= rows) return;
+  const int r_last = min(r0 + BM, rows) - 1;
+  const int32_t *ipos = p.inline_pos + (size_t)b * p.max_inline;
+  const int kmin = ipos[r0 / p.G];
+  const int kmax = ipos[r_last / p.G];
+
+  // ---- per-document metadata into shared memory (all threads)
+  const int m = min(max(fp.num_docs[b], 0), fp.max_docs);
+  for (int k = threadIdx.x; k < m; k += kThreads) {
+    const size_t i = (size_t)b * fp.max_docs + k;
+    const int id = fp.ids[i];
+    s_off[k] = fp.doc_offset[i];
+    s_delta[k] = fp.doc_delta[i];
+    s_len[k] = (id >= 0) ? fp.doc_len[id] : 0;
+    s_start[k] = (id >= 0) ? fp.doc_start[id] : 0;
+  }
+  __syncthreads();
+  Seq sq;
+  sq.seg_first = s_seg;
+  sq.off = s_off;
+  sq.len = s_len;
+  sq.delta = s_delta;
+  sq.start = s_start;
+  sq.m = m;
+  const int kend = kmax + 1;  // keys at or beyond kend are never visible here
+  sq.P = min(m > 0 ? s_off[0] : kend, kend);
+  sq.q_lo = m > 0 ? s_off[m - 1] + s_len[m - 1] : sq.P;
+  sq.q_hi = kend;
+  if (threadIdx.x == 0) {  // tiles per segment, prefix sums (m <= kMaxDocs, serial is fine)
+    int t = 0;
+    auto cache_tiles = [&](int a, int e) { return e > a ? (e - 1) / BN - a / BN + 1 : 0; };
+    s_seg[0] = 0;
+    t += cache_tiles(0, sq.P);
+    for (int k = 0; k < m; ++k) {
+      s_seg[k + 1] = t;
+      const int e = min(s_off[k] + s_len[k], kend);
+      t += e > s_off[k] ? (e - s_off[k] + BN - 1) / BN : 0;
+    }
+    s_seg[m + 1] = t;
+    t += cache_tiles(sq.q_lo, sq.q_hi);
+    s_seg[m + 2] = t;
+  }
+  __syncthreads();
+  const int n_all = s_seg[m + 2];
+  const int per = (n_all + p.num_splits - 1) / p.num_splits;
+  const int kv_begin = split * per;
+  const int n = max(0, min(per, n_all - kv_begin));
+  const size_t part_row0 =
+      ((((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * p.num_splits + split) * BM;
+  if (n == 0) {
+    if (p.num_splits > 1 && threadIdx.x < BM) {
+      p.part_ml[(part_row0 + threadIdx.x) * 2] = -INFINITY;
+      p.part_ml[(part_row0 + threadIdx.x) * 2 + 1] = 0.f;
+    }
+    return;
+  }
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < F_COUNT; ++i)
+      mbar_init(bar(i), (i == F_PFULL || i == F_PFULL + 1 || i == F_QREADY || i == F_QREADY + 1)
+                            ? 128 : 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = *tmem_slot;
+
+  if (warp == 0) {
+    // ===================================================== TMA producer
+    const int32_t *bt = p.block_table + (size_t)b * p.max_pages;
+    if (lane == 0) {
+      prefetch_tmap(&tm_q);
+      prefetch_tmap(&tm_k);
+      prefetch_tmap(&tm_v);
+      prefetch_tmap(&tm_kp);
+      prefetch_tmap(&tm_vp);
+      mbar_expect_tx(bar(F_Q), BM * D * 2);
+      const int qrow = (b * p.Hkv + hk) * p.R_pad + r0;
+      for (int pn = 0; pn < PANELS; ++pn)
+        tma_load_2d(sbase + L::kQ + pn * BM * 128, &tm_q, pn * 64, qrow, bar(F_Q));
+    }
+    int issued = 0;
+    for (int j = 0; j < n; ++j) {
+      const int st = j % NST;
+      const TileInfo ti = sq.at(kv_begin + j);
+      int y = p.oob_row;  // cache tile: lanes 0..7 look up their page
+      if (ti.doc < 0 && lane < 8) {
+        const int pidx = ti.cache_kt * 8 + lane;
+        if (pidx * 16 < ti.vhi && pidx < p.max_pages) {
+          const int page = bt[pidx];
+          if (page >= 0 && page < p.num_pages)
+            y = (int)(p.layer_row0 + ((long long)page * p.Hkv + hk) * 16);
+          else
+            dev_fail(p.status, PIC_DEV_BAD_PAGE, detail);
+        }
+      }
+      if (j >= NST) {
+        const bool ok = mbar_wait(bar(F_KVEMPTY + st), ((j / NST) - 1) & 1, abort_flag, p.status, detail);
+        if (!__all_sync(0xffffffffu, ok)) break;
+      }
+      if (lane == 0) mbar_expect_tx(bar(F_KFULL + st), L::kTile);
+      if (lane == 16) mbar_expect_tx(bar(F_VFULL + st), L::kTile);
+      __syncwarp();
+      if (ti.doc < 0) {
+        const int box = lane & 15, bpage = box / PANELS, bpanel = box % PANELS;
+        const int yb = __shfl_sync(0xffffffffu, y, bpage);
+        if (box < 8 * PANELS) {
+          const uint32_t off = st * L::kTile + bpanel * BN * 128 + bpage * 16 * 128;
+          if (lane < 16)
+            tma_load_2d(sbase + L::kK + off, &tm_k, bpanel * 64, yb, bar(F_KFULL + st));
+          else
+            tma_load_2d(sbase + L::kV + off, &tm_v, bpanel * 64, yb, bar(F_VFULL + st));
+        }
+      } else {
+        // two 128-row boxes per operand, straight from the pool rows of the document
+        const int z = (int)((long long)fp.layer * fp.pool_tokens + ti.prow);
+        if (lane < PANELS)
+          tma_load_3d(sbase + L::kK + st * L::kTile + lane * BN * 128, &tm_kp, lane * 64, hk, z,
+                      bar(F_KFULL + st));
+        else if (lane >= 16 && lane < 16 + PANELS)
+          tma_load_3d(sbase + L::kV + st * L::kTile + (lane - 16) * BN * 128, &tm_vp,
+                      (lane - 16) * 64, hk, z, bar(F_VFULL + st));
+      }
+      issued = j + 1;
+    }
+    if (lane == 0 && *abort_flag) {
+      for (int j = max(0, issued - NST); j < issued; ++j) {
+        mbar_wait(bar(F_KFULL + j % NST), (j / NST) & 1, abort_flag, p.status, detail);
+        mbar_wait(bar(F_VFULL + j % NST), (j / NST) & 1, abort_flag, p.status, detail);
+      }
+    }
+  } else if (warp == 1) {
+    // ===================================================== MMA issuer
+    if (lane == 0) {
+      const uint32_t tS0 = tbase, tO = tbase + 256, tQd = tbase + 384;
+      bool ok = mbar_wait(bar(F_Q), 0, abort_flag, p.status, detail);
+      tc_fence_after();
+      int dcount = -1;  // documents entered so far in this split
+      for (int j = 0; ok && j <= n; ++j) {
+        if (j < n) {
+          const int st = j % NST, sb = j & 1;
+          const TileInfo ti = sq.at(kv_begin + j);
+          if (ti.doc >= 0 && (ti.doc_first || j == 0)) {  // entering a document
+            ++dcount;
+            if (!mbar_wait(bar(F_QREADY + (dcount & 1)), (dcount >> 1) & 1, abort_flag, p.status, detail)) break;
+          }
+          if (!mbar_wait(bar(F_KFULL + st), (j / NST) & 1, abort_flag, p.status, detail)) break;
+          tc_fence_after();
+          const uint32_t kb = sbase + L::kK + st * L::kTile;
+          if (ti.doc < 0) {
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * (BM * 128) + (kk & 3) * 32;
+              mma_ss(tS0 + sb * 128, sdesc_sw128(sbase + L::kQ + off, 16, 1024),
+                     sdesc_sw128(kb + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024), IDESC_QK,
+                     kk > 0);
+            }
+          } else {
+            const uint32_t qa = tQd + (dcount & 1) * 64;
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk)
+              mma_ts(tS0 + sb * 128, qa + kk * 8,
+                     sdesc_sw128(kb + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024), IDESC_QK,
+                     kk > 0);
+          }
+          mma_commit(bar(F_SFULL + sb));
+        }
+        if (j >= 1) {
+          const int pj = j - 1, pst = pj % NST, pb = pj & 1;
+          if (!mbar_wait(bar(F_PFULL + pb), (pj >> 1) & 1, abort_flag, p.status, detail)) break;
+          if (!mbar_wait(bar(F_VFULL + pst), (pj / NST) & 1, abort_flag, p.status, detail)) break;
+          tc_fence_after();
+          const uint32_t vb = sbase + L::kV + pst * L::kTile;
+#pragma unroll
+          for (int kk = 0; kk < BN / 16; ++kk)
+            mma_ts(tO, tS0 + pb * 128 + kk * 8, sdesc_sw128(vb + kk * 16 * 128, BN * 128, 1024),
+                   IDESC_PV, (pj > 0 || kk > 0));
+          mma_commit(bar(F_KVEMPTY + pst));
+          mma_commit(bar(F_PFREE + pb));
+        }
+      }
+      mma_commit(bar(F_OFINAL));
+    }
+  } else {
+    // ===================================================== softmax warps
+    const int wq = warp & 3;
+    const int row = wq * 32 + lane;
+    const int rg = r0 + row;
+    const bool valid = rg < rows;
+    const int tok = rg / p.G, g = rg % p.G;
+    const int pos = valid ? ipos[tok] : -1;
+    const uint32_t tl = tbase + ((uint32_t)(wq * 32) << 16);
+    const uint32_t tQd = tl + 384;
+    const int tid128 = threadIdx.x - 64;
+    bool ok = true;
+
+    float m_used = -INFINITY, l = 0.f;
+    int dcount = -1;
+    // Q'_k = R(-delta_k) Q for this thread's row, into TMEM buffer `buf`.
+    auto make_qd = [&](int k, int buf) {
+      asm volatile("bar.sync 1, 128;" ::: "memory");  // previous table no longer read
+      if (tid128 < D / 2) {
+        const float2 cs = rope_cos_sin(s_delta[k], fp.rp.theta[tid128]);
+        s_cs[tid128] = make_float2(cs.x, -cs.y);  // R(-delta): sin changes sign
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      // my row of Q from shared memory (128-byte swizzled panels), rotate, pack
+      float x[D];
+      const uint8_t *qs = smem + L::kQ;
+#pragma unroll
+      for (int c = 0; c < D / 8; ++c) {
+        const int pn = c >> 3, ch = c & 7;
+        const uint4 v = *reinterpret_cast<const uint4 *>(
+            qs + pn * BM * 128 + row * 128 + ((ch ^ (row & 7)) << 4));
+        unpack8(v, x + 8 * c);
+      }
+      uint32_t pk[D / 2];
+      if (fp.rp.style == PIC_ROPE_HALF) {
+#pragma unroll
+        for (int i = 0; i < D / 2; ++i) {
+          const float2 cs = s_cs[i];
+          const float u = x[i], w = x[i + D / 2];
+          x[i] = fmaf(u, cs.x, -w * cs.y);
+          x[i + D / 2] = fmaf(u, cs.y, w * cs.x);
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < D / 2; ++i) {
+          const float2 cs = s_cs[i];
+          const float u = x[2 * i], w = x[2 * i + 1];
+          x[2 * i] = fmaf(u, cs.x, -w * cs.y);
+          x[2 * i + 1] = fmaf(u, cs.y, w * cs.x);
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < D / 2; ++i) pk[i] = pack2(x[2 * i], x[2 * i + 1]);
+#pragma unroll
+      for (int c = 0; c < D / 64; ++c) tmem_st32(tQd + buf * 64 + c * 32, pk + c * 32);
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(bar(F_QREADY + buf));
+    };
+
+    if (!__all_sync(0xffffffffu, mbar_wait(bar(F_Q), 0, abort_flag, p.status, detail))) ok = false;
+    // documents of this split, in order: first one prepared up front
+    int next_doc = -1;  // next document whose Q' is still to be prepared
+    if (ok) {
+      for (int j = 0; j < n; ++j) {
+        const TileInfo ti = sq.at(kv_begin + j);
+        if (ti.doc >= 0) {
+          next_doc = ti.doc;
+          break;
+        }
+      }
+      if (next_doc >= 0) {
+        make_qd(next_doc, 0);
+        ++next_doc;
+      }
+    }
+    const int last_tile_doc = ok ? sq.at(kv_begin + n - 1).doc : -1;
+    for (int j = 0; ok && j < n; ++j) {
+      const int sb = j & 1;
+      const TileInfo ti = sq.at(kv_begin + j);
+      if (!__all_sync(0xffffffffu, mbar_wait(bar(F_SFULL + sb), (j >> 1) & 1, abort_flag, p.status, detail))) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      if (ti.doc >= 0 && (ti.doc_first || j == 0)) {
+        ++dcount;
+        // S of this document's first tile is ready, so every QK of the
+        // document before it has finished: its Q' buffer may be reused.
+        if (next_doc >= 0 && next_doc < m && next_doc <= last_tile_doc && last_tile_doc >= 0) {
+          make_qd(next_doc, (dcount + 1) & 1);
+          ++next_doc;
+        }
+      }
+      float s[BN];
+#pragma unroll
+      for (int c = 0; c < BN / 32; ++c)
+        tmem_ld32(tl + sb * 128 + c * 32, reinterpret_cast<uint32_t *>(s + c * 32));
+      tmem_wait_ld();
+      {
+        const int lo = ti.vlo - ti.key_base, hi = min(ti.vhi, pos + 1) - ti.key_base;
+        if (lo > 0 || hi < BN) {
+#pragma unroll
+          for (int c = 0; c < BN; ++c)
+            if (c < lo || c >= hi) s[c] = -INFINITY;
+        }
+      }
+      float mx8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) mx8[i] = s[i];
+#pragma unroll
+      for (int c = 8; c < BN; c += 8)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) mx8[i] = fmaxf(mx8[i], s[c + i]);
+#pragma unroll
+      for (int w = 4; w; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) mx8[i] = fmaxf(mx8[i], mx8[i + w]);
+      const float m_new = fmaxf(m_used, mx8[0] * p.scale_log2);
+      float alpha = 1.f;
+      const bool resc = m_new > m_used + 8.f;
+      if (resc) {
+        alpha = ex2(m_used - m_new);
+        m_used = m_new;
+      }
+      const float mref = (m_used == -INFINITY) ? 0.f : m_used;
+      float ls8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ls8[i] = 0.f;
+      uint32_t pk[BN / 2];
+#pragma unroll
+      for (int c = 0; c < BN; c += 2) {
+        const float p0 = ex2(fmaf(s[c], p.scale_log2, -mref));
+        const float p1 = ex2(fmaf(s[c + 1], p.scale_log2, -mref));
+        ls8[(c >> 1) & 7] += p0 + p1;
+        pk[c / 2] = pack2(p0, p1);
+      }
+#pragma unroll
+      for (int w = 4; w; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) ls8[i] += ls8[i + w];
+      l = fmaf(l, alpha, ls8[0]);
+      if (j > 0 && __any_sync(0xffffffffu, resc)) {
+        const int pj = j - 1;
+        if (!__all_sync(0xffffffffu, mbar_wait(bar(F_PFREE + (pj & 1)), (pj >> 1) & 1, abort_flag, p.status, detail))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+          float o[32];
+          tmem_ld32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o));
+          tmem_wait_ld();
+#pragma unroll
+          for (int q = 0; q < 32; ++q) o[q] *= alpha;
+          tmem_st32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o));
+        }
+      }
+      tmem_st32(tl + sb * 128, pk);
+      tmem_st32(tl + sb * 128 + 32, pk + 32);
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(bar(F_PFULL + sb));
+    }
+    // ---- epilogue
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(F_OFINAL), 0, abort_flag, p.status, detail));
+    tc_fence_after();
+    if (ok) {
+      float o[D];
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) tmem_ld32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o + c * 32));
+      tmem_wait_ld();
+      if (p.num_splits == 1) {
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+        __nv_bfloat16 *dst = p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D;
+        if (valid) {
+#pragma unroll
+          for (int q = 0; q < D; ++q) o[q] *= inv;
+#pragma unroll
+          for (int q = 0; q < D / 8; ++q) st_global16(dst + q * 8, pack8(o + q * 8));
+        }
+        if (valid && p.lse)
+          p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
+              l > 0.f ? (m_used + __log2f(l)) * 0.69314718055994531f : -INFINITY;
+      } else {
+        float *dst = p.part_o + (part_row0 + row) * D;
+        if (valid) {
+#pragma unroll
+          for (int q = 0; q < D / 4; ++q)
+            reinterpret_cast<float4 *>(dst)[q] =
+                make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+        }
+        p.part_ml[(part_row0 + row) * 2] = (l > 0.f) ? m_used : -INFINITY;
+        p.part_ml[(part_row0 + row) * 2 + 1] = l;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    if (*abort_flag && lane == 0) mbar_wait(bar(F_OFINAL), 0, abort_flag, p.status, detail);
+    __syncwarp();
+    tmem_dealloc(tbase, kTmemCols);
+  }
+}
+
+}  // namespace fused
+
 // Merge the split partials (O unnormalised, m in log2 units, l) of every
 // query row by log-sum-exp: one warp per row, lanes over the d columns.  All
 // loads are issued unconditionally (an empty split's weight is zero and its
@@ -819,5 +1369,114 @@ extern "C" pic_status_t pic_attend_prefill(
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill launch");
+  return PIC_OK;
+}
+
+extern "C" pic_status_t pic_attend_prefill_fused(
+    const pic_geom_t *geom, int32_t layer, int32_t batch, int32_t max_inline,
+    const int32_t *inline_pos, const int32_t *inline_len, int32_t max_ctx,
+    const int32_t *block_table, int32_t max_pages, int64_t num_pages, const void *k_cache,
+    const void *v_cache, const void *k_pool, const void *v_pool, int64_t pool_tokens,
+    int32_t max_docs, const int64_t *doc_token_start, const int32_t *doc_len,
+    const int32_t *req_doc_ids, const int32_t *req_num_docs, const int32_t *doc_offset,
+    const int32_t *doc_delta, void *out, float *lse, int32_t num_splits, void *workspace,
+    size_t workspace_bytes, pic_stream_t stream) {
+  using namespace pic;
+  using namespace pic::prefill;
+  RopeParams rp;
+  Plan pl;
+  pic_status_t st = check_common("pic_attend_prefill_fused", geom, layer, batch, max_inline,
+                                 max_ctx, num_pages, num_splits, workspace, workspace_bytes, &rp,
+                                 &pl);
+  if (st != PIC_OK) return st;
+  if (max_pages <= 0 || pool_tokens <= 0 || max_docs < 0)
+    return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill_fused: sizes must be positive");
+  if (max_docs > fused::kMaxDocs)
+    return fail(PIC_ERR_UNSUPPORTED, "pic_attend_prefill_fused: max_docs %d > %d", max_docs,
+                fused::kMaxDocs);
+  if ((long long)geom->num_layers * pool_tokens >= (long long)INT32_MAX)
+    return fail(PIC_ERR_UNSUPPORTED, "pic_attend_prefill_fused: pool has more than 2^31 rows");
+  if (!inline_pos || !inline_len || !block_table || !k_cache || !v_cache || !k_pool || !v_pool ||
+      !out || (max_docs > 0 && (!doc_token_start || !doc_len || !req_doc_ids || !doc_offset ||
+                                !doc_delta)) || !req_num_docs)
+    return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill_fused: NULL tensor");
+  if ((reinterpret_cast<uintptr_t>(k_cache) | reinterpret_cast<uintptr_t>(v_cache) |
+       reinterpret_cast<uintptr_t>(k_pool) | reinterpret_cast<uintptr_t>(v_pool) |
+       reinterpret_cast<uintptr_t>(out)) & 15)
+    return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill_fused: bf16 tensors must be 16-byte aligned");
+  int32_t *status = device_status_ptr();
+  if (!status) return fail(PIC_ERR_CUDA, "pic_attend_prefill_fused: no device status word");
+  const int D = geom->head_dim, Hkv = geom->num_kv_heads;
+  const long long rows_total = (long long)geom->num_layers * num_pages * Hkv * 16;
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+
+  CUtensorMap tq, tk, tv, tkp, tvp;
+  st = encode_tmap_2d(&tq, ws, D, (uint64_t)batch * Hkv * pl.R_pad, (uint64_t)D * 2, 64, BM);
+  if (st == PIC_OK) st = encode_tmap_2d(&tk, k_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
+  if (st == PIC_OK) st = encode_tmap_2d(&tv, v_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
+  const uint64_t pool_rows = (uint64_t)geom->num_layers * pool_tokens;
+  if (st == PIC_OK)
+    st = encode_tmap_3d(&tkp, k_pool, D, Hkv, pool_rows, (uint64_t)D * 2, (uint64_t)Hkv * D * 2,
+                        64, 1, fused::BN);
+  if (st == PIC_OK)
+    st = encode_tmap_3d(&tvp, v_pool, D, Hkv, pool_rows, (uint64_t)D * 2, (uint64_t)Hkv * D * 2,
+                        64, 1, fused::BN);
+  if (st != PIC_OK) return st;
+
+  fused::FParams fp;
+  Params &pp = fp.base;
+  pp.batch = batch;
+  pp.Hq = geom->num_q_heads;
+  pp.Hkv = Hkv;
+  pp.G = pl.G;
+  pp.max_inline = max_inline;
+  pp.R_pad = pl.R_pad;
+  pp.m_tiles = pl.m_tiles;
+  pp.num_splits = pl.splits;
+  pp.max_pages = max_pages;
+  pp.oob_row = (int)rows_total;
+  pp.num_pages = num_pages;
+  pp.layer_row0 = (long long)layer * num_pages * Hkv * 16;
+  pp.inline_pos = inline_pos;
+  pp.inline_len = inline_len;
+  pp.block_table = block_table;
+  pp.out = static_cast<__nv_bfloat16 *>(out);
+  pp.lse = lse;
+  pp.part_o = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes) : nullptr;
+  pp.part_ml = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes + pl.po_bytes) : nullptr;
+  pp.status = status;
+  pp.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
+  fp.rp = rp;
+  fp.pool_tokens = pool_tokens;
+  fp.max_docs = max_docs;
+  fp.layer = layer;
+  fp.num_docs = req_num_docs;
+  fp.doc_offset = doc_offset;
+  fp.doc_delta = doc_delta;
+  fp.ids = req_doc_ids;
+  fp.doc_len = doc_len;
+  fp.doc_start = doc_token_start;
+
+  dim3 grid(pl.m_tiles * pl.splits, Hkv, batch);
+  cudaError_t e;
+  if (D == 128) {
+    const int smem = fused::Layout<128>::kAlloc;
+    e = cudaFuncSetAttribute(fused::attn_fused_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused smem attribute");
+    fused::attn_fused_kernel<128><<<grid, fused::kThreads, smem, stream>>>(tq, tk, tv, tkp, tvp, fp);
+  } else {
+    const int smem = fused::Layout<64>::kAlloc;
+    e = cudaFuncSetAttribute(fused::attn_fused_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused smem attribute");
+    fused::attn_fused_kernel<64><<<grid, fused::kThreads, smem, stream>>>(tq, tk, tv, tkp, tvp, fp);
+  }
+  if (pl.splits > 1) {
+    const long long crows = (long long)batch * Hkv * pl.m_tiles * BM;
+    const unsigned cgrid = (unsigned)((crows + 7) / 8);
+    if (D == 128) combine_kernel<128><<<cgrid, 256, 0, stream>>>(pp);
+    else combine_kernel<64><<<cgrid, 256, 0, stream>>>(pp);
+  }
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused launch");
   return PIC_OK;
 }

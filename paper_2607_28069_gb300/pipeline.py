@@ -9,7 +9,8 @@ from __future__ import annotations
 import torch
 
 from . import (Geometry, pic_append_inline, pic_attend_decode, pic_attend_prefill,
-               pic_compose, pic_decode_workspace_size, pic_prefill_workspace_size, pic_relocate)
+               pic_attend_prefill_fused, pic_compose, pic_decode_workspace_size,
+               pic_prefill_workspace_size, pic_relocate)
 from .workloads import Workload
 
 
@@ -87,9 +88,27 @@ class CacheHitPath:
                            self.out[layer], None if self.lse is None else self.lse[layer],
                            self.prefill_splits, self.ws_prefill)
 
+    # -- a7: prefill attention reading the documents from the pool (no relocate)
+    def attend_fused(self, layer: int):
+        wl = self.wl
+        pic_attend_prefill_fused(self.geom, layer, self.inline_pos, wl.inline_len, self.max_ctx,
+                                 wl.block_table, wl.num_pages, self.k_cache, self.v_cache,
+                                 wl.k_pool, wl.v_pool, wl.doc_token_start, wl.doc_len,
+                                 wl.req_doc_ids, wl.req_num_docs, self.doc_offset, self.doc_delta,
+                                 self.out[layer], None if self.lse is None else self.lse[layer],
+                                 self.prefill_splits, self.ws_prefill)
+
     def prefill(self, layer: int):
         self.append(layer)
         self.attend(layer)
+
+    def fused_pass(self):
+        """The cache-hit path with rotate-on-load attention: layout, then per
+        layer the inline append and the fused attention; no relocation."""
+        self.compose()
+        for layer in range(self.wl.spec.layers):
+            self.append(layer)
+            self.attend_fused(layer)
 
     # -- a6: one decode step of one layer (token position ctx_len + step)
     def decode(self, step: int, layer: int):

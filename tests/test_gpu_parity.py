@@ -249,3 +249,71 @@ def test_device_checks_report_bad_inputs(cuda_lib):
     code, _ = pic.pic_device_status()
     assert code == 6
     assert pic.pic_device_status() == (0, 0)   # cleared by the read
+
+
+# ------------------------------------------------- fused rotate-on-load (a7)
+_FUSED = {}
+
+
+def run_fused(name, splits=0, rope_style=0):
+    key = (name, splits, rope_style)
+    if key in _FUSED:
+        return _FUSED[key]
+    from paper_2607_28069_gb300.pipeline import CacheHitPath
+    import paper_2607_28069_gb300 as pic
+    wl = generate(SMALL[name], device="cuda", gen_device="cpu")
+    path = CacheHitPath(wl, prefill_splits=splits, with_lse=True, rope_style=rope_style)
+    path.fused_pass()        # compose + append + fused attention; the cache never sees a document
+    torch.cuda.synchronize()
+    assert pic.pic_device_status() == (0, 0)
+    _FUSED[key] = (wl, path)
+    return _FUSED[key]
+
+
+@pytest.mark.parametrize("name", ["tiny", "llama8b_1layer", "ragged_b3", "gqa7_decode", "d64_g8",
+                                  "no_docs"])
+@pytest.mark.parametrize("splits", [0, 1, 3])
+def test_fused_prefill_matches_oracle(cuda_lib, name, splits):
+    wl, path = run_fused(name, splits)
+    theta = theta_of(wl.spec)
+    for layer in range(wl.spec.layers):
+        for b in range(wl.spec.batch):
+            lay = oracle_layout(wl, b)
+            docs, k_docs, v_docs, q, k, v = request_inputs(wl, b, layer)
+            (o_ref, lse_ref), _, _ = O.cache_hit_prefill(
+                lay, k_docs, v_docs, wl.doc_base_pos.cpu().numpy(), q, k, v, theta,
+                return_lse=True)
+            o_gpu = f64(path.out[layer, b, :q.shape[0]])
+            ok, max_abs, row = attn_close(o_gpu, o_ref)
+            assert ok, f"layer {layer} req {b}: max-abs {max_abs:.2e} row-rel {row:.2e}"
+            assert np.abs(f64(path.lse[layer, b, :q.shape[0]]) - lse_ref).max() < 5e-2
+    # the relocated cache was never written: document slots are still zero
+    if wl.spec.docs_per_request:
+        lay = oracle_layout(wl, 0)
+        t = lay.doc_offset[0]
+        s = int(lay.slot_mapping[t])
+        assert float(path.k_cache[0].reshape(-1, wl.spec.kv_heads, 16, wl.spec.head_dim)[
+            s // 16, :, s % 16].abs().max()) == 0.0
+
+
+def test_fused_interleaved_rope(cuda_lib):
+    wl, path = run_fused("ragged_b3", 0, rope_style=1)
+    theta = theta_of(wl.spec)
+    for b in range(wl.spec.batch):
+        lay = oracle_layout(wl, b)
+        docs, k_docs, v_docs, q, k, v = request_inputs(wl, b, 1)
+        o_ref, _, _ = O.cache_hit_prefill(lay, k_docs, v_docs, wl.doc_base_pos.cpu().numpy(),
+                                          q, k, v, theta, O.INTERLEAVED)
+        ok, max_abs, row = attn_close(f64(path.out[1, b, :q.shape[0]]), o_ref)
+        assert ok, (max_abs, row)
+
+
+@pytest.mark.parametrize("name", ["llama8b_1layer", "ragged_b3"])
+def test_fused_equals_materialised(cuda_lib, name):
+    wl, path = run_path(name)
+    wlf, pathf = run_fused(name)
+    a, b = path.out.float(), pathf.out.float()
+    for bb in range(wl.spec.batch):
+        tin = int(wl.inline_len[bb])
+        d = (a[:, bb, :tin] - b[:, bb, :tin]).abs().max().item()
+        assert d <= 1e-2, d
