@@ -840,7 +840,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++next_doc;
       }
     }
-    const int last_tile_doc = ok ? sq.at(kv_begin + n - 1).doc : -1;
+    int last_tile_doc = -1;  // last document with a tile in this split
+    for (int j = n - 1; ok && j >= 0; --j) {
+      const int dj = sq.at(kv_begin + j).doc;
+      if (dj >= 0) {
+        last_tile_doc = dj;
+        break;
+      }
+    }
     for (int j = 0; ok && j < n; ++j) {
       const int sb = j & 1;
       const TileInfo ti = sq.at(kv_begin + j);
@@ -853,7 +860,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++dcount;
         // S of this document's first tile is ready, so every QK of the
         // document before it has finished: its Q' buffer may be reused.
-        if (next_doc >= 0 && next_doc < m && next_doc <= last_tile_doc && last_tile_doc >= 0) {
+        if (next_doc >= 0 && next_doc <= last_tile_doc) {
           make_qd(next_doc, (dcount + 1) & 1);
           ++next_doc;
         }
