@@ -310,7 +310,7 @@ def test_fused_interleaved_rope(cuda_lib):
 
 @pytest.mark.parametrize("name", ["llama8b_1layer", "ragged_b3"])
 def test_fused_equals_materialised(cuda_lib, name):
-    wl, path = run_path(name)
+    wl, path, _ = run_path(name)
     wlf, pathf = run_fused(name)
     a, b = path.out.float(), pathf.out.float()
     for bb in range(wl.spec.batch):
