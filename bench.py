@@ -46,6 +46,8 @@ def parse_args(argv=None):
     ap.add_argument("--decode-splits", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--fused", action="store_true",
+                    help="also time the rotate-on-load pass (default for stress_128k_b4)")
     ap.add_argument("--oracle-sample", default=None, help=argparse.SUPPRESS)
     ap.add_argument("--oracle-seconds", type=float, default=10.0, help=argparse.SUPPRESS)
     return ap.parse_args(argv)
@@ -415,6 +417,39 @@ def main_gpu(args, rank, world):
             "bytes": work["decode_bytes"], "gbs": work["decode_bytes"] / (dms * 1e6),
             "tok_s": spec.batch / (dms / 1e3)}
         rows["a6_decode"]["frac_hbm"] = rows["a6_decode"]["gbs"] / peaks["hbm_gbs"]
+
+    # fused rotate-on-load pass (a7): compose, then per layer append + fused
+    # attention reading the documents from the pool; no relocation
+    if args.fused or args.workload == "stress_128k_b4":
+        fcalls = [("compose", path.compose)]
+        for layer in range(L):
+            fcalls.append(("append", (lambda l=layer: path.append(l))))
+            fcalls.append(("fused", (lambda l=layer: path.attend_fused(l))))
+        fb = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(len(fcalls) + 1)]
+        fg = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(fg):
+            fb[0].record()
+            for i, (_, fn) in enumerate(fcalls):
+                fn()
+                fb[i + 1].record()
+        torch.cuda.synchronize()
+        f_tot, f_att = [], []
+        for k in range(W + max(2, K)):
+            flush.zero_()
+            torch.cuda._sleep(sleep_cycles)
+            fg.replay()
+            torch.cuda.synchronize()
+            ms = [fb[i].elapsed_time(fb[i + 1]) for i in range(len(fcalls))]
+            if k >= W:
+                f_tot.append(sum(ms))
+                f_att.append(sum(x for (nm, _), x in zip(fcalls, ms) if nm == "fused"))
+        fms, fatt = sum(f_tot) / len(f_tot), sum(f_att) / len(f_att)
+        rows["a7_fused"] = {
+            "ms": fms, "attend_ms": fatt, "launches": 1 + L + L * (2 if psplits > 1 else 1),
+            "flops": work["attend_flops"], "tflops": work["attend_flops"] / (fatt * 1e9),
+            "frac_bf16": work["attend_flops"] / (fatt * 1e9) / peaks["bf16_tflops"],
+            "query_tok_s": work["query_tokens"] / (fms / 1e3),
+            "speedup_vs_materialised": ms_per_step / fms}
 
     # dominant kernel of the step -> roofline object
     if per_step["attend"] >= per_step["relocate"]:

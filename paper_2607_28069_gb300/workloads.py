@@ -72,6 +72,16 @@ WORKLOADS = {
         description="32 layers, batch 4 requests of ~139k tokens: all 128 docs of a pool with "
                     "lengths U{128..2048}, each request in its own shuffled order, "
                     "512-token query chunk"),
+    # Profiling-size slices of the full workloads (same per-layer shapes, fewer
+    # layers / steps), so that one profiled launch moves more than L2 holds
+    # while the process stays at a few GB of device memory.
+    "llama8b_2layer_b8": WorkloadSpec(
+        "llama8b_2layer_b8", 2, 32, 8, 128, 5e5, 8, 64, 16, (1024, 1024), (32, 128), 256,
+        description="2 layers of llama8b_32layer_b8 (profiling slice)"),
+    "decode_1layer_b16": WorkloadSpec(
+        "decode_1layer_b16", 1, 28, 4, 128, 1e6, 16, 64, 32, (1024, 1024), (64, 64), 128,
+        decode_steps=1,
+        description="1 layer of decode_28layer_b16 with one decode step (profiling slice)"),
 }
 
 
