@@ -2,7 +2,8 @@
 // into the paged request cache; values are copied unchanged (the paper rotates
 // keys only; Background: Position-Independent Caching).
 //
-// One launch, one CTA per (16 logical positions = one page, request, layer).
+// One launch, one CTA per (one or two pages of logical positions, request,
+// layer).
 // The CTA reads the token map and slot map of its positions (written by
 // pic_compose), issues every K and V load of its page at once (16-byte
 // streaming loads; V rows are bit copies, K rows come as the two 16-byte
@@ -21,7 +22,8 @@ namespace pic {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kTok = 16;  // positions per CTA (one page)
+// Positions per CTA: one page (16) when a token carries >= 1024 K elements,
+// two pages otherwise, so every CTA moves 64 KB and amortises its set-up.
 constexpr int UV = 8;     // V tasks per thread per round
 constexpr int UK = 4;     // K tasks per thread per round
 
@@ -35,8 +37,10 @@ struct RelocArgs {
   int32_t *status;
 };
 
-template <int D>
+template <int D, int kTok>
 __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopeParams rp) {
+  static_assert(kTok == 16 || kTok == 32, "one warp scans the positions of a CTA");
+  constexpr unsigned kMask = kTok == 32 ? 0xffffffffu : 0x0000ffffu;
   constexpr int HALF = D / 2;
   constexpr int KC = D / 16;  // 8-pair chunks per K row
   constexpr int VC = D / 8;   // 16-byte pieces per V row
@@ -75,9 +79,9 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
     s_dst[tid] = slot;
     s_doc[tid] = k;
     // documents of a page are consecutive: first / last valid position's doc
-    const unsigned valid = __ballot_sync(0x0000ffffu, src >= 0);
-    const int kf = __shfl_sync(0x0000ffffu, k, valid ? __ffs(valid) - 1 : 0);
-    const int kl = __shfl_sync(0x0000ffffu, k, valid ? 31 - __clz(valid) : 0);
+    const unsigned valid = __ballot_sync(kMask, src >= 0);
+    const int kf = __shfl_sync(kMask, k, valid ? __ffs(valid) - 1 : 0);
+    const int kl = __shfl_sync(kMask, k, valid ? 31 - __clz(valid) : 0);
     if (tid == 0) {
       s_first = valid ? kf : -1;
       s_last = valid ? kl : -1;
@@ -237,11 +241,16 @@ extern "C" pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int3
   a.k_cache = static_cast<__nv_bfloat16 *>(k_cache);
   a.v_cache = static_cast<__nv_bfloat16 *>(v_cache);
   a.status = status;
-  dim3 grid((max_ctx + kTok - 1) / kTok, batch, layer_end - layer_begin);
-  if (geom->head_dim == 128)
-    relocate_kernel<128><<<grid, kThreads, 0, stream>>>(a, rp);
-  else
-    relocate_kernel<64><<<grid, kThreads, 0, stream>>>(a, rp);
+  const bool wide = geom->num_kv_heads * geom->head_dim >= 1024;
+  const int tok = wide ? 16 : 32;
+  dim3 grid((max_ctx + tok - 1) / tok, batch, layer_end - layer_begin);
+  if (geom->head_dim == 128) {
+    if (wide) relocate_kernel<128, 16><<<grid, kThreads, 0, stream>>>(a, rp);
+    else relocate_kernel<128, 32><<<grid, kThreads, 0, stream>>>(a, rp);
+  } else {
+    if (wide) relocate_kernel<64, 16><<<grid, kThreads, 0, stream>>>(a, rp);
+    else relocate_kernel<64, 32><<<grid, kThreads, 0, stream>>>(a, rp);
+  }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_relocate launch");
   return PIC_OK;
