@@ -124,6 +124,22 @@ pic_status_t encode_tmap_3d(CUtensorMap *map, const void *base, uint64_t inner, 
   return PIC_OK;
 }
 
+pic_status_t encode_tmap_pages128(CUtensorMap *map, const void *base, uint64_t n_page_heads) {
+  EncodeFn enc = get_encode();
+  if (!enc) return fail(PIC_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+  if (reinterpret_cast<uintptr_t>(base) & 15)
+    return fail(PIC_ERR_INVALID_ARG, "tensor base not 16-byte aligned");
+  cuuint64_t dims[4] = {64, 8, 2, 2 * n_page_heads};
+  cuuint64_t strides[3] = {256, 128, 2048};
+  cuuint32_t box[4] = {64, 8, 2, 2};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims,
+                   strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(PIC_ERR_CUDA, "cuTensorMapEncodeTiled (page heads) failed (%d)", (int)r);
+  return PIC_OK;
+}
+
 }  // namespace pic
 
 extern "C" {

@@ -49,6 +49,14 @@ pic_status_t encode_tmap_3d(CUtensorMap *map, const void *base, uint64_t inner, 
                             uint64_t outer, uint64_t mid_stride_bytes, uint64_t outer_stride_bytes,
                             uint32_t box_inner, uint32_t box_mid, uint32_t box_outer);
 
+// Page-head map for 128-dim caches ([..][16 rows][128 bf16] per page-head):
+// 4-D view {64 columns, 8 rows, 2 column panels, 2 * n_page_heads row halves}
+// with strides {256 B, 128 B, 2048 B}.  A box {64, 8, 2, 2} moves one whole
+// 4 KB page-head and lands as [half][panel][8 rows][128 B], so that across a
+// run of pages the 8-row groups of one panel sit at a constant 2048-byte
+// stride (the SW128 operand stride) and the two panels 1024 bytes apart.
+pic_status_t encode_tmap_pages128(CUtensorMap *map, const void *base, uint64_t n_page_heads);
+
 constexpr int kMaxHalfDim = 64;
 
 // ---------------------------------------------------------- device helpers
@@ -93,6 +101,36 @@ PIC_DEV uint4 pack8(const float *f) {
 PIC_DEV uint32_t pack2(float lo, float hi) {
   __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t *>(&h);
+}
+
+// ---- packed fp32 pairs (one 64-bit register pair, low half first)
+PIC_DEV uint64_t f2pack(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+PIC_DEV void f2unpack(uint64_t v, float &lo, float &hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+PIC_DEV uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+PIC_DEV uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+PIC_DEV uint64_t sub2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+PIC_DEV float max3f(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
 }
 
 // Streaming 16-byte load that bypasses L1 (each pool byte is read once).
@@ -247,6 +285,14 @@ PIC_DEV void tma_load_3d(uint32_t dst, const CUtensorMap *map, int x, int y, int
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
       : "memory");
 }
+PIC_DEV void tma_load_4d(uint32_t dst, const CUtensorMap *map, int x, int y, int z, int w,
+                         uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(w), "r"(bar)
+      : "memory");
+}
 PIC_DEV void prefetch_tmap(const CUtensorMap *map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
@@ -355,6 +401,11 @@ PIC_DEV float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+PIC_DEV uint64_t exp2_mufu2(uint64_t x) {
+  float x0, x1;
+  f2unpack(x, x0, x1);
+  return f2pack(ex2(x0), ex2(x1));
 }
 
 // --------------------------------------------------- warp MMA (decode path)

@@ -35,8 +35,10 @@ namespace prefill {
 constexpr int BM = 128;  // query rows per tile (TMEM lanes)
 constexpr int NQ = 2;    // query tiles per CTA, sharing every K/V tile
 constexpr int BN = 128;  // keys per KV tile
-constexpr int NST = 2;   // K/V ring stages
-constexpr int kThreads = 64 + NQ * 128;  // producer warp, MMA warp, NQ softmax warpgroups
+constexpr int NSK = 3;   // K ring stages (released after the last QK of a tile)
+constexpr int NSV = 2;   // V ring stages (released after the last PV of a tile)
+constexpr int kThreads = 96 + NQ * 128;  // K producer, MMA, NQ softmax warpgroups, V producer
+constexpr int kWarpV = 2 + 4 * NQ;       // the V producer warp
 constexpr int kMaxSplits = 32;
 constexpr uint32_t kTmemCols = 512;
 
@@ -46,8 +48,8 @@ struct Layout {
   static constexpr int kQTile = BM * D * 2;
   static constexpr int kQ = 0;
   static constexpr int kK = kQ + NQ * kQTile;
-  static constexpr int kV = kK + NST * kTile;
-  static constexpr int kBar = kV + NST * kTile;
+  static constexpr int kV = kK + NSK * kTile;
+  static constexpr int kBar = kV + NSV * kTile;
   static constexpr int kBytes = kBar + 256;
   static constexpr int kAlloc = kBytes + 1024;  // slack for 1024-byte alignment
 };
@@ -56,10 +58,11 @@ struct Layout {
 enum {
   B_Q = 0,
   B_KFULL = 1,
-  B_VFULL = B_KFULL + NST,
-  B_KVEMPTY = B_VFULL + NST,
-  B_SFULL = B_KVEMPTY + NST,  // one per query tile
-  B_PFULL = B_SFULL + NQ,     // one per query tile (128 arrivals)
+  B_KEMPTY = B_KFULL + NSK,
+  B_VFULL = B_KEMPTY + NSK,
+  B_VEMPTY = B_VFULL + NSV,
+  B_SFULL = B_VEMPTY + NSV,  // one per query tile
+  B_PFULL = B_SFULL + NQ,     // one per query tile (one arrival per softmax warp)
   B_OFINAL = B_PFULL + NQ,
   B_COUNT = B_OFINAL + 1
 };
@@ -88,6 +91,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int PANELS = D / 64;
   constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
   constexpr uint32_t IDESC_PV = idesc_bf16(BM, D, false, true);
+  // K/V ring tiles are page-major: page p of a tile at p * kPageBytes.  At
+  // d = 128 a page lands as [8-row half][64-column panel][8 rows][128 B]
+  // (8-row groups 2048 B apart, panels 1024 B apart); at d = 64 as
+  // [16 rows][128 B] (groups 1024 B apart, one panel).
+  constexpr uint32_t kPageBytes = 16 * D * 2;
+  constexpr uint32_t kGroupStride = PANELS == 2 ? 2048 : 1024;
+  constexpr uint32_t kPanelOff = PANELS == 2 ? 1024 : BN * 128;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -99,8 +109,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::kBar + 8 * B_COUNT + 8);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int pair = blockIdx.x / p.num_splits, split = blockIdx.x % p.num_splits;
-  const int hk = blockIdx.y, b = blockIdx.z;
+  // Grid (split + splits * kv head, request, pair) with pairs in reverse
+  // order: CTAs start in linear block order, so the pairs of the last query
+  // rows, which see the most keys, go first and the short prefix-row pairs
+  // fill the tail of the launch.
+  const int split = blockIdx.x % p.num_splits, hk = blockIdx.x / p.num_splits;
+  const int b = blockIdx.y, pair = (int)gridDim.z - 1 - (int)blockIdx.z;
   const int detail = b;
 
   // ---- work of this CTA (uniform across threads)
@@ -145,7 +159,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < B_COUNT; ++i)
-      mbar_init(bar(i), (i >= B_PFULL && i < B_PFULL + NQ) ? 128 : 1);
+      mbar_init(bar(i), (i >= B_PFULL && i < B_PFULL + NQ) ? 4 : 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -158,12 +172,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tbase = *tmem_slot;
 
-  if (warp == 0) {
-    // ===================================================== TMA producer
-    // All 32 lanes issue: lane l < 16 loads K box (page l / PANELS, panel
-    // l % PANELS), lane 16 + l the matching V box, so a tile's 2 * 8 * PANELS
-    // boxes go out in one instruction.  Lanes 0..7 fetch the block-table
-    // entries of the next tile one iteration ahead.
+  if (warp == 0 || warp == kWarpV) {
+    // ===================================================== TMA producers
+    // Warp 0 streams K tiles into a 3-deep ring, warp kWarpV V tiles into a
+    // 2-deep ring.  Lane l < 8 moves page l of the tile as one box (a whole
+    // page-head: 4 KB at d = 128, 2 KB at d = 64) and looks up the next
+    // tile's block-table entry one iteration ahead.
+    const bool is_k = warp == 0;
+    const int nst = is_k ? NSK : NSV;
+    const int b_full = is_k ? B_KFULL : B_VFULL, b_empty = is_k ? B_KEMPTY : B_VEMPTY;
+    const uint32_t ring = sbase + (is_k ? L::kK : L::kV);
+    const CUtensorMap *tmap = is_k ? &tm_k : &tm_v;
     const int32_t *bt = p.block_table + (size_t)b * p.max_pages;
     auto page_row = [&](int kt) -> int {  // lanes 0..7: TMA row of page `lane` of tile kt
       int y = p.oob_row;
@@ -172,15 +191,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int page = bt[pidx];
         if (page >= 0 && page < p.num_pages)
           y = (int)(p.layer_row0 + ((long long)page * p.Hkv + hk) * 16);
-        else
+        else if (is_k)
           dev_fail(p.status, PIC_DEV_BAD_PAGE, detail);
       }
       return y;
     };
-    if (lane == 0) {
+    if (is_k && lane == 0) {
       prefetch_tmap(&tm_q);
       prefetch_tmap(&tm_k);
-      prefetch_tmap(&tm_v);
       mbar_expect_tx(bar(B_Q), ntile * L::kQTile);
 #pragma unroll
       for (int t = 0; t < NQ; ++t) {
@@ -191,38 +209,32 @@ __global__ void __launch_bounds__(kThreads, 1)
           tma_load_2d(sbase + L::kQ + t * L::kQTile + pn * BM * 128, &tm_q, pn * 64, qrow, bar(B_Q));
       }
     }
-    const int box = lane & 15;  // box index within K (or V)
-    const int bpage = box / PANELS, bpanel = box % PANELS;
-    const bool issues = box < 8 * PANELS;
+    if (!is_k && lane == 0) prefetch_tmap(&tm_v);
     int y_next = page_row(kv_begin);
     int issued = 0;
     for (int j = 0; j < n; ++j) {
-      const int st = j % NST;
+      const int st = j % nst;
       const int y_mine = y_next;
       if (j + 1 < n) y_next = page_row(kv_begin + j + 1);
-      if (j >= NST) {
-        const bool ok = mbar_wait(bar(B_KVEMPTY + st), ((j / NST) - 1) & 1, abort_flag, p.status, detail);
+      if (j >= nst) {
+        const bool ok = mbar_wait(bar(b_empty + st), ((j / nst) - 1) & 1, abort_flag, p.status, detail);
         if (!__all_sync(0xffffffffu, ok)) break;
       }
-      const int y = __shfl_sync(0xffffffffu, y_mine, bpage);
-      if (lane == 0) mbar_expect_tx(bar(B_KFULL + st), L::kTile);
-      if (lane == 16) mbar_expect_tx(bar(B_VFULL + st), L::kTile);
+      if (lane == 0) mbar_expect_tx(bar(b_full + st), L::kTile);
       __syncwarp();
-      if (issues) {
-        const uint32_t off = st * L::kTile + bpanel * BN * 128 + bpage * 16 * 128;
-        if (lane < 16)
-          tma_load_2d(sbase + L::kK + off, &tm_k, bpanel * 64, y, bar(B_KFULL + st));
+      if (lane < 8) {  // one box per page-head
+        const uint32_t dst = ring + st * L::kTile + lane * kPageBytes;
+        if constexpr (PANELS == 2)
+          tma_load_4d(dst, tmap, 0, 0, 0, y_mine >> 3, bar(b_full + st));
         else
-          tma_load_2d(sbase + L::kV + off, &tm_v, bpanel * 64, y, bar(B_VFULL + st));
+          tma_load_2d(dst, tmap, 0, y_mine, bar(b_full + st));
       }
       issued = j + 1;
     }
     if (lane == 0 && *abort_flag) {
       // Let the copies already issued land before the CTA exits.
-      for (int j = max(0, issued - NST); j < issued; ++j) {
-        mbar_wait(bar(B_KFULL + j % NST), (j / NST) & 1, abort_flag, p.status, detail);
-        mbar_wait(bar(B_VFULL + j % NST), (j / NST) & 1, abort_flag, p.status, detail);
-      }
+      for (int j = max(0, issued - nst); j < issued; ++j)
+        mbar_wait(bar(b_full + j % nst), (j / nst) & 1, abort_flag, p.status, detail);
     }
   } else if (warp == 1) {
     // ===================================================== MMA issuer
@@ -237,25 +249,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t tS = tbase + t * 128, tO = tbase + 256 + t * 128;
           // O_t += P_t(j-1) V(j-1)
           if (j >= 1 && j - 1 < nt[t]) {
-            const int pj = j - 1, pst = pj % NST;
+            const int pj = j - 1, pst = pj % NSV;
             if (!mbar_wait(bar(B_PFULL + t), pj & 1, abort_flag, p.status, detail) ||
-                !mbar_wait(bar(B_VFULL + pst), (pj / NST) & 1, abort_flag, p.status, detail)) {
+                !mbar_wait(bar(B_VFULL + pst), (pj / NSV) & 1, abort_flag, p.status, detail)) {
               ok = false;
               break;
             }
             tc_fence_after();
             const uint32_t vb = sbase + L::kV + pst * L::kTile;
 #pragma unroll
-            for (int kk = 0; kk < BN / 16; ++kk)
-              mma_ts(tO, tS + kk * 8, sdesc_sw128(vb + kk * 16 * 128, BN * 128, 1024), IDESC_PV,
-                     (pj > 0 || kk > 0));
-            if (t == ntile - 1) mma_commit(bar(B_KVEMPTY + pst));  // last reader of V(j-1)
+            for (int kk = 0; kk < BN / 16; ++kk)  // one page of 16 keys per MMA
+              mma_ts(tO, tS + kk * 8, sdesc_sw128(vb + kk * kPageBytes, kPanelOff, kGroupStride),
+                     IDESC_PV, (pj > 0 || kk > 0));
+            if (t == ntile - 1) mma_commit(bar(B_VEMPTY + pst));  // last reader of V(j-1)
           }
           // S_t = Q_t K(j)^T
           if (j < nt[t]) {
-            const int st = j % NST;
+            const int st = j % NSK;
             if (!k_ready) {
-              if (!mbar_wait(bar(B_KFULL + st), (j / NST) & 1, abort_flag, p.status, detail)) {
+              if (!mbar_wait(bar(B_KFULL + st), (j / NSK) & 1, abort_flag, p.status, detail)) {
                 ok = false;
                 break;
               }
@@ -263,15 +275,16 @@ __global__ void __launch_bounds__(kThreads, 1)
               k_ready = true;
             }
             const uint32_t kb = sbase + L::kK + st * L::kTile;
-            const uint32_t qb = sbase + L::kQ + t * L::kQTile;
+            const uint32_t qb = sbase + L::kQ + t * L::kQTile;  // (st is the K ring slot)
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
               const uint32_t off = (kk >> 2) * (BM * 128) + (kk & 3) * 32;
               mma_ss(tS, sdesc_sw128(qb + off, 16, 1024),
-                     sdesc_sw128(kb + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024), IDESC_QK,
-                     kk > 0);
+                     sdesc_sw128(kb + (kk >> 2) * kPanelOff + (kk & 3) * 32, 16, kGroupStride),
+                     IDESC_QK, kk > 0);
             }
             mma_commit(bar(B_SFULL + t));
+            if (t == ntile - 1) mma_commit(bar(B_KEMPTY + st));  // last reader of K(j)
           }
         }
       }
@@ -312,19 +325,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int c = 0; c < BN; ++c)
           if (key0 + c > pos) s[c] = -INFINITY;
       }
-      // row max: 8 independent chains, then a 3-level tree
-      float mx8[8];
+      // row max: 4 independent chains of 3-input max
+      float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-      for (int i = 0; i < 8; ++i) mx8[i] = s[i];
+      for (int c = 0; c < BN; c += 8)
 #pragma unroll
-      for (int c = 8; c < BN; c += 8)
-#pragma unroll
-        for (int i = 0; i < 8; ++i) mx8[i] = fmaxf(mx8[i], s[c + i]);
-#pragma unroll
-      for (int w = 4; w; w >>= 1)
-#pragma unroll
-        for (int i = 0; i < w; ++i) mx8[i] = fmaxf(mx8[i], mx8[i + w]);
-      const float m_new = fmaxf(m_used, mx8[0] * p.scale_log2);
+        for (int i = 0; i < 4; ++i) mx[i] = max3f(mx[i], s[c + 2 * i], s[c + 2 * i + 1]);
+      const float m_new = fmaxf(m_used, max3f(mx[0], mx[1], fmaxf(mx[2], mx[3])) * p.scale_log2);
       float alpha = 1.f;
       const bool resc = m_new > m_used + 8.f;
       if (resc) {
@@ -334,27 +341,28 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float mref = (m_used == -INFINITY) ? 0.f : m_used;
       // P = exp2(s * scale - m) as bf16, written over S in 16-column chunks as
       // soon as each 32-key chunk is done (S was read completely above, so the
-      // overlap is harmless and the packed values never pile up in registers)
-      float ls8[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) ls8[i] = 0.f;
+      // overlap is harmless and the packed values never pile up in registers).
+      // Scaling and the row sum run on packed fp32 pairs (half the issue
+      // slots; the softmax is bound by instruction issue, not by MUFU).
+      const uint64_t sc2 = f2pack(p.scale_log2, p.scale_log2), nm2 = f2pack(-mref, -mref);
+      uint64_t acc[4] = {0, 0, 0, 0};
 #pragma unroll
       for (int c0 = 0; c0 < BN; c0 += 32) {
         uint32_t pk[16];
 #pragma unroll
-        for (int c = 0; c < 32; c += 2) {
-          const float p0 = ex2(fmaf(s[c0 + c], p.scale_log2, -mref));
-          const float p1 = ex2(fmaf(s[c0 + c + 1], p.scale_log2, -mref));
-          ls8[(c >> 1) & 7] += p0 + p1;
-          pk[c / 2] = pack2(p0, p1);
+        for (int q = 0; q < 16; ++q) {
+          const uint64_t e = exp2_mufu2(fma2(f2pack(s[c0 + 2 * q], s[c0 + 2 * q + 1]), sc2, nm2));
+          acc[q & 3] = add2(acc[q & 3], e);
+          float e0, e1;
+          f2unpack(e, e0, e1);
+          pk[q] = pack2(e0, e1);
         }
         tmem_st16(tS + c0 / 2, pk);
       }
-#pragma unroll
-      for (int w = 4; w; w >>= 1)
-#pragma unroll
-        for (int i = 0; i < w; ++i) ls8[i] += ls8[i + w];
-      l = fmaf(l, alpha, ls8[0]);
+      acc[0] = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
+      float l0, l1;
+      f2unpack(acc[0], l0, l1);
+      l = fmaf(l, alpha, l0 + l1);
       // O correction: PV_t(j-1) has completed (it precedes QK_t(j) in the MMA order)
       if (j > 0 && __any_sync(0xffffffffu, resc)) {
 #pragma unroll
@@ -369,44 +377,71 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(bar(B_PFULL + t));
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(B_PFULL + t));  // one arrival per warp
     }
     // ---- epilogue
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_OFINAL), 0, abort_flag, p.status, detail));
     tc_fence_after();
-    if (ok && t < ntile) {
-      if (my_n == 0) {  // this tile needs none of the split's keys
-        if (p.num_splits > 1) {
-          p.part_ml[(my_part0 + row) * 2] = -INFINITY;
-          p.part_ml[(my_part0 + row) * 2 + 1] = 0.f;
-        }
-      } else {
+    if (t < ntile && my_n == 0) {  // this tile needs none of the split's keys
+      if (ok && p.num_splits > 1) {
+        p.part_ml[(my_part0 + row) * 2] = -INFINITY;
+        p.part_ml[(my_part0 + row) * 2 + 1] = 0.f;
+      }
+    } else if (t < ntile) {
+      // Every MMA and TMA copy is finished, so the whole shared memory is free:
+      // each thread stages its finished row (padded rows keep the bank
+      // accesses at 4 wavefronts per 512 B), the warpgroup syncs on its own
+      // named barrier, and warps copy whole rows out with coalesced stores.
+      const bool single = p.num_splits == 1;
+      constexpr int kRowOut = D * 2 + 16, kRowPart = D * 4 + 16;
+      uint8_t *stage = smem + (size_t)t * BM * (single ? kRowOut : kRowPart);
+      if (ok) {
         float o[D];
 #pragma unroll
         for (int c = 0; c < D / 32; ++c) tmem_ld32(tO + c * 32, reinterpret_cast<uint32_t *>(o + c * 32));
         tmem_wait_ld();
-        if (p.num_splits == 1) {
+        if (single) {
           const float inv = l > 0.f ? 1.f / l : 0.f;
-          __nv_bfloat16 *dst = p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D;
-          if (valid) {
+          uint4 *dst = reinterpret_cast<uint4 *>(stage + row * kRowOut);
 #pragma unroll
-            for (int q = 0; q < D; ++q) o[q] *= inv;
+          for (int q = 0; q < D; ++q) o[q] *= inv;
 #pragma unroll
-            for (int q = 0; q < D / 8; ++q) st_global16(dst + q * 8, pack8(o + q * 8));
-          }
+          for (int q = 0; q < D / 8; ++q) dst[q] = pack8(o + q * 8);
           if (valid && p.lse)
             p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
                 l > 0.f ? (m_used + __log2f(l)) * 0.69314718055994531f : -INFINITY;
         } else {
-          float *dst = p.part_o + (my_part0 + row) * D;
-          if (valid) {
+          float4 *dst = reinterpret_cast<float4 *>(stage + row * kRowPart);
 #pragma unroll
-            for (int q = 0; q < D / 4; ++q)
-              reinterpret_cast<float4 *>(dst)[q] =
-                  make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
-          }
+          for (int q = 0; q < D / 4; ++q)
+            dst[q] = make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
           p.part_ml[(my_part0 + row) * 2] = (l > 0.f) ? m_used : -INFINITY;
           p.part_ml[(my_part0 + row) * 2 + 1] = l;
+        }
+      }
+      asm volatile("bar.sync %0, 128;" ::"r"(1 + t) : "memory");
+      if (ok) {
+        const int nrows = min(BM, rows - my_r0);  // valid rows of this tile
+        if (single) {
+          // 16 lanes per 256-byte row (D = 128) or 8 per 128-byte row (D = 64)
+          constexpr int LPR = D / 8, RPI = 32 / LPR;
+          for (int r = wq * RPI + lane / LPR; r < nrows; r += 4 * RPI) {
+            const int rg2 = my_r0 + r, tk = rg2 / p.G, gg = rg2 % p.G;
+            const uint4 v = *reinterpret_cast<const uint4 *>(stage + r * kRowOut + (lane % LPR) * 16);
+            st_global16(p.out + (((size_t)b * p.max_inline + tk) * p.Hq + hk * p.G + gg) * D +
+                            (lane % LPR) * 8, v);
+          }
+        } else {
+          // fp32 rows are contiguous in the partial buffer: one row per warp pass
+          constexpr int LPR = D / 4;  // 16-byte pieces per row
+          constexpr int RPI = 32 / LPR > 0 ? 32 / LPR : 1;
+          for (int r = wq * RPI + lane / LPR; r < nrows; r += 4 * RPI)
+#pragma unroll
+            for (int c = lane % LPR; c < D / 4; c += (LPR < 32 ? LPR : 32)) {
+              const float4 v = *reinterpret_cast<const float4 *>(stage + r * kRowPart + c * 16);
+              reinterpret_cast<float4 *>(p.part_o + (my_part0 + r) * D)[c] = v;
+            }
         }
       }
     }
@@ -1329,8 +1364,13 @@ extern "C" pic_status_t pic_attend_prefill(
 
   CUtensorMap tq, tk, tv;
   st = encode_tmap_2d(&tq, ws, D, (uint64_t)batch * Hkv * pl.R_pad, (uint64_t)D * 2, 64, BM);
-  if (st == PIC_OK) st = encode_tmap_2d(&tk, k_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
-  if (st == PIC_OK) st = encode_tmap_2d(&tv, v_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
+  if (D == 128) {
+    if (st == PIC_OK) st = encode_tmap_pages128(&tk, k_cache, (uint64_t)rows_total / 16);
+    if (st == PIC_OK) st = encode_tmap_pages128(&tv, v_cache, (uint64_t)rows_total / 16);
+  } else {
+    if (st == PIC_OK) st = encode_tmap_2d(&tk, k_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
+    if (st == PIC_OK) st = encode_tmap_2d(&tv, v_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
+  }
   if (st != PIC_OK) return st;
   Params pp;
   pp.batch = batch;
@@ -1355,7 +1395,7 @@ extern "C" pic_status_t pic_attend_prefill(
   pp.status = status;
   pp.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
 
-  dim3 grid(((pl.m_tiles + NQ - 1) / NQ) * pl.splits, Hkv, batch);
+  dim3 grid(pl.splits * Hkv, batch, (pl.m_tiles + NQ - 1) / NQ);
   cudaError_t e;
   if (D == 128) {
     const int smem = Layout<128>::kAlloc;
