@@ -1018,12 +1018,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace fused
 
 // Merge the split partials (O unnormalised, m in log2 units, l) of every
-// query row by log-sum-exp: one warp per row, lanes over the d columns.  All
-// loads are issued unconditionally (an empty split's weight is zero and its
-// data is discarded by a select), so a row costs two dependent L2 round trips.
+// query row by log-sum-exp: one warp per row, lanes over the d columns.  The
+// (m, l) pairs and the O rows of up to 8 splits are loaded before any of them
+// is used, so a row costs one L2 round trip for up to 8 splits (an empty
+// split's weight is zero and its data, never written, is discarded by a
+// select).  Launched as a programmatic dependent of the attention kernel: the
+// CTAs may be placed while attention drains and wait for it here.
 template <int D>
 __global__ void __launch_bounds__(256) combine_kernel(Params p) {
-  constexpr int CPL = D / 32;
+  constexpr int CPL = D / 32, U = 8;
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const long long grow = (long long)blockIdx.x * (blockDim.x >> 5) + warp;
   const long long per_b = (long long)p.Hkv * p.m_tiles * BM;
@@ -1042,24 +1046,41 @@ __global__ void __launch_bounds__(256) combine_kernel(Params p) {
     ms = p.part_ml[((base + lane) * BM + row) * 2];
     ls = p.part_ml[((base + lane) * BM + row) * 2 + 1];
   }
-  float M = ms;
-#pragma unroll
-  for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-  const float w = (ms == -INFINITY) ? 0.f : ex2(ms - M);
-  float Lsum = w * ls;
-#pragma unroll
-  for (int o = 16; o; o >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, o);
   float acc[CPL];
 #pragma unroll
   for (int q = 0; q < CPL; ++q) acc[q] = 0.f;
-  for (int sp = 0; sp < S; ++sp) {
-    const float ws = __shfl_sync(0xffffffffu, w, sp);
-    const float *src = p.part_o + ((base + sp) * BM + row) * D + lane * CPL;
-    float v[CPL];
+  float M = -INFINITY, w = 0.f, Lsum = 0.f;
+  for (int s0 = 0; s0 < S; s0 += U) {
+    float v[U][CPL];
 #pragma unroll
-    for (int q = 0; q < CPL; ++q) v[q] = src[q];
+    for (int u = 0; u < U; ++u) {
+      const int sp = min(s0 + u, S - 1);  // past the end: a harmless reload, weight 0 below
+      const float *src = p.part_o + ((base + sp) * BM + row) * D + lane * CPL;
+      if constexpr (CPL == 4) {
+        const float4 x = *reinterpret_cast<const float4 *>(src);
+        v[u][0] = x.x, v[u][1] = x.y, v[u][2] = x.z, v[u][3] = x.w;
+      } else {
+        static_assert(CPL == 2, "d = 64 or 128");
+        const float2 x = *reinterpret_cast<const float2 *>(src);
+        v[u][0] = x.x, v[u][1] = x.y;
+      }
+    }
+    if (s0 == 0) {
+      M = ms;
 #pragma unroll
-    for (int q = 0; q < CPL; ++q) acc[q] = fmaf(ws, ws == 0.f ? 0.f : v[q], acc[q]);
+      for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+      w = (ms == -INFINITY) ? 0.f : ex2(ms - M);
+      Lsum = w * ls;
+#pragma unroll
+      for (int o = 16; o; o >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, o);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const float ws = __shfl_sync(0xffffffffu, w, (s0 + u) & 31);
+      const bool use = s0 + u < S && ws != 0.f;
+#pragma unroll
+      for (int q = 0; q < CPL; ++q) acc[q] = fmaf(use ? ws : 0.f, use ? v[u][q] : 0.f, acc[q]);
+    }
   }
   const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
   const int tok = rg / p.G, g = rg % p.G;
@@ -1230,6 +1251,27 @@ inline Plan plan(const pic_geom_t *g, int batch, int max_inline, int max_ctx, in
   return pl;
 }
 
+}  // namespace prefill
+}  // namespace pic
+
+namespace pic {
+namespace prefill {
+// The merge kernel as a programmatic dependent launch of the attention
+// kernel before it on the stream (it waits with griddepcontrol.wait).
+template <int D>
+static cudaError_t launch_combine(unsigned grid, const Params &pp, cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(256);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, combine_kernel<D>, pp);
+}
 }  // namespace prefill
 }  // namespace pic
 
@@ -1411,8 +1453,8 @@ extern "C" pic_status_t pic_attend_prefill(
   if (pl.splits > 1) {
     const long long rows = (long long)batch * Hkv * pl.m_tiles * BM;
     const unsigned cgrid = (unsigned)((rows + 7) / 8);
-    if (D == 128) combine_kernel<128><<<cgrid, 256, 0, stream>>>(pp);
-    else combine_kernel<64><<<cgrid, 256, 0, stream>>>(pp);
+    e = D == 128 ? launch_combine<128>(cgrid, pp, stream) : launch_combine<64>(cgrid, pp, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "merge launch");
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill launch");
@@ -1520,8 +1562,8 @@ extern "C" pic_status_t pic_attend_prefill_fused(
   if (pl.splits > 1) {
     const long long crows = (long long)batch * Hkv * pl.m_tiles * BM;
     const unsigned cgrid = (unsigned)((crows + 7) / 8);
-    if (D == 128) combine_kernel<128><<<cgrid, 256, 0, stream>>>(pp);
-    else combine_kernel<64><<<cgrid, 256, 0, stream>>>(pp);
+    e = D == 128 ? launch_combine<128>(cgrid, pp, stream) : launch_combine<64>(cgrid, pp, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "merge launch");
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused launch");
