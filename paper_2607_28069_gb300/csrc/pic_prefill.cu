@@ -109,12 +109,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::kBar + 8 * B_COUNT + 8);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // Grid (split + splits * kv head, request, pair) with pairs in reverse
-  // order: CTAs start in linear block order, so the pairs of the last query
-  // rows, which see the most keys, go first and the short prefix-row pairs
-  // fill the tail of the launch.
-  const int split = blockIdx.x % p.num_splits, hk = blockIdx.x / p.num_splits;
-  const int b = blockIdx.y, pair = (int)gridDim.z - 1 - (int)blockIdx.z;
+  // Grid (split + splits * pair, kv head, request), pairs in reverse order.
+  // CTAs start in linear block order, so all CTAs of one (request, kv head)
+  // start together and its K/V, read by every pair, is reused from L2; within
+  // the group the pairs of the last query rows, which see the most keys, go
+  // first and the short prefix-row pairs fill in behind them.
+  const int npairs = (int)gridDim.x / p.num_splits;
+  const int split = blockIdx.x % p.num_splits;
+  const int pair = npairs - 1 - (int)blockIdx.x / p.num_splits;
+  const int hk = blockIdx.y, b = blockIdx.z;
   const int detail = b;
 
   // ---- work of this CTA (uniform across threads)
@@ -1018,80 +1021,103 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace fused
 
 // Merge the split partials (O unnormalised, m in log2 units, l) of every
-// query row by log-sum-exp: one warp per row, lanes over the d columns.  The
-// (m, l) pairs and the O rows of up to 8 splits are loaded before any of them
-// is used, so a row costs one L2 round trip for up to 8 splits (an empty
-// split's weight is zero and its data, never written, is discarded by a
-// select).  Launched as a programmatic dependent of the attention kernel: the
-// CTAs may be placed while attention drains and wait for it here.
-template <int D>
+// query row by log-sum-exp, lanes over the d columns.  A warp takes R rows
+// of one query tile and issues the (m, l) pairs and the O rows of U splits
+// for all R rows before using any of them (R * U = 8 loads of 16 bytes in
+// flight per lane), so a row costs one L2/DRAM round trip for up to U splits;
+// U is the smallest of 2, 4, 8 that covers the splits (more are merged in
+// further rounds).  An empty split's weight is zero and its data, never
+// written, is discarded by a select.  Launched as a programmatic dependent of
+// the attention kernel: the CTAs may be placed while attention drains and
+// wait for it here.
+template <int D, int U, int R>
 __global__ void __launch_bounds__(256) combine_kernel(Params p) {
-  constexpr int CPL = D / 32, U = 8;
+  constexpr int CPL = D / 32;
+  static_assert(BM % R == 0, "a warp's rows stay inside one query tile");
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long long grow = (long long)blockIdx.x * (blockDim.x >> 5) + warp;
+  const long long g0 = ((long long)blockIdx.x * (blockDim.x >> 5) + warp) * R;
   const long long per_b = (long long)p.Hkv * p.m_tiles * BM;
-  const int b = (int)(grow / per_b);
+  const int b = (int)(g0 / per_b);
   if (b >= p.batch) return;
-  const long long rem = grow % per_b;
+  const long long rem = g0 % per_b;
   const int hk = (int)(rem / ((long long)p.m_tiles * BM));
-  const int mt = (int)((rem / BM) % p.m_tiles), row = (int)(rem % BM);
+  const int mt = (int)((rem / BM) % p.m_tiles), row0 = (int)(rem % BM);
   const int tin = min(max(p.inline_len[b], 0), p.max_inline);
-  const int rg = mt * BM + row;
-  if (rg >= tin * p.G) return;
+  const int valid_rows = tin * p.G - (mt * BM + row0);  // rows of this warp that exist
+  if (valid_rows <= 0) return;
   const int S = p.num_splits;
   const size_t base = (((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * S;
-  float ms = -INFINITY, ls = 0.f;
-  if (lane < S) {
-    ms = p.part_ml[((base + lane) * BM + row) * 2];
-    ls = p.part_ml[((base + lane) * BM + row) * 2 + 1];
+  float ms[R], ls[R];
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    ms[r] = -INFINITY, ls[r] = 0.f;
+    if (lane < S) {
+      const float2 ml =
+          *reinterpret_cast<const float2 *>(p.part_ml + ((base + lane) * BM + row0 + r) * 2);
+      ms[r] = ml.x, ls[r] = ml.y;
+    }
   }
-  float acc[CPL];
+  float acc[R][CPL], M[R], w[R], Lsum[R];
 #pragma unroll
-  for (int q = 0; q < CPL; ++q) acc[q] = 0.f;
-  float M = -INFINITY, w = 0.f, Lsum = 0.f;
+  for (int r = 0; r < R; ++r)
+#pragma unroll
+    for (int q = 0; q < CPL; ++q) acc[r][q] = 0.f;
   for (int s0 = 0; s0 < S; s0 += U) {
-    float v[U][CPL];
+    float v[R][U][CPL];
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int sp = min(s0 + u, S - 1);  // past the end: a harmless reload, weight 0 below
-      const float *src = p.part_o + ((base + sp) * BM + row) * D + lane * CPL;
-      if constexpr (CPL == 4) {
-        const float4 x = *reinterpret_cast<const float4 *>(src);
-        v[u][0] = x.x, v[u][1] = x.y, v[u][2] = x.z, v[u][3] = x.w;
-      } else {
-        static_assert(CPL == 2, "d = 64 or 128");
-        const float2 x = *reinterpret_cast<const float2 *>(src);
-        v[u][0] = x.x, v[u][1] = x.y;
+    for (int r = 0; r < R; ++r)
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int sp = min(s0 + u, S - 1);  // past the end: a harmless reload, weight 0 below
+        const float *src = p.part_o + ((base + sp) * BM + row0 + r) * D + lane * CPL;
+        if constexpr (CPL == 4) {
+          const float4 x = *reinterpret_cast<const float4 *>(src);
+          v[r][u][0] = x.x, v[r][u][1] = x.y, v[r][u][2] = x.z, v[r][u][3] = x.w;
+        } else {
+          static_assert(CPL == 2, "d = 64 or 128");
+          const float2 x = *reinterpret_cast<const float2 *>(src);
+          v[r][u][0] = x.x, v[r][u][1] = x.y;
+        }
+      }
+    if (s0 == 0) {
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        M[r] = ms[r];
+#pragma unroll
+        for (int o = 16; o; o >>= 1) M[r] = fmaxf(M[r], __shfl_xor_sync(0xffffffffu, M[r], o));
+        w[r] = (ms[r] == -INFINITY) ? 0.f : ex2(ms[r] - M[r]);
+        Lsum[r] = w[r] * ls[r];
+#pragma unroll
+        for (int o = 16; o; o >>= 1) Lsum[r] += __shfl_xor_sync(0xffffffffu, Lsum[r], o);
       }
     }
-    if (s0 == 0) {
-      M = ms;
 #pragma unroll
-      for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-      w = (ms == -INFINITY) ? 0.f : ex2(ms - M);
-      Lsum = w * ls;
+    for (int r = 0; r < R; ++r)
 #pragma unroll
-      for (int o = 16; o; o >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, o);
-    }
+      for (int u = 0; u < U; ++u) {
+        const float ws = __shfl_sync(0xffffffffu, w[r], (s0 + u) & 31);
+        const bool use = s0 + u < S && ws != 0.f;
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const float ws = __shfl_sync(0xffffffffu, w, (s0 + u) & 31);
-      const bool use = s0 + u < S && ws != 0.f;
-#pragma unroll
-      for (int q = 0; q < CPL; ++q) acc[q] = fmaf(use ? ws : 0.f, use ? v[u][q] : 0.f, acc[q]);
-    }
+        for (int q = 0; q < CPL; ++q)
+          acc[r][q] = fmaf(use ? ws : 0.f, use ? v[r][u][q] : 0.f, acc[r][q]);
+      }
   }
-  const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
-  const int tok = rg / p.G, g = rg % p.G;
-  __nv_bfloat16 *dst =
-      p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D + lane * CPL;
 #pragma unroll
-  for (int q = 0; q < CPL; q += 2)
-    *reinterpret_cast<uint32_t *>(dst + q) = pack2(acc[q] * inv, acc[q + 1] * inv);
-  if (p.lse && lane == 0)
-    p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
-        Lsum > 0.f ? (M + __log2f(Lsum)) * 0.69314718055994531f : -INFINITY;
+  for (int r = 0; r < R; ++r) {
+    if (r >= valid_rows) break;
+    const int rg = mt * BM + row0 + r;
+    const float inv = Lsum[r] > 0.f ? 1.f / Lsum[r] : 0.f;
+    const int tok = rg / p.G, g = rg % p.G;
+    __nv_bfloat16 *dst =
+        p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D + lane * CPL;
+#pragma unroll
+    for (int q = 0; q < CPL; q += 2)
+      *reinterpret_cast<uint32_t *>(dst + q) = pack2(acc[r][q] * inv, acc[r][q + 1] * inv);
+    if (p.lse && lane == 0)
+      p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
+          Lsum[r] > 0.f ? (M[r] + __log2f(Lsum[r])) * 0.69314718055994531f : -INFINITY;
+  }
 }
 
 // RoPE the inline keys/queries at their logical positions; keys and values go
@@ -1259,9 +1285,11 @@ namespace prefill {
 // The merge kernel as a programmatic dependent launch of the attention
 // kernel before it on the stream (it waits with griddepcontrol.wait).
 template <int D>
-static cudaError_t launch_combine(unsigned grid, const Params &pp, cudaStream_t stream) {
+static cudaError_t launch_combine(long long rows, const Params &pp, cudaStream_t stream) {
+  const int S = pp.num_splits;
+  const int U = S <= 2 ? 2 : (S <= 4 ? 4 : 8), R = 8 / U;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
+  cfg.gridDim = dim3((unsigned)((rows + 8 * R - 1) / (8 * R)));
   cfg.blockDim = dim3(256);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
@@ -1270,7 +1298,9 @@ static cudaError_t launch_combine(unsigned grid, const Params &pp, cudaStream_t 
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, combine_kernel<D>, pp);
+  if (U == 2) return cudaLaunchKernelEx(&cfg, combine_kernel<D, 2, 4>, pp);
+  if (U == 4) return cudaLaunchKernelEx(&cfg, combine_kernel<D, 4, 2>, pp);
+  return cudaLaunchKernelEx(&cfg, combine_kernel<D, 8, 1>, pp);
 }
 }  // namespace prefill
 }  // namespace pic
@@ -1437,7 +1467,7 @@ extern "C" pic_status_t pic_attend_prefill(
   pp.status = status;
   pp.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
 
-  dim3 grid(pl.splits * Hkv, batch, (pl.m_tiles + NQ - 1) / NQ);
+  dim3 grid(((pl.m_tiles + NQ - 1) / NQ) * pl.splits, Hkv, batch);
   cudaError_t e;
   if (D == 128) {
     const int smem = Layout<128>::kAlloc;
@@ -1452,8 +1482,7 @@ extern "C" pic_status_t pic_attend_prefill(
   }
   if (pl.splits > 1) {
     const long long rows = (long long)batch * Hkv * pl.m_tiles * BM;
-    const unsigned cgrid = (unsigned)((rows + 7) / 8);
-    e = D == 128 ? launch_combine<128>(cgrid, pp, stream) : launch_combine<64>(cgrid, pp, stream);
+    e = D == 128 ? launch_combine<128>(rows, pp, stream) : launch_combine<64>(rows, pp, stream);
     if (e != cudaSuccess) return cuda_fail(e, "merge launch");
   }
   e = cudaGetLastError();
@@ -1561,8 +1590,7 @@ extern "C" pic_status_t pic_attend_prefill_fused(
   }
   if (pl.splits > 1) {
     const long long crows = (long long)batch * Hkv * pl.m_tiles * BM;
-    const unsigned cgrid = (unsigned)((crows + 7) / 8);
-    e = D == 128 ? launch_combine<128>(cgrid, pp, stream) : launch_combine<64>(cgrid, pp, stream);
+    e = D == 128 ? launch_combine<128>(crows, pp, stream) : launch_combine<64>(crows, pp, stream);
     if (e != cudaSuccess) return cuda_fail(e, "merge launch");
   }
   e = cudaGetLastError();
