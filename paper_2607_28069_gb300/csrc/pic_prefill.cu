@@ -37,8 +37,13 @@ constexpr int NQ = 2;    // query tiles per CTA, sharing every K/V tile
 constexpr int BN = 128;  // keys per KV tile
 constexpr int NSK = 3;   // K ring stages (released after the last QK of a tile)
 constexpr int NSV = 2;   // V ring stages (released after the last PV of a tile)
-constexpr int kThreads = 96 + NQ * 128;  // K producer, MMA, NQ softmax warpgroups, V producer
-constexpr int kWarpV = 2 + 4 * NQ;       // the V producer warp
+constexpr int kThreads = 128 + NQ * 128;  // K producer, MMA, NQ softmax warpgroups, V producer, relay
+constexpr int kWarpV = 2 + 4 * NQ;        // the V producer warp
+constexpr int kWarpRelay = kWarpV + 1;    // waits on behalf of the MMA issuer
+// Named barriers between the relay warp and the MMA warp (64 threads each);
+// 0 is __syncthreads, 1 and 2 belong to the softmax warpgroups' epilogue.
+constexpr int kNbPv = 3;  // + t: P_t(j-1) and V(j-1) are ready
+constexpr int kNbK = 5;   // K(j) is ready
 constexpr int kMaxSplits = 32;
 constexpr uint32_t kTmemCols = 512;
 
@@ -83,6 +88,10 @@ struct Params {
 // tcgen05 MMAs of one thread complete in order, "S_t(j) is ready" implies
 // PV_t(j-1) has finished, so softmax t may rescale O_t right away, and
 // softmax 0 runs while the tensor core works on tile 1 and vice versa.
+// The MMA issuer does no mbarrier wait inside its loop: an mbarrier wait of
+// a thread queues behind the MMAs that thread issued, so each one left the
+// tensor core idle for a while.  A relay warp waits for K(j), V(j-1) and
+// P_t(j-1) in the issuer's order and hands each over on a named barrier.
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
@@ -241,24 +250,25 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     // ===================================================== MMA issuer
-    if (lane == 0) {
-      bool ok = mbar_wait(bar(B_Q), 0, abort_flag, p.status, detail);
-      tc_fence_after();
-      for (int j = 0; ok && j <= n; ++j) {
-        bool k_ready = false;
+    // The whole warp takes part in the named barriers; lane 0 issues.  After
+    // an abort both this loop and the relay's run to the end (skipping their
+    // waits and MMAs), so every barrier sync has its arrival.
+    const bool leader = lane == 0;
+    if (leader) mbar_wait(bar(B_Q), 0, abort_flag, p.status, detail);
+    __syncwarp();
+    tc_fence_after();
+    for (int j = 0; j <= n; ++j) {
+      bool k_ready = false;
 #pragma unroll
-        for (int t = 0; t < NQ; ++t) {
-          if (t >= ntile) break;
-          const uint32_t tS = tbase + t * 128, tO = tbase + 256 + t * 128;
-          // O_t += P_t(j-1) V(j-1)
-          if (j >= 1 && j - 1 < nt[t]) {
-            const int pj = j - 1, pst = pj % NSV;
-            if (!mbar_wait(bar(B_PFULL + t), pj & 1, abort_flag, p.status, detail) ||
-                !mbar_wait(bar(B_VFULL + pst), (pj / NSV) & 1, abort_flag, p.status, detail)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
+      for (int t = 0; t < NQ; ++t) {
+        if (t >= ntile) break;
+        const uint32_t tS = tbase + t * 128, tO = tbase + 256 + t * 128;
+        // O_t += P_t(j-1) V(j-1)
+        if (j >= 1 && j - 1 < nt[t]) {
+          const int pj = j - 1, pst = pj % NSV;
+          named_bar_sync(kNbPv + t, 64);
+          tc_fence_after();
+          if (leader && !*abort_flag) {
             const uint32_t vb = sbase + L::kV + pst * L::kTile;
 #pragma unroll
             for (int kk = 0; kk < BN / 16; ++kk)  // one page of 16 keys per MMA
@@ -266,19 +276,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                      IDESC_PV, (pj > 0 || kk > 0));
             if (t == ntile - 1) mma_commit(bar(B_VEMPTY + pst));  // last reader of V(j-1)
           }
-          // S_t = Q_t K(j)^T
-          if (j < nt[t]) {
-            const int st = j % NSK;
-            if (!k_ready) {
-              if (!mbar_wait(bar(B_KFULL + st), (j / NSK) & 1, abort_flag, p.status, detail)) {
-                ok = false;
-                break;
-              }
-              tc_fence_after();
-              k_ready = true;
-            }
+        }
+        // S_t = Q_t K(j)^T
+        if (j < nt[t]) {
+          const int st = j % NSK;
+          if (!k_ready) {
+            named_bar_sync(kNbK, 64);
+            tc_fence_after();
+            k_ready = true;
+          }
+          if (leader && !*abort_flag) {
             const uint32_t kb = sbase + L::kK + st * L::kTile;
-            const uint32_t qb = sbase + L::kQ + t * L::kQTile;  // (st is the K ring slot)
+            const uint32_t qb = sbase + L::kQ + t * L::kQTile;
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
               const uint32_t off = (kk >> 2) * (BM * 128) + (kk & 3) * 32;
@@ -291,7 +300,34 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      mma_commit(bar(B_OFINAL));
+    }
+    if (leader) mma_commit(bar(B_OFINAL));
+  } else if (warp == kWarpRelay) {
+    // ===================================================== relay for the issuer
+    // Mirrors the issuer's loop: the same conditions, the same order.  Its
+    // arrival on a barrier in iteration j + 1 depends on an MMA the issuer
+    // issues only after its sync on that barrier in iteration j, so the two
+    // never get a phase apart.
+    for (int j = 0; j <= n; ++j) {
+      bool k_ready = false, v_ready = false;
+#pragma unroll
+      for (int t = 0; t < NQ; ++t) {
+        if (t >= ntile) break;
+        if (j >= 1 && j - 1 < nt[t]) {
+          const int pj = j - 1, pst = pj % NSV;
+          if (!v_ready) {
+            mbar_wait(bar(B_VFULL + pst), (pj / NSV) & 1, abort_flag, p.status, detail);
+            v_ready = true;
+          }
+          mbar_wait(bar(B_PFULL + t), pj & 1, abort_flag, p.status, detail);
+          named_bar_arrive(kNbPv + t, 64);
+        }
+        if (j < nt[t] && !k_ready) {
+          mbar_wait(bar(B_KFULL + j % NSK), (j / NSK) & 1, abort_flag, p.status, detail);
+          named_bar_arrive(kNbK, 64);
+          k_ready = true;
+        }
+      }
     }
   } else {
     // ===================================================== softmax warpgroups
