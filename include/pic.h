@@ -224,8 +224,8 @@ pic_status_t pic_attend_prefill(const pic_geom_t *geom, int32_t layer, int32_t b
 /*
  * pic_attend_prefill_fused -- pic_attend_prefill without the relocated cache:
  * the same outputs, with every document key and value read straight from the
- * pool as it was compiled (the benchmark spec's fused rotate-on-load variant of the
- * re-rotation of Eq. 3).  Because rotations are orthogonal,
+ * pool as it was compiled (a fused rotate-on-load form of the re-rotation of
+ * Eq. 3).  Because rotations are orthogonal,
  *     (R(p) q) . (R(delta_k) k) = (R(-delta_k) R(p) q) . k,
  * so per document k the 128-row query tile is rotated by -delta_k (in TMEM)
  * instead of rotating the document's keys; values are used as they are.
