@@ -48,6 +48,7 @@ class CacheHitPath:
         self.lse = torch.empty((L, B, self.max_inline, Hq), dtype=torch.float32,
                                device=dev) if with_lse else None
         self.dec_out = self.dec_lse = self.ws_decode = None
+        self._request_dev = None
         if wl.q_dec is not None:
             self.ws_decode = torch.empty(
                 pic_decode_workspace_size(self.geom, B, self.max_ctx, decode_splits),
@@ -55,6 +56,39 @@ class CacheHitPath:
             self.dec_out = torch.empty((L, B, Hq, d), dtype=bf16, device=dev)
             self.dec_lse = torch.empty((L, B, Hq), dtype=torch.float32,
                                        device=dev) if with_lse else None
+
+    # -- per-request inputs as one upload
+    REQUEST_FIELDS = ("req_doc_ids", "req_num_docs", "prefix_len", "query_len", "block_table",
+                      "inline_len", "q_inline", "k_inline", "v_inline")
+
+    def pack_request_inputs(self) -> torch.Tensor:
+        """Move the per-request inputs (document choice, lengths, block table,
+        inline projections) into one contiguous device buffer, rebinding the
+        workload's tensors to views of it, and return a pinned host mirror
+        holding the same bytes.  A serving loop then writes a request into
+        the mirror and calls ``upload`` once: one host-to-device copy per
+        step instead of one per tensor.  The document pool stays resident."""
+        wl = self.wl
+        offs, total = [], 0
+        for name in self.REQUEST_FIELDS:
+            t = getattr(wl, name)
+            offs.append(total)
+            total += (t.numel() * t.element_size() + 255) // 256 * 256
+        dev = torch.empty(total, dtype=torch.uint8, device=wl.k_pool.device)
+        host = torch.empty(total, dtype=torch.uint8, pin_memory=True)
+        for name, off in zip(self.REQUEST_FIELDS, offs):
+            t = getattr(wl, name)
+            n = t.numel() * t.element_size()
+            view = dev[off:off + n].view(t.dtype).view(t.shape)
+            view.copy_(t)
+            host[off:off + n].copy_(view.view(torch.uint8).view(-1).cpu())
+            setattr(wl, name, view)
+        self._request_dev = dev
+        return host
+
+    def upload(self, host: torch.Tensor):
+        """One asynchronous copy of a packed request (see pack_request_inputs)."""
+        self._request_dev.copy_(host, non_blocking=True)
 
     # -- a1: layout and slot map
     def compose(self):

@@ -317,3 +317,23 @@ def test_fused_equals_materialised(cuda_lib, name):
         tin = int(wl.inline_len[bb])
         d = (a[:, bb, :tin] - b[:, bb, :tin]).abs().max().item()
         assert d <= 1e-2, d
+
+
+@pytest.mark.gpu
+def test_packed_request_upload_gives_identical_results():
+    """pack_request_inputs + upload (one host-to-device copy per request)
+    must leave the pass's results bit-identical to the unpacked tensors."""
+    from paper_2607_28069_gb300.pipeline import CacheHitPath
+    wl = generate(SMALL["ragged_b3"], device="cuda", gen_device="cpu")
+    path = CacheHitPath(wl)
+    path.ttft_pass()
+    torch.cuda.synchronize()
+    ref_out, ref_k = path.out.clone(), path.k_cache.clone()
+    host = path.pack_request_inputs()
+    path.out.zero_()
+    path.k_cache.zero_()
+    path.upload(host)
+    path.ttft_pass()
+    torch.cuda.synchronize()
+    assert torch.equal(path.out, ref_out)
+    assert torch.equal(path.k_cache, ref_k)
