@@ -50,6 +50,7 @@ __device__ long long block_inclusive_scan(long long v, long long *warp_tot) {
 }
 
 __global__ void __launch_bounds__(kThreads) compose_kernel(ComposeArgs a) {
+  pdl_entry();
   const int b = blockIdx.y;
   const int tid = threadIdx.x;
   const bool lead = blockIdx.x == 0;
@@ -229,7 +230,8 @@ extern "C" pic_status_t pic_compose(const pic_geom_t *geom, int32_t batch, int32
                                          (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "pic_compose smem attribute");
   }
-  compose_kernel<<<grid, kThreads, smem, stream>>>(a);
+  cudaError_t le = launch_dependent(compose_kernel, grid, dim3(kThreads), smem, stream, a);
+  if (le != cudaSuccess) return cuda_fail(le, "pic_compose launch");
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_compose launch");
   return PIC_OK;

@@ -14,6 +14,8 @@
 #include <algorithm>
 #include <cmath>
 
+#include <utility>
+
 #include "../../include/pic.h"
 
 namespace pic {
@@ -226,6 +228,34 @@ PIC_DEV void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.clust
 PIC_DEV void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
+// Programmatic dependent launch.  A kernel launched with launch_dependent()
+// calls pdl_entry() first: it waits until the kernel before it on the stream
+// has completed and its writes are visible (before this kernel reads or
+// writes anything), then lets the next kernel's launch begin.  Because every
+// kernel of a chain waits first, completion of one implies completion of all
+// before it.  The next grid launches only once every CTA of this one has
+// run the trigger, i.e. is resident, so it never starves this one of SMs.
+PIC_DEV void pdl_entry() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                                    cudaStream_t stream, Args &&...args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 // Named CTA barriers (bar.sync / bar.arrive) shared by a fixed set of warps.
 PIC_DEV void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");

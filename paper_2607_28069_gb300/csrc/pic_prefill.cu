@@ -96,6 +96,7 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                 const __grid_constant__ CUtensorMap tm_v, Params p) {
+  pdl_entry();
   using L = Layout<D>;
   constexpr int PANELS = D / 64;
   constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
@@ -1171,6 +1172,7 @@ struct AppendArgs {
 template <int D>
 __global__ void __launch_bounds__(256) append_kernel(AppendArgs a, RopeParams rp) {
   constexpr int HALF = D / 2, KC = D / 16, VC = D / 8;
+  pdl_entry();
   const int t = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
   const int tin = min(max(a.inline_len[b], 0), a.max_inline);
   __shared__ float2 cs[HALF];
@@ -1438,8 +1440,9 @@ extern "C" pic_status_t pic_append_inline(
   if (t_slots > INT32_MAX / 2 || batch > 65535)
     return fail(PIC_ERR_UNSUPPORTED, "pic_append_inline: grid too large");
   dim3 agrid(t_slots, batch);
-  if (D == 128) append_kernel<128><<<agrid, 256, 0, stream>>>(aa, rp);
-  else append_kernel<64><<<agrid, 256, 0, stream>>>(aa, rp);
+  cudaError_t le = D == 128 ? launch_dependent(append_kernel<128>, agrid, dim3(256), 0, stream, aa, rp)
+                            : launch_dependent(append_kernel<64>, agrid, dim3(256), 0, stream, aa, rp);
+  if (le != cudaSuccess) return cuda_fail(le, "pic_append_inline launch");
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_append_inline launch");
   return PIC_OK;
@@ -1509,12 +1512,14 @@ extern "C" pic_status_t pic_attend_prefill(
     const int smem = Layout<128>::kAlloc;
     e = cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill smem attribute");
-    attn_kernel<128><<<grid, kThreads, smem, stream>>>(tq, tk, tv, pp);
+    e = launch_dependent(attn_kernel<128>, grid, dim3(kThreads), smem, stream, tq, tk, tv, pp);
+    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill launch");
   } else {
     const int smem = Layout<64>::kAlloc;
     e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill smem attribute");
-    attn_kernel<64><<<grid, kThreads, smem, stream>>>(tq, tk, tv, pp);
+    e = launch_dependent(attn_kernel<64>, grid, dim3(kThreads), smem, stream, tq, tk, tv, pp);
+    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill launch");
   }
   if (pl.splits > 1) {
     const long long rows = (long long)batch * Hkv * pl.m_tiles * BM;

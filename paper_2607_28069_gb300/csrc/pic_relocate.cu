@@ -40,6 +40,7 @@ struct RelocArgs {
 template <int D, int kTok>
 __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopeParams rp) {
   static_assert(kTok == 16 || kTok == 32, "one warp scans the positions of a CTA");
+  pdl_entry();
   constexpr unsigned kMask = kTok == 32 ? 0xffffffffu : 0x0000ffffu;
   constexpr int HALF = D / 2;
   constexpr int KC = D / 16;  // 8-pair chunks per K row
@@ -244,14 +245,15 @@ extern "C" pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int3
   const bool wide = geom->num_kv_heads * geom->head_dim >= 1024;
   const int tok = wide ? 16 : 32;
   dim3 grid((max_ctx + tok - 1) / tok, batch, layer_end - layer_begin);
-  if (geom->head_dim == 128) {
-    if (wide) relocate_kernel<128, 16><<<grid, kThreads, 0, stream>>>(a, rp);
-    else relocate_kernel<128, 32><<<grid, kThreads, 0, stream>>>(a, rp);
-  } else {
-    if (wide) relocate_kernel<64, 16><<<grid, kThreads, 0, stream>>>(a, rp);
-    else relocate_kernel<64, 32><<<grid, kThreads, 0, stream>>>(a, rp);
-  }
-  cudaError_t e = cudaGetLastError();
+  const dim3 block(kThreads);
+  cudaError_t e;
+  if (geom->head_dim == 128)
+    e = wide ? launch_dependent(relocate_kernel<128, 16>, grid, block, 0, stream, a, rp)
+             : launch_dependent(relocate_kernel<128, 32>, grid, block, 0, stream, a, rp);
+  else
+    e = wide ? launch_dependent(relocate_kernel<64, 16>, grid, block, 0, stream, a, rp)
+             : launch_dependent(relocate_kernel<64, 32>, grid, block, 0, stream, a, rp);
+  if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_relocate launch");
   return PIC_OK;
 }
