@@ -298,10 +298,17 @@ def main_gpu(args, rank, world):
     # The TTFT pass as CUDA graph(s) with timing events at every call boundary:
     # one graph with external event nodes when torch supports them, else one
     # graph per call with events between the replays.
+    # rows: the separate calls of the path; the pass (value): pic_link for the
+    # layout, every layer's relocation and the first layer's append, then the
+    # attention of every layer (and the append of the later ones)
     calls = [("compose", path.compose), ("relocate", path.relocate)]
     for layer in range(L):
         calls.append(("append", (lambda l=layer: path.append(l))))
         calls.append(("attend", (lambda l=layer: path.attend(l))))
+    pass_calls = [("link", (lambda: path.link(0))), ("attend", (lambda: path.attend(0)))]
+    for layer in range(1, L):
+        pass_calls.append(("append", (lambda l=layer: path.append(l))))
+        pass_calls.append(("attend", (lambda l=layer: path.attend(l))))
     stream = torch.cuda.current_stream()
     try:
         bounds = [torch.cuda.Event(enable_timing=True, external=True)
@@ -319,9 +326,16 @@ def main_gpu(args, rank, world):
         g_pass = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g_pass):
             ends[0].record()
-            for _, fn in calls:
+            for _, fn in pass_calls:
                 fn()
             ends[1].record()
+        # the link call alone, cold (its own row)
+        lends = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
+        g_link = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_link):
+            lends[0].record()
+            path.link(0)
+            lends[1].record()
     except (TypeError, RuntimeError):
         graphs = []
         for _, fn in calls:
@@ -349,6 +363,14 @@ def main_gpu(args, rank, world):
         torch.cuda.synchronize()
         return ends[0].elapsed_time(ends[1])
 
+    def link_step():
+        """Flush L2, then pic_link alone; returns ms."""
+        flush.zero_()
+        torch.cuda._sleep(sleep_cycles)
+        g_link.replay()
+        torch.cuda.synchronize()
+        return lends[0].elapsed_time(lends[1])
+
     def one_step():
         """Flush L2, then one pass; returns per-call ms after synchronising."""
         flush.zero_()
@@ -370,16 +392,18 @@ def main_gpu(args, rank, world):
     for _ in range(W):
         if single:
             pass_step()
+            link_step()
         one_step()
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    per_call, pass_ms = [], []
+    per_call, pass_ms, link_ms = [], [], []
     with ClockSampler(dev) as clk:
         for _ in range(K):
             if single:
                 pass_ms.append(pass_step())
+                link_ms.append(link_step())
             per_call.append(one_step())
     if world > 1:
         torch.distributed.barrier()
@@ -416,8 +440,18 @@ def main_gpu(args, rank, world):
                       "tflops": work["attend_flops"] / (per_step["attend"] * 1e9)},
     }
     rows["a2_a3_relocate"]["frac_hbm"] = rows["a2_a3_relocate"]["gbs"] / peaks["hbm_gbs"]
+    if link_ms:
+        lms = sum(link_ms) / len(link_ms)
+        link_bytes = work["relocate_bytes"] + work["append_bytes"] / L
+        rows["a1_a4_link"] = {
+            "ms": lms, "launches": 1, "bytes": link_bytes, "gbs": link_bytes / (lms * 1e6),
+            "frac_hbm": link_bytes / (lms * 1e6) / peaks["hbm_gbs"],
+            "note": "pic_link: layout, every layer's relocation and layer 0's inline append in "
+                    "one launch (what the pass runs); rows a1-a4 time the separate calls"}
     rows["a5_attend"]["frac_bf16"] = rows["a5_attend"]["tflops"] / peaks["bf16_tflops"]
-    launches = 1 + 1 + L + rows["a5_attend"]["launches"]
+    # kernels of the timed pass: pic_link, the later layers' appends, attention (+ merge)
+    launches = (1 + (L - 1) + rows["a5_attend"]["launches"]) if single else \
+        (1 + 1 + L + rows["a5_attend"]["launches"])
 
     # decode (outside the TTFT boundary), same run
     if dec_graph is not None:
@@ -505,7 +539,7 @@ def main_gpu(args, rank, world):
         d2h = host_out.numel() * host_out.element_size()
         g2 = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g2):
-            for _, fn in calls:
+            for _, fn in (pass_calls if single else calls):
                 fn()
         torch.cuda.synchronize()
         e_ms = []

@@ -167,6 +167,37 @@ pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int32_t max_doc
                           pic_stream_t stream);
 
 /*
+ * pic_link -- pic_compose, pic_relocate (layers [layer_begin, layer_end)) and
+ * pic_append_inline (layer append_layer, or none when append_layer < 0) in a
+ * single launch: the link step of a cache hit (Eqs. 1-3; appendix
+ * "Position-Independent Linking").  Every argument means what it means for
+ * those three calls, and every output -- the layout (doc_offset, doc_delta,
+ * slot_mapping, tok_map, inline_pos, ctx_len), the stitched K/V of the
+ * documents and of the appended inline tokens, and the packed queries at the
+ * start of the prefill workspace -- is bit-identical to theirs.  Each CTA
+ * handles one 16-position page of one request for one layer and derives the
+ * layout of its page itself, so the three dependent chains of memory round
+ * trips become one.  Requests with more than 256 documents (max_docs > 256)
+ * run the three calls in order instead.
+ * workspace: the prefill workspace of pic_append_inline (only its leading
+ *   packed-query part is written); may be NULL when append_layer < 0.
+ * One launch (or the three calls' launches), asynchronous on `stream`;
+ * device checks as for the three calls, reported through pic_device_status.
+ */
+pic_status_t pic_link(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
+                      int32_t n_pool_docs, const int32_t *doc_len, const int32_t *doc_base_pos,
+                      const int64_t *doc_token_start, const int32_t *req_doc_ids,
+                      const int32_t *req_num_docs, const int32_t *prefix_len,
+                      const int32_t *query_len, const int32_t *block_table, int32_t max_pages,
+                      int64_t num_pages, int32_t max_ctx, int32_t max_inline, const void *k_pool,
+                      const void *v_pool, int64_t pool_tokens, int32_t layer_begin,
+                      int32_t layer_end, int32_t append_layer, const void *q, const void *k_new,
+                      const void *v_new, const int32_t *inline_len, void *k_cache, void *v_cache,
+                      int32_t *doc_offset, int32_t *doc_delta, int64_t *slot_mapping,
+                      int64_t *tok_map, int32_t *inline_pos, int32_t *ctx_len, void *workspace,
+                      size_t workspace_bytes, pic_stream_t stream);
+
+/*
  * Prefill of one layer's inline tokens ("Cache-hit serving": only the
  * request-specific inline tokens are processed; appendix "Position-Independent
  * Linking": their KVs are interleaved with the prepared document states, and

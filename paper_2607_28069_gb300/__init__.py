@@ -16,7 +16,7 @@ from typing import Optional
 import torch
 
 __all__ = [
-    "Geometry", "load", "lib_path", "pic_abi_version", "pic_compose", "pic_relocate",
+    "Geometry", "load", "lib_path", "pic_abi_version", "pic_compose", "pic_relocate", "pic_link",
     "pic_append_inline", "pic_attend_prefill", "pic_attend_prefill_fused",
     "pic_prefill_workspace_size",
     "pic_prefill_num_splits", "pic_decode_num_splits", "pic_attend_decode_noalloc",
@@ -34,7 +34,7 @@ ROPE_INTERLEAVED = 1
 # Every symbol include/pic.h declares.
 EXPORTED_SYMBOLS = (
     "pic_abi_version", "pic_last_error", "pic_device_status", "pic_compose", "pic_relocate",
-    "pic_prefill_workspace_size", "pic_prefill_num_splits", "pic_append_inline",
+    "pic_link", "pic_prefill_workspace_size", "pic_prefill_num_splits", "pic_append_inline",
     "pic_attend_prefill", "pic_attend_prefill_fused", "pic_decode_workspace_size", "pic_decode_num_splits",
     "pic_attend_decode", "pic_attend_decode_noalloc",
 )
@@ -102,6 +102,8 @@ def load():
         "pic_compose": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, I32, I64, I32, I32,
                               P, P, P, P, P, P, P]),
         "pic_relocate": (I32, [G, I32, I32, P, P, I64, P, P, P, I32, I64, P, P, I32, I32, P]),
+        "pic_link": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, I32, I64, I32, I32, P, P, I64,
+                           I32, I32, I32, P, P, P, P, P, P, P, P, P, P, P, P, P, SZ, P]),
         "pic_prefill_workspace_size": (SZ, [G, I32, I32, I32, I32]),
         "pic_append_inline": (I32, [G, I32, I32, I32, P, P, P, P, P, P, I32, I64, P, P, P, SZ,
                                     P]),
@@ -200,6 +202,35 @@ def pic_relocate(geom: Geometry, k_pool, v_pool, tok_map, doc_delta, slot_mappin
         _ptr(k_cache, bf16, "k_cache"), _ptr(v_cache, bf16, "v_cache"), layer_begin, layer_end,
         _stream(stream))
     _check(st, "pic_relocate")
+
+
+def pic_link(geom: Geometry, doc_len, doc_base_pos, doc_token_start, req_doc_ids, req_num_docs,
+             prefix_len, query_len, block_table, num_pages: int, max_ctx: int, max_inline: int,
+             k_pool, v_pool, layer_begin: int, layer_end: int, append_layer: int, q, k_new, v_new,
+             inline_len, k_cache, v_cache, doc_offset, doc_delta, slot_mapping, tok_map, inline_pos,
+             ctx_len, workspace, stream=None):
+    """pic_compose + pic_relocate + pic_append_inline (append_layer, or none if < 0)
+    in one launch; q/k_new/v_new are the append layer's inline projections."""
+    lib = load()
+    g = geom._c()
+    B, max_docs = req_doc_ids.shape
+    app = append_layer >= 0
+    st = lib.pic_link(
+        ctypes.byref(g), B, max_docs, doc_len.numel(), _ptr(doc_len, i32, "doc_len"),
+        _ptr(doc_base_pos, i32, "doc_base_pos"), _ptr(doc_token_start, i64, "doc_token_start"),
+        _ptr(req_doc_ids, i32, "req_doc_ids"), _ptr(req_num_docs, i32, "req_num_docs"),
+        _ptr(prefix_len, i32, "prefix_len"), _ptr(query_len, i32, "query_len"),
+        _ptr(block_table, i32, "block_table"), block_table.shape[1], num_pages, max_ctx,
+        max_inline, _ptr(k_pool, bf16, "k_pool"), _ptr(v_pool, bf16, "v_pool"), k_pool.shape[1],
+        layer_begin, layer_end, append_layer, _ptr(q, bf16, "q", allow_none=not app),
+        _ptr(k_new, bf16, "k_new", allow_none=not app), _ptr(v_new, bf16, "v_new", allow_none=not app),
+        _ptr(inline_len, i32, "inline_len", allow_none=not app), _ptr(k_cache, bf16, "k_cache"),
+        _ptr(v_cache, bf16, "v_cache"), _ptr(doc_offset, i32, "doc_offset"),
+        _ptr(doc_delta, i32, "doc_delta"), _ptr(slot_mapping, i64, "slot_mapping"),
+        _ptr(tok_map, i64, "tok_map"), _ptr(inline_pos, i32, "inline_pos"),
+        _ptr(ctx_len, i32, "ctx_len"), _ptr(workspace, torch.uint8, "workspace", allow_none=not app),
+        0 if workspace is None else workspace.numel(), _stream(stream))
+    _check(st, "pic_link")
 
 
 def pic_prefill_workspace_size(geom: Geometry, batch: int, max_inline: int, max_ctx: int,

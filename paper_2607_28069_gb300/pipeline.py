@@ -9,7 +9,7 @@ from __future__ import annotations
 import torch
 
 from . import (Geometry, pic_append_inline, pic_attend_decode, pic_attend_prefill,
-               pic_attend_prefill_fused, pic_compose, pic_decode_workspace_size,
+               pic_attend_prefill_fused, pic_compose, pic_decode_workspace_size, pic_link,
                pic_prefill_workspace_size, pic_relocate)
 from .workloads import Workload
 
@@ -107,6 +107,20 @@ class CacheHitPath:
                      self.slot_mapping, wl.num_pages, self.k_cache, self.v_cache, layer_begin,
                      layer_end)
 
+    # -- a1 + a2 + a3 + a4 (first layer) in one launch
+    def link(self, append_layer: int = 0):
+        wl = self.wl
+        L = wl.spec.layers
+        app = append_layer >= 0
+        pic_link(self.geom, wl.doc_len, wl.doc_base_pos, wl.doc_token_start, wl.req_doc_ids,
+                 wl.req_num_docs, wl.prefix_len, wl.query_len, wl.block_table, wl.num_pages,
+                 self.max_ctx, self.max_inline, wl.k_pool, wl.v_pool, 0, L, append_layer,
+                 wl.q_inline[append_layer] if app else None,
+                 wl.k_inline[append_layer] if app else None,
+                 wl.v_inline[append_layer] if app else None, wl.inline_len if app else None,
+                 self.k_cache, self.v_cache, self.doc_offset, self.doc_delta, self.slot_mapping,
+                 self.tok_map, self.inline_pos, self.ctx_len, self.ws_prefill if app else None)
+
     # -- a4: RoPE + append of the inline tokens of one layer
     def append(self, layer: int):
         wl = self.wl
@@ -153,12 +167,20 @@ class CacheHitPath:
                           None if self.dec_lse is None else self.dec_lse[layer],
                           self.decode_splits, self.ws_decode, pos_offset=step)
 
-    def ttft_pass(self):
+    def ttft_pass(self, linked: bool = True):
         """The cache-hit path up to the first token: layout, re-rotation and
-        stitching of every layer, then every layer's inline prefill."""
-        self.compose()
-        self.relocate()
-        for layer in range(self.wl.spec.layers):
+        stitching of every layer, then every layer's inline prefill.  With
+        ``linked`` the layout, the relocation and the first layer's inline
+        append are one pic_link launch; otherwise the separate calls."""
+        if linked:
+            self.link(0)
+            self.attend(0)
+            first = 1
+        else:
+            self.compose()
+            self.relocate()
+            first = 0
+        for layer in range(first, self.wl.spec.layers):
             self.prefill(layer)
 
     def decode_pass(self, step: int):

@@ -337,3 +337,47 @@ def test_packed_request_upload_gives_identical_results():
     torch.cuda.synchronize()
     assert torch.equal(path.out, ref_out)
     assert torch.equal(path.k_cache, ref_k)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name,rope_style", [("tiny", 0), ("llama8b_1layer", 0), ("ragged_b3", 0),
+                                             ("ragged_b3", 1), ("d64_g8", 0), ("no_docs", 0)])
+def test_link_equals_separate_calls(name, rope_style):
+    """pic_link (layout + relocation + first-layer append in one launch) gives
+    bit-identical layout outputs, caches and prefill outputs to pic_compose,
+    pic_relocate and pic_append_inline called in turn."""
+    import paper_2607_28069_gb300 as pic
+    from paper_2607_28069_gb300.pipeline import CacheHitPath
+    wl = generate(SMALL[name], device="cuda", gen_device="cpu")
+    outs = []
+    for linked in (False, True):
+        path = CacheHitPath(wl, with_lse=True, rope_style=rope_style)
+        path.ttft_pass(linked=linked)
+        torch.cuda.synchronize()
+        assert pic.pic_device_status() == (0, 0)
+        outs.append({k: getattr(path, k).clone() for k in
+                     ("doc_offset", "doc_delta", "slot_mapping", "tok_map", "inline_pos", "ctx_len",
+                      "k_cache", "v_cache", "out", "lse")})
+    for k in ("doc_offset", "doc_delta", "slot_mapping", "tok_map", "inline_pos", "ctx_len",
+              "k_cache", "v_cache"):
+        assert torch.equal(outs[0][k], outs[1][k]), k
+    for b in range(wl.spec.batch):  # out / lse rows past a request's inline tokens are not written
+        tin = int(wl.inline_len[b])
+        assert torch.equal(outs[0]["out"][:, b, :tin], outs[1]["out"][:, b, :tin]), b
+        assert torch.equal(outs[0]["lse"][:, b, :tin], outs[1]["lse"][:, b, :tin]), b
+
+
+@pytest.mark.gpu
+def test_link_reports_bad_document_id():
+    """A document id outside the pool is a device-checked error of the link
+    launch, as of pic_compose."""
+    import paper_2607_28069_gb300 as pic
+    from paper_2607_28069_gb300.pipeline import CacheHitPath
+    wl = generate(SMALL["llama8b_1layer"], device="cuda", gen_device="cpu")
+    wl.req_doc_ids[0, 1] = wl.doc_len.numel() + 5
+    path = CacheHitPath(wl)
+    path.link(0)
+    torch.cuda.synchronize()
+    code, detail = pic.pic_device_status()
+    assert code == 1 and detail == 0
+    assert int(path.ctx_len[0]) == -1
