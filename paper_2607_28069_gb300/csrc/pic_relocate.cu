@@ -2,13 +2,14 @@
 // into the paged request cache; values are copied unchanged (the paper rotates
 // keys only; Background: Position-Independent Caching).
 //
-// One launch, one CTA per (one or two pages of logical positions, request,
-// layer).
+// One launch, one CTA per (one or two pages of logical positions, request);
+// the CTA moves its positions for every layer in turn, so its set-up (maps,
+// cos/sin) is done once and it keeps a long stream of loads in flight.
 // The CTA reads the token map and slot map of its positions (written by
-// pic_compose), issues every K and V load of its page at once (16-byte
-// streaming loads; V rows are bit copies, K rows come as the two 16-byte
-// halves of 8 RoPE pairs), and while those are in flight evaluates cos/sin of
-// delta_k * theta_i for the (one or two) documents the page touches: delta is
+// pic_compose) and evaluates cos/sin of delta_k * theta_i for the documents
+// its page touches; then, per layer, it issues every K and V load of its page
+// at once (16-byte streaming loads; V rows are bit copies, K rows come as the
+// two 16-byte halves of 8 RoPE pairs), rotates and stores.  delta is
 // constant over a document because base and target positions both advance by
 // one per token, so R(b) R(a)^-1 = R(b - a) = R(delta).  The angle is formed and
 // reduced in fp64, sin/cos evaluated in fp32 on the reduced angle; K is rotated
@@ -28,7 +29,7 @@ constexpr int UV = 8;     // V tasks per thread per round
 constexpr int UK = 4;     // K tasks per thread per round
 
 struct RelocArgs {
-  int max_docs, max_ctx, hkv, layer_begin;
+  int max_docs, max_ctx, hkv, layer_begin, layer_end;
   long long pool_tokens, num_pages;
   const __nv_bfloat16 *k_pool, *v_pool;
   const int64_t *tok_map, *slots;
@@ -47,7 +48,6 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
   constexpr int VC = D / 8;   // 16-byte pieces per V row
   const int style = rp.style;
   const int b = blockIdx.y;
-  const int layer = a.layer_begin + blockIdx.z;
   const long long t0 = (long long)blockIdx.x * kTok;
   const int tid = threadIdx.x;
 
@@ -96,6 +96,13 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
   const int n_docs = min(s_last - s_first + 1, kTok);
 
   const size_t hkv = a.hkv;
+  for (int e = tid; e < n_docs * HALF; e += kThreads) {  // cos/sin of the touched documents
+    const int j = e / HALF, i = e % HALF;
+    const int delta = a.delta[(size_t)b * a.max_docs + k_first + j];
+    s_cs[j][i] = rope_cos_sin(delta, rp.theta[i]);
+  }
+  __syncthreads();
+  for (int layer = a.layer_begin; layer < a.layer_end; ++layer) {
   const __nv_bfloat16 *kp = a.k_pool + (size_t)layer * a.pool_tokens * hkv * D;
   const __nv_bfloat16 *vp = a.v_pool + (size_t)layer * a.pool_tokens * hkv * D;
   __nv_bfloat16 *kc = a.k_cache + (size_t)layer * a.num_pages * hkv * 16 * D;
@@ -143,15 +150,6 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
         }
       }
     }
-    if (round == 0) {
-      // cos/sin of the touched documents while the loads are in flight
-      for (int e = tid; e < n_docs * HALF; e += kThreads) {
-        const int j = e / HALF, i = e % HALF;
-        const int delta = a.delta[(size_t)b * a.max_docs + k_first + j];
-        s_cs[j][i] = rope_cos_sin(delta, rp.theta[i]);
-      }
-      __syncthreads();
-    }
     // ---- V: bit copy
 #pragma unroll
     for (int u = 0; u < UV; ++u)
@@ -193,6 +191,7 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
       st_global16(kc + kdst[u] + pc.off_b, pack8(y));
     }
   }
+  }
 }
 
 }  // namespace
@@ -232,6 +231,7 @@ extern "C" pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int3
   a.max_ctx = max_ctx;
   a.hkv = geom->num_kv_heads;
   a.layer_begin = layer_begin;
+  a.layer_end = layer_end;
   a.pool_tokens = pool_tokens;
   a.num_pages = num_pages;
   a.k_pool = static_cast<const __nv_bfloat16 *>(k_pool);
@@ -244,7 +244,7 @@ extern "C" pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int3
   a.status = status;
   const bool wide = geom->num_kv_heads * geom->head_dim >= 1024;
   const int tok = wide ? 16 : 32;
-  dim3 grid((max_ctx + tok - 1) / tok, batch, layer_end - layer_begin);
+  dim3 grid((max_ctx + tok - 1) / tok, batch);
   const dim3 block(kThreads);
   cudaError_t e;
   if (geom->head_dim == 128)
