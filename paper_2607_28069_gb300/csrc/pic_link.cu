@@ -8,7 +8,9 @@
 // base to their final positions by R(delta), values are copied, and the
 // inline tokens are rotated at their own positions.
 //
-// Grid x: one CTA per 16-position page, then (with an append) one CTA per
+// Grid x: one CTA per slice of kTok positions (one page, or two when a
+// token's K row is under 1024 elements, as in pic_relocate), then (with an
+// append) one CTA per
 // inline token slot; y: request.  Each CTA derives the part of the
 // layout it needs by itself -- the request's document offsets (a block scan
 // over at most kMaxLinkDocs lengths) and the one block-table entry it needs --
@@ -27,7 +29,6 @@ namespace pic {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kTok = 16;            // positions per CTA: one page
 constexpr int kMaxLinkDocs = 256;   // documents per request handled in one launch
 constexpr int kBM = 128;            // rows per query tile of the packed-Q workspace
 constexpr int UV = 8, UK = 4;       // relocate tasks per thread per round (V, K)
@@ -248,8 +249,10 @@ __device__ void token_cta(const LinkArgs &a, const RopeParams &rp, int b, int la
   }
 }
 
-template <int D>
+template <int D, int kTok>
 __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams rp) {
+  static_assert(kTok == 16 || kTok == 32, "one warp scans the positions of a CTA");
+  constexpr unsigned kMask = kTok == 32 ? 0xffffffffu : 0x0000ffffu;
   pdl_entry();
   constexpr int HALF = D / 2, KC = D / 16, VC = D / 8;
   const int b = blockIdx.y, tid = threadIdx.x;
@@ -268,10 +271,11 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
   __shared__ int s_first, s_last;
   __shared__ float2 s_cs[kTok][HALF];       // per touched document
 
-  // ---- request scalars and this page's block-table entry, all independent
+  // ---- request scalars and the block-table entry of each position, all independent
   const int P = a.prefix[b], Tq = a.query[b], m = a.num_docs[b];
-  const long long pidx = t0 / 16;
-  const int page_raw = pidx < a.max_pages ? a.block_table[(size_t)b * a.max_pages + pidx] : -1;
+  const long long pidx = (t0 + tid) / 16;
+  const int page_raw = tid < kTok && pidx < a.max_pages
+                           ? a.block_table[(size_t)b * a.max_pages + pidx] : -1;
   const int tin = a.inline_len ? min(max(a.inline_len[b], 0), a.max_inline) : 0;
   if (tid == 0) rv.err = 0;
   __syncthreads();
@@ -322,9 +326,9 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
     s_src[tid] = tm >= 0 ? src : -1;
     s_dst[tid] = sl;
     s_doc[tid] = k;
-    const unsigned valid = __ballot_sync(0x0000ffffu, s_src[tid] >= 0);
-    const int kf = __shfl_sync(0x0000ffffu, k, valid ? __ffs(valid) - 1 : 0);
-    const int kl = __shfl_sync(0x0000ffffu, k, valid ? 31 - __clz(valid) : 0);
+    const unsigned valid = __ballot_sync(kMask, s_src[tid] >= 0);
+    const int kf = __shfl_sync(kMask, k, valid ? __ffs(valid) - 1 : 0);
+    const int kl = __shfl_sync(kMask, k, valid ? 31 - __clz(valid) : 0);
     if (tid == 0) {
       s_first = valid ? kf : -1;
       s_last = valid ? kl : -1;
@@ -501,7 +505,10 @@ extern "C" pic_status_t pic_link(
   a.G = G;
   a.R_pad = R_pad;
   a.t_slots = std::max(max_inline, (R_pad + G - 1) / G);
-  a.n_pages = (max_ctx + kTok - 1) / kTok;
+  // one page per CTA when a token carries >= 1024 K elements, else two
+  const bool wide = geom->num_kv_heads * geom->head_dim >= 1024;
+  const int tok = wide ? 16 : 32;
+  a.n_pages = (max_ctx + tok - 1) / tok;
   a.num_pages = num_pages;
   a.pool_tokens = pool_tokens;
   a.doc_len = doc_len;
@@ -530,9 +537,14 @@ extern "C" pic_status_t pic_link(
   a.status = status;
 
   dim3 grid((unsigned)(a.n_pages + (do_append ? a.t_slots : 0)), batch);
-  cudaError_t e = geom->head_dim == 128
-                      ? launch_dependent(link_kernel<128>, grid, dim3(kThreads), 0, stream, a, rp)
-                      : launch_dependent(link_kernel<64>, grid, dim3(kThreads), 0, stream, a, rp);
+  const dim3 block(kThreads);
+  cudaError_t e;
+  if (geom->head_dim == 128)
+    e = wide ? launch_dependent(link_kernel<128, 16>, grid, block, 0, stream, a, rp)
+             : launch_dependent(link_kernel<128, 32>, grid, block, 0, stream, a, rp);
+  else
+    e = wide ? launch_dependent(link_kernel<64, 16>, grid, block, 0, stream, a, rp)
+             : launch_dependent(link_kernel<64, 32>, grid, block, 0, stream, a, rp);
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_link launch");
   return PIC_OK;
