@@ -96,7 +96,6 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                 const __grid_constant__ CUtensorMap tm_v, Params p) {
-  pdl_entry();
   using L = Layout<D>;
   constexpr int PANELS = D / 64;
   constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
@@ -130,6 +129,35 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int hk = blockIdx.y, b = blockIdx.z;
   const int detail = b;
 
+  // ---- set-up that reads nothing the previous kernel writes: it runs before
+  // the programmatic-launch wait, while that kernel may still be finishing
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < B_COUNT; ++i)
+      mbar_init(bar(i), (i >= B_PFULL && i < B_PFULL + NQ) ? 4 : 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tm_q);
+    prefetch_tmap(&tm_k);
+    prefetch_tmap(&tm_v);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = *tmem_slot;
+  pdl_entry();
+  auto release_and_exit = [&]() {  // a CTA without work frees its TMEM
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+      tc_fence_after();
+      tmem_dealloc(tbase, kTmemCols);
+    }
+  };
+
   // ---- work of this CTA (uniform across threads)
   const int tin = min(max(p.inline_len[b], 0), p.max_inline);
   const int rows = tin * p.G;
@@ -145,7 +173,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       ntile = t + 1;
     }
   }
-  if (ntile == 0) return;  // no query row in this pair
+  if (ntile == 0) {  // no query row in this pair
+    release_and_exit();
+    return;
+  }
   const int kmax_all = ntile == 2 ? kmax[1] : kmax[0];
   const int n_kv_all = kmax_all >= 0 ? kmax_all / BN + 1 : 0;
   const int per = (n_kv_all + p.num_splits - 1) / p.num_splits;
@@ -167,23 +198,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         p.part_ml[(part_row0(t) + threadIdx.x) * 2] = -INFINITY;
         p.part_ml[(part_row0(t) + threadIdx.x) * 2 + 1] = 0.f;
       }
+    release_and_exit();
     return;
   }
-
-  if (threadIdx.x == 0) {
-    for (int i = 0; i < B_COUNT; ++i)
-      mbar_init(bar(i), (i >= B_PFULL && i < B_PFULL + NQ) ? 4 : 1);
-    *abort_flag = 0;
-    fence_mbar_init();
-  }
-  if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
-    tmem_relinquish();
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tbase = *tmem_slot;
 
   if (warp == 0 || warp == kWarpV) {
     // ===================================================== TMA producers
