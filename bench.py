@@ -507,8 +507,10 @@ def main_gpu(args, rank, world):
             "query_tok_s": work["query_tokens"] / (fms / 1e3),
             "speedup_vs_materialised": ms_per_step / fms}
 
-    # dominant kernel of the step -> roofline object
-    if per_step["attend"] >= per_step["relocate"]:
+    # dominant kernel of the step -> roofline object: attention, or the data
+    # movement the pass runs (pic_link when the pass is one graph, else relocate)
+    move_ms = rows["a1_a4_link"]["ms"] if "a1_a4_link" in rows else per_step["relocate"]
+    if per_step["attend"] >= move_ms:
         per_launch_ms = per_step["attend"] / L
         flops_launch = work["attend_flops"] / L
         achieved = flops_launch / (per_launch_ms * 1e9)
@@ -517,6 +519,13 @@ def main_gpu(args, rank, world):
                 "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                 "frac": achieved / peaks["bf16_tflops"], "traffic": traffic,
                 "peak_source": f"{peak_src} bf16 burst"}
+    elif "a1_a4_link" in rows:
+        achieved = rows["a1_a4_link"]["gbs"]
+        traffic = ncu_traffic(f"link_kernel|{args.workload}", "pic_link.cu")
+        roof = {"kernel": "link_kernel (pic_link)", "bound": "hbm",
+                "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / peaks["hbm_gbs"], "traffic": traffic,
+                "peak_source": f"{peak_src} copy"}
     else:
         achieved = rows["a2_a3_relocate"]["gbs"]
         traffic = ncu_traffic(f"relocate_kernel|{args.workload}", "pic_relocate.cu")
