@@ -8,21 +8,22 @@
 // base to their final positions by R(delta), values are copied, and the
 // inline tokens are rotated at their own positions.
 //
-// Grid x: one CTA per slice of kTok positions (one page, or two when a
-// token's K row is under 1024 elements, as in pic_relocate), then (with an
-// append) one CTA per
-// inline token slot; y: request.  Each CTA derives the part of the
+// Grid x: CTA x takes the slice x of kTok positions (one page, or two when a
+// token's K row is under 1024 elements, as in pic_relocate) and, with an
+// append, inline token slot x; y: request.  Each CTA derives the part of the
 // layout it needs by itself -- the request's document offsets (a block scan
-// over at most kMaxLinkDocs lengths) and the one block-table entry it needs --
+// over at most kMaxLinkDocs lengths) and the block-table entries it needs --
 // so nothing waits for another kernel: the three separate calls cost three
 // chains of dependent memory round trips and two kernel boundaries, this one a
-// single chain.  Page CTAs write the layout outputs of their page (slot map,
-// token map; the page-0 CTA also the per-document offsets and deltas, the
-// inline positions and ctx_len) exactly as pic_compose does, then relocate
-// the document positions of their page for every layer in turn as
-// pic_relocate does (the layout is derived once per page, not per layer).  Token CTAs issue their token's q/k/v loads first, then
-// find its position and slot, and rotate and store it as pic_append_inline
-// does (same arithmetic, same helpers: results bit-identical to the calls).
+// single chain.  A CTA issues its inline token's q/k/v loads first, writes
+// the layout outputs of its page (slot map, token map; the first CTA also
+// the per-document offsets and deltas, the inline positions and ctx_len)
+// exactly as pic_compose does, rotates and stores its token as
+// pic_append_inline does, then relocates the document positions of its page
+// for every layer in turn as pic_relocate does (the layout is derived once
+// per page, not per layer).  Same arithmetic, same helpers: results are
+// bit-identical to the three calls.  Folding the token slots into the page
+// CTAs keeps a one-layer link of a few thousand positions within one wave.
 #include "pic_internal.cuh"
 
 namespace pic {
@@ -153,83 +154,58 @@ __device__ long long request_view(const LinkArgs &a, int b, int P, int Tq, int m
   return ctx;
 }
 
-// One inline token slot of the append layer (pic_append_inline's work).
+// One inline token slot of the append layer (pic_append_inline's work), in
+// two halves: its loads go out at the start of the CTA, before the token's
+// position is known; its rotation and stores follow once the layout is.
+struct TokLoads {
+  uint4 qa, qb, ka, kb, vv;
+};
+
 template <int D>
-__device__ void token_cta(const LinkArgs &a, const RopeParams &rp, int b, int layer, int t,
-                          ReqView &rv) {
+__device__ void token_load(const LinkArgs &a, const RopeParams &rp, int b, int t, TokLoads &r) {
   constexpr int HALF = D / 2, KC = D / 16, VC = D / 8;
   const int tid = threadIdx.x;
-  const size_t hkv = a.hkv;
-  __shared__ float2 cs[HALF];
-  __shared__ long long s_slot;
-  __shared__ int s_pos;
-  const int tin = min(max(a.inline_len[b], 0), a.max_inline);
-  if (t >= tin) {  // zero the packed query rows of this token slot
-    for (int e = tid; e < (int)hkv * a.G * VC; e += kThreads) {
-      const int hk = e / (a.G * VC), r = e % (a.G * VC), g = r / VC, c = r % VC;
-      const int row = t * a.G + g;
-      if (row < a.R_pad)
-        st_global16(a.qpack + (((size_t)b * hkv + hk) * a.R_pad + row) * D + c * 8,
-                    make_uint4(0, 0, 0, 0));
-    }
-    return;
-  }
-  const size_t tok = (size_t)b * a.max_inline + t;
+  const size_t hkv = a.hkv, tok = (size_t)b * a.max_inline + t;
   const int nQ = a.hq * KC, nK = (int)hkv * KC, nV = (int)hkv * VC;
-  // the token's loads go out before its position is known
-  uint4 qa = make_uint4(0, 0, 0, 0), qb = qa, ka = qa, kb = qa, vv = qa;
+  r.qa = r.qb = r.ka = r.kb = r.vv = make_uint4(0, 0, 0, 0);
   const PairChunk pq = pair_chunk(tid % KC, HALF, rp.style);
   if (tid < nQ) {
     const __nv_bfloat16 *src = a.q + (tok * a.hq + tid / KC) * D;
-    qa = ld_stream(src + pq.off_a);
-    qb = ld_stream(src + pq.off_b);
+    r.qa = ld_stream(src + pq.off_a);
+    r.qb = ld_stream(src + pq.off_b);
   }
   if (tid < nK) {
     const __nv_bfloat16 *src = a.k_new + (tok * hkv + tid / KC) * D;
-    ka = ld_stream(src + pq.off_a);
-    kb = ld_stream(src + pq.off_b);
+    r.ka = ld_stream(src + pq.off_a);
+    r.kb = ld_stream(src + pq.off_b);
   }
-  if (tid < nV) vv = ld_stream(a.v_new + (tok * hkv + tid / VC) * D + (tid % VC) * 8);
-  const int P = a.prefix[b], Tq = a.query[b], m = a.num_docs[b];
-  if (tid == 0) rv.err = 0;
-  __syncthreads();
-  if (P < 0 || Tq < 0 || m < 0 || m > a.max_docs || m > kMaxLinkDocs) return;  // reported by page 0
-  const long long ctx = request_view(a, b, P, Tq, m, false, rv);
-  if (tid == 0) {
-    int pos = -1;
-    if (!rv.err && t < P) pos = t;
-    else if (!rv.err && t < P + Tq) pos = (int)(ctx - Tq + (t - P));
-    long long slot = -1;
-    if (pos < 0 || pos >= a.max_ctx) {
-      if (!rv.err) dev_fail(a.status, PIC_DEV_BAD_POSITION, b);
-      pos = -1;
-    } else {
-      const int page = a.block_table[(size_t)b * a.max_pages + pos / 16];
-      if (page < 0 || page >= a.num_pages) dev_fail(a.status, PIC_DEV_BAD_PAGE, b);
-      else slot = (long long)page * 16 + pos % 16;
-    }
-    s_pos = pos;
-    s_slot = slot;
-  }
-  __syncthreads();
-  const int pos = s_pos;
-  const long long slot = s_slot;
-  for (int i = tid; i < HALF; i += kThreads) cs[i] = rope_cos_sin(pos >= 0 ? pos : 0, rp.theta[i]);
-  __syncthreads();
-  const long long page = slot >> 4, r = slot & 15;
+  if (tid < nV) r.vv = ld_stream(a.v_new + (tok * hkv + tid / VC) * D + (tid % VC) * 8);
+}
+
+// Token t at logical position pos (-1: none) and cache slot `slot` (-1: none),
+// cos/sin of pos in cs: R(pos) q into the packed-query workspace, R(pos) k and
+// v into the cache of `layer`.
+template <int D>
+__device__ void token_store(const LinkArgs &a, const RopeParams &rp, int b, int layer, int t,
+                            long long slot, const float2 *cs, const TokLoads &r) {
+  constexpr int HALF = D / 2, KC = D / 16, VC = D / 8;
+  const int tid = threadIdx.x;
+  const size_t hkv = a.hkv, tok = (size_t)b * a.max_inline + t;
+  const int nQ = a.hq * KC, nK = (int)hkv * KC, nV = (int)hkv * VC;
+  const long long page = slot >> 4, rr = slot & 15;
   __nv_bfloat16 *kc = a.k_cache + (size_t)layer * a.num_pages * hkv * 16 * D;
   __nv_bfloat16 *vc = a.v_cache + (size_t)layer * a.num_pages * hkv * 16 * D;
   auto q_dst = [&](int h) {
     const int hk = h / a.G, g = h % a.G;
     return a.qpack + (((size_t)b * hkv + hk) * a.R_pad + (size_t)t * a.G + g) * D;
   };
-  if (tid < nQ) rot_store8(qa, qb, tid % KC, HALF, rp.style, cs + 8 * (tid % KC), q_dst(tid / KC));
+  if (tid < nQ) rot_store8(r.qa, r.qb, tid % KC, HALF, rp.style, cs + 8 * (tid % KC), q_dst(tid / KC));
   if (slot >= 0) {
     if (tid < nK)
-      rot_store8(ka, kb, tid % KC, HALF, rp.style, cs + 8 * (tid % KC),
-                 kc + ((page * (long long)hkv + tid / KC) * 16 + r) * D);
+      rot_store8(r.ka, r.kb, tid % KC, HALF, rp.style, cs + 8 * (tid % KC),
+                 kc + ((page * (long long)hkv + tid / KC) * 16 + rr) * D);
     if (tid < nV)
-      st_global16(vc + ((page * (long long)hkv + tid / VC) * 16 + r) * D + (tid % VC) * 8, vv);
+      st_global16(vc + ((page * (long long)hkv + tid / VC) * 16 + rr) * D + (tid % VC) * 8, r.vv);
   }
   for (int e = tid + kThreads; e < nQ; e += kThreads) {  // very wide models: more rounds
     const int h = e / KC, c = e % KC;
@@ -238,30 +214,43 @@ __device__ void token_cta(const LinkArgs &a, const RopeParams &rp, int b, int la
   if (slot >= 0) {
     for (int e = tid + kThreads; e < nK; e += kThreads) {
       const int h = e / KC, c = e % KC;
-      rotate_chunk(a.k_new + (tok * hkv + h) * D, kc + ((page * (long long)hkv + h) * 16 + r) * D,
+      rotate_chunk(a.k_new + (tok * hkv + h) * D, kc + ((page * (long long)hkv + h) * 16 + rr) * D,
                    c, HALF, rp.style, cs + 8 * c, true);
     }
     for (int e = tid + kThreads; e < nV; e += kThreads) {
       const int h = e / VC, c = e % VC;
-      st_global16(vc + ((page * (long long)hkv + h) * 16 + r) * D + c * 8,
+      st_global16(vc + ((page * (long long)hkv + h) * 16 + rr) * D + c * 8,
                   ld_stream(a.v_new + (tok * hkv + h) * D + c * 8));
     }
   }
 }
 
+// Token slot t >= inline_len: zero its packed query rows.
+template <int D>
+__device__ void token_zero(const LinkArgs &a, int b, int t) {
+  constexpr int VC = D / 8;
+  for (int e = threadIdx.x; e < a.hkv * a.G * VC; e += kThreads) {
+    const int hk = e / (a.G * VC), r = e % (a.G * VC), g = r / VC, c = r % VC;
+    const int row = t * a.G + g;
+    if (row < a.R_pad)
+      st_global16(a.qpack + (((size_t)b * a.hkv + hk) * a.R_pad + row) * D + c * 8,
+                  make_uint4(0, 0, 0, 0));
+  }
+}
+
+// CTA x of request y: page CTA x (its kTok positions, if x < n_pages) and,
+// with an append, inline token slot x (if x < t_slots).
 template <int D, int kTok>
 __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams rp) {
   static_assert(kTok == 16 || kTok == 32, "one warp scans the positions of a CTA");
   constexpr unsigned kMask = kTok == 32 ? 0xffffffffu : 0x0000ffffu;
-  pdl_entry();
+  // wait for the previous kernel; the dependent launch is released later
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   constexpr int HALF = D / 2, KC = D / 16, VC = D / 8;
   const int b = blockIdx.y, tid = threadIdx.x;
   __shared__ ReqView rv;
-  if ((int)blockIdx.x >= a.n_pages) {  // inline token slot of the append layer
-    token_cta<D>(a, rp, b, a.append_layer, blockIdx.x - a.n_pages, rv);
-    return;
-  }
-  const bool layout_cta = true;                          // writes the layout outputs
+  const bool has_page = (int)blockIdx.x < a.n_pages;
+  const int ti = a.append_layer >= 0 && (int)blockIdx.x < a.t_slots ? (int)blockIdx.x : -1;
   const bool lead = blockIdx.x == 0;                     // per-request outputs
   const long long t0 = (long long)blockIdx.x * kTok;
   const int style = rp.style;
@@ -270,14 +259,24 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
   __shared__ int s_doc[kTok];               // document index of each position
   __shared__ int s_first, s_last;
   __shared__ float2 s_cs[kTok][HALF];       // per touched document
+  __shared__ float2 s_tcs[HALF];            // at the inline token's position
+  __shared__ long long s_tslot;
+  __shared__ int s_tpos;
 
-  // ---- request scalars and the block-table entry of each position, all independent
+  // ---- the inline token's loads (rows past inline_len are read and dropped),
+  // the request scalars and the block-table entry of each position: all
+  // independent of one another
+  TokLoads tl;
+  if (ti >= 0 && ti < a.max_inline) token_load<D>(a, rp, b, ti, tl);
   const int P = a.prefix[b], Tq = a.query[b], m = a.num_docs[b];
   const long long pidx = (t0 + tid) / 16;
-  const int page_raw = tid < kTok && pidx < a.max_pages
+  const int page_raw = has_page && tid < kTok && pidx < a.max_pages
                            ? a.block_table[(size_t)b * a.max_pages + pidx] : -1;
   const int tin = a.inline_len ? min(max(a.inline_len[b], 0), a.max_inline) : 0;
-  if (tid == 0) rv.err = 0;
+  if (tid == 0) {
+    rv.err = 0;
+    s_first = -1;
+  }
   __syncthreads();
   if (P < 0 || Tq < 0 || m < 0 || m > a.max_docs || m > kMaxLinkDocs) {
     if (lead && tid == 0) {
@@ -288,13 +287,33 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
   }
   const long long ctx = request_view(a, b, P, Tq, m, lead, rv);
   const long long span_end = ctx - Tq;  // documents occupy [P, span_end)
-  if (lead && tid == 0 && a.append_layer >= 0 && tin > P + Tq)
-    atomicCAS(&rv.err, 0, PIC_DEV_BAD_POSITION);
-  __syncthreads();
-  const int err = rv.err;
+  const int err_view = rv.err;          // the document and size checks
+  // more inline tokens than prefix and query: reported by the lead CTA
+  const bool bad_tin = lead && a.append_layer >= 0 && tin > P + Tq;
+  const int err = err_view ? err_view : (bad_tin ? PIC_DEV_BAD_POSITION : 0);
 
-  // ---- this page: slot, token map, document of each position
-  if (tid < kTok) {
+  // ---- the inline token's position and slot (one thread of warp 1)
+  if (ti >= 0 && tid == 32) {
+    int pos = -1;
+    long long slot = -1;
+    if (ti < tin) {
+      if (!err_view && ti < P) pos = ti;
+      else if (!err_view && ti < P + Tq) pos = (int)(ctx - Tq + (ti - P));
+      if (pos < 0 || pos >= a.max_ctx) {
+        if (!err_view) dev_fail(a.status, PIC_DEV_BAD_POSITION, b);
+        pos = -1;
+      } else {
+        const int page = a.block_table[(size_t)b * a.max_pages + pos / 16];
+        if (page < 0 || page >= a.num_pages) dev_fail(a.status, PIC_DEV_BAD_PAGE, b);
+        else slot = (long long)page * 16 + pos % 16;
+      }
+    }
+    s_tpos = pos;
+    s_tslot = slot;
+  }
+
+  // ---- this page: slot, token map, document of each position (warp 0)
+  if (has_page && tid < kTok) {
     const long long t = t0 + tid;
     long long sl = -1, tm = -1, src = -1;
     int k = 0;
@@ -313,7 +332,7 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
         tm = ((long long)lo << 40) | src;
       }
     }
-    if (layout_cta && t < a.max_ctx) {
+    if (t < a.max_ctx) {
       a.slot_mapping[(size_t)b * a.max_ctx + t] = sl;
       a.tok_map[(size_t)b * a.max_ctx + t] = tm;
     }
@@ -346,15 +365,31 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
   __syncthreads();
   const size_t hkv = a.hkv;
 
+  // ---- cos/sin at the token's position and of the documents this page touches
+  if (ti >= 0 && ti < tin)
+    for (int i = tid; i < HALF; i += kThreads) s_tcs[i] = rope_cos_sin(max(s_tpos, 0), rp.theta[i]);
+  const int k_first = s_first;
+  const int n_docs = k_first >= 0 ? min(s_last - s_first + 1, kTok) : 0;
+  for (int e = tid; e < n_docs * HALF; e += kThreads) {
+    const int j = e / HALF, i = e % HALF;
+    s_cs[j][i] = rope_cos_sin(rv.delta[k_first + j], rp.theta[i]);
+  }
+  __syncthreads();
+
+  // ---- the inline token: R(p) q packed, R(p) k and v into the cache
+  if (ti >= 0) {
+    if (ti < tin) token_store<D>(a, rp, b, a.append_layer, ti, s_tslot, s_tcs, tl);
+    else token_zero<D>(a, b, ti);
+  }
+
+  // The next kernel (attention) may be launched once every CTA got here: a
+  // release at the start of the kernel made a one-layer pass slower (its
+  // CTAs were then placed while this kernel still set up), one at the end
+  // gave away the overlap with this kernel's last stores.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
   // ---- relocate the document positions of this page, layer by layer
-  if (s_first >= 0) {
-    const int k_first = s_first;
-    const int n_docs = min(s_last - s_first + 1, kTok);
-    for (int e = tid; e < n_docs * HALF; e += kThreads) {  // cos/sin of the touched documents
-      const int j = e / HALF, i = e % HALF;
-      s_cs[j][i] = rope_cos_sin(rv.delta[k_first + j], rp.theta[i]);
-    }
-    __syncthreads();
+  if (k_first >= 0) {
     for (int layer = a.layer_begin; layer < a.layer_end; ++layer) {
     const __nv_bfloat16 *kp = a.k_pool + (size_t)layer * a.pool_tokens * hkv * D;
     const __nv_bfloat16 *vp = a.v_pool + (size_t)layer * a.pool_tokens * hkv * D;
@@ -413,8 +448,9 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
   }
 
   __syncthreads();
-  if (tid == 0 && rv.err) dev_fail(a.status, rv.err, b);
-  if (lead && tid == 0) a.ctx_len[b] = rv.err ? -1 : (int32_t)ctx;
+  const int fin = rv.err ? rv.err : (bad_tin ? PIC_DEV_BAD_POSITION : 0);
+  if (tid == 0 && fin) dev_fail(a.status, fin, b);
+  if (lead && tid == 0) a.ctx_len[b] = fin ? -1 : (int32_t)ctx;
 }
 
 }  // namespace
@@ -536,7 +572,7 @@ extern "C" pic_status_t pic_link(
   a.qpack = static_cast<__nv_bfloat16 *>(workspace);
   a.status = status;
 
-  dim3 grid((unsigned)(a.n_pages + (do_append ? a.t_slots : 0)), batch);
+  dim3 grid((unsigned)(do_append ? std::max(a.n_pages, a.t_slots) : a.n_pages), batch);
   const dim3 block(kThreads);
   cudaError_t e;
   if (geom->head_dim == 128)

@@ -148,7 +148,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tbase = *tmem_slot;
-  pdl_entry();
+  asm volatile("griddepcontrol.wait;" ::: "memory");  // the kernel before has finished
   auto release_and_exit = [&]() {  // a CTA without work frees its TMEM
     tc_fence_before();
     __syncthreads();
@@ -503,6 +503,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   }
+  // Release the dependent launch (the split merge, or the next layer's
+  // append) only now: released at the start, it made the pass slower.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   tc_fence_before();
   __syncthreads();

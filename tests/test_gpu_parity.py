@@ -36,6 +36,12 @@ SMALL = {
                               head_dim=128, rope_base=5e5, batch=2, pool_docs=3,
                               docs_per_request=2, doc_len=(200, 400), prefix_len=(8, 8),
                               query_len=5, decode_steps=2),
+    # prefix rows fill four of five query pairs: the split plan gives them one
+    # CTA each and the rest to the pair that sees the documents
+    "long_prefix": custom_spec(name="long_prefix", layers=1, q_heads=32, kv_heads=8,
+                               head_dim=128, rope_base=5e5, batch=1, pool_docs=4,
+                               docs_per_request=3, doc_len=(400, 600), prefix_len=(300, 300),
+                               query_len=20, decode_steps=1),
     "no_docs": custom_spec(name="no_docs", layers=1, q_heads=4, kv_heads=1, head_dim=64,
                            rope_base=1e4, batch=2, pool_docs=1, docs_per_request=0,
                            doc_len=(10, 10), prefix_len=(3, 30), query_len=9, decode_steps=1),
