@@ -66,18 +66,26 @@ __global__ void __launch_bounds__(kThreads)
   const int split = blockIdx.x, hk = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gid = lane >> 2, tig = lane & 3;
-  const int pos = p.pos[b] + p.pos_offset;
-  const int npages = pos >= 0 ? pos / 16 + 1 : 0;
-  const int pg_begin = split * p.pages_per_split;
-  const int pg_end = min(npages, pg_begin + p.pages_per_split);
-  const int32_t *bt = p.block_table + (size_t)b * p.max_pages;
 
+  // set-up that reads nothing another kernel writes, then wait for the
+  // kernel before (programmatic dependent launch)
   if (threadIdx.x == 0) {
     for (int i = 0; i < kWarps * NSTG; ++i) mbar_init(sbase + L::kBar + 8 * i, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
+  if (lane == 0) {
+    prefetch_tmap(&tm_k);
+    prefetch_tmap(&tm_v);
+  }
   __syncthreads();
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+
+  const int pos = p.pos[b] + p.pos_offset;
+  const int npages = pos >= 0 ? pos / 16 + 1 : 0;
+  const int pg_begin = split * p.pages_per_split;
+  const int pg_end = min(npages, pg_begin + p.pages_per_split);
+  const int32_t *bt = p.block_table + (size_t)b * p.max_pages;
 
   const uint32_t wbase = sbase + warp * L::kWarpBytes;
   auto full = [&](int s) { return sbase + L::kBar + 8u * (uint32_t)(warp * NSTG + s); };
@@ -104,11 +112,8 @@ __global__ void __launch_bounds__(kThreads)
       tma_load_2d(dst + L::kPage + pn * 2048, &tm_v, pn * 64, y, full(s));
     }
   };
-  if (lane == 0) {
-    prefetch_tmap(&tm_k);
-    prefetch_tmap(&tm_v);
+  if (lane == 0)
     for (int i = 0; i < min(cw, NSTG); ++i) issue(i);
-  }
 
   // query fragments (B operand of S^T = K q^T): heads nt*8 + gid of the group
   uint32_t qb[NT][KS][2];
@@ -270,10 +275,13 @@ __global__ void __launch_bounds__(kThreads)
       }
     }
   }
+  // release the dependent launch (merge, or the next layer's append) last
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 template <int D>
 __global__ void decode_combine_kernel(Params p) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int h = blockIdx.x, b = blockIdx.y, lane = threadIdx.x;
   const size_t hrow = (size_t)b * p.Hq + h;
   const int S = p.splits;
@@ -312,6 +320,7 @@ struct AppendArgs {
 template <int D>
 __global__ void __launch_bounds__(128) decode_append_kernel(AppendArgs a, RopeParams rp) {
   constexpr int HALF = D / 2, KC = D / 16, VC = D / 8;
+  pdl_entry();
   const int b = blockIdx.x, tid = threadIdx.x;
   __shared__ float2 cs[HALF];
   const int pos = a.pos[b] + a.pos_offset;
@@ -384,7 +393,8 @@ cudaError_t launch_attn(dim3 grid, cudaStream_t stream, const CUtensorMap &tk,
   cudaError_t e = cudaFuncSetAttribute(decode_attn_kernel<D, NT>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  decode_attn_kernel<D, NT><<<grid, kThreads, smem, stream>>>(tk, tv, pp);
+  e = launch_dependent(decode_attn_kernel<D, NT>, grid, dim3(kThreads), smem, stream, tk, tv, pp);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
@@ -464,8 +474,12 @@ extern "C" pic_status_t pic_attend_decode(const pic_geom_t *geom, int32_t layer,
   aa.v_cache = static_cast<__nv_bfloat16 *>(v_cache) + (size_t)layer * layer_elems;
   aa.qrot = reinterpret_cast<__nv_bfloat16 *>(ws);
   aa.status = status;
-  if (D == 128) decode_append_kernel<128><<<batch, 128, 0, stream>>>(aa, rp);
-  else decode_append_kernel<64><<<batch, 128, 0, stream>>>(aa, rp);
+  {
+    const cudaError_t ae =
+        D == 128 ? launch_dependent(decode_append_kernel<128>, dim3(batch), dim3(128), 0, stream, aa, rp)
+                 : launch_dependent(decode_append_kernel<64>, dim3(batch), dim3(128), 0, stream, aa, rp);
+    if (ae != cudaSuccess) return cuda_fail(ae, "decode append launch");
+  }
 
   CUtensorMap tk, tv;
   st = encode_tmap_2d(&tk, k_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
@@ -499,8 +513,10 @@ extern "C" pic_status_t pic_attend_decode(const pic_geom_t *geom, int32_t layer,
   if (e != cudaSuccess) return cuda_fail(e, "pic_attend_decode attention launch");
   if (pl.splits > 1) {
     dim3 cgrid(geom->num_q_heads, batch);
-    if (D == 128) decode_combine_kernel<128><<<cgrid, 32, 0, stream>>>(pp);
-    else decode_combine_kernel<64><<<cgrid, 32, 0, stream>>>(pp);
+    const cudaError_t ce =
+        D == 128 ? launch_dependent(decode_combine_kernel<128>, cgrid, dim3(32), 0, stream, pp)
+                 : launch_dependent(decode_combine_kernel<64>, cgrid, dim3(32), 0, stream, pp);
+    if (ce != cudaSuccess) return cuda_fail(ce, "decode merge launch");
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_attend_decode launch");
@@ -630,8 +646,12 @@ extern "C" pic_status_t pic_attend_decode_noalloc(const pic_geom_t *geom, int32_
   aa.v_cache = static_cast<__nv_bfloat16 *>(v_cache) + (size_t)layer * layer_elems;
   aa.qrot = reinterpret_cast<__nv_bfloat16 *>(ws);
   aa.status = status;
-  if (D == 128) decode_append_kernel<128><<<batch, 128, 0, stream>>>(aa, rp);
-  else decode_append_kernel<64><<<batch, 128, 0, stream>>>(aa, rp);
+  {
+    const cudaError_t ae =
+        D == 128 ? launch_dependent(decode_append_kernel<128>, dim3(batch), dim3(128), 0, stream, aa, rp)
+                 : launch_dependent(decode_append_kernel<64>, dim3(batch), dim3(128), 0, stream, aa, rp);
+    if (ae != cudaSuccess) return cuda_fail(ae, "decode append launch");
+  }
 
   CUtensorMap tk, tv;
   st = encode_tmap_2d(&tk, k_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
@@ -665,8 +685,10 @@ extern "C" pic_status_t pic_attend_decode_noalloc(const pic_geom_t *geom, int32_
   if (e != cudaSuccess) return cuda_fail(e, "pic_attend_decode_noalloc attention launch");
   if (pl.splits > 1) {
     dim3 cgrid(geom->num_q_heads, batch);
-    if (D == 128) decode_combine_kernel<128><<<cgrid, 32, 0, stream>>>(pp);
-    else decode_combine_kernel<64><<<cgrid, 32, 0, stream>>>(pp);
+    const cudaError_t ce =
+        D == 128 ? launch_dependent(decode_combine_kernel<128>, cgrid, dim3(32), 0, stream, pp)
+                 : launch_dependent(decode_combine_kernel<64>, cgrid, dim3(32), 0, stream, pp);
+    if (ce != cudaSuccess) return cuda_fail(ce, "decode merge launch");
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_attend_decode_noalloc launch");

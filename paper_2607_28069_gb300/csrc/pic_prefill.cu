@@ -641,6 +641,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                       const __grid_constant__ CUtensorMap tm_v,
                       const __grid_constant__ CUtensorMap tm_kp,
                       const __grid_constant__ CUtensorMap tm_vp, FParams fp) {
+  // programmatic dependent launch: the kernel before (the append) has finished
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   using L = Layout<D>;
   const Params &p = fp.base;
   constexpr int PANELS = D / 64;
@@ -1642,12 +1644,16 @@ extern "C" pic_status_t pic_attend_prefill_fused(
     const int smem = fused::Layout<128>::kAlloc;
     e = cudaFuncSetAttribute(fused::attn_fused_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused smem attribute");
-    fused::attn_fused_kernel<128><<<grid, fused::kThreads, smem, stream>>>(tq, tk, tv, tkp, tvp, fp);
+    e = launch_dependent(fused::attn_fused_kernel<128>, grid, dim3(fused::kThreads), smem, stream,
+                         tq, tk, tv, tkp, tvp, fp);
+    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused launch");
   } else {
     const int smem = fused::Layout<64>::kAlloc;
     e = cudaFuncSetAttribute(fused::attn_fused_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused smem attribute");
-    fused::attn_fused_kernel<64><<<grid, fused::kThreads, smem, stream>>>(tq, tk, tv, tkp, tvp, fp);
+    e = launch_dependent(fused::attn_fused_kernel<64>, grid, dim3(fused::kThreads), smem, stream,
+                         tq, tk, tv, tkp, tvp, fp);
+    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused launch");
   }
   if (pl.splits > 1) {
     const long long crows = (long long)batch * Hkv * pl.m_tiles * BM;
