@@ -675,7 +675,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (r0 >= rows) return;
   const int r_last = min(r0 + BM, rows) - 1;
   const int32_t *ipos = p.inline_pos + (size_t)b * p.max_inline;
-  const int kmin = ipos[r0 / p.G];
   const int kmax = ipos[r_last / p.G];
 
   // ---- per-document metadata into shared memory (all threads)
