@@ -275,6 +275,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (leader) mbar_wait(bar(B_Q), 0, abort_flag, p.status, detail);
     __syncwarp();
     tc_fence_after();
+    // Matrix descriptors: one base per operand region.  A ring stage, a query
+    // tile or a k-step only moves the start address, which sits in the low 14
+    // bits as address >> 4; shared addresses stay below 256 KB, so adding
+    // (offset >> 4) never carries out of the field.  Built once here, each
+    // MMA costs the issuer an add instead of a full descriptor.
+    const uint64_t dQ = sdesc_sw128(sbase + L::kQ, 16, 1024);
+    const uint64_t dK = sdesc_sw128(sbase + L::kK, 16, kGroupStride);
+    const uint64_t dV = sdesc_sw128(sbase + L::kV, kPanelOff, kGroupStride);
     for (int j = 0; j <= n; ++j) {
       bool k_ready = false;
 #pragma unroll
@@ -287,11 +295,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           named_bar_sync(kNbPv + t, 64);
           tc_fence_after();
           if (leader && !*abort_flag) {
-            const uint32_t vb = sbase + L::kV + pst * L::kTile;
+            const uint64_t dv = dV + (uint64_t)((pst * L::kTile) >> 4);
 #pragma unroll
             for (int kk = 0; kk < BN / 16; ++kk)  // one page of 16 keys per MMA
-              mma_ts(tO, tS + kk * 8, sdesc_sw128(vb + kk * kPageBytes, kPanelOff, kGroupStride),
-                     IDESC_PV, (pj > 0 || kk > 0));
+              mma_ts(tO, tS + kk * 8, dv + (kk * kPageBytes) / 16, IDESC_PV, (pj > 0 || kk > 0));
             if (t == ntile - 1) mma_commit(bar(B_VEMPTY + pst));  // last reader of V(j-1)
           }
         }
@@ -304,15 +311,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             k_ready = true;
           }
           if (leader && !*abort_flag) {
-            const uint32_t kb = sbase + L::kK + st * L::kTile;
-            const uint32_t qb = sbase + L::kQ + t * L::kQTile;
+            const uint64_t dk = dK + (uint64_t)((st * L::kTile) >> 4);
+            const uint64_t dq = dQ + (uint64_t)((t * L::kQTile) >> 4);
 #pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * (BM * 128) + (kk & 3) * 32;
-              mma_ss(tS, sdesc_sw128(qb + off, 16, 1024),
-                     sdesc_sw128(kb + (kk >> 2) * kPanelOff + (kk & 3) * 32, 16, kGroupStride),
-                     IDESC_QK, kk > 0);
-            }
+            for (int kk = 0; kk < D / 16; ++kk)
+              mma_ss(tS, dq + ((kk >> 2) * (BM * 128) + (kk & 3) * 32) / 16,
+                     dk + ((kk >> 2) * kPanelOff + (kk & 3) * 32) / 16, IDESC_QK, kk > 0);
             mma_commit(bar(B_SFULL + t));
             if (t == ntile - 1) mma_commit(bar(B_KEMPTY + st));  // last reader of K(j)
           }
@@ -814,6 +818,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t tS0 = tbase, tO = tbase + 256, tQd = tbase + 384;
       bool ok = mbar_wait(bar(F_Q), 0, abort_flag, p.status, detail);
       tc_fence_after();
+      // base descriptors; stages and k-steps add (offset >> 4) to the address field
+      const uint64_t dQ = sdesc_sw128(sbase + L::kQ, 16, 1024);
+      const uint64_t dK = sdesc_sw128(sbase + L::kK, 16, 1024);
+      const uint64_t dV = sdesc_sw128(sbase + L::kV, BN * 128, 1024);
       int dcount = -1;  // documents entered so far in this split
       for (int j = 0; ok && j <= n; ++j) {
         if (j < n) {
@@ -825,22 +833,18 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (!mbar_wait(bar(F_KFULL + st), (j / NST) & 1, abort_flag, p.status, detail)) break;
           tc_fence_after();
-          const uint32_t kb = sbase + L::kK + st * L::kTile;
+          const uint64_t dk = dK + (uint64_t)((st * L::kTile) >> 4);
           if (ti.doc < 0) {
 #pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * (BM * 128) + (kk & 3) * 32;
-              mma_ss(tS0 + sb * 128, sdesc_sw128(sbase + L::kQ + off, 16, 1024),
-                     sdesc_sw128(kb + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024), IDESC_QK,
-                     kk > 0);
-            }
+            for (int kk = 0; kk < D / 16; ++kk)
+              mma_ss(tS0 + sb * 128, dQ + ((kk >> 2) * (BM * 128) + (kk & 3) * 32) / 16,
+                     dk + ((kk >> 2) * (BN * 128) + (kk & 3) * 32) / 16, IDESC_QK, kk > 0);
           } else {
             const uint32_t qa = tQd + (dcount & 1) * 64;
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk)
-              mma_ts(tS0 + sb * 128, qa + kk * 8,
-                     sdesc_sw128(kb + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024), IDESC_QK,
-                     kk > 0);
+              mma_ts(tS0 + sb * 128, qa + kk * 8, dk + ((kk >> 2) * (BN * 128) + (kk & 3) * 32) / 16,
+                     IDESC_QK, kk > 0);
           }
           mma_commit(bar(F_SFULL + sb));
         }
@@ -849,11 +853,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!mbar_wait(bar(F_PFULL + pb), (pj >> 1) & 1, abort_flag, p.status, detail)) break;
           if (!mbar_wait(bar(F_VFULL + pst), (pj / NST) & 1, abort_flag, p.status, detail)) break;
           tc_fence_after();
-          const uint32_t vb = sbase + L::kV + pst * L::kTile;
+          const uint64_t dv = dV + (uint64_t)((pst * L::kTile) >> 4);
 #pragma unroll
           for (int kk = 0; kk < BN / 16; ++kk)
-            mma_ts(tO, tS0 + pb * 128 + kk * 8, sdesc_sw128(vb + kk * 16 * 128, BN * 128, 1024),
-                   IDESC_PV, (pj > 0 || kk > 0));
+            mma_ts(tO, tS0 + pb * 128 + kk * 8, dv + (kk * 16 * 128) / 16, IDESC_PV,
+                   (pj > 0 || kk > 0));
           mma_commit(bar(F_KVEMPTY + pst));
           mma_commit(bar(F_PFREE + pb));
         }
