@@ -15,7 +15,9 @@ What the path computes (SemPIC, "Background: Position-Independent Caching" and
 "Cache-hit serving"; appendix "Position-Independent Linking"):
 
 1. ``compose_layout``   the link operator R assigns final logical positions in
-                         the canonical order P, D_1, ..., D_m, Q (Eqs. 1-2) and
+                         the canonical order P, D_1, S_1, ..., D_m, S_m, Q
+                         (Eqs. 1-2; the post-document inline spans S_k may be
+                         empty) and
                          builds the token-level map from logical positions to
                          physical paged-cache slots (appendix, "Logical Layout
                          and Re-Rotation").
@@ -142,7 +144,7 @@ def rerotate_key(k: np.ndarray, a, b, theta: np.ndarray, style: str = HALF) -> n
 # --------------------------------------------------------------------------
 @dataclass
 class RequestLayout:
-    """Logical layout of one request (canonical order P, D_1..D_m, Q)."""
+    """Logical layout of one request (canonical order P, D_1, S_1, ..., D_m, S_m, Q)."""
 
     prefix_len: int
     doc_ids: list
@@ -152,28 +154,42 @@ class RequestLayout:
     query_len: int
     ctx_len: int
     slot_mapping: np.ndarray = field(repr=False)   # [ctx_len] int64
-    inline_pos: np.ndarray = field(repr=False)     # prefix then query positions
+    inline_pos: np.ndarray = field(repr=False)     # prefix, span and query positions, in order
+    span_start: list = field(default_factory=list)  # first logical position of each span S_k
+    span_len: list = field(default_factory=list)    # |S_k| (0: no span after D_k)
 
 
 def compose_layout(doc_len, doc_base_pos, doc_ids, prefix_len, query_len,
-                   block_table, page_size=16) -> RequestLayout:
-    """Assign logical positions in the order P, D_1..D_m, Q and map them to slots.
+                   block_table, page_size=16, span_len=None) -> RequestLayout:
+    """Assign logical positions in the order P, D_1, S_1, ..., D_m, S_m, Q and
+    map them to slots.
 
     Walks the request from position 0: the prefix takes P positions, each
-    document D_k takes the next n_k positions (its target offset), the query
-    takes the final Tq positions.  A document cached at base position base_k
-    therefore moves by delta_k = offset_k - base_k.  Logical position t lives
-    in physical slot block_table[t // page_size] * page_size + t % page_size.
+    document D_k takes the next n_k positions (its target offset) and its
+    post-document inline span S_k the next |S_k| (``span_len[k]``, default 0),
+    the query takes the final Tq positions.  A document cached at base
+    position base_k therefore moves by delta_k = offset_k - base_k.  The
+    inline tokens (prefix, spans, query, in this order) keep their own
+    positions.  Logical position t lives in physical slot
+    block_table[t // page_size] * page_size + t % page_size.
     """
+    if span_len is None:
+        span_len = [0] * len(doc_ids)
+    if len(span_len) != len(doc_ids):
+        raise ValueError("one span length per document")
     pos = int(prefix_len)
-    offsets, deltas = [], []
-    for d in doc_ids:
+    offsets, deltas, span_start = [], [], []
+    for d, s in zip(doc_ids, span_len):
         n = int(doc_len[d])
         if n <= 0:
             raise ValueError("document length must be positive")
+        if int(s) < 0:
+            raise ValueError("span length must not be negative")
         offsets.append(pos)
         deltas.append(pos - int(doc_base_pos[d]))
         pos += n
+        span_start.append(pos)
+        pos += int(s)
     query_start = pos
     ctx = pos + int(query_len)
     n_pages = -(-ctx // page_size)
@@ -182,9 +198,12 @@ def compose_layout(doc_len, doc_base_pos, doc_ids, prefix_len, query_len,
     slots = np.empty(ctx, dtype=np.int64)
     for t in range(ctx):
         slots[t] = int(block_table[t // page_size]) * page_size + t % page_size
-    inline_pos = np.concatenate([np.arange(prefix_len), np.arange(query_start, ctx)]).astype(np.int64)
+    inline_pos = np.concatenate(
+        [np.arange(prefix_len)] + [np.arange(a, a + int(s)) for a, s in zip(span_start, span_len)]
+        + [np.arange(query_start, ctx)]).astype(np.int64)
     return RequestLayout(int(prefix_len), list(doc_ids), offsets, deltas, query_start,
-                         int(query_len), ctx, slots, inline_pos)
+                         int(query_len), ctx, slots, inline_pos, span_start,
+                         [int(s) for s in span_len])
 
 
 # --------------------------------------------------------------------------
@@ -196,7 +215,7 @@ def relocate_docs(layout: RequestLayout, k_docs, v_docs, doc_base_pos, theta, st
     ``k_docs[i]`` / ``v_docs[i]`` hold document layout.doc_ids[i] as compiled
     in isolation, shape [n_i, Hkv, d].  Token j of doc k sits at base position
     base_k + j and moves to offset_k + j (Eq. 3).  Returns the keys and values
-    of the document span [P, P+N) in logical order, float64.
+    of all documents in order (concatenated), float64.
     """
     ks, vs = [], []
     for i, d in enumerate(layout.doc_ids):
@@ -214,21 +233,30 @@ def dense_context(layout: RequestLayout, k_docs, v_docs, doc_base_pos,
                   k_inline, v_inline, theta, style=HALF, storage=None):
     """Keys/values of the whole request indexed by logical position.
 
-    Inline tokens (prefix then query, ``k_inline`` [P+Tq, Hkv, d] un-rotated)
-    get RoPE at their own logical positions; documents are relocated with
-    Eq. 3.  Returns (K, V) of shape [ctx, Hkv, d].  storage="bf16" rounds the
-    rotated keys to bf16, as a bf16 cache holds them (values already are).
+    Inline tokens (prefix, spans, query, ``k_inline`` [P+S+Tq, Hkv, d]
+    un-rotated) get RoPE at their own logical positions and are placed
+    there; documents are relocated with Eq. 3 and placed at their offsets.
+    Every position is filled exactly once.  Returns (K, V) of shape
+    [ctx, Hkv, d].  storage="bf16" rounds the rotated keys to bf16, as a bf16
+    cache holds them (values already are).
     """
-    P = layout.prefix_len
-    k_rot_inline = rotary(k_inline, layout.inline_pos[:, None], theta, style)
+    k_inline = np.asarray(k_inline, np.float64)
+    ctx, (_, H, d) = layout.ctx_len, k_inline.shape
+    K, V = np.zeros((ctx, H, d)), np.zeros((ctx, H, d))
+    filled = np.zeros(ctx, dtype=np.int64)
+    ip = layout.inline_pos
+    K[ip] = rotary(k_inline, ip[:, None], theta, style)
+    V[ip] = np.asarray(v_inline, np.float64)
+    filled[ip] += 1
     kd, vd = relocate_docs(layout, k_docs, v_docs, doc_base_pos, theta, style)
-    parts_k = [k_rot_inline[:P]] + ([kd] if kd is not None else []) + [k_rot_inline[P:]]
-    parts_v = [np.asarray(v_inline[:P], np.float64)] + ([vd] if vd is not None else []) \
-        + [np.asarray(v_inline[P:], np.float64)]
-    K = _store(np.concatenate(parts_k, 0), storage)
-    V = np.concatenate(parts_v, 0)
-    assert K.shape[0] == layout.ctx_len
-    return K, V
+    at = 0
+    for i, off in enumerate(layout.doc_offset):
+        n = k_docs[i].shape[0]
+        K[off:off + n], V[off:off + n] = kd[at:at + n], vd[at:at + n]
+        filled[off:off + n] += 1
+        at += n
+    assert (filled == 1).all(), "every logical position holds exactly one token"
+    return _store(K, storage), V
 
 
 def scatter_to_pages(layout: RequestLayout, K, V, k_cache, v_cache, page_size=16):
@@ -298,8 +326,8 @@ def cache_hit_prefill(layout: RequestLayout, k_docs, v_docs, doc_base_pos,
                       storage=None):
     """Cache hit: relocate the docs, RoPE the inline tokens, attend.
 
-    ``q_inline`` [P+Tq, Hq, d], ``k_inline`` / ``v_inline`` [P+Tq, Hkv, d] are
-    the un-rotated projections of the inline tokens (prefix then query).
+    ``q_inline`` [T, Hq, d], ``k_inline`` / ``v_inline`` [T, Hkv, d] are the
+    un-rotated projections of the T inline tokens (prefix, spans, query).
     Returns the attention output of every inline token, plus the dense (K, V)
     context the attention read.  storage="bf16": rotated keys and queries are
     rounded to bf16 before the (float64) attention.

@@ -226,6 +226,87 @@ def test_compose_layout_brute_force_properties():
         assert lay.doc_offset == sorted(lay.doc_offset)
 
 
+def _layout_from_golden(g, fn=None):
+    fn = fn or O.compose_layout
+    return fn(g["doc_len"], g["doc_base"], g["doc_order"], g["prefix_len"][0], g["query_len"][0],
+              g["block_table"], g["page_size"][0], span_len=g["span_len"])
+
+
+def test_compose_layout_with_spans_matches_hand_enumeration():
+    g = _read_golden("spans_layout.txt")
+    lay = _layout_from_golden(g)
+    assert lay.doc_offset == g["doc_offset"]
+    assert lay.doc_delta == g["doc_delta"]
+    assert lay.span_start == g["span_start"]
+    assert lay.query_start == g["query_start"][0]
+    assert lay.ctx_len == g["ctx"][0]
+    assert list(lay.inline_pos) == g["inline_pos"]
+    for t, s in g["slot"]:
+        assert lay.slot_mapping[t] == s
+
+
+def test_pins_catch_planted_span_layout_mistakes():
+    """Two plausible misreadings of the canonical order, planted in copies of
+    the layout: documents packed back to back with every span after the last
+    one, and spans placed before their documents."""
+    def spans_at_end(doc_len, doc_base_pos, doc_ids, P, Tq, bt, page_size=16, span_len=None):
+        # the spans' tokens treated as part of the query, after the last document
+        return PO.compose_layout(doc_len, doc_base_pos, doc_ids, P, Tq + sum(span_len), bt,
+                                 page_size)
+
+    def spans_before(doc_len, doc_base_pos, doc_ids, P, Tq, bt, page_size=16, span_len=None):
+        return PO.compose_layout(doc_len, doc_base_pos, doc_ids, P + span_len[0], Tq, bt,
+                                 page_size, span_len=list(span_len[1:]) + [0])
+
+    g = _read_golden("spans_layout.txt")
+    for mutant in (spans_at_end, spans_before):
+        lay = _layout_from_golden(g, mutant)
+        assert (lay.doc_offset != g["doc_offset"] or list(lay.inline_pos) != g["inline_pos"]), \
+            mutant.__name__
+
+
+def test_zero_spans_reduce_to_the_plain_layout():
+    rng = np.random.default_rng(11)
+    for _ in range(10):
+        n_pool = int(rng.integers(1, 7))
+        lens, base = rng.integers(1, 50, size=n_pool), rng.integers(0, 30, size=n_pool)
+        order = list(rng.permutation(n_pool))
+        P, Tq = int(rng.integers(0, 20)), int(rng.integers(1, 20))
+        bt = rng.permutation(100)
+        a = O.compose_layout(lens, base, order, P, Tq, bt, 16)
+        b = O.compose_layout(lens, base, order, P, Tq, bt, 16, span_len=[0] * len(order))
+        assert a.doc_offset == b.doc_offset and a.doc_delta == b.doc_delta
+        assert np.array_equal(a.inline_pos, b.inline_pos)
+        assert np.array_equal(a.slot_mapping, b.slot_mapping)
+
+
+def test_compose_layout_with_spans_brute_force_properties():
+    """Positions are a partition: each document holds a contiguous run right
+    after the previous document's span, and the inline positions are exactly
+    the positions no document holds, in increasing order (prefix, spans, query)."""
+    rng = np.random.default_rng(8)
+    for _ in range(20):
+        n_pool = int(rng.integers(1, 9))
+        lens, base = rng.integers(1, 70, size=n_pool), rng.integers(0, 50, size=n_pool)
+        order = list(rng.permutation(n_pool)[: int(rng.integers(1, n_pool + 1))])
+        spans = [int(x) for x in rng.integers(0, 12, size=len(order))]
+        P, Tq = int(rng.integers(0, 40)), int(rng.integers(1, 40))
+        ctx = P + int(lens[order].sum()) + sum(spans) + Tq
+        bt = rng.permutation(300)[: -(-ctx // 16) + 2]
+        lay = O.compose_layout(lens, base, order, P, Tq, bt, 16, span_len=spans)
+        assert lay.ctx_len == ctx
+        doc_at = np.zeros(ctx, bool)
+        expect = P
+        for i, d in enumerate(order):
+            assert lay.doc_offset[i] == expect
+            assert lay.doc_delta[i] == expect - base[d]
+            assert not doc_at[expect:expect + lens[d]].any()
+            doc_at[expect:expect + lens[d]] = True
+            expect += lens[d] + spans[i]
+        assert np.array_equal(lay.inline_pos, np.flatnonzero(~doc_at))
+        assert len(lay.inline_pos) == P + sum(spans) + Tq
+
+
 def test_compose_layout_rejects_bad_requests():
     with pytest.raises(ValueError):
         O.compose_layout([0], [0], [0], 4, 4, [0], 16)
@@ -295,18 +376,21 @@ def test_attention_key_permutation_invariance():
 
 
 # ----------------------------------------------------------- whole path ---
-def _tiny_request(base=(0, 0), P=16, lens=(64, 64), Tq=16, d=64, Hq=4, Hkv=1, seed=0):
+def _tiny_request(base=(0, 0), P=16, lens=(64, 64), Tq=16, d=64, Hq=4, Hkv=1, seed=0,
+                  spans=None):
     rng = np.random.default_rng(seed)
     theta = O.rope_frequencies(d, 1e4)
     raw = [rng.standard_normal((n, Hkv, d)) for n in lens]
     k_docs = [O.rotary(raw[i], (base[i] + np.arange(lens[i]))[:, None], theta) for i in range(len(lens))]
     v_docs = [rng.standard_normal((n, Hkv, d)) for n in lens]
-    ctx = P + sum(lens) + Tq
+    tin = P + (sum(spans) if spans else 0) + Tq
+    ctx = sum(lens) + tin
     bt = rng.permutation(-(-ctx // 16) + 2)
-    lay = O.compose_layout(list(lens), list(base), list(range(len(lens))), P, Tq, bt, 16)
-    q = rng.standard_normal((P + Tq, Hq, d))
-    k = rng.standard_normal((P + Tq, Hkv, d))
-    v = rng.standard_normal((P + Tq, Hkv, d))
+    lay = O.compose_layout(list(lens), list(base), list(range(len(lens))), P, Tq, bt, 16,
+                           span_len=spans)
+    q = rng.standard_normal((tin, Hq, d))
+    k = rng.standard_normal((tin, Hkv, d))
+    v = rng.standard_normal((tin, Hkv, d))
     return theta, raw, k_docs, v_docs, lay, q, k, v
 
 
@@ -323,6 +407,45 @@ def test_composed_cache_equals_cache_built_at_target_positions():
         assert np.array_equal(V[seg], v_docs[i])
     np.testing.assert_allclose(K[:16], rotary_by_complex(k[:16], np.arange(16)[:, None] + 0 * k[:16, :, 0],
                                                          theta, O.HALF), atol=1e-12)
+
+
+def test_composed_cache_with_spans_equals_direct_computation():
+    """With spans S_k between the documents, the stitched context is the
+    request computed in place: document keys rotated directly at their final
+    positions, span and query keys at theirs, values unchanged."""
+    theta, raw, k_docs, v_docs, lay, q, k, v = _tiny_request(base=(5, 11), lens=(37, 50),
+                                                             spans=[9, 4], seed=4)
+    K, V = O.dense_context(lay, k_docs, v_docs, [5, 11], k, v, theta)
+    expect_k = np.empty_like(K)
+    expect_v = np.empty_like(V)
+    for i in range(2):
+        pos = np.arange(lay.doc_offset[i], lay.doc_offset[i] + raw[i].shape[0])
+        expect_k[pos] = rotary_by_complex(raw[i], np.broadcast_to(pos[:, None], raw[i].shape[:2]),
+                                          theta, O.HALF)
+        expect_v[pos] = v_docs[i]
+    ip = lay.inline_pos
+    expect_k[ip] = rotary_by_complex(k, np.broadcast_to(ip[:, None], k.shape[:2]), theta, O.HALF)
+    expect_v[ip] = v
+    np.testing.assert_allclose(K, expect_k, atol=1e-9)
+    assert np.array_equal(V, expect_v)
+    assert list(ip[16:16 + 9]) == list(range(16 + 37, 16 + 37 + 9))    # S_1 right after D_1
+
+
+def test_span_tokens_do_not_see_later_documents():
+    """Frontier mask with spans: a span token's output does not change when a
+    later document's values change, and does change for an earlier one."""
+    theta, raw, k_docs, v_docs, lay, q, k, v = _tiny_request(lens=(30, 30), spans=[6, 3], seed=5)
+    (o1, _), _, _ = O.cache_hit_prefill(lay, k_docs, v_docs, [0, 0], q, k, v, theta, return_lse=True)
+    row = 16 + 2                                      # third token of S_1, before D_2
+    v_later = [v_docs[0], v_docs[1] + 5.0]
+    (o2, _), _, _ = O.cache_hit_prefill(lay, k_docs, v_later, [0, 0], q, k, v, theta,
+                                        return_lse=True)
+    np.testing.assert_array_equal(o1[row], o2[row])
+    v_earlier = [v_docs[0] + 5.0, v_docs[1]]
+    (o3, _), _, _ = O.cache_hit_prefill(lay, k_docs, v_earlier, [0, 0], q, k, v, theta,
+                                        return_lse=True)
+    assert np.abs(o1[row] - o3[row]).max() > 1.0
+    assert np.abs(o1[-1] - o2[-1]).max() > 1.0          # the query sees both
 
 
 def test_prefill_output_invariant_to_global_position_shift():
