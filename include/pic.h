@@ -46,7 +46,7 @@
 extern "C" {
 #endif
 
-#define PIC_ABI_VERSION 1
+#define PIC_ABI_VERSION 2
 
 typedef struct CUstream_st *pic_stream_t; /* identical to cudaStream_t */
 
@@ -106,35 +106,44 @@ pic_status_t pic_device_status(pic_stream_t stream, int32_t *code, int32_t *deta
  * token-level maps (Eqs. 1-2, "Background: Position-Independent Caching";
  * appendix "Logical Layout and Re-Rotation").
  *
- * Request b is laid out as prefix (positions 0..P_b-1), then its documents
- * in the order req_doc_ids[b][0..m_b-1], then Tq_b query tokens.  For its
- * k-th document (pool id i, length n_i):
- *     doc_offset[b][k] = P_b + sum_{k'<k} n_{ids[b][k']}
+ * Request b is laid out in the canonical order P, D_1, S_1, ..., D_m, S_m, Q
+ * (Eq. 1): the prefix (positions 0..P_b-1), then for k = 0..m_b-1 its k-th
+ * document (order req_doc_ids[b][..]) followed by that document's inline
+ * span of s_bk = span_len[b][k] tokens (a request-time span computed online,
+ * not a cached block; span_len NULL: every s_bk = 0), then Tq_b query
+ * tokens.  For its k-th document (pool id i, length n_i):
+ *     doc_offset[b][k] = P_b + sum_{k'<k} (n_{ids[b][k']} + s_bk')
  *     doc_delta[b][k]  = doc_offset[b][k] - doc_base_pos[i]
- * ctx_len[b] = P_b + sum_k n + Tq_b, and for 0 <= t < ctx_len[b]
+ * ctx_len[b] = P_b + sum_k (n + s_bk) + Tq_b, and for 0 <= t < ctx_len[b]
  *     slot_mapping[b][t] = block_table[b][t / page] * page + t % page
  *     tok_map[b][t] = (k << 40) | (doc_token_start[i] + t - doc_offset[b][k])
  *                     for a position t of the k-th document, -1 otherwise
  * (the source row in the pool and the document index of every position).
- * inline_pos[b][0..P_b+Tq_b-1] lists the inline tokens' logical positions:
- * 0..P_b-1 then ctx_len[b]-Tq_b .. ctx_len[b]-1.
+ * inline_pos[b][0..T_b-1], T_b = P_b + sum_k s_bk + Tq_b, lists the inline
+ * tokens' logical positions in this order: 0..P_b-1, then the positions of
+ * each span (doc_offset[b][k] + n .. + s_bk - 1, k ascending), then
+ * ctx_len[b]-Tq_b .. ctx_len[b]-1.  The inline projections that
+ * pic_append_inline and pic_link take are in the same order.
  *
  * Inputs (device): doc_len, doc_base_pos int32 [n_pool_docs]; doc_token_start
- *   int64 [n_pool_docs]; req_doc_ids int32 [batch][max_docs]; req_num_docs,
- *   prefix_len, query_len int32 [batch]; block_table int32 [batch][max_pages]
- *   (entries used must be in [0, num_pages)).  max_docs <= 8192.
+ *   int64 [n_pool_docs]; req_doc_ids int32 [batch][max_docs]; span_len int32
+ *   [batch][max_docs] or NULL; req_num_docs, prefix_len, query_len int32
+ *   [batch]; block_table int32 [batch][max_pages] (entries used must be in
+ *   [0, num_pages)).  max_docs <= 8192.
  * Outputs (device): doc_offset, doc_delta int32 [batch][max_docs] (entries
  *   k >= m_b are set to -1 / 0); slot_mapping, tok_map int64 [batch][max_ctx]
  *   (-1 beyond ctx_len); inline_pos int32 [batch][max_inline] (unused tail -1);
  *   ctx_len int32 [batch] (-1 for a request that failed a device check).
- * Device checks: doc id range, doc length > 0, ctx <= max_ctx,
- *   P + Tq <= max_inline, ceil(ctx / page) <= max_pages, page ids in range.
+ * Device checks: doc id range, doc length > 0, span length >= 0,
+ *   ctx <= max_ctx, T_b <= max_inline, ceil(ctx / page) <= max_pages, page ids
+ *   in range.
  */
 pic_status_t pic_compose(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
                          int32_t n_pool_docs, const int32_t *doc_len,
                          const int32_t *doc_base_pos, const int64_t *doc_token_start,
                          const int32_t *req_doc_ids, const int32_t *req_num_docs,
-                         const int32_t *prefix_len, const int32_t *query_len,
+                         const int32_t *span_len, const int32_t *prefix_len,
+                         const int32_t *query_len,
                          const int32_t *block_table, int32_t max_pages, int64_t num_pages,
                          int32_t max_ctx, int32_t max_inline, int32_t *doc_offset,
                          int32_t *doc_delta, int64_t *slot_mapping, int64_t *tok_map,
@@ -174,11 +183,13 @@ pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int32_t max_doc
  * those three calls, and every output -- the layout (doc_offset, doc_delta,
  * slot_mapping, tok_map, inline_pos, ctx_len), the stitched K/V of the
  * documents and of the appended inline tokens, and the packed queries at the
- * start of the prefill workspace -- is bit-identical to theirs.  Each CTA
- * handles one 16-position page of one request for one layer and derives the
- * layout of its page itself, so the three dependent chains of memory round
- * trips become one.  Requests with more than 256 documents (max_docs > 256)
- * run the three calls in order instead.
+ * start of the prefill workspace -- is bit-identical to theirs (span_len as
+ * for pic_compose).  Each CTA handles the positions of one page of one
+ * request (two pages when a token's K row has fewer than 1024 elements) for
+ * every layer in turn, plus one inline token slot, and derives the layout it
+ * needs itself, so the three dependent chains of memory round trips become
+ * one.  Requests with more than 256 documents (max_docs > 256) run the three
+ * calls in order instead.
  * workspace: the prefill workspace of pic_append_inline (only its leading
  *   packed-query part is written); may be NULL when append_layer < 0.
  * One launch (or the three calls' launches), asynchronous on `stream`;
@@ -187,8 +198,9 @@ pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int32_t max_doc
 pic_status_t pic_link(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
                       int32_t n_pool_docs, const int32_t *doc_len, const int32_t *doc_base_pos,
                       const int64_t *doc_token_start, const int32_t *req_doc_ids,
-                      const int32_t *req_num_docs, const int32_t *prefix_len,
-                      const int32_t *query_len, const int32_t *block_table, int32_t max_pages,
+                      const int32_t *req_num_docs, const int32_t *span_len,
+                      const int32_t *prefix_len, const int32_t *query_len,
+                      const int32_t *block_table, int32_t max_pages,
                       int64_t num_pages, int32_t max_ctx, int32_t max_inline, const void *k_pool,
                       const void *v_pool, int64_t pool_tokens, int32_t layer_begin,
                       int32_t layer_end, int32_t append_layer, const void *q, const void *k_new,

@@ -99,10 +99,10 @@ def load():
         "pic_abi_version": (I32, []),
         "pic_last_error": (ctypes.c_char_p, []),
         "pic_device_status": (I32, [P, P, P]),
-        "pic_compose": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, I32, I64, I32, I32,
+        "pic_compose": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, P, I32, I64, I32, I32,
                               P, P, P, P, P, P, P]),
         "pic_relocate": (I32, [G, I32, I32, P, P, I64, P, P, P, I32, I64, P, P, I32, I32, P]),
-        "pic_link": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, I32, I64, I32, I32, P, P, I64,
+        "pic_link": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, P, I32, I64, I32, I32, P, P, I64,
                            I32, I32, I32, P, P, P, P, P, P, P, P, P, P, P, P, P, SZ, P]),
         "pic_prefill_workspace_size": (SZ, [G, I32, I32, I32, I32]),
         "pic_append_inline": (I32, [G, I32, I32, I32, P, P, P, P, P, P, I32, I64, P, P, P, SZ,
@@ -174,7 +174,8 @@ def pic_device_status(stream=None):
 def pic_compose(geom: Geometry, doc_len, doc_base_pos, doc_token_start, req_doc_ids,
                 req_num_docs, prefix_len, query_len, block_table, num_pages: int, max_ctx: int,
                 max_inline: int, doc_offset, doc_delta, slot_mapping, tok_map, inline_pos,
-                ctx_len, stream=None):
+                ctx_len, stream=None, span_len=None):
+    """span_len: int32 [batch][max_docs] post-document inline span lengths, or None."""
     lib = load()
     g = geom._c()
     B, max_docs = req_doc_ids.shape
@@ -182,6 +183,7 @@ def pic_compose(geom: Geometry, doc_len, doc_base_pos, doc_token_start, req_doc_
         ctypes.byref(g), B, max_docs, doc_len.numel(), _ptr(doc_len, i32, "doc_len"),
         _ptr(doc_base_pos, i32, "doc_base_pos"), _ptr(doc_token_start, i64, "doc_token_start"),
         _ptr(req_doc_ids, i32, "req_doc_ids"), _ptr(req_num_docs, i32, "req_num_docs"),
+        _ptr(span_len, i32, "span_len", allow_none=True),
         _ptr(prefix_len, i32, "prefix_len"), _ptr(query_len, i32, "query_len"),
         _ptr(block_table, i32, "block_table"), block_table.shape[1], num_pages, max_ctx,
         max_inline, _ptr(doc_offset, i32, "doc_offset"), _ptr(doc_delta, i32, "doc_delta"),
@@ -208,9 +210,10 @@ def pic_link(geom: Geometry, doc_len, doc_base_pos, doc_token_start, req_doc_ids
              prefix_len, query_len, block_table, num_pages: int, max_ctx: int, max_inline: int,
              k_pool, v_pool, layer_begin: int, layer_end: int, append_layer: int, q, k_new, v_new,
              inline_len, k_cache, v_cache, doc_offset, doc_delta, slot_mapping, tok_map, inline_pos,
-             ctx_len, workspace, stream=None):
+             ctx_len, workspace, stream=None, span_len=None):
     """pic_compose + pic_relocate + pic_append_inline (append_layer, or none if < 0)
-    in one launch; q/k_new/v_new are the append layer's inline projections."""
+    in one launch; q/k_new/v_new are the append layer's inline projections;
+    span_len as for pic_compose."""
     lib = load()
     g = geom._c()
     B, max_docs = req_doc_ids.shape
@@ -219,6 +222,7 @@ def pic_link(geom: Geometry, doc_len, doc_base_pos, doc_token_start, req_doc_ids
         ctypes.byref(g), B, max_docs, doc_len.numel(), _ptr(doc_len, i32, "doc_len"),
         _ptr(doc_base_pos, i32, "doc_base_pos"), _ptr(doc_token_start, i64, "doc_token_start"),
         _ptr(req_doc_ids, i32, "req_doc_ids"), _ptr(req_num_docs, i32, "req_num_docs"),
+        _ptr(span_len, i32, "span_len", allow_none=True),
         _ptr(prefix_len, i32, "prefix_len"), _ptr(query_len, i32, "query_len"),
         _ptr(block_table, i32, "block_table"), block_table.shape[1], num_pages, max_ctx,
         max_inline, _ptr(k_pool, bf16, "k_pool"), _ptr(v_pool, bf16, "v_pool"), k_pool.shape[1],

@@ -39,7 +39,8 @@ struct LinkArgs {
   int append_layer;  // -1: no append
   int hq, hkv, G, R_pad, t_slots, n_pages;
   long long num_pages, pool_tokens;
-  const int32_t *doc_len, *doc_base, *ids, *num_docs, *prefix, *query, *block_table, *inline_len;
+  const int32_t *doc_len, *doc_base, *ids, *num_docs, *spans, *prefix, *query, *block_table,
+      *inline_len;
   const int64_t *doc_start;
   int32_t *doc_offset, *doc_delta, *inline_pos, *ctx_len;
   int64_t *slot_mapping, *tok_map;
@@ -102,19 +103,30 @@ struct ReqView {
   int off[kMaxLinkDocs];
   long long start[kMaxLinkDocs];
   int delta[kMaxLinkDocs];
-  long long total;
+  int len[kMaxLinkDocs];   // document length
+  int sin[kMaxLinkDocs];   // inline index of the first token of the span after the document
+  long long total;         // document and span tokens
+  long long n_span;        // span tokens
   int err;
 };
 
-// Document offsets and deltas of request b (one block scan, m <= kThreads),
-// with pic_compose's checks; the lead CTA writes doc_offset / doc_delta.
-// Returns ctx (P + document tokens + Tq); rv.err holds the first check failed.
+// Document offsets and deltas of request b (block scans over the document and
+// span lengths, m <= kThreads), with pic_compose's checks; the lead CTA
+// writes doc_offset / doc_delta.  Returns ctx (P + document and span tokens +
+// Tq); rv.err holds the first check failed.
 __device__ long long request_view(const LinkArgs &a, int b, int P, int Tq, int m, bool lead,
                                   ReqView &rv) {
   const int tid = threadIdx.x;
-  long long n = 0, base = 0, start = 0;
+  long long n = 0, sp = 0, base = 0, start = 0;
   if (tid < m) {
     const int id = a.ids[(size_t)b * a.max_docs + tid];
+    if (a.spans) {
+      sp = a.spans[(size_t)b * a.max_docs + tid];
+      if (sp < 0) {
+        atomicCAS(&rv.err, 0, PIC_DEV_BAD_REQUEST);
+        sp = 0;
+      }
+    }
     if (id < 0 || id >= a.n_pool) {
       atomicCAS(&rv.err, 0, PIC_DEV_BAD_DOC_ID);
     } else {
@@ -127,18 +139,24 @@ __device__ long long request_view(const LinkArgs &a, int b, int P, int Tq, int m
       }
     }
   }
-  const long long incl = scan256(n, rv.warp_tot);
-  const long long off = P + incl - n;
+  const long long incl = scan256(n + sp, rv.warp_tot);
+  const long long off = P + incl - (n + sp);
+  const long long sincl = scan256(sp, rv.warp_tot);
   if (tid < m) {
     rv.off[tid] = (int32_t)off;
     rv.start[tid] = start;
     rv.delta[tid] = (int32_t)(off - base);
+    rv.len[tid] = (int32_t)n;
+    rv.sin[tid] = (int32_t)(P + sincl - sp);
     if (lead) {
       a.doc_offset[(size_t)b * a.max_docs + tid] = (int32_t)off;
       a.doc_delta[(size_t)b * a.max_docs + tid] = (int32_t)(off - base);
     }
   }
-  if (tid == kThreads - 1) rv.total = incl;
+  if (tid == kThreads - 1) {
+    rv.total = incl;
+    rv.n_span = sincl;
+  }
   if (lead)
     for (int k = m + tid; k < a.max_docs; k += kThreads) {
       a.doc_offset[(size_t)b * a.max_docs + k] = -1;
@@ -147,11 +165,29 @@ __device__ long long request_view(const LinkArgs &a, int b, int P, int Tq, int m
   __syncthreads();
   const long long ctx = (long long)P + rv.total + Tq;
   if (tid == 0) {
-    if (ctx > a.max_ctx || P + Tq > a.max_inline) atomicCAS(&rv.err, 0, PIC_DEV_CTX_OVERFLOW);
+    if (ctx > a.max_ctx || P + rv.n_span + Tq > a.max_inline)
+      atomicCAS(&rv.err, 0, PIC_DEV_CTX_OVERFLOW);
     else if ((ctx + 15) / 16 > a.max_pages) atomicCAS(&rv.err, 0, PIC_DEV_BLOCK_TABLE_SHORT);
   }
   __syncthreads();
   return ctx;
+}
+
+// Logical position of inline token i of the request (prefix, spans S_1..S_m,
+// query in this order), -1 past the inline tokens.
+__device__ int inline_position(const ReqView &rv, int i, int P, int Tq, int m, long long ctx) {
+  if (i < P) return i;
+  if (i < P + rv.n_span) {  // the last span starting at or before i holds it
+    int lo = 0, hi = m - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (rv.sin[mid] <= i) lo = mid;
+      else hi = mid - 1;
+    }
+    return rv.off[lo] + rv.len[lo] + (i - rv.sin[lo]);
+  }
+  if (i < P + rv.n_span + Tq) return (int)(ctx - Tq + (i - P - rv.n_span));
+  return -1;
 }
 
 // One inline token slot of the append layer (pic_append_inline's work), in
@@ -286,10 +322,10 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
     return;
   }
   const long long ctx = request_view(a, b, P, Tq, m, lead, rv);
-  const long long span_end = ctx - Tq;  // documents occupy [P, span_end)
+  const long long span_end = ctx - Tq;  // documents and spans occupy [P, span_end)
   const int err_view = rv.err;          // the document and size checks
-  // more inline tokens than prefix and query: reported by the lead CTA
-  const bool bad_tin = lead && a.append_layer >= 0 && tin > P + Tq;
+  // more inline tokens than prefix, spans and query: reported by the lead CTA
+  const bool bad_tin = lead && a.append_layer >= 0 && tin > P + rv.n_span + Tq;
   const int err = err_view ? err_view : (bad_tin ? PIC_DEV_BAD_POSITION : 0);
 
   // ---- the inline token's position and slot (one thread of warp 1)
@@ -297,8 +333,7 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
     int pos = -1;
     long long slot = -1;
     if (ti < tin) {
-      if (!err_view && ti < P) pos = ti;
-      else if (!err_view && ti < P + Tq) pos = (int)(ctx - Tq + (ti - P));
+      if (!err_view) pos = inline_position(rv, ti, P, Tq, m, ctx);
       if (pos < 0 || pos >= a.max_ctx) {
         if (!err_view) dev_fail(a.status, PIC_DEV_BAD_POSITION, b);
         pos = -1;
@@ -320,16 +355,18 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
     if (t < a.max_ctx && !err && t < ctx) {
       if (page_raw < 0 || page_raw >= a.num_pages) atomicCAS(&rv.err, 0, PIC_DEV_BAD_PAGE);
       else sl = (long long)page_raw * 16 + t % 16;
-      if (t >= P && t < span_end) {  // document token: last document whose offset <= t
+      if (t >= P && t < span_end) {  // last document whose offset <= t; its token unless in its span
         int lo = 0, hi = m - 1;
         while (lo < hi) {
           const int mid = (lo + hi + 1) >> 1;
           if (rv.off[mid] <= t) lo = mid;
           else hi = mid - 1;
         }
-        k = lo;
-        src = rv.start[lo] + (t - rv.off[lo]);
-        tm = ((long long)lo << 40) | src;
+        if (t < (long long)rv.off[lo] + rv.len[lo]) {
+          k = lo;
+          src = rv.start[lo] + (t - rv.off[lo]);
+          tm = ((long long)lo << 40) | src;
+        }
       }
     }
     if (t < a.max_ctx) {
@@ -355,12 +392,8 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
   }
   if (lead) {
     int32_t *ip = a.inline_pos + (size_t)b * a.max_inline;
-    for (int i = tid; i < a.max_inline; i += kThreads) {
-      int v = -1;
-      if (!err && i < P) v = i;
-      else if (!err && i < P + Tq) v = (int)(ctx - Tq + (i - P));
-      ip[i] = v;
-    }
+    for (int i = tid; i < a.max_inline; i += kThreads)
+      ip[i] = err ? -1 : inline_position(rv, i, P, Tq, m, ctx);
   }
   __syncthreads();
   const size_t hkv = a.hkv;
@@ -459,8 +492,9 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
 extern "C" pic_status_t pic_link(
     const pic_geom_t *geom, int32_t batch, int32_t max_docs, int32_t n_pool_docs,
     const int32_t *doc_len, const int32_t *doc_base_pos, const int64_t *doc_token_start,
-    const int32_t *req_doc_ids, const int32_t *req_num_docs, const int32_t *prefix_len,
-    const int32_t *query_len, const int32_t *block_table, int32_t max_pages, int64_t num_pages,
+    const int32_t *req_doc_ids, const int32_t *req_num_docs, const int32_t *span_len,
+    const int32_t *prefix_len, const int32_t *query_len, const int32_t *block_table,
+    int32_t max_pages, int64_t num_pages,
     int32_t max_ctx, int32_t max_inline, const void *k_pool, const void *v_pool,
     int64_t pool_tokens, int32_t layer_begin, int32_t layer_end, int32_t append_layer,
     const void *q, const void *k_new, const void *v_new, const int32_t *inline_len,
@@ -490,7 +524,8 @@ extern "C" pic_status_t pic_link(
   // More documents per request than one CTA scans: the three calls in order.
   if (max_docs > kMaxLinkDocs || max_docs == 0) {
     st = pic_compose(geom, batch, max_docs, n_pool_docs, doc_len, doc_base_pos, doc_token_start,
-                     req_doc_ids, req_num_docs, prefix_len, query_len, block_table, max_pages,
+                     req_doc_ids, req_num_docs, span_len, prefix_len, query_len, block_table,
+                     max_pages,
                      num_pages, max_ctx, max_inline, doc_offset, doc_delta, slot_mapping, tok_map,
                      inline_pos, ctx_len, stream);
     if (st == PIC_OK && max_docs > 0)
@@ -551,6 +586,7 @@ extern "C" pic_status_t pic_link(
   a.doc_base = doc_base_pos;
   a.ids = req_doc_ids;
   a.num_docs = req_num_docs;
+  a.spans = max_docs > 0 ? span_len : nullptr;
   a.prefix = prefix_len;
   a.query = query_len;
   a.block_table = block_table;

@@ -556,9 +556,9 @@ struct Layout {
   static constexpr int kK = kQ + BM * D * 2;
   static constexpr int kV = kK + NST * kTile;
   static constexpr int kMeta = kV + NST * kTile;
-  // seg_first[kMaxDocs + 3] int32, off/len/delta [kMaxDocs] int32, start [kMaxDocs] int64
+  // seg_first[2 kMaxDocs + 2] int32, off/len/delta [kMaxDocs] int32, start [kMaxDocs] int64
   static constexpr int kSegFirst = kMeta;
-  static constexpr int kOff = kSegFirst + (kMaxDocs + 4) * 4;
+  static constexpr int kOff = kSegFirst + (2 * kMaxDocs + 4) * 4;
   static constexpr int kLen = kOff + kMaxDocs * 4;
   static constexpr int kDelta = kLen + kMaxDocs * 4;
   static constexpr int kStart = kDelta + kMaxDocs * 4;
@@ -601,13 +601,19 @@ struct TileInfo {
   bool doc_first;  // first tile of its document
 };
 
+// Segments of a query tile's visible keys in logical order: cache segment
+// C_0 (the prefix), document D_0, C_1 (the inline span after D_0), D_1, ...,
+// D_{m-1}, C_m (the last span and the query).  Segment 2c is C_c, 2k+1 is
+// D_k; every range is clipped to the keys below kend.
 struct Seq {
   const int32_t *seg_first, *off, *len, *delta;
   const long long *start;
-  int m, P, q_lo, q_hi;  // prefix end, query span [q_lo, q_hi)
+  int m, kend;
+  __device__ int cache_lo(int c) const { return c == 0 ? 0 : min(off[c - 1] + len[c - 1], kend); }
+  __device__ int cache_hi(int c) const { return c < m ? min(off[c], kend) : kend; }
   __device__ TileInfo at(int t) const {
-    // segment containing global tile t (binary search over seg_first[0..m+2))
-    int lo = 0, hi = m + 1;
+    // segment containing global tile t (binary search over seg_first[0..2m+1))
+    int lo = 0, hi = 2 * m;
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
       if (seg_first[mid] <= t) lo = mid;
@@ -615,8 +621,8 @@ struct Seq {
     }
     const int j = t - seg_first[lo];
     TileInfo ti;
-    if (lo == 0 || lo == m + 1) {
-      const int a = lo == 0 ? 0 : q_lo, e = lo == 0 ? P : q_hi;
+    if ((lo & 1) == 0) {
+      const int a = cache_lo(lo >> 1), e = cache_hi(lo >> 1);
       ti.doc = -1;
       ti.cache_kt = a / BN + j;
       ti.key_base = ti.cache_kt * BN;
@@ -625,7 +631,7 @@ struct Seq {
       ti.prow = 0;
       ti.doc_first = false;
     } else {
-      const int k = lo - 1;
+      const int k = lo >> 1;
       ti.doc = k;
       ti.cache_kt = -1;
       ti.key_base = off[k] + j * BN;
@@ -699,26 +705,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   sq.delta = s_delta;
   sq.start = s_start;
   sq.m = m;
-  const int kend = kmax + 1;  // keys at or beyond kend are never visible here
-  sq.P = min(m > 0 ? s_off[0] : kend, kend);
-  sq.q_lo = m > 0 ? s_off[m - 1] + s_len[m - 1] : sq.P;
-  sq.q_hi = kend;
+  sq.kend = kmax + 1;  // keys at or beyond kend are never visible here
   if (threadIdx.x == 0) {  // tiles per segment, prefix sums (m <= kMaxDocs, serial is fine)
     int t = 0;
     auto cache_tiles = [&](int a, int e) { return e > a ? (e - 1) / BN - a / BN + 1 : 0; };
-    s_seg[0] = 0;
-    t += cache_tiles(0, sq.P);
-    for (int k = 0; k < m; ++k) {
-      s_seg[k + 1] = t;
-      const int e = min(s_off[k] + s_len[k], kend);
-      t += e > s_off[k] ? (e - s_off[k] + BN - 1) / BN : 0;
+    for (int c = 0; c <= m; ++c) {
+      s_seg[2 * c] = t;
+      t += cache_tiles(sq.cache_lo(c), sq.cache_hi(c));
+      if (c == m) break;
+      s_seg[2 * c + 1] = t;
+      const int e = min(s_off[c] + s_len[c], sq.kend);
+      t += e > s_off[c] ? (e - s_off[c] + BN - 1) / BN : 0;
     }
-    s_seg[m + 1] = t;
-    t += cache_tiles(sq.q_lo, sq.q_hi);
-    s_seg[m + 2] = t;
+    s_seg[2 * m + 1] = t;
   }
   __syncthreads();
-  const int n_all = s_seg[m + 2];
+  const int n_all = s_seg[2 * m + 1];
   const int per = (n_all + p.num_splits - 1) / p.num_splits;
   const int kv_begin = split * per;
   const int n = max(0, min(per, n_all - kv_begin));

@@ -70,13 +70,14 @@ class CacheHitPath:
         step instead of one per tensor.  The document pool stays resident."""
         wl = self.wl
         offs, total = [], 0
-        for name in self.REQUEST_FIELDS:
+        fields = self.REQUEST_FIELDS + (("span_len",) if wl.span_len is not None else ())
+        for name in fields:
             t = getattr(wl, name)
             offs.append(total)
             total += (t.numel() * t.element_size() + 255) // 256 * 256
         dev = torch.empty(total, dtype=torch.uint8, device=wl.k_pool.device)
         host = torch.empty(total, dtype=torch.uint8, pin_memory=True)
-        for name, off in zip(self.REQUEST_FIELDS, offs):
+        for name, off in zip(fields, offs):
             t = getattr(wl, name)
             n = t.numel() * t.element_size()
             view = dev[off:off + n].view(t.dtype).view(t.shape)
@@ -96,7 +97,8 @@ class CacheHitPath:
         pic_compose(self.geom, wl.doc_len, wl.doc_base_pos, wl.doc_token_start, wl.req_doc_ids,
                     wl.req_num_docs, wl.prefix_len, wl.query_len, wl.block_table, wl.num_pages,
                     self.max_ctx, self.max_inline, self.doc_offset, self.doc_delta,
-                    self.slot_mapping, self.tok_map, self.inline_pos, self.ctx_len)
+                    self.slot_mapping, self.tok_map, self.inline_pos, self.ctx_len,
+                    span_len=wl.span_len)
 
     # -- a2 + a3: per-document rotation and stitching, all layers, one launch
     def relocate(self, layer_begin: int = 0, layer_end: int | None = None):
@@ -119,7 +121,8 @@ class CacheHitPath:
                  wl.k_inline[append_layer] if app else None,
                  wl.v_inline[append_layer] if app else None, wl.inline_len if app else None,
                  self.k_cache, self.v_cache, self.doc_offset, self.doc_delta, self.slot_mapping,
-                 self.tok_map, self.inline_pos, self.ctx_len, self.ws_prefill if app else None)
+                 self.tok_map, self.inline_pos, self.ctx_len, self.ws_prefill if app else None,
+                 span_len=wl.span_len)
 
     # -- a4: RoPE + append of the inline tokens of one layer
     def append(self, layer: int):

@@ -42,6 +42,7 @@ class WorkloadSpec:
     fixed_order: Optional[tuple] = None   # explicit doc order for every request
     shared_all_docs: bool = False         # every request uses the whole pool
     page_size: int = PAGE
+    span_len: tuple = (0, 0)              # (lo, hi) inclusive: inline span S_k after each doc
     description: str = ""
 
 
@@ -106,12 +107,13 @@ class Workload:
     q_inline: torch.Tensor         # [L][B][Tin_max][Hq][d] bf16
     k_inline: torch.Tensor         # [L][B][Tin_max][Hkv][d] bf16
     v_inline: torch.Tensor
-    inline_len: torch.Tensor       # [B] int32
+    inline_len: torch.Tensor       # [B] int32 (prefix + span + query tokens)
     # decode tokens
     q_dec: Optional[torch.Tensor] = None   # [steps][L][B][Hq][d]
     k_dec: Optional[torch.Tensor] = None   # [steps][L][B][Hkv][d]
     v_dec: Optional[torch.Tensor] = None
     meta: dict = field(default_factory=dict)
+    span_len: Optional[torch.Tensor] = None   # [B][max_docs] int32 (0-padded), None: no spans
 
     @property
     def tin_max(self) -> int:
@@ -154,10 +156,16 @@ def generate(spec, device="cpu", gen_device=None, value_seed=0, select_seed=1) -
             docs.append(list(rng.choice(spec.pool_docs, spec.docs_per_request, replace=False)))
     plo, phi = spec.prefix_len
     prefixes = [int(plo) if plo == phi else int(rng.integers(plo, phi + 1)) for _ in range(B)]
+    # post-document inline spans S_k (drawn only when the spec asks for them,
+    # so the other workloads keep their draws)
+    slo, shi = spec.span_len
+    spans = [[0] * len(docs[b]) for b in range(B)]
+    if shi > 0:
+        spans = [[int(x) for x in rng.integers(slo, shi + 1, size=len(docs[b]))] for b in range(B)]
 
     # Page budget per request: prompt plus decode tokens.
-    need = [prefixes[b] + int(lens[docs[b]].sum()) + spec.query_len + spec.decode_steps
-            for b in range(B)]
+    need = [prefixes[b] + int(lens[docs[b]].sum()) + sum(spans[b]) + spec.query_len
+            + spec.decode_steps for b in range(B)]
     pages_per_req = [-(-n // spec.page_size) for n in need]
     num_pages = int(sum(pages_per_req))
     perm = rng.permutation(num_pages).astype(np.int32)
@@ -176,7 +184,7 @@ def generate(spec, device="cpu", gen_device=None, value_seed=0, select_seed=1) -
     gen.manual_seed(value_seed)
     k_pool = _randn_bf16((L, pool_tokens, Hkv, d), gen, gen_device)
     v_pool = _randn_bf16((L, pool_tokens, Hkv, d), gen, gen_device)
-    tin = [prefixes[b] + spec.query_len for b in range(B)]
+    tin = [prefixes[b] + sum(spans[b]) + spec.query_len for b in range(B)]
     tin_max = max(tin)
     q_in = _randn_bf16((L, B, tin_max, Hq, d), gen, gen_device)
     k_in = _randn_bf16((L, B, tin_max, Hkv, d), gen, gen_device)
@@ -202,7 +210,8 @@ def generate(spec, device="cpu", gen_device=None, value_seed=0, select_seed=1) -
         block_table=i32(bt), num_pages=num_pages, max_ctx=max(need),
         q_inline=mv(q_in), k_inline=mv(k_in), v_inline=mv(v_in), inline_len=i32(tin),
         q_dec=mv(qd), k_dec=mv(kd), v_dec=mv(vd),
-        meta={"docs": docs, "prefix": prefixes, "pool_tokens": pool_tokens},
+        meta={"docs": docs, "prefix": prefixes, "pool_tokens": pool_tokens, "spans": spans},
+        span_len=i32([x + [0] * (max_docs - len(x)) for x in spans]) if shi > 0 else None,
     )
 
 

@@ -33,7 +33,8 @@ def oracle_layout(wl, b: int):
     spec = wl.spec
     return O.compose_layout(wl.doc_len.cpu().numpy(), wl.doc_base_pos.cpu().numpy(),
                             wl.meta["docs"][b], int(wl.prefix_len[b]), spec.query_len,
-                            wl.block_table[b].cpu().numpy(), spec.page_size)
+                            wl.block_table[b].cpu().numpy(), spec.page_size,
+                            span_len=wl.meta["spans"][b])
 
 
 def theta_of(spec):

@@ -37,7 +37,7 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_version(lib):
-    assert pic.pic_abi_version() == 1
+    assert pic.pic_abi_version() == 2
 
 
 def _geom(**kw):
@@ -67,8 +67,8 @@ def _call_compose_with(geom):
     g = geom._c()
     null = ctypes.c_void_p(0)
     return pic.load().pic_compose(ctypes.byref(g), 1, 1, 1, null, null, null, null, null, null,
-                                  null, null, 1, 1, 16, 16, null, null, null, null, null, null,
-                                  null)
+                                  null, null, null, 1, 1, 16, 16, null, null, null, null, null,
+                                  null, null)
 
 
 def test_invalid_geometry_rejected_before_launch(lib):

@@ -42,6 +42,16 @@ SMALL = {
                                head_dim=128, rope_base=5e5, batch=1, pool_docs=4,
                                docs_per_request=3, doc_len=(400, 600), prefix_len=(300, 300),
                                query_len=20, decode_steps=1),
+    # post-document inline spans S_k (canonical order P, D_1, S_1, ..., D_m,
+    # S_m, Q), some of them empty
+    "spans_b2": custom_spec(name="spans_b2", layers=2, q_heads=8, kv_heads=2, head_dim=128,
+                            rope_base=5e5, batch=2, pool_docs=5, docs_per_request=4,
+                            doc_len=(20, 300), prefix_len=(0, 40), query_len=24,
+                            span_len=(0, 3), decode_steps=2),
+    "spans_d64": custom_spec(name="spans_d64", layers=1, q_heads=16, kv_heads=2, head_dim=64,
+                             rope_base=1e4, batch=2, pool_docs=6, docs_per_request=6,
+                             doc_len=(5, 130), prefix_len=(3, 17), query_len=9,
+                             span_len=(0, 150), decode_steps=1),
     "no_docs": custom_spec(name="no_docs", layers=1, q_heads=4, kv_heads=1, head_dim=64,
                            rope_base=1e4, batch=2, pool_docs=1, docs_per_request=0,
                            doc_len=(10, 10), prefix_len=(3, 30), query_len=9, decode_steps=1),
@@ -96,7 +106,8 @@ def test_compose_bit_exact(cuda_lib, name):
 
 
 @pytest.mark.parametrize("rope_style", [0, 1])
-@pytest.mark.parametrize("name", ["tiny", "llama8b_1layer", "ragged_b3", "d64_g8"])
+@pytest.mark.parametrize("name", ["tiny", "llama8b_1layer", "ragged_b3", "d64_g8", "spans_b2",
+                                  "spans_d64"])
 def test_stitched_cache(cuda_lib, name, rope_style):
     """Relocated doc keys within the K bar, values bit-exact, inline K rotated
     at their positions, inline V bit-exact -- all read back through the slots."""
@@ -170,7 +181,7 @@ def test_prefill_split_count_invariance(cuda_lib, splits):
     assert d <= 1e-2
 
 
-@pytest.mark.parametrize("name", ["gqa7_decode", "d64_g8", "g16_decode", "no_docs"])
+@pytest.mark.parametrize("name", ["gqa7_decode", "d64_g8", "g16_decode", "no_docs", "spans_b2"])
 @pytest.mark.parametrize("splits", [0, 1, 3])
 def test_decode_steps(cuda_lib, name, splits):
     wl, path, dec = run_path(name, decode_splits=splits)
@@ -277,7 +288,7 @@ def run_fused(name, splits=0, rope_style=0):
 
 
 @pytest.mark.parametrize("name", ["tiny", "llama8b_1layer", "ragged_b3", "gqa7_decode", "d64_g8",
-                                  "no_docs"])
+                                  "no_docs", "spans_b2", "spans_d64"])
 @pytest.mark.parametrize("splits", [0, 1, 3])
 def test_fused_prefill_matches_oracle(cuda_lib, name, splits):
     wl, path = run_fused(name, splits)
@@ -330,7 +341,7 @@ def test_packed_request_upload_gives_identical_results():
     """pack_request_inputs + upload (one host-to-device copy per request)
     must leave the pass's results bit-identical to the unpacked tensors."""
     from paper_2607_28069_gb300.pipeline import CacheHitPath
-    wl = generate(SMALL["ragged_b3"], device="cuda", gen_device="cpu")
+    wl = generate(SMALL["spans_b2"], device="cuda", gen_device="cpu")
     path = CacheHitPath(wl)
     path.ttft_pass()
     torch.cuda.synchronize()
@@ -347,7 +358,8 @@ def test_packed_request_upload_gives_identical_results():
 
 @pytest.mark.gpu
 @pytest.mark.parametrize("name,rope_style", [("tiny", 0), ("llama8b_1layer", 0), ("ragged_b3", 0),
-                                             ("ragged_b3", 1), ("d64_g8", 0), ("no_docs", 0)])
+                                             ("ragged_b3", 1), ("d64_g8", 0), ("no_docs", 0),
+                                             ("spans_b2", 0), ("spans_d64", 1)])
 def test_link_equals_separate_calls(name, rope_style):
     """pic_link (layout + relocation + first-layer append in one launch) gives
     bit-identical layout outputs, caches and prefill outputs to pic_compose,
