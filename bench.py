@@ -169,24 +169,31 @@ class ClockSampler:
 # ---------------------------------------------------------- work accounting
 def work_of(wl):
     """Algorithmic work of one TTFT pass (and one decode step), from the
-    request description: bytes for the HBM-bound rows, FLOPs for attention."""
+    request description: bytes for the HBM-bound rows, FLOPs for attention.
+    An inline token (prefix, post-document span or query) at logical position
+    p sees the p + 1 keys before and at it."""
     spec = wl.spec
     L, Hq, Hkv, d = spec.layers, spec.q_heads, spec.kv_heads, spec.head_dim
     lens = wl.doc_len.cpu().tolist()
     doc_tokens = sum(sum(lens[i] for i in docs) for docs in wl.meta["docs"])
     pairs = 0
     query_tokens = 0
+    inline_tokens = 0
     ctx = []
     for b, docs in enumerate(wl.meta["docs"]):
         P = wl.meta["prefix"][b]
-        N = sum(lens[i] for i in docs)
+        spans = wl.meta["spans"][b]
         Tq = spec.query_len
-        c = P + N + Tq
-        ctx.append(c)
         pairs += P * (P + 1) // 2                       # prefix rows see the prefix
-        pairs += Tq * (P + N) + Tq * (Tq + 1) // 2      # query rows see all before them
+        pos = P
+        for i, s in zip(docs, spans):
+            pos += lens[i]                              # the document, then its span
+            pairs += s * pos + s * (s + 1) // 2
+            pos += s
+        pairs += Tq * pos + Tq * (Tq + 1) // 2          # query rows see all before them
+        ctx.append(pos + Tq)
         query_tokens += Tq
-    inline_tokens = sum(wl.meta["prefix"]) + spec.batch * spec.query_len
+        inline_tokens += P + sum(spans) + Tq
     row_bytes = Hkv * d * 2
     return {
         "query_tokens": query_tokens,
@@ -224,7 +231,8 @@ def oracle_sample(workload, seconds):
         tin = int(wl.inline_len[b])
         t0 = time.perf_counter()
         lay = O.compose_layout(lens, wl.doc_base_pos.numpy(), docs, int(wl.prefix_len[b]),
-                               spec.query_len, wl.block_table[b].numpy(), spec.page_size)
+                               spec.query_len, wl.block_table[b].numpy(), spec.page_size,
+                               span_len=wl.meta["spans"][b])
         k_docs = [f64(wl.k_pool[0, starts[x]:starts[x] + lens[x]]) for x in docs]
         v_docs = [f64(wl.v_pool[0, starts[x]:starts[x] + lens[x]]) for x in docs]
         O.cache_hit_prefill(lay, k_docs, v_docs, wl.doc_base_pos.numpy(),

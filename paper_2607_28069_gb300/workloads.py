@@ -73,6 +73,14 @@ WORKLOADS = {
         description="32 layers, batch 4 requests of ~139k tokens: all 128 docs of a pool with "
                     "lengths U{128..2048}, each request in its own shuffled order, "
                     "512-token query chunk"),
+    # The 32-layer batch-8 workload with a request-time inline span S_k of
+    # 16-64 tokens after every document (canonical order P, D_1, S_1, ...,
+    # D_m, S_m, Q): ~640 more inline tokens per request.
+    "llama8b_32layer_b8_spans": WorkloadSpec(
+        "llama8b_32layer_b8_spans", 32, 32, 8, 128, 5e5, 8, 64, 16, (1024, 1024), (32, 128), 256,
+        span_len=(16, 64),
+        description="llama8b_32layer_b8 with an inline span of U{16..64} tokens after each "
+                    "document"),
     # Profiling-size slices of the full workloads (same per-layer shapes, fewer
     # layers / steps), so that one profiled launch moves more than L2 holds
     # while the process stays at a few GB of device memory.
