@@ -52,6 +52,14 @@ SMALL = {
                              rope_base=1e4, batch=2, pool_docs=6, docs_per_request=6,
                              doc_len=(5, 130), prefix_len=(3, 17), query_len=9,
                              span_len=(0, 150), decode_steps=1),
+    # boundary states around every document (header and trailer blocks of
+    # a boundary-conditioned cache), supplied as pool entries 0 and 1 and
+    # repeated in the request's order: H, D, T, H, D, T, ...
+    "boundary_blocks": custom_spec(name="boundary_blocks", layers=1, q_heads=8, kv_heads=2,
+                                   head_dim=128, rope_base=5e5, batch=2, pool_docs=5,
+                                   docs_per_request=9, doc_len=(3, 90), prefix_len=(5, 20),
+                                   query_len=12, fixed_order=(0, 2, 1, 0, 3, 1, 0, 4, 1),
+                                   span_len=(0, 4), decode_steps=1),
     "no_docs": custom_spec(name="no_docs", layers=1, q_heads=4, kv_heads=1, head_dim=64,
                            rope_base=1e4, batch=2, pool_docs=1, docs_per_request=0,
                            doc_len=(10, 10), prefix_len=(3, 30), query_len=9, decode_steps=1),
@@ -107,7 +115,7 @@ def test_compose_bit_exact(cuda_lib, name):
 
 @pytest.mark.parametrize("rope_style", [0, 1])
 @pytest.mark.parametrize("name", ["tiny", "llama8b_1layer", "ragged_b3", "d64_g8", "spans_b2",
-                                  "spans_d64"])
+                                  "spans_d64", "boundary_blocks"])
 def test_stitched_cache(cuda_lib, name, rope_style):
     """Relocated doc keys within the K bar, values bit-exact, inline K rotated
     at their positions, inline V bit-exact -- all read back through the slots."""
@@ -288,7 +296,7 @@ def run_fused(name, splits=0, rope_style=0):
 
 
 @pytest.mark.parametrize("name", ["tiny", "llama8b_1layer", "ragged_b3", "gqa7_decode", "d64_g8",
-                                  "no_docs", "spans_b2", "spans_d64"])
+                                  "no_docs", "spans_b2", "spans_d64", "boundary_blocks"])
 @pytest.mark.parametrize("splits", [0, 1, 3])
 def test_fused_prefill_matches_oracle(cuda_lib, name, splits):
     wl, path = run_fused(name, splits)
@@ -359,7 +367,8 @@ def test_packed_request_upload_gives_identical_results():
 @pytest.mark.gpu
 @pytest.mark.parametrize("name,rope_style", [("tiny", 0), ("llama8b_1layer", 0), ("ragged_b3", 0),
                                              ("ragged_b3", 1), ("d64_g8", 0), ("no_docs", 0),
-                                             ("spans_b2", 0), ("spans_d64", 1)])
+                                             ("spans_b2", 0), ("spans_d64", 1),
+                                             ("boundary_blocks", 0)])
 def test_link_equals_separate_calls(name, rope_style):
     """pic_link (layout + relocation + first-layer append in one launch) gives
     bit-identical layout outputs, caches and prefill outputs to pic_compose,
