@@ -85,6 +85,12 @@ typedef struct {
   double rope_base;      /* theta_i = rope_base^(-2i/d)                    */
   const double *inv_freq;/* nullable HOST pointer to d/2 frequencies that
                             replace rope_base^(-2i/d) (scaled RoPE)        */
+  const double *layer_inv_freq; /* nullable DEVICE pointer to [num_layers][d/2]
+                            frequencies, row l for layer l (a layer-specific
+                            rotary transform R_l, Eq. 3); overrides rope_base
+                            and inv_freq.  Values must be positive and finite
+                            (not checked); the caller keeps it alive while
+                            calls that use the geometry run.             */
 } pic_geom_t;
 
 /* Library version (PIC_ABI_VERSION of the build). */

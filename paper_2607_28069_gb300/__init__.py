@@ -57,6 +57,7 @@ class _Geom(ctypes.Structure):
         ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
         ("page_size", ctypes.c_int32), ("rope_style", ctypes.c_int32),
         ("rope_base", ctypes.c_double), ("inv_freq", ctypes.POINTER(ctypes.c_double)),
+        ("layer_inv_freq", ctypes.c_void_p),
     ]
 
 
@@ -70,14 +71,21 @@ class Geometry:
     page_size: int = 16
     rope_style: int = ROPE_HALF
     inv_freq: Optional[list] = None
+    # device float64 [num_layers][head_dim / 2]: a rotary table per layer
+    layer_inv_freq: Optional[torch.Tensor] = None
 
     def _c(self):
         g = _Geom(self.num_layers, self.num_q_heads, self.num_kv_heads, self.head_dim,
-                  self.page_size, self.rope_style, float(self.rope_base), None)
+                  self.page_size, self.rope_style, float(self.rope_base), None, None)
         if self.inv_freq is not None:
             arr = (ctypes.c_double * len(self.inv_freq))(*[float(x) for x in self.inv_freq])
             g.inv_freq = ctypes.cast(arr, ctypes.POINTER(ctypes.c_double))
             g._keep = arr  # keep the array alive with the struct
+        if self.layer_inv_freq is not None:
+            t = self.layer_inv_freq
+            if tuple(t.shape) != (self.num_layers, self.head_dim // 2):
+                raise ValueError("layer_inv_freq must be [num_layers][head_dim / 2]")
+            g.layer_inv_freq = _ptr(t, torch.float64, "layer_inv_freq")
         return g
 
 

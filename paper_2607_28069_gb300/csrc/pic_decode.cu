@@ -309,7 +309,7 @@ __global__ void decode_combine_kernel(Params p) {
 }
 
 struct AppendArgs {
-  int Hq, Hkv, max_pages, pos_offset;
+  int Hq, Hkv, max_pages, pos_offset, layer;
   long long num_pages;
   const __nv_bfloat16 *q, *k, *v;
   const int32_t *pos, *block_table;
@@ -334,7 +334,8 @@ __global__ void __launch_bounds__(128) decode_append_kernel(AppendArgs a, RopePa
       page = -1;
     }
   }
-  for (int i = tid; i < HALF; i += blockDim.x) cs[i] = rope_cos_sin(pos > 0 ? pos : 0, rp.theta[i]);
+  for (int i = tid; i < HALF; i += blockDim.x)
+    cs[i] = rope_cos_sin(pos > 0 ? pos : 0, rope_theta(rp, a.layer, i));
   __syncthreads();
   if (page >= 0) {
     const int r = pos & 15;
@@ -464,6 +465,7 @@ extern "C" pic_status_t pic_attend_decode(const pic_geom_t *geom, int32_t layer,
   aa.Hkv = Hkv;
   aa.max_pages = max_pages;
   aa.pos_offset = pos_offset;
+  aa.layer = layer;
   aa.num_pages = num_pages;
   aa.q = static_cast<const __nv_bfloat16 *>(q);
   aa.k = static_cast<const __nv_bfloat16 *>(k_new);
@@ -636,6 +638,7 @@ extern "C" pic_status_t pic_attend_decode_noalloc(const pic_geom_t *geom, int32_
   aa.Hkv = Hkv;
   aa.max_pages = max_pages;
   aa.pos_offset = pos_offset;
+  aa.layer = layer;
   aa.num_pages = num_pages;
   aa.q = static_cast<const __nv_bfloat16 *>(q);
   aa.k = static_cast<const __nv_bfloat16 *>(k_new);

@@ -30,13 +30,15 @@ pic_status_t check_geom(const pic_geom_t *g, double *theta);
 
 // RoPE parameters passed by value to kernels.
 struct RopeParams {
-  double theta[64];  // frequencies, d/2 <= 64
-  int half;          // d / 2
-  int style;         // PIC_ROPE_HALF / PIC_ROPE_INTERLEAVED
+  double theta[64];            // frequencies, d/2 <= 64
+  const double *layer_theta;   // device [num_layers][d/2] per-layer frequencies, or null
+  int half;                    // d / 2
+  int style;                   // PIC_ROPE_HALF / PIC_ROPE_INTERLEAVED
 };
 
 inline pic_status_t make_rope(const pic_geom_t *g, RopeParams *rp) {
   pic_status_t s = check_geom(g, rp->theta);
+  rp->layer_theta = g->layer_inv_freq;
   rp->half = g->head_dim / 2;
   rp->style = g->rope_style;
   return s;
@@ -80,6 +82,12 @@ PIC_DEV float2 rope_cos_sin(long long pos, double theta) {
   float s, c;
   sincosf((float)r, &s, &c);
   return make_float2(c, s);
+}
+
+// Frequency i of layer `layer`: the per-layer table when the geometry has
+// one, else the table shared by all layers.
+PIC_DEV double rope_theta(const RopeParams &rp, int layer, int i) {
+  return rp.layer_theta ? rp.layer_theta[(size_t)layer * rp.half + i] : rp.theta[i];
 }
 
 PIC_DEV void unpack8(const uint4 &v, float *f) {

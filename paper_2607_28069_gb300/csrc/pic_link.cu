@@ -400,13 +400,17 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
 
   // ---- cos/sin at the token's position and of the documents this page touches
   if (ti >= 0 && ti < tin)
-    for (int i = tid; i < HALF; i += kThreads) s_tcs[i] = rope_cos_sin(max(s_tpos, 0), rp.theta[i]);
+    for (int i = tid; i < HALF; i += kThreads)
+      s_tcs[i] = rope_cos_sin(max(s_tpos, 0), rope_theta(rp, a.append_layer, i));
   const int k_first = s_first;
   const int n_docs = k_first >= 0 ? min(s_last - s_first + 1, kTok) : 0;
-  for (int e = tid; e < n_docs * HALF; e += kThreads) {
-    const int j = e / HALF, i = e % HALF;
-    s_cs[j][i] = rope_cos_sin(rv.delta[k_first + j], rp.theta[i]);
-  }
+  auto fill_cs = [&](int layer) {  // cos/sin of the documents this page touches
+    for (int e = tid; e < n_docs * HALF; e += kThreads) {
+      const int j = e / HALF, i = e % HALF;
+      s_cs[j][i] = rope_cos_sin(rv.delta[k_first + j], rope_theta(rp, layer, i));
+    }
+  };
+  fill_cs(a.layer_begin);
   __syncthreads();
 
   // ---- the inline token: R(p) q packed, R(p) k and v into the cache
@@ -424,6 +428,11 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
   // ---- relocate the document positions of this page, layer by layer
   if (k_first >= 0) {
     for (int layer = a.layer_begin; layer < a.layer_end; ++layer) {
+    if (rp.layer_theta && layer > a.layer_begin) {  // a rotary table per layer
+      __syncthreads();
+      fill_cs(layer);
+      __syncthreads();
+    }
     const __nv_bfloat16 *kp = a.k_pool + (size_t)layer * a.pool_tokens * hkv * D;
     const __nv_bfloat16 *vp = a.v_pool + (size_t)layer * a.pool_tokens * hkv * D;
     __nv_bfloat16 *kc = a.k_cache + (size_t)layer * a.num_pages * hkv * 16 * D;

@@ -885,7 +885,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto make_qd = [&](int k, int buf) {
       asm volatile("bar.sync 1, 128;" ::: "memory");  // previous table no longer read
       if (tid128 < D / 2) {
-        const float2 cs = rope_cos_sin(s_delta[k], fp.rp.theta[tid128]);
+        const float2 cs = rope_cos_sin(s_delta[k], rope_theta(fp.rp, fp.layer, tid128));
         s_cs[tid128] = make_float2(cs.x, -cs.y);  // R(-delta): sin changes sign
       }
       asm volatile("bar.sync 1, 128;" ::: "memory");
@@ -1187,7 +1187,7 @@ __global__ void __launch_bounds__(256) combine_kernel(Params p) {
 // RoPE the inline keys/queries at their logical positions; keys and values go
 // to their cache slots, queries to the GQA-packed workspace.
 struct AppendArgs {
-  int Hq, Hkv, G, max_inline, max_ctx, R_pad;
+  int Hq, Hkv, G, max_inline, max_ctx, R_pad, layer;
   long long num_pages;
   const __nv_bfloat16 *q, *k, *v;
   const int32_t *inline_pos, *inline_len;
@@ -1239,7 +1239,8 @@ __global__ void __launch_bounds__(256) append_kernel(AppendArgs a, RopeParams rp
     if (tid == 0) dev_fail(a.status, PIC_DEV_BAD_PAGE, b);
     slot = -1;
   }
-  for (int i = tid; i < HALF; i += blockDim.x) cs[i] = rope_cos_sin(pos_ok ? pos : 0, rp.theta[i]);
+  for (int i = tid; i < HALF; i += blockDim.x)
+    cs[i] = rope_cos_sin(pos_ok ? pos : 0, rope_theta(rp, a.layer, i));
   __syncthreads();
   const long long page = slot >> 4, r = slot & 15;
 
@@ -1452,6 +1453,7 @@ extern "C" pic_status_t pic_append_inline(
   aa.max_inline = max_inline;
   aa.max_ctx = max_ctx;
   aa.R_pad = pl.R_pad;
+  aa.layer = layer;
   aa.num_pages = num_pages;
   aa.q = static_cast<const __nv_bfloat16 *>(q);
   aa.k = static_cast<const __nv_bfloat16 *>(k_new);

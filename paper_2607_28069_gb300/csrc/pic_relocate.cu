@@ -96,13 +96,21 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
   const int n_docs = min(s_last - s_first + 1, kTok);
 
   const size_t hkv = a.hkv;
-  for (int e = tid; e < n_docs * HALF; e += kThreads) {  // cos/sin of the touched documents
-    const int j = e / HALF, i = e % HALF;
-    const int delta = a.delta[(size_t)b * a.max_docs + k_first + j];
-    s_cs[j][i] = rope_cos_sin(delta, rp.theta[i]);
-  }
+  auto fill_cs = [&](int layer) {  // cos/sin of the touched documents
+    for (int e = tid; e < n_docs * HALF; e += kThreads) {
+      const int j = e / HALF, i = e % HALF;
+      const int delta = a.delta[(size_t)b * a.max_docs + k_first + j];
+      s_cs[j][i] = rope_cos_sin(delta, rope_theta(rp, layer, i));
+    }
+  };
+  fill_cs(a.layer_begin);
   __syncthreads();
   for (int layer = a.layer_begin; layer < a.layer_end; ++layer) {
+  if (rp.layer_theta && layer > a.layer_begin) {  // a rotary table per layer
+    __syncthreads();
+    fill_cs(layer);
+    __syncthreads();
+  }
   const __nv_bfloat16 *kp = a.k_pool + (size_t)layer * a.pool_tokens * hkv * D;
   const __nv_bfloat16 *vp = a.v_pool + (size_t)layer * a.pool_tokens * hkv * D;
   __nv_bfloat16 *kc = a.k_cache + (size_t)layer * a.num_pages * hkv * 16 * D;

@@ -16,13 +16,14 @@ from .workloads import Workload
 
 class CacheHitPath:
     def __init__(self, wl: Workload, prefill_splits: int = 0, decode_splits: int = 0,
-                 with_lse: bool = False, rope_style: int = 0, inv_freq=None):
+                 with_lse: bool = False, rope_style: int = 0, inv_freq=None,
+                 layer_inv_freq=None):
         spec = wl.spec
         dev = wl.k_pool.device
         self.wl = wl
         self.geom = Geometry(spec.layers, spec.q_heads, spec.kv_heads, spec.head_dim,
                              spec.rope_base, page_size=spec.page_size, rope_style=rope_style,
-                             inv_freq=inv_freq)
+                             inv_freq=inv_freq, layer_inv_freq=layer_inv_freq)
         B, md = wl.req_doc_ids.shape
         L, Hq, Hkv, d = spec.layers, spec.q_heads, spec.kv_heads, spec.head_dim
         self.B, self.max_docs = B, md

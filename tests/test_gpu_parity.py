@@ -408,3 +408,55 @@ def test_link_reports_bad_document_id():
     code, detail = pic.pic_device_status()
     assert code == 1 and detail == 0
     assert int(path.ctx_len[0]) == -1
+
+
+def test_per_layer_rotary_tables(cuda_lib):
+    """A rotary table per layer (the layer-specific R_l of Eq. 3, e.g. models
+    whose layers use different RoPE bases): each layer's relocated keys,
+    prefill and decode outputs follow that layer's frequencies, through the
+    linked pass and through the fused rotate-on-load pass."""
+    from paper_2607_28069_gb300.pipeline import CacheHitPath
+    spec = custom_spec(name="rope_layers", layers=3, q_heads=8, kv_heads=2, head_dim=128,
+                       rope_base=1e4, batch=2, pool_docs=4, docs_per_request=3,
+                       doc_len=(40, 300), prefix_len=(4, 30), query_len=20, span_len=(0, 5),
+                       decode_steps=1)
+    thetas = [O.rope_frequencies(128, base) for base in (1e4, 5e5, 1e6)]
+    table = torch.tensor(np.stack(thetas), dtype=torch.float64, device="cuda")
+    wl = generate(spec, device="cuda", gen_device="cpu")
+    # materialised, linked pass + one decode step
+    path = CacheHitPath(wl, with_lse=True, layer_inv_freq=table)
+    path.ttft_pass()
+    path.decode_pass(0)
+    # fused rotate-on-load pass
+    pathf = CacheHitPath(wl, with_lse=True, layer_inv_freq=table)
+    pathf.compose()
+    for layer in range(spec.layers):
+        pathf.append(layer)
+        pathf.attend_fused(layer)
+    torch.cuda.synchronize()
+    import paper_2607_28069_gb300 as pic
+    assert pic.pic_device_status() == (0, 0)
+    for layer in range(spec.layers):
+        th = thetas[layer]
+        for b in range(spec.batch):
+            lay = oracle_layout(wl, b)
+            docs, k_docs, v_docs, q, k, v = request_inputs(wl, b, layer)
+            base = wl.doc_base_pos.cpu().numpy()
+            (o_ref, _), K, V = O.cache_hit_prefill(lay, k_docs, v_docs, base, q, k, v, th,
+                                                   return_lse=True)
+            slots = torch.as_tensor(lay.slot_mapping, device="cuda")
+            kc = path.k_cache[layer].reshape(-1, spec.kv_heads, 16, spec.head_dim)
+            Kg = f64(kc[slots // 16, :, slots % 16])
+            ok, ratio = kv_tolerance_ok(Kg, K)
+            assert ok, f"K layer {layer} req {b}: worst err/bound {ratio:.3f}"
+            if layer > 0:  # the layer's own table, not layer 0's
+                K0, _ = O.dense_context(lay, k_docs, v_docs, base, k, v, thetas[0])
+                assert not kv_tolerance_ok(Kg, K0)[0]
+            tin = q.shape[0]
+            for pp in (path, pathf):
+                ok, max_abs, row = attn_close(f64(pp.out[layer, b, :tin]), o_ref)
+                assert ok, f"layer {layer} req {b}: max-abs {max_abs:.2e} row-rel {row:.2e}"
+            o_dec, _, _ = O.decode_step(K, V, f64(wl.q_dec[0, layer, b]), f64(wl.k_dec[0, layer, b]),
+                                        f64(wl.v_dec[0, layer, b]), lay.ctx_len, th)
+            ok, max_abs, row = attn_close(f64(path.dec_out[layer, b]), o_dec)
+            assert ok, f"decode layer {layer} req {b}: {max_abs:.2e} {row:.2e}"
