@@ -46,6 +46,8 @@ def parse_args(argv=None):
     ap.add_argument("--decode-splits", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--deviation", action="store_true",
+                    help="also time the attention-deviation diagnostic on layer 0")
     ap.add_argument("--fused", action="store_true",
                     help="also time the rotate-on-load pass (default for stress_128k_b4)")
     ap.add_argument("--oracle-sample", default=None, help=argparse.SUPPRESS)
@@ -514,6 +516,55 @@ def main_gpu(args, rank, world):
             "frac_bf16": work["attend_flops"] / (fatt * 1e9) / peaks["bf16_tflops"],
             "query_tok_s": work["query_tokens"] / (fms / 1e3),
             "speedup_vs_materialised": ms_per_step / fms}
+
+    # attention-deviation diagnostic (off the serving path): D_r between the
+    # relocated cache and the documents copied without re-rotation, layer 0
+    if args.deviation:
+        pathB = CacheHitPath(wl, prefill_splits=args.prefill_splits)
+        pathB.compose()
+        pic.pic_relocate(pathB.geom, wl.k_pool, wl.v_pool, pathB.tok_map,
+                         torch.zeros_like(pathB.doc_delta), pathB.slot_mapping, wl.num_pages,
+                         pathB.k_cache, pathB.v_cache, 0, 1)
+        pathA = CacheHitPath(wl, prefill_splits=args.prefill_splits, with_lse=True)
+        pathA.compose()
+        pathA.relocate(0, 1)
+        pathB.lse = torch.empty_like(pathA.lse)
+        for pth in (pathA, pathB):
+            pth.append(0)
+            pic.pic_attend_prefill(pth.geom, 0, pth.inline_pos, wl.inline_len, pth.max_ctx,
+                                   wl.block_table, wl.num_pages, pth.k_cache, pth.v_cache,
+                                   pth.out[0], pth.lse[0], args.prefill_splits, pth.ws_prefill)
+        qlen = torch.full((spec.batch,), spec.query_len, dtype=torch.int32, device=dev)
+        dsum = torch.empty((spec.batch, 2), dtype=torch.float64, device=dev)
+        dcnt = torch.empty((spec.batch, 2), dtype=torch.int64, device=dev)
+
+        def dev_call():
+            pic.pic_attention_deviation(pathA.geom, 0, pathA.inline_pos, wl.inline_len, qlen,
+                                        wl.req_doc_ids, wl.doc_len, pathA.doc_offset,
+                                        pathA.slot_mapping, pathA.tok_map, wl.num_pages,
+                                        pathA.k_cache, pathB.k_cache, pathA.lse[0], pathB.lse[0],
+                                        pathA.ws_prefill, dsum, dcnt, (0.0, 0.1, 0.9))
+        dts = []
+        for k in range(W + max(3, K // 2)):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            dev_call()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if k >= W:
+                dts.append(e0.elapsed_time(e1))
+        dv_ms = sum(dts) / len(dts)
+        terms = int(dcnt.sum().item())          # (row, head, key) terms in the regions
+        flops = 2 * 2 * spec.head_dim * terms   # two dot products per term
+        fp32_peak = 152 * 128 * 2 * 2.07e9 / 1e12
+        d_r = (dsum.sum(0) / dcnt.sum(0).clamp(min=1)).tolist()
+        rows["next4_deviation"] = {
+            "ms": dv_ms, "launches": 1, "terms": terms, "tflops_fp32": flops / (dv_ms * 1e9),
+            "frac_fp32_fma": flops / (dv_ms * 1e9) / fp32_peak, "D_pre": d_r[0], "D_int": d_r[1],
+            "note": "layer 0: relocated cache vs documents copied without re-rotation; "
+                    "fp32 FMA peak 152 SMs x 128 lanes x 2 x 2.07 GHz"}
+        del pathA, pathB
 
     # dominant kernel of the step -> roofline object: attention, or the data
     # movement the pass runs (pic_link when the pass is one graph, else relocate)

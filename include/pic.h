@@ -300,6 +300,45 @@ pic_status_t pic_attend_prefill_fused(const pic_geom_t *geom, int32_t layer, int
                                       pic_stream_t stream);
 
 /*
+ * pic_attention_deviation -- the attention-deviation diagnostic of the
+ * paper's "Motivating Analysis": D_r(A, B), the mean absolute deviation
+ * between the post-softmax attention probabilities of two configurations A
+ * and B within normalized block region r.  Here A and B are two stitched key
+ * caches of the same requests with the same slot map (for example the
+ * relocated cache and one whose documents were copied at their compiled
+ * positions), read by the same rotated queries, for one layer.
+ * For request b the query rows are its last query_len[b] inline tokens and
+ * every query head; the blocks are its documents: token j of document k
+ * (n_k tokens) lies in region i when ceil(edges[i] n_k) <= j <
+ * ceil(edges[i+1] n_k) (double-precision products), i.e. edges[i] <= j / n_k
+ * < edges[i+1].  With p_X = exp(q.k_X / sqrt(d) - lse_X), lse_X the
+ * natural-log LSE output of pic_attend_prefill for configuration X:
+ *     sums[b][i]   = sum over those rows, heads and keys of |p_A - p_B|
+ *     counts[b][i] = the number of terms          (D_i = sums / counts)
+ * Inputs (device): inline_pos, inline_len, query_len, req_doc_ids, doc_len,
+ *   doc_offset, slot_mapping, tok_map as from pic_compose / pic_link;
+ *   k_cache_a, k_cache_b bf16 paged caches (layout of pic_relocate); lse_a,
+ *   lse_b float [batch][max_inline][Hq]; workspace: the prefill workspace
+ *   after pic_append_inline (its packed rotated queries are read).
+ * edges: HOST array of n_regions + 1 ascending fractions in [0, 1],
+ *   1 <= n_regions <= 8 (e.g. {0, 0.1, 0.9}: the paper's pre and int regions).
+ * Outputs (device, overwritten): sums double [batch][n_regions], counts
+ *   int64 [batch][n_regions].  Two memsets and one launch on `stream`; a
+ *   CUDA-core kernel (a diagnostic, off the serving path).
+ */
+pic_status_t pic_attention_deviation(const pic_geom_t *geom, int32_t layer, int32_t batch,
+                                     int32_t max_inline, int32_t max_docs, int32_t max_ctx,
+                                     int64_t num_pages, const int32_t *inline_pos,
+                                     const int32_t *inline_len, const int32_t *query_len,
+                                     const int32_t *req_doc_ids, const int32_t *doc_len,
+                                     const int32_t *doc_offset, const int64_t *slot_mapping,
+                                     const int64_t *tok_map, const void *k_cache_a,
+                                     const void *k_cache_b, const float *lse_a,
+                                     const float *lse_b, const double *edges, int32_t n_regions,
+                                     const void *workspace, size_t workspace_bytes, double *sums,
+                                     int64_t *counts, pic_stream_t stream);
+
+/*
  * pic_attend_decode -- one layer of one plain autoregressive decoding step over
  * the completed cache (appendix "Position-Independent Linking": after the first
  * token, generation proceeds as usual on the linked cache).

@@ -356,3 +356,63 @@ def decode_step(K, V, q_new, k_new, v_new, pos, theta, style=HALF, return_lse=Fa
     if return_lse:
         return (res[0][0], res[1][0]), K2, V2
     return res[0], K2, V2
+
+
+# --------------------------------------------------------------------------
+# Attention-deviation diagnostic ("Motivating Analysis")
+# --------------------------------------------------------------------------
+def attention_probabilities(q, q_pos, K, k_pos=None, scale=None):
+    """Post-softmax attention probabilities [T, Hq, S] of rotated queries q
+    [T, Hq, d] at positions q_pos over keys K [S, Hkv, d] at k_pos (default
+    0..S-1), frontier mask and GQA as in ``attention``; masked keys get 0."""
+    q = np.asarray(q, np.float64)
+    K = np.asarray(K, np.float64)
+    T, Hq, d = q.shape
+    S, Hkv, _ = K.shape
+    G = Hq // Hkv
+    scale = 1.0 / math.sqrt(d) if scale is None else scale
+    k_pos = np.arange(S) if k_pos is None else np.asarray(k_pos)
+    visible = k_pos[None, :] <= np.asarray(q_pos)[:, None]
+    out = np.zeros((T, Hq, S))
+    for h in range(Hq):
+        s = (q[:, h, :] @ K[:, h // G, :].T) * scale
+        s = np.where(visible, s, -np.inf)
+        p = np.exp(s - s.max(axis=1, keepdims=True))
+        out[:, h, :] = p / p.sum(axis=1, keepdims=True)
+    return out
+
+
+def block_region_bounds(n, edges):
+    """Token index bounds of the normalized regions of a block of n tokens:
+    region i holds the tokens j with edges[i] <= j / n < edges[i+1], i.e.
+    ceil(edges[i] * n) <= j < ceil(edges[i+1] * n) (products in double
+    precision)."""
+    return [int(math.ceil(float(e) * n)) for e in edges]
+
+
+def attention_deviation(q, q_pos, K_a, K_b, layout: RequestLayout, doc_lens, edges=(0.0, 0.1, 0.9)):
+    """D_r(A, B) of the paper's diagnostic: the mean absolute deviation between
+    the post-softmax attention probabilities of two configurations A and B
+    (the same rotated queries over two key sets of one request, e.g. a
+    relocated cache and one built another way) within normalized block
+    region r.  Key t of the k-th block (document) lies at normalized
+    position (t - offset_k) / n_k; region i is [edges[i], edges[i+1]) (the
+    paper's pre = [0, 0.1), int = [0.1, 0.9)).
+
+    Returns (sums, counts) per region: the sum over query rows, query heads
+    and block keys in the region of |p_A - p_B|, and the number of terms; the
+    deviation is sums / counts.
+    """
+    pa = attention_probabilities(q, q_pos, K_a)
+    pb = attention_probabilities(q, q_pos, K_b)
+    diff = np.abs(pa - pb)                      # [T, Hq, S]
+    R = len(edges) - 1
+    sums, counts = np.zeros(R), np.zeros(R, dtype=np.int64)
+    T, Hq = diff.shape[:2]
+    for off, n in zip(layout.doc_offset, doc_lens):
+        b = block_region_bounds(n, edges)
+        for i in range(R):
+            lo, hi = off + b[i], off + max(b[i], b[i + 1])
+            sums[i] += diff[:, :, lo:hi].sum()
+            counts[i] += T * Hq * (hi - lo)
+    return sums, counts

@@ -460,3 +460,56 @@ def test_per_layer_rotary_tables(cuda_lib):
                                         f64(wl.v_dec[0, layer, b]), lay.ctx_len, th)
             ok, max_abs, row = attn_close(f64(path.dec_out[layer, b]), o_dec)
             assert ok, f"decode layer {layer} req {b}: {max_abs:.2e} {row:.2e}"
+
+
+@pytest.mark.parametrize("name", ["spans_b2", "llama8b_1layer"])
+def test_attention_deviation_matches_oracle(cuda_lib, name):
+    """D_r(A, B) of the diagnostic on the GPU against the oracle, with A = the
+    relocated cache and B = the same documents copied at their compiled
+    positions (no re-rotation: every delta 0), over the paper's pre / int
+    regions and a four-region split."""
+    import paper_2607_28069_gb300 as pic
+    from paper_2607_28069_gb300.pipeline import CacheHitPath
+    wl = generate(SMALL[name], device="cuda", gen_device="cpu")
+    spec = wl.spec
+    A = CacheHitPath(wl, with_lse=True)
+    Bp = CacheHitPath(wl, with_lse=True)
+    A.compose()
+    A.relocate()
+    Bp.compose()
+    pic.pic_relocate(Bp.geom, wl.k_pool, wl.v_pool, Bp.tok_map, torch.zeros_like(Bp.doc_delta),
+                     Bp.slot_mapping, wl.num_pages, Bp.k_cache, Bp.v_cache, 0, spec.layers)
+    theta = theta_of(spec)
+    query_len = torch.full((spec.batch,), spec.query_len, dtype=torch.int32, device="cuda")
+    for edges in ((0.0, 0.1, 0.9), (0.0, 0.25, 0.5, 0.75, 1.0)):
+        R = len(edges) - 1
+        for layer in range(spec.layers):
+            for p in (A, Bp):
+                p.append(layer)
+                p.attend(layer)
+            sums = torch.empty((spec.batch, R), dtype=torch.float64, device="cuda")
+            counts = torch.empty((spec.batch, R), dtype=torch.int64, device="cuda")
+            pic.pic_attention_deviation(A.geom, layer, A.inline_pos, wl.inline_len, query_len,
+                                        wl.req_doc_ids, wl.doc_len, A.doc_offset, A.slot_mapping,
+                                        A.tok_map, wl.num_pages, A.k_cache, Bp.k_cache,
+                                        A.lse[layer], Bp.lse[layer], A.ws_prefill, sums, counts,
+                                        edges)
+            torch.cuda.synchronize()
+            assert pic.pic_device_status() == (0, 0)
+            for b in range(spec.batch):
+                lay = oracle_layout(wl, b)
+                docs, k_docs, v_docs, q, k, v = request_inputs(wl, b, layer)
+                base = wl.doc_base_pos.cpu().numpy().copy()
+                Ka, _ = O.dense_context(lay, k_docs, v_docs, base, k, v, theta, storage="bf16")
+                for i, dd in enumerate(docs):       # B: every document left where it was compiled
+                    base[dd] = lay.doc_offset[i]
+                Kb, _ = O.dense_context(lay, k_docs, v_docs, base, k, v, theta, storage="bf16")
+                tq = spec.query_len
+                qp = lay.inline_pos[-tq:]
+                qr = O.round_bf16(O.rotary(q[-tq:], qp[:, None], theta))
+                lens = [int(wl.doc_len[dd]) for dd in docs]
+                s_ref, c_ref = O.attention_deviation(qr, qp, Ka, Kb, lay, lens, edges)
+                assert np.array_equal(counts[b].cpu().numpy(), c_ref), (layer, b)
+                got = sums[b].cpu().numpy()
+                np.testing.assert_allclose(got, s_ref, rtol=2e-2, atol=1e-6 * c_ref.max())
+                assert (s_ref > 0).all()

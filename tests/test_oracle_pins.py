@@ -587,3 +587,84 @@ def test_bf16_storage_only_rounds_rotated_keys_and_queries():
     assert np.array_equal(Kb, O.round_bf16(K)) and np.array_equal(Vb, V)
     # unit roundoff of an 8-bit significand: |round(x) - x| <= 2^-8 |x|
     assert (np.abs(Kb - K) <= 2.0 ** -8 * np.abs(K)).all()
+
+
+# ------------------------------------------- attention-deviation diagnostic ---
+def _deviation_brute_force(q, q_pos, Ka, Kb, offsets, lens, edges):
+    """Scalar loops: probabilities with math.exp per row, regions by the
+    exact rational test e_i <= j / n < e_(i+1)."""
+    from fractions import Fraction
+    T, Hq, d = q.shape
+    G = Hq // Ka.shape[1]
+    scale = 1 / math.sqrt(d)
+
+    def probs(K, t, h):
+        vis = [s for s in range(K.shape[0]) if s <= q_pos[t]]
+        sc = {s: scale * sum(q[t, h, i] * K[s, h // G, i] for i in range(d)) for s in vis}
+        m = max(sc.values())
+        w = {s: math.exp(x - m) for s, x in sc.items()}
+        z = sum(w.values())
+        return {s: w[s] / z for s in vis}
+
+    R = len(edges) - 1
+    sums, counts = [0.0] * R, [0] * R
+    E = [Fraction(e) for e in edges]
+    for t in range(T):
+        for h in range(Hq):
+            pa, pb = probs(Ka, t, h), probs(Kb, t, h)
+            for off, n in zip(offsets, lens):
+                for j in range(n):
+                    u = Fraction(j, n)
+                    for i in range(R):
+                        if E[i] <= u < E[i + 1]:
+                            sums[i] += abs(pa.get(off + j, 0.0) - pb.get(off + j, 0.0))
+                            counts[i] += 1
+    return np.array(sums), np.array(counts)
+
+
+def _deviation_case(seed=0, lens=(7, 13, 23), P=3, Tq=4, d=8, Hq=4, Hkv=2):
+    rng = np.random.default_rng(seed)
+    ctx = P + sum(lens) + Tq
+    lay = O.compose_layout(list(lens), [0] * len(lens), list(range(len(lens))), P, Tq,
+                           np.arange(-(-ctx // 16)), 16)
+    q = rng.standard_normal((Tq, Hq, d))
+    q_pos = lay.inline_pos[P:]
+    Ka = rng.standard_normal((ctx, Hkv, d))
+    Kb = Ka.copy()
+    Kb[lay.doc_offset[1]:lay.doc_offset[1] + lens[1]] *= -0.5     # B differs in doc 1
+    Kb[lay.doc_offset[2] + 2] += 1.0                              # and one key of doc 2
+    return q, q_pos, Ka, Kb, lay, lens
+
+
+def test_attention_deviation_pinned_to_brute_force():
+    for edges in ((0.0, 0.1, 0.9), (0.0, 0.25, 0.5, 1.0)):
+        q, q_pos, Ka, Kb, lay, lens = _deviation_case()
+        s, c = O.attention_deviation(q, q_pos, Ka, Kb, lay, lens, edges)
+        sb, cb = _deviation_brute_force(q, q_pos, Ka, Kb, lay.doc_offset, lens, edges)
+        np.testing.assert_allclose(s, sb, rtol=1e-12, atol=1e-15)
+        assert np.array_equal(c, cb)
+
+
+def test_attention_deviation_identity_symmetry_and_bound():
+    q, q_pos, Ka, Kb, lay, lens = _deviation_case(seed=3)
+    s0, c0 = O.attention_deviation(q, q_pos, Ka, Ka, lay, lens)
+    assert (s0 == 0).all() and c0.sum() > 0                  # D(A, A) = 0
+    s1, _ = O.attention_deviation(q, q_pos, Ka, Kb, lay, lens)
+    s2, _ = O.attention_deviation(q, q_pos, Kb, Ka, lay, lens)
+    np.testing.assert_allclose(s1, s2, rtol=1e-14)           # symmetric
+    assert s1.sum() <= 2 * q.shape[0] * q.shape[1] + 1e-12   # total variation <= 2 per row
+    assert (s1 > 0).all()
+
+
+def test_pins_catch_planted_deviation_mistakes():
+    q, q_pos, Ka, Kb, lay, lens = _deviation_case(seed=5)
+    edges = (0.0, 0.1, 0.9)
+    ref = _deviation_brute_force(q, q_pos, Ka, Kb, lay.doc_offset, lens, edges)[0]
+
+    class Shifted:  # regions taken one document off
+        doc_offset = lay.doc_offset[1:] + [lay.doc_offset[0]]
+    s_shift, _ = O.attention_deviation(q, q_pos, Ka, Kb, Shifted, lens, edges)
+    # unnormalised region edges (fractions of the longest block)
+    s_abs, _ = O.attention_deviation(q, q_pos, Ka, Kb, lay, [max(lens)] * len(lens), edges)
+    for s in (s_shift, s_abs):
+        assert not np.allclose(s, ref, rtol=1e-6)
