@@ -46,6 +46,8 @@ def parse_args(argv=None):
     ap.add_argument("--decode-splits", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--layer-rope", action="store_true",
+                    help="a rotary table per layer (bases 1e4 and the workload's, alternating)")
     ap.add_argument("--deviation", action="store_true",
                     help="also time the attention-deviation diagnostic on layer 0")
     ap.add_argument("--fused", action="store_true",
@@ -289,7 +291,15 @@ def main_gpu(args, rank, world):
     import dataclasses
     spec1 = spec if spec.decode_steps <= 1 else dataclasses.replace(spec, decode_steps=1)
     wl = generate(spec1, device=dev, gen_device=GPU_GEN.get(args.workload, "cuda"))
-    path = CacheHitPath(wl, prefill_splits=args.prefill_splits, decode_splits=args.decode_splits)
+    layer_table = None
+    if args.layer_rope:  # alternate a local-attention base (1e4) with the workload's base
+        half = spec.head_dim // 2
+        i = torch.arange(half, dtype=torch.float64)
+        rows = [torch.pow(torch.tensor(1e4 if l % 2 == 0 else spec.rope_base, dtype=torch.float64),
+                          -2.0 * i / spec.head_dim) for l in range(spec.layers)]
+        layer_table = torch.stack(rows).to(dev)
+    path = CacheHitPath(wl, prefill_splits=args.prefill_splits, decode_splits=args.decode_splits,
+                        layer_inv_freq=layer_table)
     work = work_of(wl)
     L = spec.layers
     geom = path.geom

@@ -276,7 +276,7 @@ __device__ void token_zero(const LinkArgs &a, int b, int t) {
 
 // CTA x of request y: page CTA x (its kTok positions, if x < n_pages) and,
 // with an append, inline token slot x (if x < t_slots).
-template <int D, int kTok>
+template <int D, int kTok, bool kLayerRope>
 __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams rp) {
   static_assert(kTok == 16 || kTok == 32, "one warp scans the positions of a CTA");
   constexpr unsigned kMask = kTok == 32 ? 0xffffffffu : 0x0000ffffu;
@@ -294,7 +294,9 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
   __shared__ long long s_src[kTok], s_dst[kTok];
   __shared__ int s_doc[kTok];               // document index of each position
   __shared__ int s_first, s_last;
-  __shared__ float2 s_cs[kTok][HALF];       // per touched document
+  // per touched document; with a table per layer, two buffers (this layer's
+  // and the next one's, computed while this layer's loads are in flight)
+  __shared__ float2 s_cs[kLayerRope ? 2 : 1][kTok][HALF];
   __shared__ float2 s_tcs[HALF];            // at the inline token's position
   __shared__ long long s_tslot;
   __shared__ int s_tpos;
@@ -404,13 +406,13 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
       s_tcs[i] = rope_cos_sin(max(s_tpos, 0), rope_theta(rp, a.append_layer, i));
   const int k_first = s_first;
   const int n_docs = k_first >= 0 ? min(s_last - s_first + 1, kTok) : 0;
-  auto fill_cs = [&](int layer) {  // cos/sin of the documents this page touches
+  auto fill_cs = [&](int layer, int buf) {  // cos/sin of the documents this page touches
     for (int e = tid; e < n_docs * HALF; e += kThreads) {
       const int j = e / HALF, i = e % HALF;
-      s_cs[j][i] = rope_cos_sin(rv.delta[k_first + j], rope_theta(rp, layer, i));
+      s_cs[buf][j][i] = rope_cos_sin(rv.delta[k_first + j], rope_theta(rp, layer, i));
     }
   };
-  fill_cs(a.layer_begin);
+  fill_cs(a.layer_begin, 0);
   __syncthreads();
 
   // ---- the inline token: R(p) q packed, R(p) k and v into the cache
@@ -425,14 +427,13 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
   // gave away the overlap with this kernel's last stores.
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-  // ---- relocate the document positions of this page, layer by layer
+  // ---- relocate the document positions of this page, layer by layer (with
+  // a rotary table per layer, the cos/sin are recomputed for each layer;
+  // that form is a separate instantiation so the common one keeps its
+  // tighter loop)
   if (k_first >= 0) {
     for (int layer = a.layer_begin; layer < a.layer_end; ++layer) {
-    if (rp.layer_theta && layer > a.layer_begin) {  // a rotary table per layer
-      __syncthreads();
-      fill_cs(layer);
-      __syncthreads();
-    }
+    const int cur = kLayerRope ? (layer - a.layer_begin) & 1 : 0;
     const __nv_bfloat16 *kp = a.k_pool + (size_t)layer * a.pool_tokens * hkv * D;
     const __nv_bfloat16 *vp = a.v_pool + (size_t)layer * a.pool_tokens * hkv * D;
     __nv_bfloat16 *kc = a.k_cache + (size_t)layer * a.num_pages * hkv * 16 * D;
@@ -478,14 +479,19 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
           }
         }
       }
+      if constexpr (kLayerRope) {  // next layer's table while the loads are in flight
+        if (round == 0 && layer + 1 < a.layer_end) fill_cs(layer + 1, cur ^ 1);
+      }
 #pragma unroll
       for (int u = 0; u < UV; ++u)
         if (vdst[u] >= 0) st_global16(vc + vdst[u], v[u]);
 #pragma unroll
       for (int u = 0; u < UK; ++u)
-        if (kdst[u] >= 0) rot_store8(ka[u], kb[u], kch[u], HALF, style, &s_cs[kdoc[u]][8 * kch[u]],
-                                     kc + kdst[u]);
+        if (kdst[u] >= 0)
+          rot_store8(ka[u], kb[u], kch[u], HALF, style, &s_cs[cur][kdoc[u]][8 * kch[u]],
+                     kc + kdst[u]);
     }
+    if constexpr (kLayerRope) __syncthreads();  // next table written; this one read
     }
   }
 
@@ -620,12 +626,22 @@ extern "C" pic_status_t pic_link(
   dim3 grid((unsigned)(do_append ? std::max(a.n_pages, a.t_slots) : a.n_pages), batch);
   const dim3 block(kThreads);
   cudaError_t e;
-  if (geom->head_dim == 128)
-    e = wide ? launch_dependent(link_kernel<128, 16>, grid, block, 0, stream, a, rp)
-             : launch_dependent(link_kernel<128, 32>, grid, block, 0, stream, a, rp);
-  else
-    e = wide ? launch_dependent(link_kernel<64, 16>, grid, block, 0, stream, a, rp)
-             : launch_dependent(link_kernel<64, 32>, grid, block, 0, stream, a, rp);
+  const bool per_layer = rp.layer_theta != nullptr;
+  if (geom->head_dim == 128) {
+    if (per_layer)
+      e = wide ? launch_dependent(link_kernel<128, 16, true>, grid, block, 0, stream, a, rp)
+               : launch_dependent(link_kernel<128, 32, true>, grid, block, 0, stream, a, rp);
+    else
+      e = wide ? launch_dependent(link_kernel<128, 16, false>, grid, block, 0, stream, a, rp)
+               : launch_dependent(link_kernel<128, 32, false>, grid, block, 0, stream, a, rp);
+  } else {
+    if (per_layer)
+      e = wide ? launch_dependent(link_kernel<64, 16, true>, grid, block, 0, stream, a, rp)
+               : launch_dependent(link_kernel<64, 32, true>, grid, block, 0, stream, a, rp);
+    else
+      e = wide ? launch_dependent(link_kernel<64, 16, false>, grid, block, 0, stream, a, rp)
+               : launch_dependent(link_kernel<64, 32, false>, grid, block, 0, stream, a, rp);
+  }
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_link launch");
   return PIC_OK;

@@ -38,7 +38,9 @@ struct RelocArgs {
   int32_t *status;
 };
 
-template <int D, int kTok>
+// kLayerRope: a rotary table per layer (its cos/sin double-buffered: the next
+// layer's table is computed while this layer's loads are in flight)
+template <int D, int kTok, bool kLayerRope>
 __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopeParams rp) {
   static_assert(kTok == 16 || kTok == 32, "one warp scans the positions of a CTA");
   pdl_entry();
@@ -55,7 +57,7 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
   __shared__ long long s_dst[kTok];  // cache slot
   __shared__ int s_doc[kTok];        // document index k within the request
   __shared__ int s_first, s_last;    // document range touched by this page
-  __shared__ float2 s_cs[kTok][HALF];
+  __shared__ float2 s_cs[kLayerRope ? 2 : 1][kTok][HALF];
 
   if (tid < kTok) {
     const long long t = t0 + tid;
@@ -96,21 +98,17 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
   const int n_docs = min(s_last - s_first + 1, kTok);
 
   const size_t hkv = a.hkv;
-  auto fill_cs = [&](int layer) {  // cos/sin of the touched documents
+  auto fill_cs = [&](int layer, int buf) {  // cos/sin of the touched documents
     for (int e = tid; e < n_docs * HALF; e += kThreads) {
       const int j = e / HALF, i = e % HALF;
       const int delta = a.delta[(size_t)b * a.max_docs + k_first + j];
-      s_cs[j][i] = rope_cos_sin(delta, rope_theta(rp, layer, i));
+      s_cs[buf][j][i] = rope_cos_sin(delta, rope_theta(rp, layer, i));
     }
   };
-  fill_cs(a.layer_begin);
+  fill_cs(a.layer_begin, 0);
   __syncthreads();
   for (int layer = a.layer_begin; layer < a.layer_end; ++layer) {
-  if (rp.layer_theta && layer > a.layer_begin) {  // a rotary table per layer
-    __syncthreads();
-    fill_cs(layer);
-    __syncthreads();
-  }
+  const int cur = kLayerRope ? (layer - a.layer_begin) & 1 : 0;
   const __nv_bfloat16 *kp = a.k_pool + (size_t)layer * a.pool_tokens * hkv * D;
   const __nv_bfloat16 *vp = a.v_pool + (size_t)layer * a.pool_tokens * hkv * D;
   __nv_bfloat16 *kc = a.k_cache + (size_t)layer * a.num_pages * hkv * 16 * D;
@@ -158,6 +156,9 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
         }
       }
     }
+    if constexpr (kLayerRope) {  // next layer's table while the loads are in flight
+      if (round == 0 && layer + 1 < a.layer_end) fill_cs(layer + 1, cur ^ 1);
+    }
     // ---- V: bit copy
 #pragma unroll
     for (int u = 0; u < UV; ++u)
@@ -169,7 +170,7 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
       const int c = kch[u];
       float2 cs[8];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) cs[q] = s_cs[kdoc[u]][8 * c + q];
+      for (int q = 0; q < 8; ++q) cs[q] = s_cs[cur][kdoc[u]][8 * c + q];
       float x[8], y[8], uu[8], ww[8];
       unpack8(ka[u], x);
       unpack8(kb[u], y);
@@ -199,6 +200,7 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
       st_global16(kc + kdst[u] + pc.off_b, pack8(y));
     }
   }
+  if constexpr (kLayerRope) __syncthreads();  // next table written; this one read
   }
 }
 
@@ -256,11 +258,17 @@ extern "C" pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int3
   const dim3 block(kThreads);
   cudaError_t e;
   if (geom->head_dim == 128)
-    e = wide ? launch_dependent(relocate_kernel<128, 16>, grid, block, 0, stream, a, rp)
-             : launch_dependent(relocate_kernel<128, 32>, grid, block, 0, stream, a, rp);
+    e = rp.layer_theta
+            ? (wide ? launch_dependent(relocate_kernel<128, 16, true>, grid, block, 0, stream, a, rp)
+                    : launch_dependent(relocate_kernel<128, 32, true>, grid, block, 0, stream, a, rp))
+            : (wide ? launch_dependent(relocate_kernel<128, 16, false>, grid, block, 0, stream, a, rp)
+                    : launch_dependent(relocate_kernel<128, 32, false>, grid, block, 0, stream, a, rp));
   else
-    e = wide ? launch_dependent(relocate_kernel<64, 16>, grid, block, 0, stream, a, rp)
-             : launch_dependent(relocate_kernel<64, 32>, grid, block, 0, stream, a, rp);
+    e = rp.layer_theta
+            ? (wide ? launch_dependent(relocate_kernel<64, 16, true>, grid, block, 0, stream, a, rp)
+                    : launch_dependent(relocate_kernel<64, 32, true>, grid, block, 0, stream, a, rp))
+            : (wide ? launch_dependent(relocate_kernel<64, 16, false>, grid, block, 0, stream, a, rp)
+                    : launch_dependent(relocate_kernel<64, 32, false>, grid, block, 0, stream, a, rp));
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_relocate launch");
   return PIC_OK;
