@@ -102,3 +102,41 @@ def test_product_path_does_not_import_the_oracle():
             if f.endswith((".py", ".cu", ".cuh", ".h")):
                 src = open(os.path.join(dirpath, f)).read()
                 assert "import oracle" not in src and "from oracle" not in src, f
+
+
+def _call_deviation_with(geom, edges, n_regions, layer=0, tensors=True):
+    g = geom._c()
+    null = ctypes.c_void_p(0)
+    fake = ctypes.c_void_p(256) if tensors else null   # never dereferenced: rejected first
+    arr = (ctypes.c_double * len(edges))(*edges)
+    return pic.load().pic_attention_deviation(
+        ctypes.byref(g), layer, 1, 16, 2, 64, 8, fake, fake, fake, fake, fake, fake, fake, fake,
+        fake, fake, fake, fake, ctypes.cast(arr, ctypes.c_void_p), n_regions, fake, 1 << 20, fake,
+        fake, null)
+
+
+def test_attention_deviation_arguments_checked_on_the_host(lib):
+    g = _geom()
+    assert _call_deviation_with(g, [0.0, 0.1, 0.9], 0) == 1        # no region
+    assert _call_deviation_with(g, [0.0] * 10, 9) == 1              # more than 8 regions
+    assert _call_deviation_with(g, [0.0, 0.9, 0.1], 2) == 1         # edges not ascending
+    assert b"edges" in pic.load().pic_last_error()
+    assert _call_deviation_with(g, [0.0, 1.5], 1) == 1              # outside [0, 1]
+    assert _call_deviation_with(g, [0.0, 0.1, 0.9], 2, layer=2) == 1  # layer outside the model
+    assert _call_deviation_with(g, [0.0, 0.1, 0.9], 2, tensors=False) == 1
+    assert b"NULL" in pic.load().pic_last_error()
+
+
+def test_geometry_binding_carries_the_per_layer_table_pointer():
+    import torch
+    g = _geom()
+    assert g._c().layer_inv_freq is None
+    with pytest.raises(ValueError):   # wrong shape is refused before any call
+        pic.Geometry(2, 32, 8, 128, 5e5, layer_inv_freq=torch.zeros((3, 64),
+                                                                     dtype=torch.float64))._c()
+
+
+def test_compose_span_input_is_optional_in_the_binding():
+    import inspect
+    for fn in (pic.pic_compose, pic.pic_link):
+        assert inspect.signature(fn).parameters["span_len"].default is None
