@@ -553,7 +553,8 @@ def main_gpu(args, rank, world):
                                         wl.req_doc_ids, wl.doc_len, pathA.doc_offset,
                                         pathA.slot_mapping, pathA.tok_map, wl.num_pages,
                                         pathA.k_cache, pathB.k_cache, pathA.lse[0], pathB.lse[0],
-                                        pathA.ws_prefill, dsum, dcnt, (0.0, 0.1, 0.9))
+                                        pathA.ws_prefill, dsum, dcnt, (0.0, 0.1, 0.9),
+                                        max_query_len=spec.query_len)
         dts = []
         for k in range(W + max(3, K // 2)):
             flush.zero_()
@@ -566,14 +567,14 @@ def main_gpu(args, rank, world):
                 dts.append(e0.elapsed_time(e1))
         dv_ms = sum(dts) / len(dts)
         terms = int(dcnt.sum().item())          # (row, head, key) terms in the regions
-        flops = 2 * 2 * spec.head_dim * terms   # two dot products per term
-        fp32_peak = 152 * 128 * 2 * 2.07e9 / 1e12
+        flops = 2 * 2 * spec.head_dim * terms   # two dot products (QK^T of A and of B) per term
         d_r = (dsum.sum(0) / dcnt.sum(0).clamp(min=1)).tolist()
         rows["next4_deviation"] = {
-            "ms": dv_ms, "launches": 1, "terms": terms, "tflops_fp32": flops / (dv_ms * 1e9),
-            "frac_fp32_fma": flops / (dv_ms * 1e9) / fp32_peak, "D_pre": d_r[0], "D_int": d_r[1],
-            "note": "layer 0: relocated cache vs documents copied without re-rotation; "
-                    "fp32 FMA peak 152 SMs x 128 lanes x 2 x 2.07 GHz"}
+            "ms": dv_ms, "launches": 1, "terms": terms, "tflops": flops / (dv_ms * 1e9),
+            "frac_bf16": flops / (dv_ms * 1e9) / peaks["bf16_tflops"], "D_pre": d_r[0],
+            "D_int": d_r[1],
+            "note": "layer 0: relocated cache vs documents copied without re-rotation; FLOPs "
+                    "count the region terms only (two 2-d dot products each)"}
         del pathA, pathB
 
     # dominant kernel of the step -> roofline object: attention, or the data

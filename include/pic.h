@@ -322,15 +322,18 @@ pic_status_t pic_attend_prefill_fused(const pic_geom_t *geom, int32_t layer, int
  *   after pic_append_inline (its packed rotated queries are read).
  * edges: HOST array of n_regions + 1 ascending fractions in [0, 1],
  *   1 <= n_regions <= 8 (e.g. {0, 0.1, 0.9}: the paper's pre and int regions).
+ * max_query_len: the largest query_len[b] (host value; sizes the grid).
  * Outputs (device, overwritten): sums double [batch][n_regions], counts
- *   int64 [batch][n_regions].  Two memsets and one launch on `stream`; a
- *   CUDA-core kernel (a diagnostic, off the serving path).
+ *   int64 [batch][n_regions].  Two memsets and one launch on `stream`: a
+ *   tcgen05 kernel (both score matrices on the tensor cores; a diagnostic,
+ *   off the serving path).
  */
 pic_status_t pic_attention_deviation(const pic_geom_t *geom, int32_t layer, int32_t batch,
                                      int32_t max_inline, int32_t max_docs, int32_t max_ctx,
                                      int64_t num_pages, const int32_t *inline_pos,
                                      const int32_t *inline_len, const int32_t *query_len,
-                                     const int32_t *req_doc_ids, const int32_t *doc_len,
+                                     int32_t max_query_len, const int32_t *req_doc_ids,
+                                     const int32_t *doc_len,
                                      const int32_t *doc_offset, const int64_t *slot_mapping,
                                      const int64_t *tok_map, const void *k_cache_a,
                                      const void *k_cache_b, const float *lse_a,

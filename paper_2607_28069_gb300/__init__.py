@@ -115,8 +115,8 @@ def load():
         "pic_link": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, P, I32, I64, I32, I32, P, P, I64,
                            I32, I32, I32, P, P, P, P, P, P, P, P, P, P, P, P, P, SZ, P]),
         "pic_prefill_workspace_size": (SZ, [G, I32, I32, I32, I32]),
-        "pic_attention_deviation": (I32, [G, I32, I32, I32, I32, I32, I64, P, P, P, P, P, P, P, P,
-                                          P, P, P, P, P, I32, P, SZ, P, P, P]),
+        "pic_attention_deviation": (I32, [G, I32, I32, I32, I32, I32, I64, P, P, P, I32, P, P, P,
+                                          P, P, P, P, P, P, P, I32, P, SZ, P, P, P]),
         "pic_append_inline": (I32, [G, I32, I32, I32, P, P, P, P, P, P, I32, I64, P, P, P, SZ,
                                     P]),
         "pic_attend_prefill": (I32, [G, I32, I32, I32, P, P, I32, P, I32, I64, P, P, P, P, I32,
@@ -363,18 +363,21 @@ def pic_attend_decode_noalloc(geom: Geometry, layer: int, q, k_new, v_new, pos, 
 def pic_attention_deviation(geom: Geometry, layer: int, inline_pos, inline_len, query_len,
                             req_doc_ids, doc_len, doc_offset, slot_mapping, tok_map,
                             num_pages: int, k_cache_a, k_cache_b, lse_a, lse_b, workspace,
-                            sums, counts, edges=(0.0, 0.1, 0.9), stream=None):
+                            sums, counts, edges=(0.0, 0.1, 0.9), max_query_len=None,
+                            stream=None):
     """D_r(A, B) of two stitched key caches (see include/pic.h): fills
     sums [B][R] (float64) and counts [B][R] (int64) for the regions between
     consecutive ``edges``."""
     lib = load()
     g = geom._c()
     B, max_inline = inline_pos.shape
+    if max_query_len is None:
+        max_query_len = int(query_len.max().item())
     arr = (ctypes.c_double * len(edges))(*[float(e) for e in edges])
     st = lib.pic_attention_deviation(
         ctypes.byref(g), layer, B, max_inline, req_doc_ids.shape[1], slot_mapping.shape[1],
         num_pages, _ptr(inline_pos, i32, "inline_pos"), _ptr(inline_len, i32, "inline_len"),
-        _ptr(query_len, i32, "query_len"), _ptr(req_doc_ids, i32, "req_doc_ids"),
+        _ptr(query_len, i32, "query_len"), int(max_query_len), _ptr(req_doc_ids, i32, "req_doc_ids"),
         _ptr(doc_len, i32, "doc_len"), _ptr(doc_offset, i32, "doc_offset"),
         _ptr(slot_mapping, i64, "slot_mapping"), _ptr(tok_map, i64, "tok_map"),
         _ptr(k_cache_a, bf16, "k_cache_a"), _ptr(k_cache_b, bf16, "k_cache_b"),

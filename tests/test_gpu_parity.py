@@ -462,12 +462,16 @@ def test_per_layer_rotary_tables(cuda_lib):
             assert ok, f"decode layer {layer} req {b}: {max_abs:.2e} {row:.2e}"
 
 
-@pytest.mark.parametrize("name", ["spans_b2", "llama8b_1layer"])
-def test_attention_deviation_matches_oracle(cuda_lib, name):
+@pytest.mark.parametrize("name,rows", [("spans_b2", "query"), ("llama8b_1layer", "query"),
+                                       ("spans_d64", "query"), ("boundary_blocks", "query"),
+                                       ("spans_b2", "inline"), ("boundary_blocks", "inline")])
+def test_attention_deviation_matches_oracle(cuda_lib, name, rows):
     """D_r(A, B) of the diagnostic on the GPU against the oracle, with A = the
     relocated cache and B = the same documents copied at their compiled
     positions (no re-rotation: every delta 0), over the paper's pre / int
-    regions and a four-region split."""
+    regions and a four-region split.  rows="inline" takes every inline token
+    as a query row: prefix and span rows come before later documents, whose
+    keys they do not see."""
     import paper_2607_28069_gb300 as pic
     from paper_2607_28069_gb300.pipeline import CacheHitPath
     wl = generate(SMALL[name], device="cuda", gen_device="cpu")
@@ -480,7 +484,10 @@ def test_attention_deviation_matches_oracle(cuda_lib, name):
     pic.pic_relocate(Bp.geom, wl.k_pool, wl.v_pool, Bp.tok_map, torch.zeros_like(Bp.doc_delta),
                      Bp.slot_mapping, wl.num_pages, Bp.k_cache, Bp.v_cache, 0, spec.layers)
     theta = theta_of(spec)
-    query_len = torch.full((spec.batch,), spec.query_len, dtype=torch.int32, device="cuda")
+    if rows == "query":
+        query_len = torch.full((spec.batch,), spec.query_len, dtype=torch.int32, device="cuda")
+    else:
+        query_len = wl.inline_len.to(torch.int32).clone()
     for edges in ((0.0, 0.1, 0.9), (0.0, 0.25, 0.5, 0.75, 1.0)):
         R = len(edges) - 1
         for layer in range(spec.layers):
@@ -499,12 +506,12 @@ def test_attention_deviation_matches_oracle(cuda_lib, name):
             for b in range(spec.batch):
                 lay = oracle_layout(wl, b)
                 docs, k_docs, v_docs, q, k, v = request_inputs(wl, b, layer)
-                base = wl.doc_base_pos.cpu().numpy().copy()
+                base = wl.doc_base_pos.cpu().numpy()
                 Ka, _ = O.dense_context(lay, k_docs, v_docs, base, k, v, theta, storage="bf16")
-                for i, dd in enumerate(docs):       # B: every document left where it was compiled
-                    base[dd] = lay.doc_offset[i]
-                Kb, _ = O.dense_context(lay, k_docs, v_docs, base, k, v, theta, storage="bf16")
-                tq = spec.query_len
+                Kb = Ka.copy()       # B: every document occurrence as compiled (delta 0)
+                for i, kd in enumerate(k_docs):
+                    Kb[lay.doc_offset[i]:lay.doc_offset[i] + kd.shape[0]] = kd
+                tq = int(query_len[b])
                 qp = lay.inline_pos[-tq:]
                 qr = O.round_bf16(O.rotary(q[-tq:], qp[:, None], theta))
                 lens = [int(wl.doc_len[dd]) for dd in docs]
