@@ -551,7 +551,7 @@ def main_gpu(args, rank, world):
         def dev_call():
             pic.pic_attention_deviation(pathA.geom, 0, pathA.inline_pos, wl.inline_len, qlen,
                                         wl.req_doc_ids, wl.doc_len, pathA.doc_offset,
-                                        pathA.slot_mapping, pathA.tok_map, wl.num_pages,
+                                        pathA.slot_mapping, wl.num_pages,
                                         pathA.k_cache, pathB.k_cache, pathA.lse[0], pathB.lse[0],
                                         pathA.ws_prefill, dsum, dcnt, (0.0, 0.1, 0.9),
                                         max_query_len=spec.query_len)

@@ -316,7 +316,8 @@ pic_status_t pic_attend_prefill_fused(const pic_geom_t *geom, int32_t layer, int
  *     sums[b][i]   = sum over those rows, heads and keys of |p_A - p_B|
  *     counts[b][i] = the number of terms          (D_i = sums / counts)
  * Inputs (device): inline_pos, inline_len, query_len, req_doc_ids, doc_len,
- *   doc_offset, slot_mapping, tok_map as from pic_compose / pic_link;
+ *   doc_offset (ascending, -1 past the request's documents), slot_mapping as
+ *   from pic_compose / pic_link;
  *   k_cache_a, k_cache_b bf16 paged caches (layout of pic_relocate); lse_a,
  *   lse_b float [batch][max_inline][Hq]; workspace: the prefill workspace
  *   after pic_append_inline (its packed rotated queries are read).
@@ -326,7 +327,9 @@ pic_status_t pic_attend_prefill_fused(const pic_geom_t *geom, int32_t layer, int
  * Outputs (device, overwritten): sums double [batch][n_regions], counts
  *   int64 [batch][n_regions].  Two memsets and one launch on `stream`: a
  *   tcgen05 kernel (both score matrices on the tensor cores; a diagnostic,
- *   off the serving path).
+ *   off the serving path).  Each CTA keeps its request's document table in
+ *   shared memory: PIC_ERR_UNSUPPORTED when max_docs x 4 (n_regions + 3)
+ *   bytes do not fit beside the tiles (about 60 KB: 1500-3000 documents).
  */
 pic_status_t pic_attention_deviation(const pic_geom_t *geom, int32_t layer, int32_t batch,
                                      int32_t max_inline, int32_t max_docs, int32_t max_ctx,
@@ -335,7 +338,7 @@ pic_status_t pic_attention_deviation(const pic_geom_t *geom, int32_t layer, int3
                                      int32_t max_query_len, const int32_t *req_doc_ids,
                                      const int32_t *doc_len,
                                      const int32_t *doc_offset, const int64_t *slot_mapping,
-                                     const int64_t *tok_map, const void *k_cache_a,
+                                     const void *k_cache_a,
                                      const void *k_cache_b, const float *lse_a,
                                      const float *lse_b, const double *edges, int32_t n_regions,
                                      const void *workspace, size_t workspace_bytes, double *sums,

@@ -116,7 +116,7 @@ def load():
                            I32, I32, I32, P, P, P, P, P, P, P, P, P, P, P, P, P, SZ, P]),
         "pic_prefill_workspace_size": (SZ, [G, I32, I32, I32, I32]),
         "pic_attention_deviation": (I32, [G, I32, I32, I32, I32, I32, I64, P, P, P, I32, P, P, P,
-                                          P, P, P, P, P, P, P, I32, P, SZ, P, P, P]),
+                                          P, P, P, P, P, P, I32, P, SZ, P, P, P]),
         "pic_append_inline": (I32, [G, I32, I32, I32, P, P, P, P, P, P, I32, I64, P, P, P, SZ,
                                     P]),
         "pic_attend_prefill": (I32, [G, I32, I32, I32, P, P, I32, P, I32, I64, P, P, P, P, I32,
@@ -361,7 +361,7 @@ def pic_attend_decode_noalloc(geom: Geometry, layer: int, q, k_new, v_new, pos, 
 
 
 def pic_attention_deviation(geom: Geometry, layer: int, inline_pos, inline_len, query_len,
-                            req_doc_ids, doc_len, doc_offset, slot_mapping, tok_map,
+                            req_doc_ids, doc_len, doc_offset, slot_mapping,
                             num_pages: int, k_cache_a, k_cache_b, lse_a, lse_b, workspace,
                             sums, counts, edges=(0.0, 0.1, 0.9), max_query_len=None,
                             stream=None):
@@ -379,7 +379,7 @@ def pic_attention_deviation(geom: Geometry, layer: int, inline_pos, inline_len, 
         num_pages, _ptr(inline_pos, i32, "inline_pos"), _ptr(inline_len, i32, "inline_len"),
         _ptr(query_len, i32, "query_len"), int(max_query_len), _ptr(req_doc_ids, i32, "req_doc_ids"),
         _ptr(doc_len, i32, "doc_len"), _ptr(doc_offset, i32, "doc_offset"),
-        _ptr(slot_mapping, i64, "slot_mapping"), _ptr(tok_map, i64, "tok_map"),
+        _ptr(slot_mapping, i64, "slot_mapping"),
         _ptr(k_cache_a, bf16, "k_cache_a"), _ptr(k_cache_b, bf16, "k_cache_b"),
         _ptr(lse_a, f32, "lse_a"), _ptr(lse_b, f32, "lse_b"), ctypes.cast(arr, ctypes.c_void_p),
         len(edges) - 1,

@@ -19,8 +19,10 @@
 namespace pic {
 namespace {
 
-constexpr int kThreads = 320;  // warp 0 TMA producer, warp 1 MMA issuer, warps 2-9 compute
+// warp 0 TMA producer, warp 1 MMA issuer, warps 2-9 compute, warp 10 key regions
+constexpr int kThreads = 352;
 constexpr int kComputeWarps = 8;  // two per TMEM lane quarter, each on half the key columns
+constexpr int kRegionWarp = 10;
 constexpr int BM = 128;        // query rows per tile (TMEM lanes)
 constexpr int BN = 128;        // key positions per tile
 constexpr int NS = 2;          // K stages, each a tile of cache A and one of cache B
@@ -34,8 +36,12 @@ struct DLayout {
   static constexpr int kK = kQ + BM * D * 2;      // stage st: A at kK + 2 st kTile, B after it
   static constexpr int kReg = kK + NS * 2 * kTile;  // int8 region of each key, [2][BN]
   static constexpr int kBar = kReg + 2 * BN;
-  static constexpr int kBytes = kBar + 256;
-  static constexpr int kAlloc = kBytes + 1024;
+  static constexpr int kTable = kBar + 256;  // document table, sized at launch
+  // offsets and lengths int32 [max_docs] each, then the region bounds
+  // int32 [max_docs][n_regions + 1]
+  static size_t alloc(int max_docs, int n_regions) {
+    return 1024 + kTable + (size_t)max_docs * 4 * (n_regions + 3);
+  }
 };
 
 enum {
@@ -44,7 +50,8 @@ enum {
   DB_KEMPTY = DB_KFULL + NS,
   DB_SFULL = DB_KEMPTY + NS,  // per S buffer
   DB_SFREE = DB_SFULL + 2,    // per S buffer, one arrival per compute warp
-  DB_FINAL = DB_SFREE + 2,
+  DB_RFULL = DB_SFREE + 2,    // per region buffer (the region bytes of a tile)
+  DB_FINAL = DB_RFULL + 2,
   DB_COUNT = DB_FINAL + 1
 };
 
@@ -52,7 +59,7 @@ struct DevArgs {
   int Hq, Hkv, G, max_inline, max_docs, max_ctx, R_pad, n_regions, splits;
   long long num_pages, layer_row0, oob_row;
   const int32_t *inline_pos, *inline_len, *query_len, *ids, *doc_len, *doc_offset;
-  const int64_t *slots, *tok_map;
+  const int64_t *slots;
   const float *lse_a, *lse_b;
   double edges[kMaxRegions + 1];
   double *sums;
@@ -61,37 +68,69 @@ struct DevArgs {
   float scale_log2;
 };
 
-// Region of the document token at logical position t of request b (-1: not
-// a document token, or in no region).
-__device__ int key_region(const DevArgs &a, int b, long long t) {
-  if (t < 0 || t >= a.max_ctx) return -1;
-  const long long tm = a.tok_map[(size_t)b * a.max_ctx + t];
-  if (tm < 0) return -1;
-  const int k = (int)(tm >> 40);
-  if (k >= a.max_docs) return -1;
-  const int id = a.ids[(size_t)b * a.max_docs + k];
-  const int n = id >= 0 ? a.doc_len[id] : 0;
-  const long long j = t - a.doc_offset[(size_t)b * a.max_docs + k];
-  int reg = -1;
-  for (int i = 0; i < a.n_regions && n > 0; ++i)
-    if (j >= (long long)ceil(a.edges[i] * n) && j < (long long)ceil(a.edges[i + 1] * n)) reg = i;
-  return reg;
+// The request's document table in shared memory: the documents' offsets
+// ascend (canonical order), so the document holding a logical position t is
+// the last one starting at or before t, and t - offset is its token index.
+// doc_at: that document (0 when t precedes every document), by bisection.
+__device__ int doc_at(const int32_t *s_off, int m, long long t) {
+  int lo = 0, hi = m - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (s_off[mid] <= t) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+// Regions of the keys at logical positions t .. t+3 (-1: not a document
+// token, or in no region), packed one byte per key, searching forward from
+// document k, which starts at or before t (or is document 0).  One document
+// lookup serves the four keys unless the next document starts among them.
+__device__ uint32_t four_regions(const int32_t *s_off, const int32_t *s_bnd, int m, int R1, int k,
+                                 long long t) {
+  if (m == 0) return 0xffffffffu;
+  while (k + 1 < m && s_off[k + 1] <= t) ++k;
+  long long off = s_off[k], nxt = k + 1 < m ? s_off[k + 1] : LLONG_MAX;
+  int bd[kMaxRegions + 1];
+#pragma unroll
+  for (int i = 0; i <= kMaxRegions; ++i) bd[i] = i < R1 ? s_bnd[k * R1 + i] : 0;
+  uint32_t packed = 0;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const long long te = t + e;
+    if (te >= nxt) {
+      while (k + 1 < m && s_off[k + 1] <= te) ++k;
+      off = s_off[k];
+      nxt = k + 1 < m ? s_off[k + 1] : LLONG_MAX;
+#pragma unroll
+      for (int i = 0; i <= kMaxRegions; ++i) bd[i] = i < R1 ? s_bnd[k * R1 + i] : 0;
+    }
+    int reg = -1;
+    const long long jj = te - off;  // negative before the first document
+#pragma unroll
+    for (int i = 0; i < kMaxRegions; ++i)
+      if (i + 1 < R1 && jj >= bd[i] && jj < bd[i + 1]) reg = i;
+    packed |= (uint32_t)(uint8_t)(int8_t)reg << (8 * e);
+  }
+  return packed;
 }
 
 // CTA = (128-row query tile, key split, kv head, request).  Per 128-key tile
 // of the documents' span: the producer loads the tile of both caches (page
-// boxes through the block layout, as the prefill attention does) and writes
-// the key regions; the issuer computes S_A = Q K_A^T and S_B = Q K_B^T into a
-// TMEM buffer (two buffers, so the next tile's MMAs overlap this one's
-// exponentials); each compute thread owns one query row, reads both rows of
-// scores from TMEM 32 columns at a time and adds |p_A - p_B| to its region.
+// boxes through the block layout, as the prefill attention does), one after
+// the other, and the region warp writes the tile's key regions; the issuer
+// computes [S_A S_B] = Q [K_A; K_B]^T, one N = 256 MMA per 16-deep slice,
+// into a TMEM buffer (two buffers, so the next tile's MMAs overlap this
+// one's exponentials); each compute thread owns one query row, reads both
+// rows of scores from TMEM 32 columns at a time and adds |p_A - p_B| to its
+// region.
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     deviation_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_ka,
                      const __grid_constant__ CUtensorMap tm_kb, DevArgs a) {
   using L = DLayout<D>;
   constexpr int PANELS = D / 64;
-  constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
+  constexpr uint32_t IDESC_QK = idesc_bf16(BM, 2 * BN, false, false);
   constexpr uint32_t kPageBytes = 16 * D * 2;
   constexpr uint32_t kGroupStride = PANELS == 2 ? 2048 : 1024;
   constexpr uint32_t kPanelOff = PANELS == 2 ? 1024 : BN * 128;
@@ -115,9 +154,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(bar(i), (i == DB_SFREE || i == DB_SFREE + 1) ? kComputeWarps : 1);
     *abort_flag = 0;
     fence_mbar_init();
-    int m = 0;  // documents of the request: doc_offset is -1 past them
-    while (m < a.max_docs && a.doc_offset[(size_t)b * a.max_docs + m] >= 0) ++m;
-    s_m = m;
+    s_m = a.max_docs;
   }
   if (tid < kMaxRegions) s_sum[tid] = 0.0;
   if (warp == 1) {
@@ -129,6 +166,27 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tbase = *tmem_slot;
 
+  // ---- the request's document table: offset, length and region bounds
+  // ceil(e_i n) (double-precision products) of each document; the request's
+  // documents end at the first doc_offset of -1
+  const int R1 = a.n_regions + 1;
+  int32_t *s_off = reinterpret_cast<int32_t *>(smem + L::kTable);
+  int32_t *s_len = s_off + a.max_docs;
+  int32_t *s_bnd = s_len + a.max_docs;
+  for (int k = tid; k < a.max_docs; k += kThreads) {
+    const int off = a.doc_offset[(size_t)b * a.max_docs + k];
+    if (off < 0) {
+      atomicMin(&s_m, k);
+      continue;
+    }
+    const int id = a.ids[(size_t)b * a.max_docs + k];
+    const int nk = id >= 0 ? a.doc_len[id] : 0;
+    s_off[k] = off;
+    s_len[k] = nk;
+    for (int i = 0; i < R1; ++i) s_bnd[k * R1 + i] = (int)ceil(a.edges[i] * nk);
+  }
+  __syncthreads();
+
   // ---- the work of this CTA (uniform)
   const int tin = min(max(a.inline_len[b], 0), a.max_inline);
   const int tq = min(max(a.query_len[b], 0), tin);
@@ -137,9 +195,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int m = s_m;
   long long key_lo = 0, key_hi = 0;
   if (m > 0) {
-    key_lo = a.doc_offset[(size_t)b * a.max_docs];
-    const int id = a.ids[(size_t)b * a.max_docs + m - 1];
-    key_hi = a.doc_offset[(size_t)b * a.max_docs + m - 1] + (id >= 0 ? a.doc_len[id] : 0);
+    key_lo = s_off[0];
+    key_hi = (long long)s_off[m - 1] + s_len[m - 1];
   }
   const int kt0 = (int)(key_lo / BN);
   const int n_kt = key_hi > key_lo ? (int)((key_hi - 1) / BN) - kt0 + 1 : 0;
@@ -148,16 +205,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int n = max(0, min(per, n_kt - kv_begin));
 
   // the number of terms of each region: one CTA per request
-  if (qt == 0 && split == 0 && hk == 0 && warp >= 2)
-    for (int k = tid - 64; k < m; k += 32 * kComputeWarps) {
-      const int id = a.ids[(size_t)b * a.max_docs + k];
-      const int nk = id >= 0 ? a.doc_len[id] : 0;
-      for (int i = 0; i < a.n_regions && nk > 0; ++i) {
-        const long long lo = (long long)ceil(a.edges[i] * nk), hi = (long long)ceil(a.edges[i + 1] * nk);
+  if (qt == 0 && split == 0 && hk == 0 && warp >= 2 && warp < 2 + kComputeWarps)
+    for (int k = tid - 64; k < m; k += 32 * kComputeWarps)
+      for (int i = 0; i < a.n_regions; ++i) {
+        const long long lo = s_bnd[k * R1 + i], hi = s_bnd[k * R1 + i + 1];
         if (hi > lo)
           atomicAdd(&a.counts[(size_t)b * a.n_regions + i], (unsigned long long)(hi - lo) * tq * a.Hq);
       }
-    }
 
   if (r0 < row_end && n > 0) {
     if (warp == 0) {
@@ -172,22 +226,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int pn = 0; pn < PANELS; ++pn)
           tma_load_2d(sbase + L::kQ + pn * BM * 128, &tm_q, pn * 64, qrow, bar(DB_Q));
       }
+      // lanes 0..7: the slot of the first position of page `lane` of tile
+      // jj, loaded one tile ahead so that the TMA issue never waits on it
+      auto load_slot = [&](int jj) -> long long {
+        if (lane >= 8 || jj >= n) return -1;
+        const long long t = ((long long)(kt0 + kv_begin + jj) * 8 + lane) * 16;
+        return t < a.max_ctx ? a.slots[(size_t)b * a.max_ctx + t] : -1;
+      };
+      long long slot_next = load_slot(0);
       for (int j = 0; j < n; ++j) {
-        const int st = j % NS, kt = kt0 + kv_begin + j;
+        const int st = j % NS;
+        const long long slot = slot_next;
+        slot_next = load_slot(j + 1);
+        int y = (int)a.oob_row;  // lanes 0..7: page row of page `lane` of the tile
+        if (slot >= 0 && (slot >> 4) < a.num_pages)
+          y = (int)(a.layer_row0 + ((slot >> 4) * a.Hkv + hk) * 16);
         bool ok = true;
         if (j >= NS) ok = mbar_wait(bar(DB_KEMPTY + st), ((j / NS) - 1) & 1, abort_flag, a.status, b);
-        if (ok && j >= 2) ok = mbar_wait(bar(DB_SFREE + (j & 1)), ((j >> 1) - 1) & 1, abort_flag, a.status, b);
         if (!__all_sync(0xffffffffu, ok)) break;
-        for (int c = lane; c < BN; c += 32)
-          s_reg[(j & 1) * BN + c] = (int8_t)key_region(a, b, (long long)kt * BN + c);
-        int y = (int)a.oob_row;  // lanes 0..7: page row of page `lane` of the tile
-        if (lane < 8) {
-          const long long t = ((long long)kt * 8 + lane) * 16;
-          const long long slot = t < a.max_ctx ? a.slots[(size_t)b * a.max_ctx + t] : -1;
-          if (slot >= 0 && (slot >> 4) < a.num_pages)
-            y = (int)(a.layer_row0 + ((slot >> 4) * a.Hkv + hk) * 16);
-        }
-        __syncwarp();
         if (lane == 0) mbar_expect_tx(bar(DB_KFULL + st), 2 * L::kTile);
         __syncwarp();
         if (lane < 8) {
@@ -200,6 +256,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_2d(dst + L::kTile, &tm_kb, 0, y, bar(DB_KFULL + st));
           }
         }
+      }
+    } else if (warp == kRegionWarp) {
+      // ================================================ key regions
+      // Lane l writes the regions of keys 4l .. 4l+3 of each tile; the bytes
+      // go where tile j - 2's were, once its scores are consumed.
+      int kc = m > 0 ? doc_at(s_off, m, (long long)(kt0 + kv_begin) * BN) : 0;
+      for (int j = 0; j < n; ++j) {
+        const long long t0 = (long long)(kt0 + kv_begin + j) * BN;
+        const uint32_t packed = four_regions(s_off, s_bnd, m, R1, kc, t0 + 4 * lane);
+        while (kc + 1 < m && s_off[kc + 1] <= t0 + BN) ++kc;
+        bool ok = true;
+        if (j >= 2) ok = mbar_wait(bar(DB_SFREE + (j & 1)), ((j >> 1) - 1) & 1, abort_flag, a.status, b);
+        if (!__all_sync(0xffffffffu, ok)) break;
+        reinterpret_cast<uint32_t *>(s_reg + (j & 1) * BN)[lane] = packed;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(DB_RFULL + (j & 1)));
       }
     } else if (warp == 1) {
       // ================================================ MMA issuer
@@ -214,15 +286,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (ok && j >= 2) ok = mbar_wait(bar(DB_SFREE + buf), ((j >> 1) - 1) & 1, abort_flag, a.status, b);
           if (!ok) break;
           tc_fence_after();
-          const uint32_t tSA = tbase + buf * 256, tSB = tSA + 128;
-          const uint64_t dka = dK + (uint64_t)((st * 2 * L::kTile) >> 4);
-          const uint64_t dkb = dka + (uint64_t)(L::kTile >> 4);
+          // K_B's tile follows K_A's with the same 8-row group stride, so
+          // one 256-row operand covers both: S_A in columns 0..127 of the
+          // buffer, S_B in 128..255
+          const uint32_t tS = tbase + buf * 256;
+          const uint64_t dk = dK + (uint64_t)((st * 2 * L::kTile) >> 4);
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
             const uint64_t qd = dQ + ((kk >> 2) * (BM * 128) + (kk & 3) * 32) / 16;
             const uint64_t ko = ((kk >> 2) * kPanelOff + (kk & 3) * 32) / 16;
-            mma_ss(tSA, qd, dka + ko, IDESC_QK, kk > 0);
-            mma_ss(tSB, qd, dkb + ko, IDESC_QK, kk > 0);
+            mma_ss(tS, qd, dk + ko, IDESC_QK, kk > 0);
           }
           mma_commit(bar(DB_SFULL + buf));
           mma_commit(bar(DB_KEMPTY + st));
@@ -231,13 +304,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     } else {
       // ================================================ compute warps
-      // Two warps per TMEM lane quarter, each on 64 of the 128 key columns.
-      // Keys come in runs of one region (the producer's bytes, the same for
-      // every row): |p_A - p_B| is summed per run and added to the run's
-      // region when the region changes.  A key after a row's position (an
-      // inline span taken as a query row before a later document) has
-      // p_A = p_B = 0; 32-key chunks that every row of the warp sees skip
-      // that test.
+      // Two warps per TMEM lane quarter, each on 64 of the 128 key columns,
+      // 32 at a time.  The 32 terms of a chunk are computed without branches
+      // (the exponentials pipeline); a chunk whose keys all lie in one region
+      // (the region bytes are the same for every row) is summed at once, one
+      // in no region is skipped, and only a chunk across a region or
+      // document boundary is summed key by key.  A key after a row's
+      // position (an inline span taken as a query row before a later
+      // document) has p_A = p_B = 0.
       const int wq = warp & 3, half = (warp - 2) >> 2;
       const int row = wq * 32 + lane, rg = r0 + row;
       float la = INFINITY, lb = INFINITY;  // rows past the query rows add nothing
@@ -249,57 +323,72 @@ __global__ void __launch_bounds__(kThreads, 1)
         lb = a.lse_b[li] * 1.4426950408889634f;
         qpos = a.inline_pos[(size_t)b * a.max_inline + tok];
       }
-      long long wmin = qpos;
-#pragma unroll
-      for (int o = 16; o; o >>= 1) wmin = min(wmin, __shfl_xor_sync(0xffffffffu, wmin, o));
       const uint32_t tl = tbase + ((uint32_t)(wq * 32) << 16) + half * 64;
       float acc[kMaxRegions];
 #pragma unroll
       for (int i = 0; i < kMaxRegions; ++i) acc[i] = 0.f;
-      int cur = -1;
-      float run = 0.f;
-      auto flush = [&]() {
+      auto add_to = [&](int reg, float v) {
 #pragma unroll
         for (int i = 0; i < kMaxRegions; ++i)
-          if (i == cur) acc[i] += run;
-        run = 0.f;
+          if (i == reg) acc[i] += v;
       };
       for (int j = 0; j < n; ++j) {
-        const int st = j % NS, buf = j & 1;
-        // K(j) landed (also publishes the producer's region bytes), S(j) ready
-        bool ok = mbar_wait(bar(DB_KFULL + st), (j / NS) & 1, abort_flag, a.status, b);
+        const int buf = j & 1;
+        // the region bytes of tile j written, S(j) ready
+        bool ok = mbar_wait(bar(DB_RFULL + buf), (j >> 1) & 1, abort_flag, a.status, b);
         if (ok) ok = mbar_wait(bar(DB_SFULL + buf), (j >> 1) & 1, abort_flag, a.status, b);
         if (!__all_sync(0xffffffffu, ok)) break;
         tc_fence_after();
 #pragma unroll 1
         for (int c0 = 0; c0 < 64; c0 += 32) {
+          const int8_t *rr = s_reg + buf * BN + half * 64 + c0;
+          const uint4 w0 = *reinterpret_cast<const uint4 *>(rr);
+          const uint4 w1 = *reinterpret_cast<const uint4 *>(rr + 16);
+          const int reg0 = rr[0];
+          const uint32_t rep = (uint32_t)(uint8_t)rr[0] * 0x01010101u;
+          const bool uniform = w0.x == rep && w0.y == rep && w0.z == rep && w0.w == rep &&
+                               w1.x == rep && w1.y == rep && w1.z == rep && w1.w == rep;
+          if (uniform && reg0 < 0) continue;  // no key of the chunk is in a region
           float sa[32], sb[32];
           tmem_ld32(tl + buf * 256 + c0, reinterpret_cast<uint32_t *>(sa));
           tmem_ld32(tl + buf * 256 + 128 + c0, reinterpret_cast<uint32_t *>(sb));
           tmem_wait_ld();
-          const int8_t *rr = s_reg + buf * BN + half * 64 + c0;
+          // keys 0..lim of the chunk are at or before this row's position;
+          // chunks every row of the warp sees skip the test
           const long long t0 = (long long)(kt0 + kv_begin + j) * BN + half * 64 + c0;
-          if (t0 + 31 <= wmin) {
+          const int lim = (int)min(max(qpos - t0, -1ll), 31ll);
 #pragma unroll
-            for (int c = 0; c < 32; ++c) {
-              const int reg = rr[c];
-              if (reg != cur) {  // the same for every thread: no divergence
-                flush();
-                cur = reg;
-              }
-              if (reg >= 0)
-                run += fabsf(ex2(fmaf(sa[c], a.scale_log2, -la)) - ex2(fmaf(sb[c], a.scale_log2, -lb)));
+          for (int c = 0; c < 32; ++c) {
+            const float d = fabsf(ex2(fmaf(sa[c], a.scale_log2, -la)) - ex2(fmaf(sb[c], a.scale_log2, -lb)));
+            sa[c] = c <= lim ? d : 0.f;
+          }
+          if (uniform) {
+            float v0 = 0.f, v1 = 0.f, v2 = 0.f, v3 = 0.f;
+#pragma unroll
+            for (int c = 0; c < 32; c += 4) {
+              v0 += sa[c];
+              v1 += sa[c + 1];
+              v2 += sa[c + 2];
+              v3 += sa[c + 3];
             }
+            add_to(reg0, (v0 + v1) + (v2 + v3));
           } else {
+            // a region or document boundary inside the chunk: one masked
+            // sum per region, with no branch between the terms (a branch per
+            // key would serialise the exponentials above)
+            int rg[32];
 #pragma unroll
-            for (int c = 0; c < 32; ++c) {
-              const int reg = rr[c];
-              if (reg != cur) {
-                flush();
-                cur = reg;
+            for (int c = 0; c < 32; ++c) rg[c] = rr[c];
+#pragma unroll
+            for (int i = 0; i < kMaxRegions; ++i) {
+              if (i >= a.n_regions) break;
+              float v0 = 0.f, v1 = 0.f;
+#pragma unroll
+              for (int c = 0; c < 32; c += 2) {
+                v0 += rg[c] == i ? sa[c] : 0.f;
+                v1 += rg[c + 1] == i ? sa[c + 1] : 0.f;
               }
-              if (reg >= 0 && t0 + c <= qpos)
-                run += fabsf(ex2(fmaf(sa[c], a.scale_log2, -la)) - ex2(fmaf(sb[c], a.scale_log2, -lb)));
+              acc[i] += v0 + v1;
             }
           }
         }
@@ -307,7 +396,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(bar(DB_SFREE + buf));
       }
-      flush();
 #pragma unroll
       for (int i = 0; i < kMaxRegions; ++i) {
         double v = acc[i];
@@ -336,7 +424,7 @@ extern "C" pic_status_t pic_attention_deviation(
     int32_t max_ctx, int64_t num_pages, const int32_t *inline_pos, const int32_t *inline_len,
     const int32_t *query_len, int32_t max_query_len, const int32_t *req_doc_ids,
     const int32_t *doc_len,
-    const int32_t *doc_offset, const int64_t *slot_mapping, const int64_t *tok_map,
+    const int32_t *doc_offset, const int64_t *slot_mapping,
     const void *k_cache_a, const void *k_cache_b, const float *lse_a, const float *lse_b,
     const double *edges, int32_t n_regions, const void *workspace, size_t workspace_bytes,
     double *sums, int64_t *counts, pic_stream_t stream) {
@@ -358,7 +446,7 @@ extern "C" pic_status_t pic_attention_deviation(
       return fail(PIC_ERR_INVALID_ARG, "pic_attention_deviation: edges must ascend in [0, 1]");
   }
   if (!inline_pos || !inline_len || !query_len || !req_doc_ids || !doc_len || !doc_offset ||
-      !slot_mapping || !tok_map || !k_cache_a || !k_cache_b || !lse_a || !lse_b || !workspace ||
+      !slot_mapping || !k_cache_a || !k_cache_b || !lse_a || !lse_b || !workspace ||
       !sums || !counts)
     return fail(PIC_ERR_INVALID_ARG, "pic_attention_deviation: NULL tensor");
   const int Hkv = geom->num_kv_heads, G = geom->num_q_heads / Hkv, D = geom->head_dim;
@@ -405,7 +493,6 @@ extern "C" pic_status_t pic_attention_deviation(
   a.doc_len = doc_len;
   a.doc_offset = doc_offset;
   a.slots = slot_mapping;
-  a.tok_map = tok_map;
   a.lse_a = lse_a;
   a.lse_b = lse_b;
   for (int i = 0; i <= kMaxRegions; ++i) a.edges[i] = i <= n_regions ? edges[i] : 1.0;
@@ -414,13 +501,19 @@ extern "C" pic_status_t pic_attention_deviation(
   a.status = status;
   a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
   // query tiles: the query rows of a request are its last query_len inline
-  // tokens times G; key splits: enough CTAs for two waves of the GPU (every
-  // split adds its own partial sums)
+  // tokens times G.  Key splits (every split adds its own partial sums): one
+  // CTA per SM, so a launch takes ceil(CTAs / 152) rounds of one CTA's key
+  // tiles plus about two tiles of pipeline fill; take the split count that
+  // minimises that
   const int q_tiles = (int)(((long long)max_query_len * G + BM - 1) / BM);
   const int kt_max = (max_ctx + BN - 1) / BN;
   const long long groups = (long long)batch * Hkv * std::max(q_tiles, 1);
-  a.splits = (int)std::max<long long>(1, std::min<long long>(std::min(kt_max, 64),
-                                                             (2 * 152 + groups - 1) / groups));
+  a.splits = 1;
+  long long best = -1;
+  for (int sp = 1; sp <= std::min(kt_max, 64); ++sp) {
+    const long long cost = ((groups * sp + 151) / 152) * ((kt_max + sp - 1) / sp + 2);
+    if (best < 0 || cost < best) best = cost, a.splits = sp;
+  }
   cudaError_t e = cudaMemsetAsync(sums, 0, sizeof(double) * batch * n_regions, stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(counts, 0, sizeof(int64_t) * batch * n_regions, stream);
   if (e != cudaSuccess) return cuda_fail(e, "pic_attention_deviation clear");
@@ -428,12 +521,17 @@ extern "C" pic_status_t pic_attention_deviation(
   if ((long long)q_tiles * a.splits > 65535 || batch > 65535 || Hkv > 65535)
     return fail(PIC_ERR_INVALID_ARG, "pic_attention_deviation: grid too large");
   const dim3 grid((unsigned)(q_tiles * a.splits), Hkv, batch);
+  const size_t smem_need = D == 128 ? DLayout<128>::alloc(max_docs, n_regions)
+                                     : DLayout<64>::alloc(max_docs, n_regions);
+  if (smem_need > 227 * 1024)
+    return fail(PIC_ERR_UNSUPPORTED, "pic_attention_deviation: %d documents per request do not fit the "
+                "shared-memory document table", max_docs);
   if (D == 128) {
-    const int smem = DLayout<128>::kAlloc;
+    const int smem = (int)smem_need;
     e = cudaFuncSetAttribute(deviation_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e == cudaSuccess) deviation_kernel<128><<<grid, kThreads, smem, stream>>>(tq, tka, tkb, a);
   } else {
-    const int smem = DLayout<64>::kAlloc;
+    const int smem = (int)smem_need;
     e = cudaFuncSetAttribute(deviation_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e == cudaSuccess) deviation_kernel<64><<<grid, kThreads, smem, stream>>>(tq, tka, tkb, a);
   }

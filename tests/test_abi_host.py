@@ -112,7 +112,7 @@ def _call_deviation_with(geom, edges, n_regions, layer=0, tensors=True):
     return pic.load().pic_attention_deviation(
         ctypes.byref(g), layer, 1, 16, 2, 64, 8,
         fake, fake, fake, 4,                      # inline_pos, inline_len, query_len, max_query_len
-        fake, fake, fake, fake, fake,             # req_doc_ids, doc_len, doc_offset, slots, tok_map
+        fake, fake, fake, fake,                   # req_doc_ids, doc_len, doc_offset, slots
         fake, fake, fake, fake,                   # k_cache_a, k_cache_b, lse_a, lse_b
         ctypes.cast(arr, ctypes.c_void_p), n_regions, fake, 1 << 20, fake, fake, null)
 

@@ -498,7 +498,7 @@ def test_attention_deviation_matches_oracle(cuda_lib, name, rows):
             counts = torch.empty((spec.batch, R), dtype=torch.int64, device="cuda")
             pic.pic_attention_deviation(A.geom, layer, A.inline_pos, wl.inline_len, query_len,
                                         wl.req_doc_ids, wl.doc_len, A.doc_offset, A.slot_mapping,
-                                        A.tok_map, wl.num_pages, A.k_cache, Bp.k_cache,
+                                        wl.num_pages, A.k_cache, Bp.k_cache,
                                         A.lse[layer], Bp.lse[layer], A.ws_prefill, sums, counts,
                                         edges)
             torch.cuda.synchronize()
