@@ -353,42 +353,43 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_ld32(tl + buf * 256 + c0, reinterpret_cast<uint32_t *>(sa));
           tmem_ld32(tl + buf * 256 + 128 + c0, reinterpret_cast<uint32_t *>(sb));
           tmem_wait_ld();
-          // keys 0..lim of the chunk are at or before this row's position;
-          // chunks every row of the warp sees skip the test
+          // keys 0..lim of the chunk are at or before this row's position
           const long long t0 = (long long)(kt0 + kv_begin + j) * BN + half * 64 + c0;
           const int lim = (int)min(max(qpos - t0, -1ll), 31ll);
-#pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            const float d = fabsf(ex2(fmaf(sa[c], a.scale_log2, -la)) - ex2(fmaf(sb[c], a.scale_log2, -lb)));
-            sa[c] = c <= lim ? d : 0.f;
-          }
-          if (uniform) {
+          if (uniform && __all_sync(0xffffffffu, lim == 31)) {
+            // one region, every key visible to every row of the warp: six
+            // instructions a term (two FFMA, two EX2, two FADD)
             float v0 = 0.f, v1 = 0.f, v2 = 0.f, v3 = 0.f;
 #pragma unroll
             for (int c = 0; c < 32; c += 4) {
-              v0 += sa[c];
-              v1 += sa[c + 1];
-              v2 += sa[c + 2];
-              v3 += sa[c + 3];
+              v0 += fabsf(ex2(fmaf(sa[c], a.scale_log2, -la)) - ex2(fmaf(sb[c], a.scale_log2, -lb)));
+              v1 += fabsf(ex2(fmaf(sa[c + 1], a.scale_log2, -la)) - ex2(fmaf(sb[c + 1], a.scale_log2, -lb)));
+              v2 += fabsf(ex2(fmaf(sa[c + 2], a.scale_log2, -la)) - ex2(fmaf(sb[c + 2], a.scale_log2, -lb)));
+              v3 += fabsf(ex2(fmaf(sa[c + 3], a.scale_log2, -la)) - ex2(fmaf(sb[c + 3], a.scale_log2, -lb)));
             }
             add_to(reg0, (v0 + v1) + (v2 + v3));
           } else {
-            // a region or document boundary inside the chunk: one masked
+            // a region or document boundary inside the chunk, or keys after
+            // some row's position: the masked terms first, then one masked
             // sum per region, with no branch between the terms (a branch per
-            // key would serialise the exponentials above)
+            // key would serialise the exponentials)
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+              const float d = fabsf(ex2(fmaf(sa[c], a.scale_log2, -la)) - ex2(fmaf(sb[c], a.scale_log2, -lb)));
+              sa[c] = c <= lim ? d : 0.f;
+            }
             int rg[32];
 #pragma unroll
             for (int c = 0; c < 32; ++c) rg[c] = rr[c];
-#pragma unroll
-            for (int i = 0; i < kMaxRegions; ++i) {
-              if (i >= a.n_regions) break;
+#pragma unroll 1
+            for (int i = 0; i < a.n_regions; ++i) {
               float v0 = 0.f, v1 = 0.f;
 #pragma unroll
               for (int c = 0; c < 32; c += 2) {
                 v0 += rg[c] == i ? sa[c] : 0.f;
                 v1 += rg[c + 1] == i ? sa[c + 1] : 0.f;
               }
-              acc[i] += v0 + v1;
+              add_to(i, v0 + v1);
             }
           }
         }

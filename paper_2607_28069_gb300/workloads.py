@@ -91,6 +91,10 @@ WORKLOADS = {
         "decode_1layer_b16", 1, 28, 4, 128, 1e6, 16, 64, 32, (1024, 1024), (64, 64), 128,
         decode_steps=1,
         description="1 layer of decode_28layer_b16 with one decode step (profiling slice)"),
+    "stress_1layer_b4": WorkloadSpec(
+        "stress_1layer_b4", 1, 32, 8, 128, 5e5, 4, 128, 128, (128, 2048), (64, 64), 512,
+        shared_all_docs=True,
+        description="1 layer of stress_128k_b4 (profiling slice)"),
 }
 
 

@@ -60,6 +60,11 @@ SMALL = {
                                    docs_per_request=9, doc_len=(3, 90), prefix_len=(5, 20),
                                    query_len=12, fixed_order=(0, 2, 1, 0, 3, 1, 0, 4, 1),
                                    span_len=(0, 4), decode_steps=1),
+    # more documents than the three-stage form of the deviation kernel has
+    # room for in its shared-memory document table
+    "many_docs": custom_spec(name="many_docs", layers=1, q_heads=8, kv_heads=2, head_dim=128,
+                             rope_base=5e5, batch=1, pool_docs=80, docs_per_request=80,
+                             doc_len=(4, 40), prefix_len=(2, 8), query_len=16, decode_steps=1),
     "no_docs": custom_spec(name="no_docs", layers=1, q_heads=4, kv_heads=1, head_dim=64,
                            rope_base=1e4, batch=2, pool_docs=1, docs_per_request=0,
                            doc_len=(10, 10), prefix_len=(3, 30), query_len=9, decode_steps=1),
@@ -464,7 +469,8 @@ def test_per_layer_rotary_tables(cuda_lib):
 
 @pytest.mark.parametrize("name,rows", [("spans_b2", "query"), ("llama8b_1layer", "query"),
                                        ("spans_d64", "query"), ("boundary_blocks", "query"),
-                                       ("spans_b2", "inline"), ("boundary_blocks", "inline")])
+                                       ("spans_b2", "inline"), ("boundary_blocks", "inline"),
+                                       ("many_docs", "query")])
 def test_attention_deviation_matches_oracle(cuda_lib, name, rows):
     """D_r(A, B) of the diagnostic on the GPU against the oracle, with A = the
     relocated cache and B = the same documents copied at their compiled
