@@ -607,19 +607,22 @@ def main_gpu(args, rank, world):
     # end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
-        # Per-request inputs packed into one buffer (pipeline API): each step
-        # copies the whole request from pinned host memory in one transfer,
-        # runs the pass and reads the output back.  The graphs captured above
-        # read the same device tensors, now views of the packed buffer, so
-        # they are captured again.
+        # Per-request inputs packed into one pinned host buffer (pipeline
+        # API): every step copies the whole request in and every layer's
+        # attention output back out, overlapped with the compute
+        # (CacheHitPath.served_pass: the per-request fields and layer 0's
+        # projections by the library's copy kernel, later layers' inputs and
+        # earlier layers' outputs on two copy-engine streams, the last
+        # layer's output by the copy kernel), captured as one graph that
+        # reads and writes the same host buffers on every replay.
         host_req = path.pack_request_inputs()
         host_out = torch.empty(path.out.shape, dtype=path.out.dtype, pin_memory=True)
         h2d = host_req.numel()
         d2h = host_out.numel() * host_out.element_size()
+        up_stream, down_stream = torch.cuda.Stream(), torch.cuda.Stream()
         g2 = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g2):
-            for _, fn in (pass_calls if single else calls):
-                fn()
+            path.served_pass(host_req, host_out, up_stream, down_stream)
         torch.cuda.synchronize()
         e_ms = []
         for k in range(W + K):
@@ -627,9 +630,7 @@ def main_gpu(args, rank, world):
             torch.cuda.synchronize()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-            path.upload(host_req)
             g2.replay()
-            host_out.copy_(path.out, non_blocking=True)
             e1.record(stream)
             torch.cuda.synchronize()
             if k >= W:

@@ -108,6 +108,22 @@ const char *pic_last_error(void);
 pic_status_t pic_device_status(pic_stream_t stream, int32_t *code, int32_t *detail);
 
 /*
+ * pic_copy_async -- copy `bytes` from src to dst on `stream`, where each of
+ * src and dst is memory of the current device or page-locked host memory
+ * (cudaHostAlloc, cudaHostRegister, a pinned torch tensor).  Not an
+ * operation of the paper: the transfer of a request's inputs and outputs
+ * that a serving loop performs around the cache-hit path.  The bytes are
+ * moved by a kernel (16-byte loads and stores; host memory is reached over
+ * the chip-to-chip link of a Grace-Blackwell node), which for transfers of a
+ * few megabytes is faster than the copy engines; when either address is not
+ * 16-byte aligned the copy engine moves them instead.  Asynchronous: the
+ * caller keeps both buffers alive and unmodified until the stream reaches
+ * the copy.  Errors: PIC_ERR_INVALID_ARG for NULL, pageable host memory,
+ * another device's memory or overlapping ranges; bytes = 0 does nothing.
+ */
+pic_status_t pic_copy_async(void *dst, const void *src, size_t bytes, pic_stream_t stream);
+
+/*
  * pic_compose -- link operator R: logical layout of each request and its
  * token-level maps (Eqs. 1-2, "Background: Position-Independent Caching";
  * appendix "Logical Layout and Re-Rotation").

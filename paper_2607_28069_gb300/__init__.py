@@ -17,7 +17,7 @@ import torch
 
 __all__ = [
     "Geometry", "load", "lib_path", "pic_abi_version", "pic_compose", "pic_relocate", "pic_link",
-    "pic_attention_deviation",
+    "pic_attention_deviation", "pic_copy_async",
     "pic_append_inline", "pic_attend_prefill", "pic_attend_prefill_fused",
     "pic_prefill_workspace_size",
     "pic_prefill_num_splits", "pic_decode_num_splits", "pic_attend_decode_noalloc",
@@ -38,7 +38,7 @@ EXPORTED_SYMBOLS = (
     "pic_link", "pic_attention_deviation", "pic_prefill_workspace_size", "pic_prefill_num_splits",
     "pic_append_inline",
     "pic_attend_prefill", "pic_attend_prefill_fused", "pic_decode_workspace_size", "pic_decode_num_splits",
-    "pic_attend_decode", "pic_attend_decode_noalloc",
+    "pic_attend_decode", "pic_attend_decode_noalloc", "pic_copy_async",
 )
 
 DEVICE_CODES = {
@@ -109,6 +109,7 @@ def load():
         "pic_abi_version": (I32, []),
         "pic_last_error": (ctypes.c_char_p, []),
         "pic_device_status": (I32, [P, P, P]),
+        "pic_copy_async": (I32, [P, P, SZ, P]),
         "pic_compose": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, P, I32, I64, I32, I32,
                               P, P, P, P, P, P, P]),
         "pic_relocate": (I32, [G, I32, I32, P, P, I64, P, P, P, I32, I64, P, P, I32, I32, P]),
@@ -181,6 +182,23 @@ def pic_device_status(stream=None):
     if st not in (0, 5):
         _check(st, "pic_device_status")
     return code.value, detail.value
+
+
+def pic_copy_async(dst: torch.Tensor, src: torch.Tensor, stream=None):
+    """Copy the bytes of src into dst (see include/pic.h): each a contiguous
+    CUDA tensor of the current device or a pinned CPU tensor, of the same
+    size in bytes.  The GPU's own loads and stores move them."""
+    for t, name in ((dst, "dst"), (src, "src")):
+        if not t.is_contiguous():
+            raise ValueError(f"{name} must be contiguous")
+        if not t.is_cuda and not t.is_pinned():
+            raise ValueError(f"{name} must be a CUDA tensor or pinned host memory")
+    nbytes = dst.numel() * dst.element_size()
+    if src.numel() * src.element_size() != nbytes:
+        raise ValueError("dst and src differ in size")
+    st = load().pic_copy_async(ctypes.c_void_p(dst.data_ptr()), ctypes.c_void_p(src.data_ptr()),
+                               nbytes, _stream(stream))
+    _check(st, "pic_copy_async")
 
 
 def pic_compose(geom: Geometry, doc_len, doc_base_pos, doc_token_start, req_doc_ids,

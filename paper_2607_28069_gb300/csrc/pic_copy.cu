@@ -1,0 +1,95 @@
+// pic_copy_async: host <-> device transfers of a request's inputs and
+// outputs moved by the GPU's own loads and stores.  On a Grace-Blackwell
+// node page-locked host memory is reachable from kernels over the coherent
+// chip-to-chip link, which a kernel with many 16-byte requests in flight
+// drives well above the rate the copy engines reach for transfers of a few
+// megabytes.  Either side may be device memory of the current device or
+// page-locked host memory (cudaHostAlloc / cudaHostRegister, e.g. a pinned
+// torch tensor); the kernel addresses host memory through its device
+// pointer.
+#include "pic_internal.cuh"
+
+namespace pic {
+namespace {
+
+constexpr int kCopyThreads = 256;
+constexpr int kCopyUnroll = 4;  // 16-byte loads in flight per thread
+
+// dst[i] = src[i] for i < n16 (16-byte words), then the tail bytes.
+__global__ void __launch_bounds__(kCopyThreads) copy_kernel(uint4 *__restrict__ dst,
+                                                            const uint4 *__restrict__ src,
+                                                            size_t n16, uint8_t *__restrict__ dst_tail,
+                                                            const uint8_t *__restrict__ src_tail,
+                                                            int tail) {
+  const size_t per_block = (size_t)kCopyThreads * kCopyUnroll;
+  const size_t stride = (size_t)gridDim.x * per_block;
+  for (size_t base = (size_t)blockIdx.x * per_block + threadIdx.x; base < n16; base += stride) {
+    uint4 v[kCopyUnroll];
+#pragma unroll
+    for (int u = 0; u < kCopyUnroll; ++u) {
+      const size_t k = base + (size_t)u * kCopyThreads;
+      if (k < n16) v[u] = src[k];
+    }
+#pragma unroll
+    for (int u = 0; u < kCopyUnroll; ++u) {
+      const size_t k = base + (size_t)u * kCopyThreads;
+      if (k < n16) dst[k] = v[u];
+    }
+  }
+  if (blockIdx.x == 0 && (int)threadIdx.x < tail) dst_tail[threadIdx.x] = src_tail[threadIdx.x];
+}
+
+// The device-side address of p: itself for device memory of the current
+// device, the mapped address for page-locked or managed host memory; NULL
+// for pageable host memory or another device's memory.
+void *device_address(const void *p, int dev) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();  // clear the error the failed query recorded
+    return nullptr;
+  }
+  switch (at.type) {
+    case cudaMemoryTypeDevice:
+      return at.device == dev ? const_cast<void *>(p) : nullptr;
+    case cudaMemoryTypeHost:
+    case cudaMemoryTypeManaged:
+      return at.devicePointer;
+    default:
+      return nullptr;
+  }
+}
+
+}  // namespace
+}  // namespace pic
+
+extern "C" pic_status_t pic_copy_async(void *dst, const void *src, size_t bytes, pic_stream_t stream) {
+  using namespace pic;
+  if (bytes == 0) return PIC_OK;
+  if (!dst || !src) return fail(PIC_ERR_INVALID_ARG, "pic_copy_async: NULL pointer");
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "pic_copy_async device");
+  void *d = device_address(dst, dev);
+  const void *s = device_address(src, dev);
+  if (!d || !s)
+    return fail(PIC_ERR_INVALID_ARG,
+                "pic_copy_async: %s is neither memory of the current device nor page-locked host memory",
+                !d ? "dst" : "src");
+  const uintptr_t du = reinterpret_cast<uintptr_t>(d), su = reinterpret_cast<uintptr_t>(s);
+  if (du < su ? su - du < bytes : du - su < bytes)
+    return fail(PIC_ERR_INVALID_ARG, "pic_copy_async: overlapping ranges");
+  if ((du | su) & 15) {
+    // unaligned: the copy engine moves it
+    e = cudaMemcpyAsync(d, s, bytes, cudaMemcpyDefault, stream);
+    return e == cudaSuccess ? PIC_OK : cuda_fail(e, "pic_copy_async (unaligned)");
+  }
+  const size_t n16 = bytes / 16;
+  const int tail = (int)(bytes % 16);
+  const size_t per_block = (size_t)kCopyThreads * kCopyUnroll;
+  const size_t blocks = std::max<size_t>(1, std::min<size_t>((n16 + per_block - 1) / per_block, 152 * 8));
+  copy_kernel<<<(unsigned)blocks, kCopyThreads, 0, stream>>>(
+      static_cast<uint4 *>(d), static_cast<const uint4 *>(s), n16,
+      static_cast<uint8_t *>(d) + n16 * 16, static_cast<const uint8_t *>(s) + n16 * 16, tail);
+  e = cudaGetLastError();
+  return e == cudaSuccess ? PIC_OK : cuda_fail(e, "pic_copy_async launch");
+}

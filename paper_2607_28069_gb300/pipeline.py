@@ -9,8 +9,8 @@ from __future__ import annotations
 import torch
 
 from . import (Geometry, pic_append_inline, pic_attend_decode, pic_attend_prefill,
-               pic_attend_prefill_fused, pic_compose, pic_decode_workspace_size, pic_link,
-               pic_prefill_workspace_size, pic_relocate)
+               pic_attend_prefill_fused, pic_compose, pic_copy_async, pic_decode_workspace_size,
+               pic_link, pic_prefill_workspace_size, pic_relocate)
 from .workloads import Workload
 
 
@@ -60,7 +60,8 @@ class CacheHitPath:
 
     # -- per-request inputs as one upload
     REQUEST_FIELDS = ("req_doc_ids", "req_num_docs", "prefix_len", "query_len", "block_table",
-                      "inline_len", "q_inline", "k_inline", "v_inline")
+                      "inline_len")
+    LAYER_FIELDS = ("q_inline", "k_inline", "v_inline")
 
     def pack_request_inputs(self) -> torch.Tensor:
         """Move the per-request inputs (document choice, lengths, block table,
@@ -68,14 +69,25 @@ class CacheHitPath:
         workload's tensors to views of it, and return a pinned host mirror
         holding the same bytes.  A serving loop then writes a request into
         the mirror and calls ``upload`` once: one host-to-device copy per
-        step instead of one per tensor.  The document pool stays resident."""
+        step instead of one per tensor.  The document pool stays resident.
+
+        Layout: the per-request fields first, then layer by layer that
+        layer's q, k and v, so that the bytes layer 0 needs are one prefix
+        and each later layer one contiguous range (``served_pass`` streams
+        them)."""
         wl = self.wl
-        offs, total = [], 0
+        L = wl.spec.layers
+        align = lambda n: (n + 255) // 256 * 256  # noqa: E731
         fields = self.REQUEST_FIELDS + (("span_len",) if wl.span_len is not None else ())
+        offs, total = [], 0
         for name in fields:
             t = getattr(wl, name)
             offs.append(total)
-            total += (t.numel() * t.element_size() + 255) // 256 * 256
+            total += align(t.numel() * t.element_size())
+        per_layer = [align(getattr(wl, f)[0].numel() * 2) for f in self.LAYER_FIELDS]
+        layer0 = total
+        layer_bytes = sum(per_layer)
+        total += L * layer_bytes
         dev = torch.empty(total, dtype=torch.uint8, device=wl.k_pool.device)
         host = torch.empty(total, dtype=torch.uint8, pin_memory=True)
         for name, off in zip(fields, offs):
@@ -83,14 +95,75 @@ class CacheHitPath:
             n = t.numel() * t.element_size()
             view = dev[off:off + n].view(t.dtype).view(t.shape)
             view.copy_(t)
-            host[off:off + n].copy_(view.view(torch.uint8).view(-1).cpu())
             setattr(wl, name, view)
+        buf16 = dev.view(torch.bfloat16)
+        off = layer0
+        for f, nb in zip(self.LAYER_FIELDS, per_layer):
+            t = getattr(wl, f)
+            assert t.dtype == torch.bfloat16 and t.is_contiguous()
+            view = torch.as_strided(buf16, t.shape, (layer_bytes // 2,) + t.stride()[1:], off // 2)
+            view.copy_(t)
+            setattr(wl, f, view)
+            off += nb
+        host.copy_(dev.cpu())
         self._request_dev = dev
+        self._layer_ranges = [(layer0 + l * layer_bytes, layer0 + (l + 1) * layer_bytes)
+                              for l in range(L)]
         return host
 
     def upload(self, host: torch.Tensor):
-        """One asynchronous copy of a packed request (see pack_request_inputs)."""
-        self._request_dev.copy_(host, non_blocking=True)
+        """One asynchronous copy of a packed request (see pack_request_inputs),
+        moved by the library's copy kernel (pic_copy_async)."""
+        pic_copy_async(self._request_dev, host)
+
+    def download(self, host_out: torch.Tensor, dev: torch.Tensor | None = None):
+        """Asynchronous copy of the attention outputs (or `dev`) into the pinned
+        host tensor host_out, by the library's copy kernel."""
+        pic_copy_async(host_out, self.out if dev is None else dev)
+
+    def served_pass(self, host: torch.Tensor, host_out: torch.Tensor,
+                    up_stream: torch.cuda.Stream, down_stream: torch.cuda.Stream):
+        """One TTFT pass (as ``ttft_pass``) with the request's inputs taken
+        from the pinned host mirror ``host`` and every layer's attention
+        output written to the pinned ``host_out`` [L][B][T][Hq][d], the
+        copies overlapping the compute: the per-request fields and layer 0's
+        projections go first by the copy kernel; the projections of layers
+        1.. stream in on ``up_stream`` (copy engine; layer l's append waits
+        for its range), and the output of each layer but the last streams
+        out on ``down_stream`` once its attention is done; the last layer's
+        output comes back by the copy kernel.  Returns with the current
+        stream ordered after every copy.  Capturable in a CUDA graph."""
+        L = self.wl.spec.layers
+        main = torch.cuda.current_stream()
+        dev = self._request_dev
+        first = self._layer_ranges[0][1]
+        pic_copy_async(dev[:first], host[:first])
+        up_done = [None] * L
+        if L > 1:
+            up_stream.wait_stream(main)
+            down_stream.wait_stream(main)
+            with torch.cuda.stream(up_stream):
+                for l in range(1, L):
+                    lo, hi = self._layer_ranges[l]
+                    dev[lo:hi].copy_(host[lo:hi], non_blocking=True)
+                    up_done[l] = torch.cuda.Event()
+                    up_done[l].record(up_stream)
+        for l in range(L):
+            if l == 0:
+                self.link(0)
+            else:
+                main.wait_event(up_done[l])
+                self.append(l)
+            self.attend(l)
+            if l < L - 1:
+                down_stream.wait_stream(main)
+                with torch.cuda.stream(down_stream):
+                    host_out[l].copy_(self.out[l], non_blocking=True)
+            else:
+                pic_copy_async(host_out[l], self.out[l])
+        if L > 1:
+            main.wait_stream(up_stream)
+            main.wait_stream(down_stream)
 
     # -- a1: layout and slot map
     def compose(self):

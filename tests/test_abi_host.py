@@ -142,3 +142,12 @@ def test_compose_span_input_is_optional_in_the_binding():
     import inspect
     for fn in (pic.pic_compose, pic.pic_link):
         assert inspect.signature(fn).parameters["span_len"].default is None
+
+
+def test_copy_binding_refuses_pageable_and_mismatched_tensors():
+    import torch
+    a = torch.zeros(64, dtype=torch.uint8)           # pageable host memory
+    with pytest.raises(ValueError):
+        pic.pic_copy_async(a, torch.zeros(64, dtype=torch.uint8))
+    with pytest.raises(ValueError):
+        pic.pic_copy_async(a[::2], a[1::2])            # not contiguous

@@ -370,6 +370,45 @@ def test_packed_request_upload_gives_identical_results():
 
 
 @pytest.mark.gpu
+@pytest.mark.parametrize("name", ["spans_b2", "gqa7_decode", "tiny"])
+@pytest.mark.parametrize("graph", [False, True])
+def test_served_pass_streams_inputs_and_outputs(cuda_lib, name, graph):
+    """served_pass (inputs uploaded and outputs read back per layer, on side
+    streams, overlapping the compute) gives the host the outputs of
+    ttft_pass bit for bit, run eagerly and replayed from a CUDA graph."""
+    from paper_2607_28069_gb300.pipeline import CacheHitPath
+    wl = generate(SMALL[name], device="cuda", gen_device="cpu")
+    path = CacheHitPath(wl)
+    path.ttft_pass()
+    torch.cuda.synchronize()
+    ref_out, ref_k = path.out.clone(), path.k_cache.clone()
+    host = path.pack_request_inputs()
+    host_out = torch.zeros(path.out.shape, dtype=path.out.dtype, pin_memory=True)
+    up, down = torch.cuda.Stream(), torch.cuda.Stream()
+    path.out.zero_()
+    path.k_cache.zero_()
+    path._request_dev.zero_()        # every input must come from the host mirror
+    if graph:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            path.served_pass(host, host_out, up, down)
+        torch.cuda.synchronize()
+        path.out.zero_()
+        path._request_dev.zero_()
+        host_out.zero_()
+        g.replay()
+    else:
+        path.served_pass(host, host_out, up, down)
+    torch.cuda.synchronize()
+    L, B = wl.spec.layers, wl.spec.batch
+    for b in range(B):
+        tin = int(wl.inline_len[b])
+        assert torch.equal(host_out[:, b, :tin], ref_out[:, b, :tin].cpu())
+    assert torch.equal(path.k_cache, ref_k)
+    assert L == host_out.shape[0]
+
+
+@pytest.mark.gpu
 @pytest.mark.parametrize("name,rope_style", [("tiny", 0), ("llama8b_1layer", 0), ("ragged_b3", 0),
                                              ("ragged_b3", 1), ("d64_g8", 0), ("no_docs", 0),
                                              ("spans_b2", 0), ("spans_d64", 1),
