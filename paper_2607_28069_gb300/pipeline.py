@@ -126,34 +126,37 @@ class CacheHitPath:
         """One TTFT pass (as ``ttft_pass``) with the request's inputs taken
         from the pinned host mirror ``host`` and every layer's attention
         output written to the pinned ``host_out`` [L][B][T][Hq][d], the
-        copies overlapping the compute: the per-request fields and layer 0's
-        projections go first by the copy kernel; the projections of layers
-        1.. stream in on ``up_stream`` (copy engine; layer l's append waits
-        for its range), and the output of each layer but the last streams
-        out on ``down_stream`` once its attention is done; the last layer's
-        output comes back by the copy kernel.  Returns with the current
-        stream ordered after every copy.  Capturable in a CUDA graph."""
+        copies overlapping the compute: the per-request fields go first (copy
+        kernel), then the link runs without its append (layout and every
+        layer's relocation need no projections) while layer 0's projections
+        arrive on ``up_stream`` by the copy kernel and those of layers 1..
+        follow by the copy engine; layer l's append waits for its range.
+        The output of each layer but the last streams out on
+        ``down_stream`` once its attention is done; the last layer's output
+        comes back by the copy kernel.  Returns with the current stream
+        ordered after every copy.  Capturable in a CUDA graph."""
         L = self.wl.spec.layers
         main = torch.cuda.current_stream()
         dev = self._request_dev
-        first = self._layer_ranges[0][1]
-        pic_copy_async(dev[:first], host[:first])
-        up_done = [None] * L
-        if L > 1:
-            up_stream.wait_stream(main)
-            down_stream.wait_stream(main)
-            with torch.cuda.stream(up_stream):
-                for l in range(1, L):
-                    lo, hi = self._layer_ranges[l]
+        fields_end = self._layer_ranges[0][0]
+        pic_copy_async(dev[:fields_end], host[:fields_end])
+        up_stream.wait_stream(main)
+        down_stream.wait_stream(main)
+        up_done = []
+        with torch.cuda.stream(up_stream):
+            for l in range(L):
+                lo, hi = self._layer_ranges[l]
+                if l == 0:
+                    pic_copy_async(dev[lo:hi], host[lo:hi])
+                else:
                     dev[lo:hi].copy_(host[lo:hi], non_blocking=True)
-                    up_done[l] = torch.cuda.Event()
-                    up_done[l].record(up_stream)
+                up_done.append(torch.cuda.Event())
+                up_done[l].record(up_stream)
         for l in range(L):
             if l == 0:
-                self.link(0)
-            else:
-                main.wait_event(up_done[l])
-                self.append(l)
+                self.link(-1)
+            main.wait_event(up_done[l])
+            self.append(l)
             self.attend(l)
             if l < L - 1:
                 down_stream.wait_stream(main)
@@ -161,9 +164,8 @@ class CacheHitPath:
                     host_out[l].copy_(self.out[l], non_blocking=True)
             else:
                 pic_copy_async(host_out[l], self.out[l])
-        if L > 1:
-            main.wait_stream(up_stream)
-            main.wait_stream(down_stream)
+        main.wait_stream(up_stream)
+        main.wait_stream(down_stream)
 
     # -- a1: layout and slot map
     def compose(self):
