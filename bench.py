@@ -72,6 +72,23 @@ def src_sha(name):
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
 
+def max_over_ranks(x: float, world: int, device) -> float:
+    """The largest value of x over the ranks of the job (x itself when alone):
+    the job's time is its slowest rank's."""
+    if world <= 1:
+        return x
+    import torch
+    t = torch.tensor([x], device=device, dtype=torch.float64)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(units_per_step: float, steps: int, world: int, total_ms: float) -> float:
+    """Whole-job throughput: the units every rank processed (each rank runs its
+    own replica of the step) over the slowest rank's time."""
+    return units_per_step * steps * world / (total_ms / 1e3)
+
+
 def ncu_traffic(kernel_key, src_file):
     """DRAM bytes per launch from a committed ncu summary, if it was taken on
     the current source of the kernel; else None."""
@@ -435,13 +452,9 @@ def main_gpu(args, rank, world):
     for x in per_call:
         for (name, _), ms in zip(calls, x):
             phase_ms.setdefault(name, []).append(ms)
-    total_ms = sum(step_ms)
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev, dtype=torch.float64)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(sum(step_ms), world, dev)
     ms_per_step = total_ms / K
-    value = work["query_tokens"] * K * world / (total_ms / 1e3)
+    value = job_rate(work["query_tokens"], K, world, total_ms)
 
     # per-row averages over the timed steps (ms per step)
     per_step = {name: sum(v) / K for name, v in phase_ms.items()}
@@ -635,12 +648,8 @@ def main_gpu(args, rank, world):
             torch.cuda.synchronize()
             if k >= W:
                 e_ms.append(e0.elapsed_time(e1))
-        e_total = sum(e_ms)
-        if world > 1:
-            t = torch.tensor([e_total], device=dev, dtype=torch.float64)
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            e_total = float(t.item())
-        e2e = {"value": work["query_tokens"] * K * world / (e_total / 1e3),
+        e_total = max_over_ranks(sum(e_ms), world, dev)
+        e2e = {"value": job_rate(work["query_tokens"], K, world, e_total),
                "unit": "query_tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
     code, detail = pic.pic_device_status()
