@@ -409,7 +409,9 @@ __global__ void __launch_bounds__(kThreads) link_kernel(LinkArgs a, RopeParams r
   auto fill_cs = [&](int layer, int buf) {  // cos/sin of the documents this page touches
     for (int e = tid; e < n_docs * HALF; e += kThreads) {
       const int j = e / HALF, i = e % HALF;
-      s_cs[buf][j][i] = rope_cos_sin(rv.delta[k_first + j], rope_theta(rp, layer, i));
+      const long long dl = rv.delta[k_first + j];
+      s_cs[buf][j][i] = kLayerRope ? rope_cos_sin_fast(dl, rope_theta(rp, layer, i))
+                                   : rope_cos_sin(dl, rope_theta(rp, layer, i));
     }
   };
   fill_cs(a.layer_begin, 0);

@@ -102,7 +102,8 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
     for (int e = tid; e < n_docs * HALF; e += kThreads) {
       const int j = e / HALF, i = e % HALF;
       const int delta = a.delta[(size_t)b * a.max_docs + k_first + j];
-      s_cs[buf][j][i] = rope_cos_sin(delta, rope_theta(rp, layer, i));
+      s_cs[buf][j][i] = kLayerRope ? rope_cos_sin_fast(delta, rope_theta(rp, layer, i))
+                                   : rope_cos_sin(delta, rope_theta(rp, layer, i));
     }
   };
   fill_cs(a.layer_begin, 0);
