@@ -12,8 +12,10 @@
  *
  * Conventions shared by every call
  * --------------------------------
- * - Every tensor pointer is DEVICE memory owned by the caller; the library
- *   allocates nothing and keeps no pointer after a call returns.
+ * - Every tensor pointer is DEVICE memory owned by the caller, except where a
+ *   call says it may also be page-locked host memory (pic_copy_async, the
+ *   output of pic_attend_prefill); the library allocates nothing and keeps no
+ *   pointer after a call returns.
  * - Every call is asynchronous on `stream` (NULL = legacy default stream).
  *   Outputs are valid once the stream has reached the call.
  * - bf16 tensors are IEEE bfloat16, row-major, densely packed, in the layouts
@@ -259,6 +261,10 @@ pic_status_t pic_link(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
  *   per request; inline_len: int32 [batch]; slot_mapping: int64 [batch][max_ctx];
  *   block_table: int32 [batch][max_pages].  Every position must be < max_ctx.
  * out: bf16 [batch][max_inline][Hq][d]; lse: float [batch][max_inline][Hq] or NULL.
+ *   out may be page-locked host memory (cudaHostAlloc, cudaHostRegister): the
+ *   kernels then store the rows there directly (over the chip-to-chip link of
+ *   a Grace-Blackwell node), so a caller that wants the result on the host
+ *   needs no copy; PIC_ERR_INVALID_ARG for pageable memory.
  * workspace: >= pic_prefill_workspace_size(... num_splits ...) bytes, 256-byte
  *   aligned, the same buffer for both calls (pic_append_inline only uses its
  *   leading pic_prefill_workspace_size(..., 1) bytes).

@@ -153,6 +153,15 @@ def _stream(stream) -> ctypes.c_void_p:
     return ctypes.c_void_p(stream.cuda_stream)
 
 
+def _ptr_or_pinned(t: torch.Tensor, dtype, name: str):
+    """Like _ptr, for an output that may also live in pinned host memory."""
+    if not t.is_cuda and t.is_pinned():
+        if t.dtype != dtype or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous {dtype} tensor")
+        return ctypes.c_void_p(t.data_ptr())
+    return _ptr(t, dtype, name)
+
+
 def _ptr(t: Optional[torch.Tensor], dtype, name: str, allow_none=False):
     if t is None:
         if allow_none:
@@ -310,7 +319,7 @@ def pic_attend_prefill(geom: Geometry, layer: int, inline_pos, inline_len, max_c
         ctypes.byref(g), layer, B, max_inline, _ptr(inline_pos, i32, "inline_pos"),
         _ptr(inline_len, i32, "inline_len"), max_ctx, _ptr(block_table, i32, "block_table"),
         block_table.shape[1], num_pages, _ptr(k_cache, bf16, "k_cache"),
-        _ptr(v_cache, bf16, "v_cache"), _ptr(out, bf16, "out"),
+        _ptr(v_cache, bf16, "v_cache"), _ptr_or_pinned(out, bf16, "out"),
         _ptr(lse, f32, "lse", allow_none=True), num_splits,
         _ptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream))
     _check(st, "pic_attend_prefill")

@@ -26,6 +26,25 @@ pic_status_t cuda_fail(cudaError_t e, const char *what) {
   return fail(PIC_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
 }
 
+void *device_address(const void *p) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();  // clear the error the failed query recorded
+    return nullptr;
+  }
+  switch (at.type) {
+    case cudaMemoryTypeDevice:
+      return at.device == dev ? const_cast<void *>(p) : nullptr;
+    case cudaMemoryTypeHost:
+    case cudaMemoryTypeManaged:
+      return at.devicePointer;
+    default:
+      return nullptr;
+  }
+}
+
 int32_t *device_status_ptr() {
   constexpr int kMaxDev = 64;
   static int32_t *ptrs[kMaxDev] = {nullptr};

@@ -39,26 +39,6 @@ __global__ void __launch_bounds__(kCopyThreads) copy_kernel(uint4 *__restrict__ 
   if (blockIdx.x == 0 && (int)threadIdx.x < tail) dst_tail[threadIdx.x] = src_tail[threadIdx.x];
 }
 
-// The device-side address of p: itself for device memory of the current
-// device, the mapped address for page-locked or managed host memory; NULL
-// for pageable host memory or another device's memory.
-void *device_address(const void *p, int dev) {
-  cudaPointerAttributes at;
-  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
-    cudaGetLastError();  // clear the error the failed query recorded
-    return nullptr;
-  }
-  switch (at.type) {
-    case cudaMemoryTypeDevice:
-      return at.device == dev ? const_cast<void *>(p) : nullptr;
-    case cudaMemoryTypeHost:
-    case cudaMemoryTypeManaged:
-      return at.devicePointer;
-    default:
-      return nullptr;
-  }
-}
-
 }  // namespace
 }  // namespace pic
 
@@ -66,15 +46,13 @@ extern "C" pic_status_t pic_copy_async(void *dst, const void *src, size_t bytes,
   using namespace pic;
   if (bytes == 0) return PIC_OK;
   if (!dst || !src) return fail(PIC_ERR_INVALID_ARG, "pic_copy_async: NULL pointer");
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return cuda_fail(e, "pic_copy_async device");
-  void *d = device_address(dst, dev);
-  const void *s = device_address(src, dev);
+  void *d = device_address(dst);
+  const void *s = device_address(src);
   if (!d || !s)
     return fail(PIC_ERR_INVALID_ARG,
                 "pic_copy_async: %s is neither memory of the current device nor page-locked host memory",
                 !d ? "dst" : "src");
+  cudaError_t e;
   const uintptr_t du = reinterpret_cast<uintptr_t>(d), su = reinterpret_cast<uintptr_t>(s);
   if (du < su ? su - du < bytes : du - su < bytes)
     return fail(PIC_ERR_INVALID_ARG, "pic_copy_async: overlapping ranges");

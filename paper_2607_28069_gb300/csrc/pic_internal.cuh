@@ -23,6 +23,10 @@ namespace pic {
 // ---------------------------------------------------------------- host side
 pic_status_t fail(pic_status_t s, const char *fmt, ...);
 pic_status_t cuda_fail(cudaError_t e, const char *what);
+// The address kernels use for p: p itself for memory of the current device,
+// the mapped address for page-locked (or managed) host memory; NULL for
+// pageable host memory or another device's memory.
+void *device_address(const void *p);
 // Address of the current device's status word ({code, detail}).
 int32_t *device_status_ptr();
 // Validates the geometry and fills theta[0..d/2) (fp64 frequencies).

@@ -1493,6 +1493,11 @@ extern "C" pic_status_t pic_attend_prefill(
   if (max_pages <= 0) return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill: max_pages <= 0");
   if (!inline_pos || !inline_len || !block_table || !k_cache || !v_cache || !out)
     return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill: NULL tensor");
+  // out may be page-locked host memory: the kernels then store the rows there
+  out = device_address(out);
+  if (!out)
+    return fail(PIC_ERR_INVALID_ARG,
+                "pic_attend_prefill: out is neither memory of the current device nor page-locked host memory");
   if ((reinterpret_cast<uintptr_t>(k_cache) | reinterpret_cast<uintptr_t>(v_cache) |
        reinterpret_cast<uintptr_t>(out)) & 15)
     return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill: bf16 tensors must be 16-byte aligned");

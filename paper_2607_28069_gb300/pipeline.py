@@ -132,8 +132,9 @@ class CacheHitPath:
         arrive on ``up_stream`` by the copy kernel and those of layers 1..
         follow by the copy engine; layer l's append waits for its range.
         The output of each layer but the last streams out on
-        ``down_stream`` once its attention is done; the last layer's output
-        comes back by the copy kernel.  Returns with the current stream
+        ``down_stream`` once its attention is done; the last layer's
+        attention writes its rows into ``host_out`` itself (pinned host
+        memory, reached over the chip-to-chip link).  Returns with the current stream
         ordered after every copy.  Capturable in a CUDA graph."""
         L = self.wl.spec.layers
         main = torch.cuda.current_stream()
@@ -157,13 +158,13 @@ class CacheHitPath:
                 self.link(-1)
             main.wait_event(up_done[l])
             self.append(l)
-            self.attend(l)
             if l < L - 1:
+                self.attend(l)
                 down_stream.wait_stream(main)
                 with torch.cuda.stream(down_stream):
                     host_out[l].copy_(self.out[l], non_blocking=True)
             else:
-                pic_copy_async(host_out[l], self.out[l])
+                self.attend(l, out=host_out[l])  # the last layer's rows go straight to the host
         main.wait_stream(up_stream)
         main.wait_stream(down_stream)
 
@@ -208,11 +209,14 @@ class CacheHitPath:
                           wl.num_pages, self.k_cache, self.v_cache, self.ws_prefill)
 
     # -- a5: prefill attention of one layer
-    def attend(self, layer: int):
+    def attend(self, layer: int, out: torch.Tensor | None = None):
+        """Prefill attention of one layer into self.out[layer], or into `out`
+        (for instance a pinned host tensor, written by the kernels directly)."""
         wl = self.wl
         pic_attend_prefill(self.geom, layer, self.inline_pos, wl.inline_len, self.max_ctx,
                            wl.block_table, wl.num_pages, self.k_cache, self.v_cache,
-                           self.out[layer], None if self.lse is None else self.lse[layer],
+                           self.out[layer] if out is None else out,
+                           None if self.lse is None else self.lse[layer],
                            self.prefill_splits, self.ws_prefill)
 
     # -- a7: prefill attention reading the documents from the pool (no relocate)

@@ -60,8 +60,8 @@ SMALL = {
                                    docs_per_request=9, doc_len=(3, 90), prefix_len=(5, 20),
                                    query_len=12, fixed_order=(0, 2, 1, 0, 3, 1, 0, 4, 1),
                                    span_len=(0, 4), decode_steps=1),
-    # more documents than the three-stage form of the deviation kernel has
-    # room for in its shared-memory document table
+    # 80 short documents per request: a long document table (the deviation
+    # kernel keeps it in shared memory)
     "many_docs": custom_spec(name="many_docs", layers=1, q_heads=8, kv_heads=2, head_dim=128,
                              rope_base=5e5, batch=1, pool_docs=80, docs_per_request=80,
                              doc_len=(4, 40), prefix_len=(2, 8), query_len=16, decode_steps=1),
@@ -565,3 +565,25 @@ def test_attention_deviation_matches_oracle(cuda_lib, name, rows):
                 got = sums[b].cpu().numpy()
                 np.testing.assert_allclose(got, s_ref, rtol=2e-2, atol=1e-6 * c_ref.max())
                 assert (s_ref > 0).all()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("splits", [1, 0])
+def test_prefill_output_into_pinned_host_memory(cuda_lib, splits):
+    """pic_attend_prefill with `out` in page-locked host memory: the kernels
+    (the attention epilogue with one split, the merge kernel with several)
+    store the rows there, bit for bit the rows they store on the device."""
+    from paper_2607_28069_gb300.pipeline import CacheHitPath
+    wl = generate(SMALL["spans_b2"], device="cuda", gen_device="cpu")
+    path = CacheHitPath(wl, prefill_splits=splits)
+    path.ttft_pass()
+    host = torch.zeros(path.out[0].shape, dtype=path.out.dtype, pin_memory=True)
+    for layer in range(wl.spec.layers):
+        path.append(layer)      # the workspace holds one layer's rotated queries
+        path.attend(layer)
+        host.zero_()
+        path.attend(layer, out=host)
+        torch.cuda.synchronize()
+        for b in range(wl.spec.batch):
+            tin = int(wl.inline_len[b])
+            assert torch.equal(host[b, :tin], path.out[layer, b, :tin].cpu())
