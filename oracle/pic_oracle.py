@@ -36,7 +36,7 @@ What the path computes (SemPIC, "Background: Position-Independent Caching" and
                          one layer: layout, re-rotation, inline RoPE, attention
                          over the stitched context, then ordinary decoding.
 
-Readings where the paper is silent (each is restated in the design doc):
+Readings where the paper is silent:
 * R(p) pairs element i with i + d/2 ("half-split", the convention of the
   Llama/Qwen decoders the paper evaluates); ``style="interleaved"`` pairs
   (2i, 2i+1).  Frequencies theta_i = base^(-2i/d), no scaling, one table for

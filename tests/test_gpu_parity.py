@@ -1,7 +1,7 @@
 """GPU parity: every step of the cache-hit path through the C ABI against the
 CPU oracle on the same seeded inputs.
 
-Bars (written here, derived in the design doc):
+Bars (written here; derived from bf16 rounding and the fp32 arithmetic):
 * layout, slot map, inline positions, ctx: bit-exact;
 * V and every copied value: bit-exact;
 * relocated / rotated K: |g - r| <= 4e-3 max(|r|, 2^-8 rowmax) and row rel-L2 <= 4e-3;
