@@ -587,3 +587,19 @@ def test_prefill_output_into_pinned_host_memory(cuda_lib, splits):
         for b in range(wl.spec.batch):
             tin = int(wl.inline_len[b])
             assert torch.equal(host[b, :tin], path.out[layer, b, :tin].cpu())
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name", ["gqa7_decode", "g16_decode", "spans_b2"])
+def test_decode_split_count_invariance(cuda_lib, name):
+    """Every split of the key range gives the same decode output: the LSE
+    merge is exact up to rounding, so outputs for 1, 3 and the automatic
+    number of splits agree within 1e-3 (max-abs)."""
+    outs = []
+    for splits in (1, 3, 0):
+        wl, path, dec = run_path(name, decode_splits=splits)
+        outs.append([d[0].float() for d in dec])
+    for s in range(len(outs[0])):
+        for other in outs[1:]:
+            diff = (other[s] - outs[0][s]).abs().max().item()
+            assert diff <= 1e-3, f"{name} step {s}: split-count difference {diff:.2e}"
