@@ -603,3 +603,21 @@ def test_decode_split_count_invariance(cuda_lib, name):
         for other in outs[1:]:
             diff = (other[s] - outs[0][s]).abs().max().item()
             assert diff <= 1e-3, f"{name} step {s}: split-count difference {diff:.2e}"
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name,splits", [("tiny", 0), ("llama8b_1layer", 0), ("llama8b_1layer", 5),
+                                         ("gqa7_decode", 0), ("d64_g8", 0), ("long_prefix", 0),
+                                         ("no_docs", 0), ("boundary_blocks", 0)])
+def test_single_visible_key_returns_its_value_bit_exact(cuda_lib, name, splits):
+    """The first prefix token sees only itself (position 0), so its softmax
+    has one term, p = 1, and its output is its own value, bit for bit: every
+    layer and query head, with and without key splits."""
+    wl, path, _ = run_path(name, prefill_splits=splits)
+    G = wl.spec.q_heads // wl.spec.kv_heads
+    for b in range(wl.spec.batch):
+        if int(wl.prefix_len[b]) < 1:
+            continue
+        out = path.out[:, b, 0]                                    # [L][Hq][d]
+        v0 = wl.v_inline[:, b, 0].repeat_interleave(G, dim=1)      # [L][Hq][d]
+        assert torch.equal(out, v0), f"request {b}: {(out.float() - v0.float()).abs().max():.2e}"
