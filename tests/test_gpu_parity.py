@@ -621,3 +621,32 @@ def test_single_visible_key_returns_its_value_bit_exact(cuda_lib, name, splits):
         out = path.out[:, b, 0]                                    # [L][Hq][d]
         v0 = wl.v_inline[:, b, 0].repeat_interleave(G, dim=1)      # [L][Hq][d]
         assert torch.equal(out, v0), f"request {b}: {(out.float() - v0.float()).abs().max():.2e}"
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("splits", [1, 0])
+def test_zero_keys_give_the_mean_of_visible_values(cuda_lib, splits):
+    """With every key zero the scores are all zero and the softmax uniform:
+    each output row is the mean of the values at or before its position
+    (computed here in fp64 from the inputs), through spans, documents and
+    the split merge."""
+    from paper_2607_28069_gb300.pipeline import CacheHitPath
+    wl = generate(SMALL["spans_b2"], device="cuda", gen_device="cpu")
+    wl.k_pool.zero_()
+    wl.k_inline.zero_()
+    path = CacheHitPath(wl, prefill_splits=splits)
+    path.ttft_pass()
+    torch.cuda.synchronize()
+    theta = theta_of(wl.spec)
+    G = wl.spec.q_heads // wl.spec.kv_heads
+    for layer in range(wl.spec.layers):
+        for b in range(wl.spec.batch):
+            lay = oracle_layout(wl, b)
+            docs, k_docs, v_docs, q, k, v = request_inputs(wl, b, layer)
+            _, V = O.dense_context(lay, k_docs, v_docs, wl.doc_base_pos.cpu().numpy(), k, v, theta)
+            pos = np.asarray(lay.inline_pos)
+            csum = np.cumsum(V, axis=0)                               # [ctx][Hkv][d]
+            ref = csum[pos] / (pos + 1)[:, None, None]                # [T][Hkv][d]
+            ref = np.repeat(ref, G, axis=1)                           # [T][Hq][d]
+            ok, max_abs, row = attn_close(f64(path.out[layer, b, :len(pos)]), ref)
+            assert ok, f"layer {layer} req {b}: max-abs {max_abs:.2e} row-rel {row:.2e}"
