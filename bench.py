@@ -40,7 +40,8 @@ def parse_args(argv=None):
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--workload", default="llama8b_1layer")
+    ap.add_argument("--workload", default="stress_128k_b4",
+                    help="default: the largest single-GPU workload (4 requests of ~139k tokens)")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--prefill-splits", type=int, default=0)
     ap.add_argument("--decode-splits", type=int, default=0)
@@ -54,6 +55,7 @@ def parse_args(argv=None):
                     help="also time the rotate-on-load pass (default for stress_128k_b4)")
     ap.add_argument("--oracle-sample", default=None, help=argparse.SUPPRESS)
     ap.add_argument("--oracle-seconds", type=float, default=10.0, help=argparse.SUPPRESS)
+    ap.add_argument("--oracle-passes", type=int, default=0, help=argparse.SUPPRESS)
     return ap.parse_args(argv)
 
 
@@ -188,22 +190,21 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------- work accounting
-def work_of(wl):
+def work_of(spec, st):
     """Algorithmic work of one TTFT pass (and one decode step), from the
-    request description: bytes for the HBM-bound rows, FLOPs for attention.
-    An inline token (prefix, post-document span or query) at logical position
-    p sees the p + 1 keys before and at it."""
-    spec = wl.spec
+    request description (``workloads.Structure``): bytes for the HBM-bound
+    rows, FLOPs for attention.  An inline token (prefix, post-document span
+    or query) at logical position p sees the p + 1 keys before and at it."""
     L, Hq, Hkv, d = spec.layers, spec.q_heads, spec.kv_heads, spec.head_dim
-    lens = wl.doc_len.cpu().tolist()
-    doc_tokens = sum(sum(lens[i] for i in docs) for docs in wl.meta["docs"])
+    lens = [int(x) for x in st.lens]
+    doc_tokens = sum(sum(lens[i] for i in docs) for docs in st.docs)
     pairs = 0
     query_tokens = 0
     inline_tokens = 0
     ctx = []
-    for b, docs in enumerate(wl.meta["docs"]):
-        P = wl.meta["prefix"][b]
-        spans = wl.meta["spans"][b]
+    for b, docs in enumerate(st.docs):
+        P = st.prefixes[b]
+        spans = st.spans[b]
         Tq = spec.query_len
         pairs += P * (P + 1) // 2                       # prefix rows see the prefix
         pos = P
@@ -226,57 +227,133 @@ def work_of(wl):
     }
 
 
+METRIC = ("cache-hit prefill query tok/s (TTFT path: compose + relocate + append + prefill "
+          "attention, all layers)")
+
+
+def bench_config(workload, world):
+    """The ``config`` object of the JSON line, the same for both arms: the
+    workload by name and shape, computed from its selections alone."""
+    from paper_2607_28069_gb300.workloads import WORKLOADS, draw_structure
+    spec = WORKLOADS[workload]
+    work = work_of(spec, draw_structure(spec))
+    return {"workload": workload, "description": spec.description,
+            "batch": spec.batch, "layers": spec.layers, "q_heads": spec.q_heads,
+            "kv_heads": spec.kv_heads, "head_dim": spec.head_dim,
+            "query_len": spec.query_len, "ctx_tokens": work["ctx"],
+            "l2_policy": "L2 flushed before every step (a write of max(2 x L2, 256 MiB))",
+            "timing": "value: one CUDA graph per pass, CUDA events at its two ends only; rows: "
+                      "a second graph with event nodes at every call boundary, run in "
+                      "alternate steps",
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU"}
+
+
 # ------------------------------------------------------------- oracle arms
-def oracle_sample(workload, seconds):
-    """Run the CPU oracle on a bounded sample of the workload (one request,
-    one layer per pass) until `seconds` elapse.  Returns the rate in query
-    tokens per second of the full workload (a request needs every layer)."""
-    import numpy as np  # noqa: F401
+ORACLE_ROWS = 32   # query rows timed per oracle pass when a request has more
+ORACLE_DOCS = 8    # documents re-rotated per oracle pass when a request has more
+
+
+def oracle_sample(workload, seconds, passes=0):
+    """Time the CPU oracle on bounded samples of the workload.
+
+    A full oracle pass is one request through one layer: the layout
+    (compose_layout), the re-rotation of every document (relocate_docs), the
+    inline tokens' RoPE (rotary), the prefix rows' attention over the prefix
+    and the query rows' attention over the whole stitched context
+    (attention).  A sample times the layout, the inline RoPE and the prefix
+    rows in full, and of the two large parts a seeded subset: ORACLE_DOCS of
+    the request's documents (their time scaled by the request's document
+    tokens over theirs) and ORACLE_ROWS of its query rows over the full
+    context (scaled by query_len / ORACLE_ROWS; every query row sees the
+    whole context, so their costs are equal).  The stitched context the
+    attention reads is built once per request, untimed; requests of 50k
+    positions or more use request 0 only (their set-up alone takes minutes).  Samples run until `seconds`
+    elapse, or exactly `passes` of them.  Returns the per-sample estimates
+    of a full pass and the rate in query tokens per second of the full
+    workload (a request needs every layer)."""
+    import dataclasses
+
+    import numpy as np
 
     import oracle as O
     from paper_2607_28069_gb300.workloads import WORKLOADS, generate
-    spec = WORKLOADS[workload]
-    small = workload in GPU_GEN
-    if not small:
-        import dataclasses
-        # same shapes per layer; one layer is enough for a per-layer sample
-        spec = dataclasses.replace(spec, layers=1, decode_steps=0)
+    full = WORKLOADS[workload]
+    # same selections and shapes per layer; one layer is enough for a sample
+    spec = dataclasses.replace(full, layers=1, decode_steps=0)
     wl = generate(spec, device="cpu", gen_device="cpu")
     theta = O.rope_frequencies(spec.head_dim, spec.rope_base)
     f64 = lambda t: t.float().numpy().astype("float64")  # noqa: E731
     starts, lens = wl.doc_token_start.numpy(), wl.doc_len.numpy()
-    passes, t_total = 0, 0.0
-    b = 0
-    while t_total < seconds or passes == 0:
-        docs = wl.meta["docs"][b]
-        tin = int(wl.inline_len[b])
+    base = wl.doc_base_pos.numpy()
+    rng = np.random.default_rng(28069)
+    Tq = spec.query_len
+    ctx = {}
+
+    def request(b):
+        """Untimed set-up of request b: its inputs and its stitched context."""
+        if b not in ctx:
+            docs = wl.meta["docs"][b]
+            tin = int(wl.inline_len[b])
+            k_docs = [f64(wl.k_pool[0, starts[x]:starts[x] + lens[x]]) for x in docs]
+            v_docs = [f64(wl.v_pool[0, starts[x]:starts[x] + lens[x]]) for x in docs]
+            q, k, v = (f64(t[0, b, :tin]) for t in (wl.q_inline, wl.k_inline, wl.v_inline))
+            lay = O.compose_layout(lens, base, docs, int(wl.prefix_len[b]), Tq,
+                                   wl.block_table[b].numpy(), spec.page_size,
+                                   span_len=wl.meta["spans"][b])
+            K, V = O.dense_context(lay, k_docs, v_docs, base, k, v, theta)
+            ctx[b] = (docs, k_docs, v_docs, q, k, K, V)
+        return ctx[b]
+
+    per_pass, b = [], 0
+    while (passes and len(per_pass) < passes) or (not passes and (sum(per_pass) < seconds
+                                                                  or not per_pass)):
+        docs, k_docs, v_docs, q, k, K, V = request(b)
+        tin = q.shape[0]
+        n_rows = min(Tq, ORACLE_ROWS)
+        rows = np.sort(rng.choice(Tq, size=n_rows, replace=False)) + (tin - Tq)
+        pick = np.sort(rng.choice(len(docs), size=min(len(docs), ORACLE_DOCS), replace=False)) \
+            if docs else np.zeros(0, np.int64)
         t0 = time.perf_counter()
-        lay = O.compose_layout(lens, wl.doc_base_pos.numpy(), docs, int(wl.prefix_len[b]),
-                               spec.query_len, wl.block_table[b].numpy(), spec.page_size,
+        lay = O.compose_layout(lens, base, docs, int(wl.prefix_len[b]), Tq,
+                               wl.block_table[b].numpy(), spec.page_size,
                                span_len=wl.meta["spans"][b])
-        k_docs = [f64(wl.k_pool[0, starts[x]:starts[x] + lens[x]]) for x in docs]
-        v_docs = [f64(wl.v_pool[0, starts[x]:starts[x] + lens[x]]) for x in docs]
-        O.cache_hit_prefill(lay, k_docs, v_docs, wl.doc_base_pos.numpy(),
-                            f64(wl.q_inline[0, b, :tin]), f64(wl.k_inline[0, b, :tin]),
-                            f64(wl.v_inline[0, b, :tin]), theta)
-        t_total += time.perf_counter() - t0
-        passes += 1
-        b = (b + 1) % spec.batch
-    full = WORKLOADS[workload]
-    # each pass = one request through one layer; a request needs `layers` of them
-    rate = passes * full.query_len / (t_total * full.layers)
-    return {"value": rate, "passes": passes, "seconds": t_total}
+        t1 = time.perf_counter()
+        sub = dataclasses.replace(lay, doc_ids=[docs[i] for i in pick],
+                                  doc_offset=[lay.doc_offset[i] for i in pick])
+        if len(pick):
+            O.relocate_docs(sub, [k_docs[i] for i in pick], [v_docs[i] for i in pick], base,
+                            theta)
+        t2 = time.perf_counter()
+        ip = lay.inline_pos
+        O.rotary(k, ip[:, None], theta)
+        q_rot = O.rotary(q, ip[:, None], theta)
+        lead = tin - Tq     # prefix and span rows, over the keys they can see
+        if lead:
+            O.attention(q_rot[:lead], ip[:lead], K[:ip[lead - 1] + 1], V[:ip[lead - 1] + 1])
+        t3 = time.perf_counter()
+        O.attention(q_rot[rows], ip[rows], K, V)
+        t4 = time.perf_counter()
+        doc_tok = sum(int(lens[x]) for x in docs)
+        sub_tok = sum(int(lens[docs[i]]) for i in pick)
+        reloc = (t2 - t1) * doc_tok / sub_tok if sub_tok else 0.0
+        per_pass.append((t1 - t0) + reloc + (t3 - t2) + (t4 - t3) * Tq / n_rows)
+        if K.shape[0] < 50_000:
+            b = (b + 1) % spec.batch   # short requests: cycle over the batch
+    t_total = sum(per_pass)
+    rate = len(per_pass) * full.query_len / (t_total * full.layers)
+    return {"value": rate, "passes": len(per_pass), "seconds": t_total, "per_pass": per_pass}
 
 
-def run_oracle_subprocess(workload, seconds):
+def run_oracle_subprocess(workload, seconds, passes=0):
     cores = len(os.sched_getaffinity(0))
     env = dict(os.environ)
     for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
         env[k] = str(cores)
     env["CUDA_VISIBLE_DEVICES"] = ""
     r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--oracle-sample",
-                        workload, "--oracle-seconds", str(seconds)],
-                       capture_output=True, text=True, env=env, timeout=600)
+                        workload, "--oracle-seconds", str(seconds), "--oracle-passes",
+                        str(passes)],
+                       capture_output=True, text=True, env=env, timeout=1200)
     if r.returncode != 0:
         raise RuntimeError(f"oracle sample failed: {r.stderr[-2000:]}")
     d = json.loads(r.stdout.strip().splitlines()[-1])
@@ -285,11 +362,18 @@ def run_oracle_subprocess(workload, seconds):
 
 
 def sample_desc(workload):
-    from paper_2607_28069_gb300.workloads import WORKLOADS
+    from paper_2607_28069_gb300.workloads import WORKLOADS, draw_structure
     s = WORKLOADS[workload]
-    return (f"fp64 numpy oracle, one request x one layer per pass ({s.query_len} query tokens "
-            f"over the full stitched context), repeated for >= the stated seconds; rate scaled to "
-            f"{s.layers} layer(s) per request")
+    m = len(draw_structure(s).docs[0])
+    docs = (f"{ORACLE_DOCS} seeded documents of {m} re-rotated (time scaled by the request's "
+            f"document tokens over theirs)" if m > ORACLE_DOCS else "every document re-rotated")
+    rows = (f"{ORACLE_ROWS} seeded query rows of {s.query_len} over the full stitched context "
+            f"(time scaled by {s.query_len}/{ORACLE_ROWS})" if s.query_len > ORACLE_ROWS else
+            f"all {s.query_len} query rows over the full stitched context")
+    one = "request 0" if sum(draw_structure(s).need) / s.batch >= 50_000 else "one request"
+    return (f"fp64 numpy oracle, {one} x one layer per pass: layout, {docs}, inline RoPE, "
+            f"prefix rows over the prefix, {rows}; rate scaled to {s.layers} layer(s) per "
+            f"request")
 
 
 # --------------------------------------------------------------- GPU arm
@@ -317,7 +401,8 @@ def main_gpu(args, rank, world):
         layer_table = torch.stack(rows).to(dev)
     path = CacheHitPath(wl, prefill_splits=args.prefill_splits, decode_splits=args.decode_splits,
                         layer_inv_freq=layer_table)
-    work = work_of(wl)
+    from paper_2607_28069_gb300.workloads import draw_structure
+    work = work_of(spec, draw_structure(spec))
     L = spec.layers
     geom = path.geom
     psplits = pic.pic_prefill_num_splits(geom, spec.batch, path.max_inline, path.max_ctx,
@@ -656,22 +741,15 @@ def main_gpu(args, rank, world):
     if code:
         raise RuntimeError(f"device status {code} detail {detail} after the timed run")
 
+    config = bench_config(args.workload, world)
+    if not single:
+        config["timing"] = "one CUDA graph per call, events between replays"
     out = {
-        "metric": "cache-hit prefill query tok/s (TTFT path: compose + relocate + append + "
-                  "prefill attention, all layers)",
+        "metric": METRIC,
         "value": value, "unit": "query_tokens/s", "n_gpus": world, "steps": K, "warmup": W,
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": args.workload, "description": spec.description,
-                   "batch": spec.batch, "layers": L, "q_heads": spec.q_heads,
-                   "kv_heads": spec.kv_heads, "head_dim": spec.head_dim,
-                   "query_len": spec.query_len, "ctx_tokens": work["ctx"],
-                   "l2_policy": f"L2 flushed before every step ({flush.numel() >> 20} MiB write)",
-                   "timing": ("value: one CUDA graph per pass, events at its two ends only; rows: "
-                              "a second graph with event nodes at every call boundary, run in "
-                              "alternate steps" if single else
-                              "one CUDA graph per call, events between replays"),
-                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "config": config,
         "gpu_launches": launches,
         "rows": rows,
         "rows_ms_per_step": sum(per_step.values()),  # the row graph, with its event nodes
@@ -683,27 +761,26 @@ def main_gpu(args, rank, world):
 
 
 def main_reference(args):
+    """The reference arm: the CPU oracle on the machine's host cores, W untimed
+    and K timed passes (one subprocess, the workload generated once), each a
+    bounded sample of the workload (see oracle_sample)."""
+    cores = len(os.sched_getaffinity(0))
+    W, K = args.warmup, args.steps
+    d = run_oracle_subprocess(args.workload, 0.0, passes=W + K)
+    timed = d["per_pass"][W:]
     from paper_2607_28069_gb300.workloads import WORKLOADS
     spec = WORKLOADS[args.workload]
-    cores = len(os.sched_getaffinity(0))
-    rates = []
-    per = max(1.0, min(10.0, 150.0 / max(1, args.steps + args.warmup)))
-    for k in range(args.warmup + args.steps):
-        d = run_oracle_subprocess(args.workload, per)
-        if k >= args.warmup:
-            rates.append(d)
-    tot_tokens = sum(d["value"] * d["seconds"] for d in rates)
-    tot_s = sum(d["seconds"] for d in rates)
-    value = tot_tokens / tot_s
+    value = len(timed) * spec.query_len / (sum(timed) * spec.layers)
     return {
-        "impl": "reference", "metric": "cache-hit prefill query tok/s (TTFT path: compose + "
-        "relocate + append + prefill attention, all layers)", "value": value,
-        "unit": "query_tokens/s", "n_gpus": args.gpus, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": 1e3 * spec.batch * spec.query_len / value,
+        "impl": "reference", "metric": METRIC, "value": value,
+        "unit": "query_tokens/s", "n_gpus": args.gpus, "steps": K,
+        "warmup": W, "ms_per_step": 1e3 * spec.batch * spec.query_len / value,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": args.workload},
+        "data": "synthetic", "config": bench_config(args.workload, args.gpus),
         "cpu_baseline": {"value": value, "unit": "query_tokens/s", "cores": cores,
-                         "kind": "oracle", "sample": sample_desc(args.workload)},
+                         "kind": "oracle",
+                         "sample": sample_desc(args.workload) +
+                         f"; {K} timed passes after {W} untimed, one per step"},
         "e2e": {"value": value, "unit": "query_tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -712,7 +789,8 @@ def main_reference(args):
 def main(argv=None):
     args = parse_args(argv)
     if args.oracle_sample:
-        print(json.dumps(oracle_sample(args.oracle_sample, args.oracle_seconds)))
+        print(json.dumps(oracle_sample(args.oracle_sample, args.oracle_seconds,
+                                       args.oracle_passes)))
         return 0
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))

@@ -378,7 +378,9 @@ pic_status_t pic_attention_deviation(const pic_geom_t *geom, int32_t layer, int3
  * q: bf16 [batch][Hq][d]; k_new, v_new: bf16 [batch][Hkv][d]; pos: int32 [batch]
  * (e.g. ctx_len from pic_compose) plus the scalar pos_offset (e.g. the step index);
  * out: bf16 [batch][Hq][d]; lse: float [batch][Hq] or NULL.
- * max_ctx: an upper bound on pos[b] + pos_offset + 1 (sizes the grid).
+ * max_ctx: an upper bound on pos[b] + pos_offset + 1 (sizes the grid); a
+ * request whose keys reach past it is reported as PIC_DEV_CTX_OVERFLOW by
+ * pic_device_status (its output then misses those keys).
  * num_splits: key-range splits per (request, kv head) (0 = automatic); the
  * partial softmax states are merged by log-sum-exp.  Hq / Hkv <= 16.
  * workspace: >= pic_decode_workspace_size(... same num_splits ...) bytes.
@@ -410,8 +412,9 @@ pic_status_t pic_attend_decode(const pic_geom_t *geom, int32_t layer, int32_t ba
  * 8 MiB array inside the library that every GPU which loads it holds until
  * the process exits.  The call allocates nothing.
  *  - The first call on a device (with that device current) looks the array
- *    up with cudaGetSymbolAddress; make that first call before any stream
- *    capture.
+ *    up with cudaGetSymbolAddress (and again after a device reset, which
+ *    gives the device a new context); make that first call before any
+ *    stream capture.
  *  - Every call on a device shares the array: calls that overlap on the GPU
  *    (e.g. on two streams) race.  No scratch value needs to start at zero.
  *  - num_splits 0 picks the automatic split count, lowered until the scratch

@@ -45,17 +45,47 @@ void *device_address(const void *p) {
   }
 }
 
+unsigned long long current_context_id() {
+  using GetCurrentFn = CUresult (*)(CUcontext *);
+  using GetIdFn = CUresult (*)(CUcontext, unsigned long long *);
+  static GetCurrentFn get_current = nullptr;
+  static GetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<GetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<GetIdFn>(p);
+  });
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx ||
+      get_id(ctx, &id) != CUDA_SUCCESS)
+    return 0;
+  return id;
+}
+
 int32_t *device_status_ptr() {
   constexpr int kMaxDev = 64;
   static int32_t *ptrs[kMaxDev] = {nullptr};
+  static unsigned long long ctx_ids[kMaxDev] = {0};
   static std::mutex mu;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return nullptr;
   std::lock_guard<std::mutex> lk(mu);
-  if (!ptrs[dev]) {
+  // looked up once per device context: a device reset makes a new context
+  // (and a new copy of the word), so the address is looked up again
+  const unsigned long long id = current_context_id();
+  if (!ptrs[dev] || id == 0 || id != ctx_ids[dev]) {
     void *p = nullptr;
     if (cudaGetSymbolAddress(&p, g_device_status) != cudaSuccess) return nullptr;
     ptrs[dev] = static_cast<int32_t *>(p);
+    ctx_ids[dev] = current_context_id();
   }
   return ptrs[dev];
 }

@@ -83,6 +83,11 @@ __global__ void __launch_bounds__(kThreads)
 
   const int pos = p.pos[b] + p.pos_offset;
   const int npages = pos >= 0 ? pos / 16 + 1 : 0;
+  // max_ctx sized the split plan: keys past the last split's pages would be
+  // left out, so that is a device-checked error (the step's output for the
+  // request is then incomplete)
+  if (split == p.splits - 1 && threadIdx.x == 0 && npages > p.splits * p.pages_per_split)
+    dev_fail(p.status, PIC_DEV_CTX_OVERFLOW, b);
   const int pg_begin = split * p.pages_per_split;
   const int pg_end = min(npages, pg_begin + p.pages_per_split);
   const int32_t *bt = p.block_table + (size_t)b * p.max_pages;
@@ -416,48 +421,57 @@ extern "C" int32_t pic_decode_num_splits(const pic_geom_t *geom, int32_t batch, 
   return pic::decode::plan(geom, batch, max_ctx, num_splits).splits;
 }
 
-extern "C" pic_status_t pic_attend_decode(const pic_geom_t *geom, int32_t layer, int32_t batch,
-                                          const void *q, const void *k_new, const void *v_new,
-                                          const int32_t *pos, int32_t pos_offset,
-                                          const int32_t *block_table,
-                                          int32_t max_pages, int64_t num_pages, void *k_cache,
-                                          void *v_cache, void *out, float *lse, int32_t max_ctx,
-                                          int32_t num_splits, void *workspace,
-                                          size_t workspace_bytes, pic_stream_t stream) {
-  using namespace pic;
-  using namespace pic::decode;
-  RopeParams rp;
-  pic_status_t st = make_rope(geom, &rp);
+namespace pic {
+namespace decode {
+
+// Host checks shared by pic_attend_decode and pic_attend_decode_noalloc
+// (everything but the scratch); fills the rotary parameters.
+static pic_status_t check_step(const char *who, const pic_geom_t *geom, RopeParams *rp,
+                               int32_t layer, int32_t batch, const void *q, const void *k_new,
+                               const void *v_new, const int32_t *pos, const int32_t *block_table,
+                               int32_t max_pages, int64_t num_pages, const void *k_cache,
+                               const void *v_cache, const void *out, int32_t max_ctx,
+                               int32_t num_splits) {
+  pic_status_t st = make_rope(geom, rp);
   if (st != PIC_OK) return st;
   if (layer < 0 || layer >= geom->num_layers)
-    return fail(PIC_ERR_INVALID_ARG, "pic_attend_decode: layer %d outside [0, %d)", layer,
+    return fail(PIC_ERR_INVALID_ARG, "%s: layer %d outside [0, %d)", who, layer,
                 geom->num_layers);
   if (batch <= 0 || max_pages <= 0 || num_pages <= 0 || max_ctx <= 0)
-    return fail(PIC_ERR_INVALID_ARG, "pic_attend_decode: sizes must be positive");
+    return fail(PIC_ERR_INVALID_ARG, "%s: sizes must be positive", who);
   if (num_splits < 0 || num_splits > kMaxSplits)
-    return fail(PIC_ERR_INVALID_ARG, "pic_attend_decode: num_splits %d outside [0, %d]", num_splits,
+    return fail(PIC_ERR_INVALID_ARG, "%s: num_splits %d outside [0, %d]", who, num_splits,
                 kMaxSplits);
-  const int G = geom->num_q_heads / geom->num_kv_heads;
-  if (G > 16) return fail(PIC_ERR_UNSUPPORTED, "pic_attend_decode: more than 16 query heads per kv head");
+  if (geom->num_q_heads / geom->num_kv_heads > 16)
+    return fail(PIC_ERR_UNSUPPORTED, "%s: more than 16 query heads per kv head", who);
   if (!q || !k_new || !v_new || !pos || !block_table || !k_cache || !v_cache || !out)
-    return fail(PIC_ERR_INVALID_ARG, "pic_attend_decode: NULL tensor");
+    return fail(PIC_ERR_INVALID_ARG, "%s: NULL tensor", who);
   if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k_new) |
        reinterpret_cast<uintptr_t>(v_new) | reinterpret_cast<uintptr_t>(k_cache) |
        reinterpret_cast<uintptr_t>(v_cache)) & 15)
-    return fail(PIC_ERR_INVALID_ARG, "pic_attend_decode: bf16 tensors must be 16-byte aligned");
-  const int D = geom->head_dim, Hkv = geom->num_kv_heads;
-  const long long rows_total = (long long)geom->num_layers * num_pages * Hkv * 16;
+    return fail(PIC_ERR_INVALID_ARG, "%s: bf16 tensors must be 16-byte aligned", who);
+  const long long rows_total =
+      (long long)geom->num_layers * num_pages * geom->num_kv_heads * 16;
   if (rows_total + 16 >= 0x7fffff00LL)
-    return fail(PIC_ERR_UNSUPPORTED, "pic_attend_decode: cache has more than 2^31 rows");
-  if (batch > 65535 || Hkv > 65535)
-    return fail(PIC_ERR_UNSUPPORTED, "pic_attend_decode: grid too large");
-  Plan pl = plan(geom, batch, max_ctx, num_splits);
-  if (!workspace || workspace_bytes < pl.total || (reinterpret_cast<uintptr_t>(workspace) & 255))
-    return fail(PIC_ERR_WORKSPACE, "pic_attend_decode: workspace needs %zu bytes, 256-aligned",
-                pl.total);
+    return fail(PIC_ERR_UNSUPPORTED, "%s: cache has more than 2^31 rows", who);
+  if (batch > 65535 || geom->num_kv_heads > 65535)
+    return fail(PIC_ERR_UNSUPPORTED, "%s: grid too large", who);
+  return PIC_OK;
+}
+
+// The launches of one decoding step of one layer (append, attention, merge
+// when split) with the scratch at `ws` laid out by `pl`.
+static pic_status_t launch_step(const char *who, const pic_geom_t *geom, const RopeParams &rp,
+                                int32_t layer, int32_t batch, const void *q, const void *k_new,
+                                const void *v_new, const int32_t *pos, int32_t pos_offset,
+                                const int32_t *block_table, int32_t max_pages, int64_t num_pages,
+                                void *k_cache, void *v_cache, void *out, float *lse,
+                                const Plan &pl, uint8_t *ws, pic_stream_t stream) {
   int32_t *status = device_status_ptr();
-  if (!status) return fail(PIC_ERR_CUDA, "pic_attend_decode: no device status word");
-  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  if (!status) return fail(PIC_ERR_CUDA, "%s: no device status word", who);
+  const int D = geom->head_dim, Hkv = geom->num_kv_heads;
+  const int G = geom->num_q_heads / Hkv;
+  const long long rows_total = (long long)geom->num_layers * num_pages * Hkv * 16;
   const size_t layer_elems = (size_t)num_pages * Hkv * 16 * D;
 
   AppendArgs aa;
@@ -484,7 +498,7 @@ extern "C" pic_status_t pic_attend_decode(const pic_geom_t *geom, int32_t layer,
   }
 
   CUtensorMap tk, tv;
-  st = encode_tmap_2d(&tk, k_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
+  pic_status_t st = encode_tmap_2d(&tk, k_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
   if (st == PIC_OK) st = encode_tmap_2d(&tv, v_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
   if (st != PIC_OK) return st;
 
@@ -512,7 +526,7 @@ extern "C" pic_status_t pic_attend_decode(const pic_geom_t *geom, int32_t layer,
   cudaError_t e;
   if (D == 128) e = G <= 8 ? launch_attn<128, 1>(grid, stream, tk, tv, pp) : launch_attn<128, 2>(grid, stream, tk, tv, pp);
   else e = G <= 8 ? launch_attn<64, 1>(grid, stream, tk, tv, pp) : launch_attn<64, 2>(grid, stream, tk, tv, pp);
-  if (e != cudaSuccess) return cuda_fail(e, "pic_attend_decode attention launch");
+  if (e != cudaSuccess) return cuda_fail(e, "decode attention launch");
   if (pl.splits > 1) {
     dim3 cgrid(geom->num_q_heads, batch);
     const cudaError_t ce =
@@ -521,8 +535,35 @@ extern "C" pic_status_t pic_attend_decode(const pic_geom_t *geom, int32_t layer,
     if (ce != cudaSuccess) return cuda_fail(ce, "decode merge launch");
   }
   e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_fail(e, "pic_attend_decode launch");
+  if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   return PIC_OK;
+}
+
+}  // namespace decode
+}  // namespace pic
+
+extern "C" pic_status_t pic_attend_decode(const pic_geom_t *geom, int32_t layer, int32_t batch,
+                                          const void *q, const void *k_new, const void *v_new,
+                                          const int32_t *pos, int32_t pos_offset,
+                                          const int32_t *block_table,
+                                          int32_t max_pages, int64_t num_pages, void *k_cache,
+                                          void *v_cache, void *out, float *lse, int32_t max_ctx,
+                                          int32_t num_splits, void *workspace,
+                                          size_t workspace_bytes, pic_stream_t stream) {
+  using namespace pic;
+  using namespace pic::decode;
+  static const char *who = "pic_attend_decode";
+  RopeParams rp;
+  pic_status_t st = check_step(who, geom, &rp, layer, batch, q, k_new, v_new, pos, block_table,
+                               max_pages, num_pages, k_cache, v_cache, out, max_ctx, num_splits);
+  if (st != PIC_OK) return st;
+  const Plan pl = plan(geom, batch, max_ctx, num_splits);
+  if (!workspace || workspace_bytes < pl.total || (reinterpret_cast<uintptr_t>(workspace) & 255))
+    return fail(PIC_ERR_WORKSPACE, "pic_attend_decode: workspace needs %zu bytes, 256-aligned",
+                pl.total);
+  return launch_step(who, geom, rp, layer, batch, q, k_new, v_new, pos, pos_offset, block_table,
+                     max_pages, num_pages, k_cache, v_cache, out, lse, pl,
+                     static_cast<uint8_t *>(workspace), stream);
 }
 
 // ---------------------------------------------------------------------------
@@ -538,8 +579,9 @@ extern "C" pic_status_t pic_attend_decode(const pic_geom_t *geom, int32_t layer,
 // holds until the process exits.
 //
 // Set-up: the first call on each device (with that device current) looks up
-// the array's device address with cudaGetSymbolAddress and caches it; make
-// that first call before any stream capture.  The array is shared by every
+// the array's device address with cudaGetSymbolAddress and caches it, per
+// device context (a device reset replaces the context, and the address is
+// looked up again); make that first call before any stream capture.  The array is shared by every
 // call on the device and keeps the last call's contents: calls that overlap on
 // the GPU (for example on two streams) race on it.  Nothing in it needs to
 // start at zero: each call writes every scratch value before reading it.
@@ -552,6 +594,7 @@ static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocScratchBytes]
 static uint8_t *noalloc_scratch_ptr(pic_status_t *st) {
   constexpr int kMaxDev = 64;
   static uint8_t *ptrs[kMaxDev] = {nullptr};
+  static unsigned long long ctx_ids[kMaxDev] = {0};
   static std::mutex mu;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -561,7 +604,10 @@ static uint8_t *noalloc_scratch_ptr(pic_status_t *st) {
     return nullptr;
   }
   std::lock_guard<std::mutex> lk(mu);
-  if (!ptrs[dev]) {
+  // Set-up once per device (per device context: after a device reset the
+  // array has a new address in the new context, so it is looked up again).
+  const unsigned long long id = current_context_id();
+  if (!ptrs[dev] || id == 0 || id != ctx_ids[dev]) {
     void *p = nullptr;
     e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (e != cudaSuccess) {
@@ -569,6 +615,7 @@ static uint8_t *noalloc_scratch_ptr(pic_status_t *st) {
       return nullptr;
     }
     ptrs[dev] = static_cast<uint8_t *>(p);
+    ctx_ids[dev] = current_context_id();
   }
   *st = PIC_OK;
   return ptrs[dev];
@@ -587,34 +634,11 @@ extern "C" pic_status_t pic_attend_decode_noalloc(const pic_geom_t *geom, int32_
                                                   pic_stream_t stream) {
   using namespace pic;
   using namespace pic::decode;
+  static const char *who = "pic_attend_decode_noalloc";
   RopeParams rp;
-  pic_status_t st = make_rope(geom, &rp);
+  pic_status_t st = check_step(who, geom, &rp, layer, batch, q, k_new, v_new, pos, block_table,
+                               max_pages, num_pages, k_cache, v_cache, out, max_ctx, num_splits);
   if (st != PIC_OK) return st;
-  if (layer < 0 || layer >= geom->num_layers)
-    return fail(PIC_ERR_INVALID_ARG, "pic_attend_decode_noalloc: layer %d outside [0, %d)", layer,
-                geom->num_layers);
-  if (batch <= 0 || max_pages <= 0 || num_pages <= 0 || max_ctx <= 0)
-    return fail(PIC_ERR_INVALID_ARG, "pic_attend_decode_noalloc: sizes must be positive");
-  if (num_splits < 0 || num_splits > kMaxSplits)
-    return fail(PIC_ERR_INVALID_ARG, "pic_attend_decode_noalloc: num_splits %d outside [0, %d]",
-                num_splits, kMaxSplits);
-  const int G = geom->num_q_heads / geom->num_kv_heads;
-  if (G > 16)
-    return fail(PIC_ERR_UNSUPPORTED,
-                "pic_attend_decode_noalloc: more than 16 query heads per kv head");
-  if (!q || !k_new || !v_new || !pos || !block_table || !k_cache || !v_cache || !out)
-    return fail(PIC_ERR_INVALID_ARG, "pic_attend_decode_noalloc: NULL tensor");
-  if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k_new) |
-       reinterpret_cast<uintptr_t>(v_new) | reinterpret_cast<uintptr_t>(k_cache) |
-       reinterpret_cast<uintptr_t>(v_cache)) & 15)
-    return fail(PIC_ERR_INVALID_ARG,
-                "pic_attend_decode_noalloc: bf16 tensors must be 16-byte aligned");
-  const int D = geom->head_dim, Hkv = geom->num_kv_heads;
-  const long long rows_total = (long long)geom->num_layers * num_pages * Hkv * 16;
-  if (rows_total + 16 >= 0x7fffff00LL)
-    return fail(PIC_ERR_UNSUPPORTED, "pic_attend_decode_noalloc: cache has more than 2^31 rows");
-  if (batch > 65535 || Hkv > 65535)
-    return fail(PIC_ERR_UNSUPPORTED, "pic_attend_decode_noalloc: grid too large");
   // Scratch must fit the built-in array: the automatic split count is lowered
   // until it does; an explicit split count that does not fit is rejected.
   Plan pl = plan(geom, batch, max_ctx, num_splits);
@@ -629,71 +653,6 @@ extern "C" pic_status_t pic_attend_decode_noalloc(const pic_geom_t *geom, int32_
                 pl.total, kNoAllocScratchBytes);
   uint8_t *ws = noalloc_scratch_ptr(&st);
   if (!ws) return st;
-  int32_t *status = device_status_ptr();
-  if (!status) return fail(PIC_ERR_CUDA, "pic_attend_decode_noalloc: no device status word");
-  const size_t layer_elems = (size_t)num_pages * Hkv * 16 * D;
-
-  AppendArgs aa;
-  aa.Hq = geom->num_q_heads;
-  aa.Hkv = Hkv;
-  aa.max_pages = max_pages;
-  aa.pos_offset = pos_offset;
-  aa.layer = layer;
-  aa.num_pages = num_pages;
-  aa.q = static_cast<const __nv_bfloat16 *>(q);
-  aa.k = static_cast<const __nv_bfloat16 *>(k_new);
-  aa.v = static_cast<const __nv_bfloat16 *>(v_new);
-  aa.pos = pos;
-  aa.block_table = block_table;
-  aa.k_cache = static_cast<__nv_bfloat16 *>(k_cache) + (size_t)layer * layer_elems;
-  aa.v_cache = static_cast<__nv_bfloat16 *>(v_cache) + (size_t)layer * layer_elems;
-  aa.qrot = reinterpret_cast<__nv_bfloat16 *>(ws);
-  aa.status = status;
-  {
-    const cudaError_t ae =
-        D == 128 ? launch_dependent(decode_append_kernel<128>, dim3(batch), dim3(128), 0, stream, aa, rp)
-                 : launch_dependent(decode_append_kernel<64>, dim3(batch), dim3(128), 0, stream, aa, rp);
-    if (ae != cudaSuccess) return cuda_fail(ae, "decode append launch");
-  }
-
-  CUtensorMap tk, tv;
-  st = encode_tmap_2d(&tk, k_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
-  if (st == PIC_OK) st = encode_tmap_2d(&tv, v_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
-  if (st != PIC_OK) return st;
-
-  Params pp;
-  pp.Hq = geom->num_q_heads;
-  pp.Hkv = Hkv;
-  pp.G = G;
-  pp.max_pages = max_pages;
-  pp.splits = pl.splits;
-  pp.pages_per_split = pl.pages_per_split;
-  pp.pos_offset = pos_offset;
-  pp.num_pages = num_pages;
-  pp.layer_row0 = (long long)layer * num_pages * Hkv * 16;
-  pp.pos = pos;
-  pp.block_table = block_table;
-  pp.qrot = aa.qrot;
-  pp.out = static_cast<__nv_bfloat16 *>(out);
-  pp.lse = lse;
-  pp.part_o = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes) : nullptr;
-  pp.part_ml = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes + pl.po_bytes) : nullptr;
-  pp.status = status;
-  pp.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
-
-  dim3 grid(pl.splits, Hkv, batch);
-  cudaError_t e;
-  if (D == 128) e = G <= 8 ? launch_attn<128, 1>(grid, stream, tk, tv, pp) : launch_attn<128, 2>(grid, stream, tk, tv, pp);
-  else e = G <= 8 ? launch_attn<64, 1>(grid, stream, tk, tv, pp) : launch_attn<64, 2>(grid, stream, tk, tv, pp);
-  if (e != cudaSuccess) return cuda_fail(e, "pic_attend_decode_noalloc attention launch");
-  if (pl.splits > 1) {
-    dim3 cgrid(geom->num_q_heads, batch);
-    const cudaError_t ce =
-        D == 128 ? launch_dependent(decode_combine_kernel<128>, cgrid, dim3(32), 0, stream, pp)
-                 : launch_dependent(decode_combine_kernel<64>, cgrid, dim3(32), 0, stream, pp);
-    if (ce != cudaSuccess) return cuda_fail(ce, "decode merge launch");
-  }
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_fail(e, "pic_attend_decode_noalloc launch");
-  return PIC_OK;
+  return launch_step(who, geom, rp, layer, batch, q, k_new, v_new, pos, pos_offset, block_table,
+                     max_pages, num_pages, k_cache, v_cache, out, lse, pl, ws, stream);
 }

@@ -29,6 +29,10 @@ pic_status_t cuda_fail(cudaError_t e, const char *what);
 void *device_address(const void *p);
 // Address of the current device's status word ({code, detail}).
 int32_t *device_status_ptr();
+// Unique identity of the calling thread's current CUDA context (0 when it has
+// none or the driver cannot say): device addresses of module variables are
+// valid for one context, and a device reset replaces it.
+unsigned long long current_context_id();
 // Validates the geometry and fills theta[0..d/2) (fp64 frequencies).
 pic_status_t check_geom(const pic_geom_t *g, double *theta);
 

@@ -4,8 +4,10 @@ This module draws random numbers and sizes buffers; it holds none of the
 method's arithmetic (no positions, rotations, slots or attention).  Both the
 CUDA path and the CPU oracle receive the tensors made here.
 
-Recipe (per workload): document K/V compiled at base position 0 (the paper's
-Writer is out of scope, so the cached values are N(0,1) bf16 draws), a pool
+Recipe (per workload): document K/V compiled at a base position (0 for the
+five benchmark workloads; a per-document draw for parity cases that move
+documents backwards as well as forwards; the paper's Writer is out of scope,
+so the cached values are N(0,1) bf16 draws), a pool
 of documents stored token-major ``[L][pool_tokens][Hkv][d]``, per-request
 document choices in random order, an uncached inline prefix, a query chunk and
 (optionally) decode tokens.  Physical pages are a seeded random permutation so
@@ -43,6 +45,7 @@ class WorkloadSpec:
     shared_all_docs: bool = False         # every request uses the whole pool
     page_size: int = PAGE
     span_len: tuple = (0, 0)              # (lo, hi) inclusive: inline span S_k after each doc
+    base_pos: tuple = (0, 0)              # (lo, hi) inclusive: compiled base position per pool doc
     description: str = ""
 
 
@@ -142,21 +145,38 @@ def _randn_bf16(shape, gen, device):
     return out
 
 
-def generate(spec, device="cpu", gen_device=None, value_seed=0, select_seed=1) -> Workload:
-    """Materialise a workload.  ``gen_device`` selects the random generator
-    ('cpu' for sizes the oracle handles, 'cuda' for the full-size ones);
-    tensors end up on ``device``."""
+@dataclass
+class Structure:
+    """The selections of a workload, without any tensor: pool document
+    lengths, rows and base positions, each request's documents, prefix and
+    spans, and its block table.  Cheap at every size (the bench's CPU arm
+    reads its shape from here)."""
+    lens: np.ndarray          # [n_pool] int64
+    starts: np.ndarray        # [n_pool] int64 first pool row of each document
+    bases: np.ndarray         # [n_pool] int64 compiled base position
+    docs: list                # per request: pool ids in request order
+    prefixes: list            # per request: prefix length
+    spans: list               # per request: span length after each document
+    block_table: np.ndarray   # [B][max_pages] int32 (-1 padded)
+    num_pages: int
+    need: list                # per request: positions incl. decode tokens
+    tin: list                 # per request: inline tokens (prefix + spans + query)
+
+    @property
+    def pool_tokens(self) -> int:
+        return int(self.lens.sum())
+
+
+def draw_structure(spec, select_seed=1) -> Structure:
+    """Draw the selections of a workload with the selection seed."""
     if isinstance(spec, str):
         spec = WORKLOADS[spec]
-    gen_device = gen_device or device
     rng = np.random.default_rng(select_seed)
-    L, Hq, Hkv, d, B = spec.layers, spec.q_heads, spec.kv_heads, spec.head_dim, spec.batch
-
+    B = spec.batch
     lo, hi = spec.doc_len
     lens = np.full(spec.pool_docs, lo, np.int64) if lo == hi else \
         rng.integers(lo, hi + 1, size=spec.pool_docs)
     starts = np.concatenate([[0], np.cumsum(lens)[:-1]]).astype(np.int64)
-    pool_tokens = int(lens.sum())
 
     docs = []
     for b in range(B):
@@ -187,6 +207,27 @@ def generate(spec, device="cpu", gen_device=None, value_seed=0, select_seed=1) -
     for b in range(B):
         bt[b, :pages_per_req[b]] = perm[o:o + pages_per_req[b]]
         o += pages_per_req[b]
+    # compiled base positions, drawn last and only when asked for (the other
+    # workloads keep every draw above)
+    blo, bhi = spec.base_pos
+    bases = np.zeros(spec.pool_docs, np.int64)
+    if (blo, bhi) != (0, 0):
+        bases = rng.integers(blo, bhi + 1, size=spec.pool_docs).astype(np.int64)
+    tin = [prefixes[b] + sum(spans[b]) + spec.query_len for b in range(B)]
+    return Structure(lens, starts, bases, docs, prefixes, spans, bt, num_pages, need, tin)
+
+
+def generate(spec, device="cpu", gen_device=None, value_seed=0, select_seed=1) -> Workload:
+    """Materialise a workload.  ``gen_device`` selects the random generator
+    ('cpu' for sizes the oracle handles, 'cuda' for the full-size ones);
+    tensors end up on ``device``."""
+    if isinstance(spec, str):
+        spec = WORKLOADS[spec]
+    gen_device = gen_device or device
+    st = draw_structure(spec, select_seed)
+    L, Hq, Hkv, d, B = spec.layers, spec.q_heads, spec.kv_heads, spec.head_dim, spec.batch
+    docs, spans, lens = st.docs, st.spans, st.lens
+    pool_tokens = st.pool_tokens
     max_docs = max(len(x) for x in docs)
     ids = np.full((B, max_docs), -1, np.int32)
     for b in range(B):
@@ -196,8 +237,7 @@ def generate(spec, device="cpu", gen_device=None, value_seed=0, select_seed=1) -
     gen.manual_seed(value_seed)
     k_pool = _randn_bf16((L, pool_tokens, Hkv, d), gen, gen_device)
     v_pool = _randn_bf16((L, pool_tokens, Hkv, d), gen, gen_device)
-    tin = [prefixes[b] + sum(spans[b]) + spec.query_len for b in range(B)]
-    tin_max = max(tin)
+    tin_max = max(st.tin)
     q_in = _randn_bf16((L, B, tin_max, Hq, d), gen, gen_device)
     k_in = _randn_bf16((L, B, tin_max, Hkv, d), gen, gen_device)
     v_in = _randn_bf16((L, B, tin_max, Hkv, d), gen, gen_device)
@@ -214,16 +254,17 @@ def generate(spec, device="cpu", gen_device=None, value_seed=0, select_seed=1) -
     mv = lambda t: None if t is None else t.to(device)  # noqa: E731
     return Workload(
         spec=spec,
-        doc_len=i32(lens), doc_base_pos=i32(np.zeros(spec.pool_docs)),
-        doc_token_start=torch.as_tensor(starts, dtype=torch.int64).to(device),
+        doc_len=i32(lens), doc_base_pos=i32(st.bases),
+        doc_token_start=torch.as_tensor(st.starts, dtype=torch.int64).to(device),
         k_pool=mv(k_pool), v_pool=mv(v_pool),
         req_doc_ids=i32(ids), req_num_docs=i32([len(x) for x in docs]),
-        prefix_len=i32(prefixes), query_len=i32([spec.query_len] * B),
-        block_table=i32(bt), num_pages=num_pages, max_ctx=max(need),
-        q_inline=mv(q_in), k_inline=mv(k_in), v_inline=mv(v_in), inline_len=i32(tin),
+        prefix_len=i32(st.prefixes), query_len=i32([spec.query_len] * B),
+        block_table=i32(st.block_table), num_pages=st.num_pages, max_ctx=max(st.need),
+        q_inline=mv(q_in), k_inline=mv(k_in), v_inline=mv(v_in), inline_len=i32(st.tin),
         q_dec=mv(qd), k_dec=mv(kd), v_dec=mv(vd),
-        meta={"docs": docs, "prefix": prefixes, "pool_tokens": pool_tokens, "spans": spans},
-        span_len=i32([x + [0] * (max_docs - len(x)) for x in spans]) if shi > 0 else None,
+        meta={"docs": docs, "prefix": st.prefixes, "pool_tokens": pool_tokens, "spans": spans},
+        span_len=i32([x + [0] * (max_docs - len(x)) for x in spans])
+        if spec.span_len[1] > 0 else None,
     )
 
 

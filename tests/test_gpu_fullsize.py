@@ -11,7 +11,11 @@ oracle computes one by one:
 * the prefill attention of sampled (request, layer) pairs for 64 sampled
   inline rows including the last one (every head; one kv-head group for the
   ~139k-token contexts);
-* for the decode workload, one decode step of a sampled request and layer.
+* for the decode workload, one decode step of a sampled request and layer;
+* for the 32-layer batch-8 and the stress workloads, the fused rotate-on-load
+  attention of the same two layers (their caches cleared first, so that the
+  documents can only come from the pool), on the same sampled rows of one
+  kv-head group per sampled request.
 
 Each case frees its device memory when it ends.
 """
@@ -94,14 +98,41 @@ def _check_attention(wl, path, b, layer, lay, q, K, V, theta, rng, kv_groups):
         heads = slice(g * G, (g + 1) * G)
         o_ref = O.attention(qr[:, heads], qp, K[:, g:g + 1], V[:, g:g + 1])
         ok, max_abs, row = attn_close(out[:, heads], o_ref)
-        assert ok, f"layer {layer} req {b} kv group {g}: max-abs {max_abs:.2e} row-rel {row:.2e}"
+        assert ok, f"layer {layer} req {b} kv group {g}: err/bound {max_abs:.2f} row-rel {row:.2e}"
 
 
 def _check_decode(wl, path, b, layer, lay, K, V, theta):
     o_ref, _, _ = O.decode_step(K, V, f64(wl.q_dec[0, layer, b]), f64(wl.k_dec[0, layer, b]),
                                 f64(wl.v_dec[0, layer, b]), lay.ctx_len, theta)
     ok, max_abs, row = attn_close(f64(path.dec_out[layer, b]), o_ref)
-    assert ok, f"decode layer {layer} req {b}: max-abs {max_abs:.2e} row-rel {row:.2e}"
+    assert ok, f"decode layer {layer} req {b}: err/bound {max_abs:.2f} row-rel {row:.2e}"
+
+
+FUSED = ["llama8b_32layer_b8", "stress_128k_b4"]
+
+
+def _check_fused(wl, path, layers, reqs, theta):
+    """Fused rotate-on-load attention at full size: the sampled layers'
+    caches are zeroed and refilled with the inline tokens only, so every
+    document key and value must come from the pool, rotated by -delta on
+    the query side."""
+    import paper_2607_28069_gb300 as pic
+    spec = wl.spec
+    rng = np.random.default_rng(28069)
+    for layer in layers:
+        path.k_cache[layer].zero_()
+        path.v_cache[layer].zero_()
+        path.out[layer].zero_()
+        path.append(layer)
+        path.attend_fused(layer)
+        torch.cuda.synchronize()
+        code, detail = pic.pic_device_status()
+        assert code == 0, f"device status {code} detail {detail}"
+        for b in reqs:
+            lay, q, K, V = _dense(wl, b, layer, theta)
+            groups = [int(rng.integers(spec.kv_heads))]
+            _check_attention(wl, path, b, layer, lay, q, K, V, theta, rng, groups)
+            del K, V
 
 
 @pytest.mark.parametrize("name", FULL)
@@ -126,6 +157,8 @@ def test_full_size_sampled_parity(cuda_lib, name):
                 if wl.q_dec is not None:
                     _check_decode(wl, path, b, layer, lay, K, V, theta)
                 del K, V
+        if name in FUSED:
+            _check_fused(wl, path, layers, reqs, theta)
     finally:
         del path, wl
         gc.collect()

@@ -8,8 +8,11 @@ import numpy as np
 import pytest
 import torch
 
+import oracle as O
 from paper_2607_28069_gb300.workloads import custom_spec, generate
-from tests.helpers import attn_close, f64
+from tests.helpers import attn_close, f64, oracle_layout, request_inputs, theta_of
+
+SCRATCH_BYTES = 8 << 20   # the size of the library's built-in scratch array
 
 pytestmark = pytest.mark.gpu
 
@@ -44,9 +47,59 @@ def test_noalloc_decode_matches_workspace_decode_twice(cuda_lib):
             lse=lse, pos_offset=0)
         torch.cuda.synchronize()
         ok, max_abs, row = attn_close(f64(out), ref_out)
-        assert ok, f"call {call}: max-abs {max_abs:.2e} row-rel {row:.2e}"
+        assert ok, f"call {call}: err/bound {max_abs:.2f} row-rel {row:.2e}"
         assert np.abs(f64(lse) - ref_lse).max() < 5e-2
+        # and against the oracle's decoding step over the same stitched context
+        theta = theta_of(wl.spec)
+        for b in range(wl.spec.batch):
+            lay = oracle_layout(wl, b)
+            docs, k_docs, v_docs, q, k, v = request_inputs(wl, b, 0)
+            K, V = O.dense_context(lay, k_docs, v_docs, wl.doc_base_pos.cpu().numpy(), k, v,
+                                   theta)
+            (o_ref, lse_ref), _, _ = O.decode_step(
+                K, V, f64(wl.q_dec[0, 0, b]), f64(wl.k_dec[0, 0, b]), f64(wl.v_dec[0, 0, b]),
+                lay.ctx_len, theta, return_lse=True)
+            ok, max_abs, row = attn_close(f64(out[b]), o_ref)
+            assert ok, f"call {call} req {b}: err/bound {max_abs:.2f} row-rel {row:.2e}"
+            assert np.abs(f64(lse[b]) - lse_ref).max() < 5e-2
     assert pic.pic_device_status() == (0, 0)
+
+
+def test_noalloc_lowers_the_automatic_split_count_to_fit(cuda_lib):
+    """16 query heads over one kv head at batch 32 and a ~10k-position
+    context: the automatic split plan needs more partial states than the
+    built-in array holds, so the allocation-free call lowers the split
+    count to the largest that fits, and then gives exactly what the
+    workspace entry point gives with that split count."""
+    import paper_2607_28069_gb300 as pic
+    from paper_2607_28069_gb300.pipeline import CacheHitPath
+    spec = custom_spec(name="noalloc_g16", layers=1, q_heads=16, kv_heads=1, head_dim=128,
+                       rope_base=5e5, batch=32, pool_docs=4, docs_per_request=4,
+                       doc_len=(2500, 2500), prefix_len=(16, 16), query_len=8, decode_steps=1)
+    wl = generate(spec, device="cuda", gen_device="cpu")
+    path = CacheHitPath(wl, with_lse=True)
+    path.ttft_pass()
+    B, mc = spec.batch, path.max_ctx
+    auto = pic.pic_decode_num_splits(path.geom, B, mc, 0)
+    fits = [s for s in range(1, auto + 1)
+            if pic.pic_decode_workspace_size(path.geom, B, mc, s) <= SCRATCH_BYTES]
+    assert fits and max(fits) < auto, (auto, fits[-3:])
+    lowered = max(fits)
+    ref_out = torch.empty_like(path.dec_out[0])
+    ref_lse = torch.empty_like(path.dec_lse[0])
+    ws = torch.empty(pic.pic_decode_workspace_size(path.geom, B, mc, lowered), dtype=torch.uint8,
+                     device="cuda")
+    pic.pic_attend_decode(path.geom, 0, wl.q_dec[0, 0], wl.k_dec[0, 0], wl.v_dec[0, 0],
+                          path.ctx_len, wl.block_table, wl.num_pages, path.k_cache, path.v_cache,
+                          ref_out, mc, ref_lse, lowered, ws, pos_offset=0)
+    out = torch.full_like(ref_out, float("nan"))
+    lse = torch.full_like(ref_lse, float("nan"))
+    pic.pic_attend_decode_noalloc(path.geom, 0, wl.q_dec[0, 0], wl.k_dec[0, 0], wl.v_dec[0, 0],
+                                  path.ctx_len, wl.block_table, wl.num_pages, path.k_cache,
+                                  path.v_cache, out, mc, lse=lse, pos_offset=0)
+    torch.cuda.synchronize()
+    assert pic.pic_device_status() == (0, 0)
+    assert torch.equal(out, ref_out) and torch.equal(lse, ref_lse)
 
 
 def test_noalloc_rejects_scratch_beyond_its_array(cuda_lib):
