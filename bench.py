@@ -630,7 +630,7 @@ def main_gpu(args, rank, world):
     if args.deviation:
         pathB = CacheHitPath(wl, prefill_splits=args.prefill_splits)
         pathB.compose()
-        pic.pic_relocate(pathB.geom, wl.k_pool, wl.v_pool, pathB.tok_map,
+        pic.pic_relocate_mapped(pathB.geom, wl.k_pool, wl.v_pool, pathB.tok_map,
                          torch.zeros_like(pathB.doc_delta), pathB.slot_mapping, wl.num_pages,
                          pathB.k_cache, pathB.v_cache, 0, 1)
         pathA = CacheHitPath(wl, prefill_splits=args.prefill_splits, with_lse=True)

@@ -48,7 +48,7 @@
 extern "C" {
 #endif
 
-#define PIC_ABI_VERSION 2
+#define PIC_ABI_VERSION 3
 
 typedef struct CUstream_st *pic_stream_t; /* identical to cudaStream_t */
 
@@ -175,32 +175,68 @@ pic_status_t pic_compose(const pic_geom_t *geom, int32_t batch, int32_t max_docs
 
 /*
  * pic_relocate -- key re-rotation and stitching of the cached documents
- * (Eq. 3; only keys are rotated, values are copied as they are).
+ * (Eq. 3, "Background: Position-Independent Caching"; appendix "Logical
+ * Layout and Re-Rotation": only keys are rotated, values are reused as they
+ * are).  The arguments are the problem as the paper states it: per document
+ * its prepared KV block (pool rows), base position and target position.
  *
- * For every layer l in [layer_begin, layer_end), request b and position t
- * with tok_map[b][t] = (k << 40) | row (written by pic_compose):
- *     k_cache[l][slot(t)] = R(doc_delta[b][k]) * k_pool[l][row]
- *     v_cache[l][slot(t)] = v_pool[l][row]                      (bit copy)
- * with slot(t) = slot_mapping[b][t].  R(delta) rotates each RoPE pair by
- * delta * theta_i (delta is the same for every token of a document, since
- * base and target both advance by one per token, so R(b) R(a)^-1 = R(b - a)).
- * cos/sin come from the angle delta * theta_i formed and reduced in fp64; the
- * rotation is fp32; K' is rounded to bf16 (round to nearest even).
- * delta == 0 reproduces k bit-exactly.
+ * For every layer l in [layer_begin, layer_end), request b and its k-th
+ * listed document (k < req_num_docs[b], pool id i = req_doc_ids[b][k],
+ * n_i = doc_len[i] tokens, compiled at base position a_i = doc_base_pos[i])
+ * placed at target position t_bk = doc_target[b][k], each token j < n_i:
+ *     k_cache[l][slot(t_bk + j)] = R(t_bk - a_i) * k_pool[l][doc_token_start[i] + j]
+ *     v_cache[l][slot(t_bk + j)] = v_pool[l][doc_token_start[i] + j]   (bit copy)
+ * with slot(t) = block_table[b][t / page] * page + t % page.  R(delta)
+ * rotates each RoPE pair by delta * theta_i: moving a key from a + j to
+ * t + j is R(t + j) R(a + j)^-1 = R(t - a), one rotation per document.
+ * cos/sin come from the angle formed and reduced in fp64; the rotation is
+ * fp32; K' is rounded to bf16 (round to nearest even).  delta == 0
+ * reproduces k bit-exactly.  The canonical placement of pic_compose is
+ * doc_target = its doc_offset output, but any placement is accepted.
  *
- * Inputs: k_pool, v_pool (layout above) with pool_tokens rows per layer;
- *   tok_map, slot_mapping int64 [batch][max_ctx]; doc_delta int32 [batch][max_docs].
+ * Inputs (device): k_pool, v_pool (pool layout above) with pool_tokens rows
+ *   per layer; doc_token_start int64, doc_len, doc_base_pos int32
+ *   [n_pool_docs]; req_doc_ids, doc_target int32 [batch][max_docs];
+ *   req_num_docs int32 [batch]; block_table int32 [batch][max_pages].
+ * Device checks (pic_device_status; the failing document is skipped):
+ *   document id outside the pool, length <= 0 or rows past the pool,
+ *   negative target, target + n beyond max_pages pages, a page id outside
+ *   [0, num_pages); two documents of a request whose target ranges overlap
+ *   are reported as PIC_DEV_BAD_POSITION (both are still written, so the
+ *   overlap holds one of them).
  * One launch, no workspace.  max_docs == 0 returns PIC_OK without launching.
  */
 pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
-                          const void *k_pool, const void *v_pool, int64_t pool_tokens,
-                          const int64_t *tok_map, const int32_t *doc_delta,
-                          const int64_t *slot_mapping, int32_t max_ctx, int64_t num_pages,
-                          void *k_cache, void *v_cache, int32_t layer_begin, int32_t layer_end,
-                          pic_stream_t stream);
+                          int32_t n_pool_docs, const void *k_pool, const void *v_pool,
+                          int64_t pool_tokens, const int64_t *doc_token_start,
+                          const int32_t *doc_len, const int32_t *doc_base_pos,
+                          const int32_t *req_doc_ids, const int32_t *req_num_docs,
+                          const int32_t *doc_target, const int32_t *block_table,
+                          int32_t max_pages, int64_t num_pages, void *k_cache, void *v_cache,
+                          int32_t layer_begin, int32_t layer_end, pic_stream_t stream);
 
 /*
- * pic_link -- pic_compose, pic_relocate (layers [layer_begin, layer_end)) and
+ * pic_relocate_mapped -- pic_relocate driven by pic_compose's token-level
+ * maps instead of the per-document description (the same relocation, a
+ * CTA per page of logical positions).  For every layer l in [layer_begin,
+ * layer_end), request b and position t with tok_map[b][t] = (k << 40) | row:
+ *     k_cache[l][slot(t)] = R(doc_delta[b][k]) * k_pool[l][row]
+ *     v_cache[l][slot(t)] = v_pool[l][row]                      (bit copy)
+ * with slot(t) = slot_mapping[b][t]; arithmetic as pic_relocate, so for the
+ * same placement the two give bit-identical caches.
+ * Inputs: k_pool, v_pool with pool_tokens rows per layer; tok_map,
+ *   slot_mapping int64 [batch][max_ctx]; doc_delta int32 [batch][max_docs].
+ * One launch, no workspace.  max_docs == 0 returns PIC_OK without launching.
+ */
+pic_status_t pic_relocate_mapped(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
+                                 const void *k_pool, const void *v_pool, int64_t pool_tokens,
+                                 const int64_t *tok_map, const int32_t *doc_delta,
+                                 const int64_t *slot_mapping, int32_t max_ctx, int64_t num_pages,
+                                 void *k_cache, void *v_cache, int32_t layer_begin,
+                                 int32_t layer_end, pic_stream_t stream);
+
+/*
+ * pic_link -- pic_compose, pic_relocate_mapped (layers [layer_begin, layer_end)) and
  * pic_append_inline (layer append_layer, or none when append_layer < 0) in a
  * single launch: the link step of a cache hit (Eqs. 1-3; appendix
  * "Position-Independent Linking").  Every argument means what it means for
@@ -238,23 +274,31 @@ pic_status_t pic_link(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
  * request-specific inline tokens are processed; appendix "Position-Independent
  * Linking": their KVs are interleaved with the prepared document states, and
  * a frontier causal mask stops an inline token from attending to any later
- * logical position).  Two calls, made in this order on the same workspace:
+ * logical position).
  *
- * pic_append_inline -- each inline token t of request b (logical position
- *   p = inline_pos[b][t], t < inline_len[b]) gets its key R(p) k_new and value
- *   v_new written to slot(p) = slot_mapping[b][p] of `layer`, and its rotated
- *   query R(p) q written into the workspace (GQA-packed: the query heads that
- *   share a kv head are adjacent rows).  One launch.
+ * pic_attend_prefill -- given the layer's inline projections q, k_new, v_new
+ *   (un-rotated), each inline token t of request b (logical position
+ *   p = inline_pos[b][t], t < inline_len[b]) first gets its key R(p) k_new and
+ *   value v_new written to slot(p) = block_table[b][p / page] * page + p % page
+ *   of `layer` and its query rotated to R(p) q; then for every inline token
+ *   and query head h (kv head g = h / G, G = Hq / Hkv):
+ *       out[b][t][h] = sum_{s <= p} softmax_s(R(p) q . k_s / sqrt(d)) v_s
+ *   over the keys of logical positions 0..p of the stitched cache of `layer`
+ *   (the documents relocated there by pic_relocate or pic_link, the inline
+ *   tokens just appended).  lse[b][t][h] (nullable) = natural-log sum-exp of
+ *   those scaled scores.  Runs on the tensor cores (tcgen05.mma, TMEM
+ *   accumulators, TMA loads of the paged K/V through block_table).
+ *   num_splits: key-range splits per 128-row query tile (0 = automatic);
+ *   splits are merged by log-sum-exp.  Launches: the append, the attention,
+ *   the merge when split.
+ *   q, k_new, v_new may all be NULL: the append of this layer was already
+ *   done into the same workspace by pic_append_inline or pic_link (a fast
+ *   path that lets the append overlap other work); the call then only
+ *   attends.
  *
- * pic_attend_prefill -- for every inline token and query head h (kv head
- *   g = h / G, G = Hq / Hkv):
- *       out[b][t][h] = sum_{s <= p} softmax_s(q.k_s / sqrt(d)) v_s
- *   over the keys of logical positions 0..p of the stitched cache of `layer`,
- *   reading the rotated queries pic_append_inline left in the workspace.
- *   lse[b][t][h] (nullable) = natural-log sum-exp of those scaled scores.
- *   Runs on the tensor cores (tcgen05.mma, TMEM accumulators, TMA loads of
- *   the paged K/V through block_table).  num_splits: key-range splits per
- *   128-row query tile (0 = automatic); splits are merged by log-sum-exp.
+ * pic_append_inline -- the append alone (R(p) k_new, v_new into slot(p) =
+ *   slot_mapping[b][p], the rotated queries into the workspace, GQA-packed:
+ *   the query heads that share a kv head are adjacent rows).  One launch.
  *
  * q: bf16 [batch][max_inline][Hq][d]; k_new, v_new: bf16 [batch][max_inline][Hkv][d]
  *   (un-rotated projections); inline_pos: int32 [batch][max_inline], ascending
@@ -266,8 +310,9 @@ pic_status_t pic_link(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
  *   a Grace-Blackwell node), so a caller that wants the result on the host
  *   needs no copy; PIC_ERR_INVALID_ARG for pageable memory.
  * workspace: >= pic_prefill_workspace_size(... num_splits ...) bytes, 256-byte
- *   aligned, the same buffer for both calls (pic_append_inline only uses its
- *   leading pic_prefill_workspace_size(..., 1) bytes).
+ *   aligned (pic_append_inline only uses its leading
+ *   pic_prefill_workspace_size(..., 1) bytes).  Device checks: positions in
+ *   [0, max_ctx), pages in range, block table long enough.
  */
 size_t pic_prefill_workspace_size(const pic_geom_t *geom, int32_t batch, int32_t max_inline,
                                   int32_t max_ctx, int32_t num_splits);
@@ -285,10 +330,11 @@ pic_status_t pic_append_inline(const pic_geom_t *geom, int32_t layer, int32_t ba
                                void *workspace, size_t workspace_bytes, pic_stream_t stream);
 
 pic_status_t pic_attend_prefill(const pic_geom_t *geom, int32_t layer, int32_t batch,
-                                int32_t max_inline, const int32_t *inline_pos,
+                                int32_t max_inline, const void *q, const void *k_new,
+                                const void *v_new, const int32_t *inline_pos,
                                 const int32_t *inline_len, int32_t max_ctx,
                                 const int32_t *block_table, int32_t max_pages, int64_t num_pages,
-                                const void *k_cache, const void *v_cache, void *out, float *lse,
+                                void *k_cache, void *v_cache, void *out, float *lse,
                                 int32_t num_splits, void *workspace, size_t workspace_bytes,
                                 pic_stream_t stream);
 
@@ -300,8 +346,10 @@ pic_status_t pic_attend_prefill(const pic_geom_t *geom, int32_t layer, int32_t b
  *     (R(p) q) . (R(delta_k) k) = (R(-delta_k) R(p) q) . k,
  * so per document k the 128-row query tile is rotated by -delta_k (in TMEM)
  * instead of rotating the document's keys; values are used as they are.
- * Prefix and query keys come from the paged cache, so pic_compose and
- * pic_append_inline must have run for this layer; pic_relocate is not needed.
+ * Prefix and query keys come from the paged cache: pass the layer's inline
+ * projections q, k_new, v_new to append them first (as pic_attend_prefill
+ * does), or NULL when pic_append_inline already ran for this layer; no
+ * relocation is needed.
  * Extra inputs: k_pool, v_pool, pool_tokens (layout above), doc_token_start
  *   int64 [n_pool_docs], doc_len int32 [n_pool_docs], and, from the request,
  *   req_doc_ids, doc_offset, doc_delta [batch][max_docs] (max_docs <= 1024),
@@ -309,10 +357,11 @@ pic_status_t pic_attend_prefill(const pic_geom_t *geom, int32_t layer, int32_t b
  *   workspace is the one pic_append_inline filled.
  */
 pic_status_t pic_attend_prefill_fused(const pic_geom_t *geom, int32_t layer, int32_t batch,
-                                      int32_t max_inline, const int32_t *inline_pos,
+                                      int32_t max_inline, const void *q, const void *k_new,
+                                      const void *v_new, const int32_t *inline_pos,
                                       const int32_t *inline_len, int32_t max_ctx,
                                       const int32_t *block_table, int32_t max_pages,
-                                      int64_t num_pages, const void *k_cache, const void *v_cache,
+                                      int64_t num_pages, void *k_cache, void *v_cache,
                                       const void *k_pool, const void *v_pool, int64_t pool_tokens,
                                       int32_t max_docs, const int64_t *doc_token_start,
                                       const int32_t *doc_len, const int32_t *req_doc_ids,

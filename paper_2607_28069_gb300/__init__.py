@@ -16,7 +16,8 @@ from typing import Optional
 import torch
 
 __all__ = [
-    "Geometry", "load", "lib_path", "pic_abi_version", "pic_compose", "pic_relocate", "pic_link",
+    "Geometry", "load", "lib_path", "pic_abi_version", "pic_compose", "pic_relocate",
+    "pic_relocate_mapped", "pic_link",
     "pic_attention_deviation", "pic_copy_async",
     "pic_append_inline", "pic_attend_prefill", "pic_attend_prefill_fused",
     "pic_prefill_workspace_size",
@@ -35,7 +36,7 @@ ROPE_INTERLEAVED = 1
 # Every symbol include/pic.h declares.
 EXPORTED_SYMBOLS = (
     "pic_abi_version", "pic_last_error", "pic_device_status", "pic_compose", "pic_relocate",
-    "pic_link", "pic_attention_deviation", "pic_prefill_workspace_size", "pic_prefill_num_splits",
+    "pic_relocate_mapped", "pic_link", "pic_attention_deviation", "pic_prefill_workspace_size", "pic_prefill_num_splits",
     "pic_append_inline",
     "pic_attend_prefill", "pic_attend_prefill_fused", "pic_decode_workspace_size", "pic_decode_num_splits",
     "pic_attend_decode", "pic_attend_decode_noalloc", "pic_copy_async",
@@ -112,7 +113,10 @@ def load():
         "pic_copy_async": (I32, [P, P, SZ, P]),
         "pic_compose": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, P, I32, I64, I32, I32,
                               P, P, P, P, P, P, P]),
-        "pic_relocate": (I32, [G, I32, I32, P, P, I64, P, P, P, I32, I64, P, P, I32, I32, P]),
+        "pic_relocate": (I32, [G, I32, I32, I32, P, P, I64, P, P, P, P, P, P, P, I32, I64, P, P,
+                               I32, I32, P]),
+        "pic_relocate_mapped": (I32, [G, I32, I32, P, P, I64, P, P, P, I32, I64, P, P, I32, I32,
+                                      P]),
         "pic_link": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, P, I32, I64, I32, I32, P, P, I64,
                            I32, I32, I32, P, P, P, P, P, P, P, P, P, P, P, P, P, SZ, P]),
         "pic_prefill_workspace_size": (SZ, [G, I32, I32, I32, I32]),
@@ -120,10 +124,11 @@ def load():
                                           P, P, P, P, P, P, I32, P, SZ, P, P, P]),
         "pic_append_inline": (I32, [G, I32, I32, I32, P, P, P, P, P, P, I32, I64, P, P, P, SZ,
                                     P]),
-        "pic_attend_prefill": (I32, [G, I32, I32, I32, P, P, I32, P, I32, I64, P, P, P, P, I32,
-                                     P, SZ, P]),
-        "pic_attend_prefill_fused": (I32, [G, I32, I32, I32, P, P, I32, P, I32, I64, P, P, P, P,
-                                           I64, I32, P, P, P, P, P, P, P, P, I32, P, SZ, P]),
+        "pic_attend_prefill": (I32, [G, I32, I32, I32, P, P, P, P, P, I32, P, I32, I64, P, P, P,
+                                     P, I32, P, SZ, P]),
+        "pic_attend_prefill_fused": (I32, [G, I32, I32, I32, P, P, P, P, P, I32, P, I32, I64, P,
+                                           P, P, P, I64, I32, P, P, P, P, P, P, P, P, I32, P, SZ,
+                                           P]),
         "pic_decode_workspace_size": (SZ, [G, I32, I32, I32]),
         "pic_attend_decode_noalloc": (I32, [G, I32, I32, P, P, P, P, I32, P, I32, I64, P, P, P, P,
                                             I32, I32, P]),
@@ -231,18 +236,42 @@ def pic_compose(geom: Geometry, doc_len, doc_base_pos, doc_token_start, req_doc_
     _check(st, "pic_compose")
 
 
-def pic_relocate(geom: Geometry, k_pool, v_pool, tok_map, doc_delta, slot_mapping,
-                 num_pages: int, k_cache, v_cache, layer_begin: int, layer_end: int, stream=None):
+def pic_relocate(geom: Geometry, k_pool, v_pool, doc_token_start, doc_len, doc_base_pos,
+                 req_doc_ids, req_num_docs, doc_target, block_table, num_pages: int, k_cache,
+                 v_cache, layer_begin: int, layer_end: int, stream=None):
+    """Per-document relocation: request b's k-th listed document moves from
+    its base position to doc_target[b][k] (e.g. pic_compose's doc_offset)."""
+    lib = load()
+    g = geom._c()
+    B, max_docs = req_doc_ids.shape
+    if tuple(doc_target.shape) != (B, max_docs):
+        raise ValueError("doc_target must be [batch][max_docs] like req_doc_ids")
+    st = lib.pic_relocate(
+        ctypes.byref(g), B, max_docs, doc_len.numel(), _ptr(k_pool, bf16, "k_pool"),
+        _ptr(v_pool, bf16, "v_pool"), k_pool.shape[1],
+        _ptr(doc_token_start, i64, "doc_token_start"), _ptr(doc_len, i32, "doc_len"),
+        _ptr(doc_base_pos, i32, "doc_base_pos"), _ptr(req_doc_ids, i32, "req_doc_ids"),
+        _ptr(req_num_docs, i32, "req_num_docs"), _ptr(doc_target, i32, "doc_target"),
+        _ptr(block_table, i32, "block_table"), block_table.shape[1], num_pages,
+        _ptr(k_cache, bf16, "k_cache"), _ptr(v_cache, bf16, "v_cache"), layer_begin, layer_end,
+        _stream(stream))
+    _check(st, "pic_relocate")
+
+
+def pic_relocate_mapped(geom: Geometry, k_pool, v_pool, tok_map, doc_delta, slot_mapping,
+                        num_pages: int, k_cache, v_cache, layer_begin: int, layer_end: int,
+                        stream=None):
+    """Relocation driven by pic_compose's token and slot maps."""
     lib = load()
     g = geom._c()
     B, max_docs = doc_delta.shape
-    st = lib.pic_relocate(
+    st = lib.pic_relocate_mapped(
         ctypes.byref(g), B, max_docs, _ptr(k_pool, bf16, "k_pool"), _ptr(v_pool, bf16, "v_pool"),
         k_pool.shape[1], _ptr(tok_map, i64, "tok_map"), _ptr(doc_delta, i32, "doc_delta"),
         _ptr(slot_mapping, i64, "slot_mapping"), slot_mapping.shape[1], num_pages,
         _ptr(k_cache, bf16, "k_cache"), _ptr(v_cache, bf16, "v_cache"), layer_begin, layer_end,
         _stream(stream))
-    _check(st, "pic_relocate")
+    _check(st, "pic_relocate_mapped")
 
 
 def pic_link(geom: Geometry, doc_len, doc_base_pos, doc_token_start, req_doc_ids, req_num_docs,
@@ -309,14 +338,28 @@ def pic_append_inline(geom: Geometry, layer: int, q, k_new, v_new, inline_pos, i
     _check(st, "pic_append_inline")
 
 
+def _projections(q, k_new, v_new):
+    given = [t is not None for t in (q, k_new, v_new)]
+    if any(given) and not all(given):
+        raise ValueError("give q, k_new and v_new together, or none")
+    return (_ptr(q, bf16, "q", allow_none=True), _ptr(k_new, bf16, "k_new", allow_none=True),
+            _ptr(v_new, bf16, "v_new", allow_none=True))
+
+
 def pic_attend_prefill(geom: Geometry, layer: int, inline_pos, inline_len, max_ctx: int,
                        block_table, num_pages: int, k_cache, v_cache, out, lse=None,
-                       num_splits: int = 0, workspace=None, stream=None):
+                       num_splits: int = 0, workspace=None, stream=None, q=None, k_new=None,
+                       v_new=None):
+    """Prefill attention of one layer.  With q, k_new and v_new (the layer's
+    un-rotated inline projections) the call appends them itself first;
+    without, the workspace must hold this layer's append (pic_append_inline
+    or pic_link)."""
     lib = load()
     g = geom._c()
     B, max_inline = inline_pos.shape
     st = lib.pic_attend_prefill(
-        ctypes.byref(g), layer, B, max_inline, _ptr(inline_pos, i32, "inline_pos"),
+        ctypes.byref(g), layer, B, max_inline, *_projections(q, k_new, v_new),
+        _ptr(inline_pos, i32, "inline_pos"),
         _ptr(inline_len, i32, "inline_len"), max_ctx, _ptr(block_table, i32, "block_table"),
         block_table.shape[1], num_pages, _ptr(k_cache, bf16, "k_cache"),
         _ptr(v_cache, bf16, "v_cache"), _ptr_or_pinned(out, bf16, "out"),
@@ -329,13 +372,16 @@ def pic_attend_prefill_fused(geom: Geometry, layer: int, inline_pos, inline_len,
                              block_table, num_pages: int, k_cache, v_cache, k_pool, v_pool,
                              doc_token_start, doc_len, req_doc_ids, req_num_docs, doc_offset,
                              doc_delta, out, lse=None, num_splits: int = 0, workspace=None,
-                             stream=None):
+                             stream=None, q=None, k_new=None, v_new=None):
+    """Rotate-on-load prefill attention (documents read from the pool); q,
+    k_new, v_new as for pic_attend_prefill."""
     lib = load()
     g = geom._c()
     B, max_inline = inline_pos.shape
     max_docs = req_doc_ids.shape[1]
     st = lib.pic_attend_prefill_fused(
-        ctypes.byref(g), layer, B, max_inline, _ptr(inline_pos, i32, "inline_pos"),
+        ctypes.byref(g), layer, B, max_inline, *_projections(q, k_new, v_new),
+        _ptr(inline_pos, i32, "inline_pos"),
         _ptr(inline_len, i32, "inline_len"), max_ctx, _ptr(block_table, i32, "block_table"),
         block_table.shape[1], num_pages, _ptr(k_cache, bf16, "k_cache"),
         _ptr(v_cache, bf16, "v_cache"), _ptr(k_pool, bf16, "k_pool"), _ptr(v_pool, bf16, "v_pool"),

@@ -546,7 +546,7 @@ extern "C" pic_status_t pic_link(
                      num_pages, max_ctx, max_inline, doc_offset, doc_delta, slot_mapping, tok_map,
                      inline_pos, ctx_len, stream);
     if (st == PIC_OK && max_docs > 0)
-      st = pic_relocate(geom, batch, max_docs, k_pool, v_pool, pool_tokens, tok_map, doc_delta,
+      st = pic_relocate_mapped(geom, batch, max_docs, k_pool, v_pool, pool_tokens, tok_map, doc_delta,
                         slot_mapping, max_ctx, num_pages, k_cache, v_cache, layer_begin, layer_end,
                         stream);
     if (st == PIC_OK && do_append)

@@ -1187,11 +1187,12 @@ __global__ void __launch_bounds__(256) combine_kernel(Params p) {
 // RoPE the inline keys/queries at their logical positions; keys and values go
 // to their cache slots, queries to the GQA-packed workspace.
 struct AppendArgs {
-  int Hq, Hkv, G, max_inline, max_ctx, R_pad, layer;
+  int Hq, Hkv, G, max_inline, max_ctx, R_pad, layer, max_pages;
   long long num_pages;
   const __nv_bfloat16 *q, *k, *v;
   const int32_t *inline_pos, *inline_len;
-  const int64_t *slots;
+  const int64_t *slots;          // slot map, or NULL: slots from the block table
+  const int32_t *block_table;
   __nv_bfloat16 *k_cache, *v_cache, *qpack;  // cache pointers already at the layer
   int32_t *status;
 };
@@ -1232,9 +1233,21 @@ __global__ void __launch_bounds__(256) append_kernel(AppendArgs a, RopeParams rp
 
   const int pos = a.inline_pos[tok];
   const bool pos_ok = pos >= 0 && pos < a.max_ctx;
-  long long slot = pos_ok ? a.slots[(size_t)b * a.max_ctx + pos] : -1;
+  long long slot = -1;
+  if (pos_ok) {
+    if (a.slots) {
+      slot = a.slots[(size_t)b * a.max_ctx + pos];
+    } else if ((pos >> 4) < a.max_pages) {
+      slot = (long long)a.block_table[(size_t)b * a.max_pages + (pos >> 4)] * 16 + (pos & 15);
+    } else {
+      if (tid == 0) dev_fail(a.status, PIC_DEV_BLOCK_TABLE_SHORT, b);
+      slot = -2;
+    }
+  }
   if (!pos_ok) {
     if (tid == 0) dev_fail(a.status, PIC_DEV_BAD_POSITION, b);
+  } else if (slot == -2) {
+    slot = -1;
   } else if (slot < 0 || slot >= a.num_pages * 16) {
     if (tid == 0) dev_fail(a.status, PIC_DEV_BAD_PAGE, b);
     slot = -1;
@@ -1422,6 +1435,74 @@ extern "C" int32_t pic_prefill_num_splits(const pic_geom_t *geom, int32_t batch,
   return pic::prefill::plan(geom, batch, max_inline, max_ctx, num_splits).splits;
 }
 
+namespace pic {
+namespace prefill {
+
+// One layer's inline append (append_kernel) into the packed-query part of
+// the workspace; slots from slot_mapping, or from the block table when it is
+// NULL.  Shared by pic_append_inline and the prefill calls that are given
+// the projections.
+static pic_status_t launch_append(const char *who, const pic_geom_t *geom, const RopeParams &rp,
+                                  const Plan &pl, int32_t layer, int32_t batch, int32_t max_inline,
+                                  const void *q, const void *k_new, const void *v_new,
+                                  const int32_t *inline_pos, const int32_t *inline_len,
+                                  const int64_t *slot_mapping, const int32_t *block_table,
+                                  int32_t max_pages, int32_t max_ctx, int64_t num_pages,
+                                  void *k_cache, void *v_cache, void *workspace,
+                                  pic_stream_t stream) {
+  if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k_new) |
+       reinterpret_cast<uintptr_t>(v_new) | reinterpret_cast<uintptr_t>(k_cache) |
+       reinterpret_cast<uintptr_t>(v_cache)) & 15)
+    return fail(PIC_ERR_INVALID_ARG, "%s: bf16 tensors must be 16-byte aligned", who);
+  int32_t *status = device_status_ptr();
+  if (!status) return fail(PIC_ERR_CUDA, "%s: no device status word", who);
+  const int D = geom->head_dim, Hkv = geom->num_kv_heads;
+  const size_t layer_elems = (size_t)num_pages * Hkv * 16 * D;
+  AppendArgs aa;
+  aa.Hq = geom->num_q_heads;
+  aa.Hkv = Hkv;
+  aa.G = pl.G;
+  aa.max_inline = max_inline;
+  aa.max_ctx = max_ctx;
+  aa.R_pad = pl.R_pad;
+  aa.layer = layer;
+  aa.max_pages = max_pages;
+  aa.num_pages = num_pages;
+  aa.q = static_cast<const __nv_bfloat16 *>(q);
+  aa.k = static_cast<const __nv_bfloat16 *>(k_new);
+  aa.v = static_cast<const __nv_bfloat16 *>(v_new);
+  aa.inline_pos = inline_pos;
+  aa.inline_len = inline_len;
+  aa.slots = slot_mapping;
+  aa.block_table = block_table;
+  aa.k_cache = static_cast<__nv_bfloat16 *>(k_cache) + (size_t)layer * layer_elems;
+  aa.v_cache = static_cast<__nv_bfloat16 *>(v_cache) + (size_t)layer * layer_elems;
+  aa.qpack = static_cast<__nv_bfloat16 *>(workspace);
+  aa.status = status;
+  const int t_slots = std::max(max_inline, (pl.R_pad + pl.G - 1) / pl.G);
+  if (t_slots > INT32_MAX / 2 || batch > 65535)
+    return fail(PIC_ERR_UNSUPPORTED, "%s: grid too large", who);
+  dim3 agrid(t_slots, batch);
+  cudaError_t le = D == 128 ? launch_dependent(append_kernel<128>, agrid, dim3(256), 0, stream, aa, rp)
+                            : launch_dependent(append_kernel<64>, agrid, dim3(256), 0, stream, aa, rp);
+  if (le != cudaSuccess) return cuda_fail(le, "append launch");
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "append launch");
+  return PIC_OK;
+}
+
+// The inline projections of a prefill call: all three or none.
+static pic_status_t check_projections(const char *who, const void *q, const void *k_new,
+                                      const void *v_new) {
+  const int given = (q != nullptr) + (k_new != nullptr) + (v_new != nullptr);
+  if (given != 0 && given != 3)
+    return fail(PIC_ERR_INVALID_ARG, "%s: give q, k_new and v_new together, or none", who);
+  return PIC_OK;
+}
+
+}  // namespace prefill
+}  // namespace pic
+
 extern "C" pic_status_t pic_append_inline(
     const pic_geom_t *geom, int32_t layer, int32_t batch, int32_t max_inline, const void *q,
     const void *k_new, const void *v_new, const int32_t *inline_pos, const int32_t *inline_len,
@@ -1438,50 +1519,16 @@ extern "C" pic_status_t pic_append_inline(
   if (!q || !k_new || !v_new || !inline_pos || !inline_len || !slot_mapping || !k_cache ||
       !v_cache)
     return fail(PIC_ERR_INVALID_ARG, "pic_append_inline: NULL tensor");
-  if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k_new) |
-       reinterpret_cast<uintptr_t>(v_new) | reinterpret_cast<uintptr_t>(k_cache) |
-       reinterpret_cast<uintptr_t>(v_cache)) & 15)
-    return fail(PIC_ERR_INVALID_ARG, "pic_append_inline: bf16 tensors must be 16-byte aligned");
-  int32_t *status = device_status_ptr();
-  if (!status) return fail(PIC_ERR_CUDA, "pic_append_inline: no device status word");
-  const int D = geom->head_dim, Hkv = geom->num_kv_heads;
-  const size_t layer_elems = (size_t)num_pages * Hkv * 16 * D;
-  AppendArgs aa;
-  aa.Hq = geom->num_q_heads;
-  aa.Hkv = Hkv;
-  aa.G = pl.G;
-  aa.max_inline = max_inline;
-  aa.max_ctx = max_ctx;
-  aa.R_pad = pl.R_pad;
-  aa.layer = layer;
-  aa.num_pages = num_pages;
-  aa.q = static_cast<const __nv_bfloat16 *>(q);
-  aa.k = static_cast<const __nv_bfloat16 *>(k_new);
-  aa.v = static_cast<const __nv_bfloat16 *>(v_new);
-  aa.inline_pos = inline_pos;
-  aa.inline_len = inline_len;
-  aa.slots = slot_mapping;
-  aa.k_cache = static_cast<__nv_bfloat16 *>(k_cache) + (size_t)layer * layer_elems;
-  aa.v_cache = static_cast<__nv_bfloat16 *>(v_cache) + (size_t)layer * layer_elems;
-  aa.qpack = static_cast<__nv_bfloat16 *>(workspace);
-  aa.status = status;
-  const int t_slots = std::max(max_inline, (pl.R_pad + pl.G - 1) / pl.G);
-  if (t_slots > INT32_MAX / 2 || batch > 65535)
-    return fail(PIC_ERR_UNSUPPORTED, "pic_append_inline: grid too large");
-  dim3 agrid(t_slots, batch);
-  cudaError_t le = D == 128 ? launch_dependent(append_kernel<128>, agrid, dim3(256), 0, stream, aa, rp)
-                            : launch_dependent(append_kernel<64>, agrid, dim3(256), 0, stream, aa, rp);
-  if (le != cudaSuccess) return cuda_fail(le, "pic_append_inline launch");
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_fail(e, "pic_append_inline launch");
-  return PIC_OK;
+  return launch_append("pic_append_inline", geom, rp, pl, layer, batch, max_inline, q, k_new,
+                       v_new, inline_pos, inline_len, slot_mapping, nullptr, 0, max_ctx,
+                       num_pages, k_cache, v_cache, workspace, stream);
 }
 
 extern "C" pic_status_t pic_attend_prefill(
-    const pic_geom_t *geom, int32_t layer, int32_t batch, int32_t max_inline,
-    const int32_t *inline_pos, const int32_t *inline_len, int32_t max_ctx,
-    const int32_t *block_table, int32_t max_pages, int64_t num_pages, const void *k_cache,
-    const void *v_cache, void *out, float *lse, int32_t num_splits, void *workspace,
+    const pic_geom_t *geom, int32_t layer, int32_t batch, int32_t max_inline, const void *q,
+    const void *k_new, const void *v_new, const int32_t *inline_pos, const int32_t *inline_len,
+    int32_t max_ctx, const int32_t *block_table, int32_t max_pages, int64_t num_pages,
+    void *k_cache, void *v_cache, void *out, float *lse, int32_t num_splits, void *workspace,
     size_t workspace_bytes, pic_stream_t stream) {
   using namespace pic;
   using namespace pic::prefill;
@@ -1493,6 +1540,8 @@ extern "C" pic_status_t pic_attend_prefill(
   if (max_pages <= 0) return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill: max_pages <= 0");
   if (!inline_pos || !inline_len || !block_table || !k_cache || !v_cache || !out)
     return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill: NULL tensor");
+  st = check_projections("pic_attend_prefill", q, k_new, v_new);
+  if (st != PIC_OK) return st;
   // out may be page-locked host memory: the kernels then store the rows there
   out = device_address(out);
   if (!out)
@@ -1503,6 +1552,12 @@ extern "C" pic_status_t pic_attend_prefill(
     return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill: bf16 tensors must be 16-byte aligned");
   int32_t *status = device_status_ptr();
   if (!status) return fail(PIC_ERR_CUDA, "pic_attend_prefill: no device status word");
+  if (q) {  // the inline tokens' RoPE and append first (slots from the block table)
+    st = launch_append("pic_attend_prefill", geom, rp, pl, layer, batch, max_inline, q, k_new,
+                       v_new, inline_pos, inline_len, nullptr, block_table, max_pages, max_ctx,
+                       num_pages, k_cache, v_cache, workspace, stream);
+    if (st != PIC_OK) return st;
+  }
   const int D = geom->head_dim, Hkv = geom->num_kv_heads;
   const long long rows_total = (long long)geom->num_layers * num_pages * Hkv * 16;
   uint8_t *ws = static_cast<uint8_t *>(workspace);
@@ -1566,10 +1621,10 @@ extern "C" pic_status_t pic_attend_prefill(
 }
 
 extern "C" pic_status_t pic_attend_prefill_fused(
-    const pic_geom_t *geom, int32_t layer, int32_t batch, int32_t max_inline,
-    const int32_t *inline_pos, const int32_t *inline_len, int32_t max_ctx,
-    const int32_t *block_table, int32_t max_pages, int64_t num_pages, const void *k_cache,
-    const void *v_cache, const void *k_pool, const void *v_pool, int64_t pool_tokens,
+    const pic_geom_t *geom, int32_t layer, int32_t batch, int32_t max_inline, const void *q,
+    const void *k_new, const void *v_new, const int32_t *inline_pos, const int32_t *inline_len,
+    int32_t max_ctx, const int32_t *block_table, int32_t max_pages, int64_t num_pages,
+    void *k_cache, void *v_cache, const void *k_pool, const void *v_pool, int64_t pool_tokens,
     int32_t max_docs, const int64_t *doc_token_start, const int32_t *doc_len,
     const int32_t *req_doc_ids, const int32_t *req_num_docs, const int32_t *doc_offset,
     const int32_t *doc_delta, void *out, float *lse, int32_t num_splits, void *workspace,
@@ -1597,8 +1652,16 @@ extern "C" pic_status_t pic_attend_prefill_fused(
        reinterpret_cast<uintptr_t>(k_pool) | reinterpret_cast<uintptr_t>(v_pool) |
        reinterpret_cast<uintptr_t>(out)) & 15)
     return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill_fused: bf16 tensors must be 16-byte aligned");
+  st = check_projections("pic_attend_prefill_fused", q, k_new, v_new);
+  if (st != PIC_OK) return st;
   int32_t *status = device_status_ptr();
   if (!status) return fail(PIC_ERR_CUDA, "pic_attend_prefill_fused: no device status word");
+  if (q) {  // the inline tokens' RoPE and append first (slots from the block table)
+    st = launch_append("pic_attend_prefill_fused", geom, rp, pl, layer, batch, max_inline, q,
+                       k_new, v_new, inline_pos, inline_len, nullptr, block_table, max_pages,
+                       max_ctx, num_pages, k_cache, v_cache, workspace, stream);
+    if (st != PIC_OK) return st;
+  }
   const int D = geom->head_dim, Hkv = geom->num_kv_heads;
   const long long rows_total = (long long)geom->num_layers * num_pages * Hkv * 16;
   uint8_t *ws = static_cast<uint8_t *>(workspace);

@@ -1,8 +1,17 @@
-// pic_relocate: key re-rotation (Eq. 3) and stitching of cached documents
-// into the paged request cache; values are copied unchanged (the paper rotates
-// keys only; Background: Position-Independent Caching).
+// pic_relocate / pic_relocate_mapped: key re-rotation (Eq. 3) and stitching
+// of cached documents into the paged request cache; values are copied
+// unchanged (the paper rotates keys only; Background: Position-Independent
+// Caching).
 //
-// One launch, one CTA per (one or two pages of logical positions, request);
+// pic_relocate takes the problem as the paper states it: per listed document
+// its pool rows, base position and target position, and the request's block
+// table (relocate_docs_kernel: a CTA per chunk of a document's tokens).
+// pic_relocate_mapped takes pic_compose's token and slot maps instead
+// (relocate_kernel, described below); both share the mover of the second
+// half, so for the same placement their caches are bit-identical.
+//
+// relocate_kernel: one launch, one CTA per (one or two pages of logical
+// positions, request);
 // the CTA moves its positions for every layer in turn, so its set-up (maps,
 // cos/sin) is done once and it keeps a long stream of loads in flight.
 // The CTA reads the token map and slot map of its positions (written by
@@ -17,6 +26,8 @@
 // rows are d contiguous bf16 and consecutive threads take consecutive 16-byte
 // pieces of the same row, so every warp access is fully coalesced.
 // HBM-bound: 4 * Hkv * d * 2 bytes move per document token.
+#include <algorithm>
+
 #include "pic_internal.cuh"
 
 namespace pic {
@@ -36,7 +47,22 @@ struct RelocArgs {
   const int32_t *delta;
   __nv_bfloat16 *k_cache, *v_cache;
   int32_t *status;
+  // per-document form (pic_relocate): the documents' pool rows, base and
+  // target positions, and the block table instead of the two maps
+  int n_pool_docs, max_pages;
+  const int64_t *doc_start;
+  const int32_t *doc_len, *doc_base, *ids, *num_docs, *target, *block_table;
 };
+
+// Moves the positions a CTA set up (s_src / s_dst / s_doc, the documents'
+// deltas in s_delta) for every layer of [layer_begin, layer_end): the
+// shared second half of both relocation kernels.
+template <int D, int kTok, bool kLayerRope>
+__device__ __forceinline__ void move_positions(const RelocArgs &a, const RopeParams &rp, int b,
+                                               const long long *s_src, const long long *s_dst,
+                                               const int *s_doc, const int *s_delta,
+                                               int k_first, int n_docs,
+                                               float2 (*s_cs)[kTok][D / 2]);
 
 // kLayerRope: a rotary table per layer (its cos/sin double-buffered: the next
 // layer's table is computed while this layer's loads are in flight)
@@ -46,9 +72,6 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
   pdl_entry();
   constexpr unsigned kMask = kTok == 32 ? 0xffffffffu : 0x0000ffffu;
   constexpr int HALF = D / 2;
-  constexpr int KC = D / 16;  // 8-pair chunks per K row
-  constexpr int VC = D / 8;   // 16-byte pieces per V row
-  const int style = rp.style;
   const int b = blockIdx.y;
   const long long t0 = (long long)blockIdx.x * kTok;
   const int tid = threadIdx.x;
@@ -56,6 +79,7 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
   __shared__ long long s_src[kTok];  // pool row of position t0 + i, -1 = not a doc token
   __shared__ long long s_dst[kTok];  // cache slot
   __shared__ int s_doc[kTok];        // document index k within the request
+  __shared__ int s_delta[kTok];      // delta of documents k_first .. k_first + n_docs - 1
   __shared__ int s_first, s_last;    // document range touched by this page
   __shared__ float2 s_cs[kLayerRope ? 2 : 1][kTok][HALF];
 
@@ -96,12 +120,106 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
   // every document between the first and last one here owns >= 1 position,
   // so at most kTok rows; anything else is a malformed token map
   const int n_docs = min(s_last - s_first + 1, kTok);
+  if (tid < n_docs) s_delta[tid] = a.delta[(size_t)b * a.max_docs + k_first + tid];
+  __syncthreads();
+  move_positions<D, kTok, kLayerRope>(a, rp, b, s_src, s_dst, s_doc, s_delta, k_first, n_docs,
+                                      s_cs);
+}
 
+// The per-document form: CTA (slice, k, b) moves the kTok-token chunks
+// slice, slice + S, ... of the k-th listed document of request b (S =
+// gridDim.x): token j of the document (pool row doc_start + j, compiled at
+// base + j) goes to logical position target + j, i.e. to slot
+// block_table[b][(target + j) / 16] * 16 + (target + j) % 16, rotated by
+// delta = target - base.
+template <int D, int kTok, bool kLayerRope>
+__global__ void __launch_bounds__(kThreads) relocate_docs_kernel(RelocArgs a, RopeParams rp) {
+  pdl_entry();
+  constexpr int HALF = D / 2;
+  const int k = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
+  __shared__ long long s_src[kTok];
+  __shared__ long long s_dst[kTok];
+  __shared__ int s_doc[kTok];
+  __shared__ int s_delta[1];
+  __shared__ float2 s_cs[kLayerRope ? 2 : 1][kTok][HALF];
+  const int m = a.num_docs[b];
+  if (m < 0 || m > a.max_docs) {
+    if (tid == 0 && blockIdx.x == 0 && k == 0) dev_fail(a.status, PIC_DEV_BAD_REQUEST, b);
+    return;
+  }
+  if (k >= m) return;
+  const int id = a.ids[(size_t)b * a.max_docs + k];
+  if (id < 0 || id >= a.n_pool_docs) {
+    if (tid == 0 && blockIdx.x == 0) dev_fail(a.status, PIC_DEV_BAD_DOC_ID, b);
+    return;
+  }
+  const int n = a.doc_len[id];
+  const long long start = a.doc_start[id];
+  if (n <= 0 || start < 0 || start + n > a.pool_tokens) {
+    if (tid == 0 && blockIdx.x == 0) dev_fail(a.status, PIC_DEV_BAD_DOC_LEN, b);
+    return;
+  }
+  const long long target = a.target[(size_t)b * a.max_docs + k];
+  if (target < 0 || target + n > (long long)a.max_pages * 16) {
+    if (tid == 0 && blockIdx.x == 0)
+      dev_fail(a.status, target < 0 ? PIC_DEV_BAD_POSITION : PIC_DEV_BLOCK_TABLE_SHORT, b);
+    return;
+  }
+  if (blockIdx.x == 0 && tid < 32) {  // targets of two listed documents must not overlap
+    bool clash = false;
+    for (int k2 = tid; k2 < m; k2 += 32) {
+      if (k2 == k) continue;
+      const int id2 = a.ids[(size_t)b * a.max_docs + k2];
+      if (id2 < 0 || id2 >= a.n_pool_docs) continue;
+      const long long t2 = a.target[(size_t)b * a.max_docs + k2];
+      const long long n2 = a.doc_len[id2];
+      clash |= t2 < target + n && target < t2 + n2;
+    }
+    if (__any_sync(0xffffffffu, clash) && tid == 0) dev_fail(a.status, PIC_DEV_BAD_POSITION, b);
+  }
+  if (tid == 0) s_delta[0] = (int)(target - a.doc_base[id]);
+  const int32_t *bt = a.block_table + (size_t)b * a.max_pages;
+  const int chunks = (n + kTok - 1) / kTok;
+  for (int c = blockIdx.x; c < chunks; c += gridDim.x) {
+    __syncthreads();  // the previous chunk's maps are no longer read
+    if (tid < kTok) {
+      const int j = c * kTok + tid;
+      long long src = -1, slot = -1;
+      if (j < n) {
+        const long long t = target + j;
+        const int page = bt[t >> 4];
+        if (page < 0 || page >= a.num_pages) {
+          dev_fail(a.status, PIC_DEV_BAD_PAGE, b);
+        } else {
+          src = start + j;
+          slot = (long long)page * 16 + (t & 15);
+        }
+      }
+      s_src[tid] = src;
+      s_dst[tid] = slot;
+      s_doc[tid] = 0;
+    }
+    __syncthreads();
+    move_positions<D, kTok, kLayerRope>(a, rp, b, s_src, s_dst, s_doc, s_delta, 0, 1, s_cs);
+  }
+}
+
+template <int D, int kTok, bool kLayerRope>
+__device__ __forceinline__ void move_positions(const RelocArgs &a, const RopeParams &rp, int b,
+                                               const long long *s_src, const long long *s_dst,
+                                               const int *s_doc, const int *s_delta,
+                                               int k_first, int n_docs,
+                                               float2 (*s_cs)[kTok][D / 2]) {
+  constexpr int HALF = D / 2;
+  constexpr int KC = D / 16;  // 8-pair chunks per K row
+  constexpr int VC = D / 8;   // 16-byte pieces per V row
+  const int style = rp.style;
+  const int tid = threadIdx.x;
   const size_t hkv = a.hkv;
   auto fill_cs = [&](int layer, int buf) {  // cos/sin of the touched documents
     for (int e = tid; e < n_docs * HALF; e += kThreads) {
       const int j = e / HALF, i = e % HALF;
-      const int delta = a.delta[(size_t)b * a.max_docs + k_first + j];
+      const int delta = s_delta[j];
       s_cs[buf][j][i] = kLayerRope ? rope_cos_sin_fast(delta, rope_theta(rp, layer, i))
                                    : rope_cos_sin(delta, rope_theta(rp, layer, i));
     }
@@ -208,34 +326,35 @@ __global__ void __launch_bounds__(kThreads) relocate_kernel(RelocArgs a, RopePar
 }  // namespace
 }  // namespace pic
 
-extern "C" pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
-                                     const void *k_pool, const void *v_pool, int64_t pool_tokens,
-                                     const int64_t *tok_map, const int32_t *doc_delta,
-                                     const int64_t *slot_mapping, int32_t max_ctx,
-                                     int64_t num_pages, void *k_cache, void *v_cache,
-                                     int32_t layer_begin, int32_t layer_end,
-                                     pic_stream_t stream) {
+extern "C" pic_status_t pic_relocate_mapped(const pic_geom_t *geom, int32_t batch,
+                                            int32_t max_docs, const void *k_pool,
+                                            const void *v_pool, int64_t pool_tokens,
+                                            const int64_t *tok_map, const int32_t *doc_delta,
+                                            const int64_t *slot_mapping, int32_t max_ctx,
+                                            int64_t num_pages, void *k_cache, void *v_cache,
+                                            int32_t layer_begin, int32_t layer_end,
+                                            pic_stream_t stream) {
   using namespace pic;
   RopeParams rp;
   pic_status_t st = make_rope(geom, &rp);
   if (st != PIC_OK) return st;
   if (max_docs == 0 && batch > 0) return PIC_OK;  // no document to move
   if (batch <= 0 || max_docs < 0 || pool_tokens <= 0 || max_ctx <= 0 || num_pages <= 0)
-    return fail(PIC_ERR_INVALID_ARG, "pic_relocate: sizes must be positive");
+    return fail(PIC_ERR_INVALID_ARG, "pic_relocate_mapped: sizes must be positive");
   if (pool_tokens >= (1LL << 40))
-    return fail(PIC_ERR_UNSUPPORTED, "pic_relocate: pool has 2^40 rows or more");
+    return fail(PIC_ERR_UNSUPPORTED, "pic_relocate_mapped: pool has 2^40 rows or more");
   if (layer_begin < 0 || layer_end > geom->num_layers || layer_begin >= layer_end)
-    return fail(PIC_ERR_INVALID_ARG, "pic_relocate: layer range [%d, %d) outside [0, %d)",
+    return fail(PIC_ERR_INVALID_ARG, "pic_relocate_mapped: layer range [%d, %d) outside [0, %d)",
                 layer_begin, layer_end, geom->num_layers);
   if (layer_end - layer_begin > 65535 || batch > 65535)
-    return fail(PIC_ERR_INVALID_ARG, "pic_relocate: grid too large");
+    return fail(PIC_ERR_INVALID_ARG, "pic_relocate_mapped: grid too large");
   if (!k_pool || !v_pool || !tok_map || !doc_delta || !slot_mapping || !k_cache || !v_cache)
-    return fail(PIC_ERR_INVALID_ARG, "pic_relocate: NULL tensor");
+    return fail(PIC_ERR_INVALID_ARG, "pic_relocate_mapped: NULL tensor");
   if ((reinterpret_cast<uintptr_t>(k_pool) | reinterpret_cast<uintptr_t>(v_pool) |
        reinterpret_cast<uintptr_t>(k_cache) | reinterpret_cast<uintptr_t>(v_cache)) & 15)
-    return fail(PIC_ERR_INVALID_ARG, "pic_relocate: K/V tensors must be 16-byte aligned");
+    return fail(PIC_ERR_INVALID_ARG, "pic_relocate_mapped: K/V tensors must be 16-byte aligned");
   int32_t *status = device_status_ptr();
-  if (!status) return fail(PIC_ERR_CUDA, "pic_relocate: no device status word");
+  if (!status) return fail(PIC_ERR_CUDA, "pic_relocate_mapped: no device status word");
 
   RelocArgs a;
   a.max_docs = max_docs;
@@ -270,6 +389,86 @@ extern "C" pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int3
                     : launch_dependent(relocate_kernel<64, 32, true>, grid, block, 0, stream, a, rp))
             : (wide ? launch_dependent(relocate_kernel<64, 16, false>, grid, block, 0, stream, a, rp)
                     : launch_dependent(relocate_kernel<64, 32, false>, grid, block, 0, stream, a, rp));
+  if (e == cudaSuccess) e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "pic_relocate_mapped launch");
+  return PIC_OK;
+}
+
+extern "C" pic_status_t pic_relocate(const pic_geom_t *geom, int32_t batch, int32_t max_docs,
+                                     int32_t n_pool_docs, const void *k_pool, const void *v_pool,
+                                     int64_t pool_tokens, const int64_t *doc_token_start,
+                                     const int32_t *doc_len, const int32_t *doc_base_pos,
+                                     const int32_t *req_doc_ids, const int32_t *req_num_docs,
+                                     const int32_t *doc_target, const int32_t *block_table,
+                                     int32_t max_pages, int64_t num_pages, void *k_cache,
+                                     void *v_cache, int32_t layer_begin, int32_t layer_end,
+                                     pic_stream_t stream) {
+  using namespace pic;
+  RopeParams rp;
+  pic_status_t st = make_rope(geom, &rp);
+  if (st != PIC_OK) return st;
+  if (max_docs == 0 && batch > 0) return PIC_OK;  // no document to move
+  if (batch <= 0 || max_docs < 0 || n_pool_docs <= 0 || pool_tokens <= 0 || max_pages <= 0 ||
+      num_pages <= 0)
+    return fail(PIC_ERR_INVALID_ARG, "pic_relocate: sizes must be positive");
+  if (layer_begin < 0 || layer_end > geom->num_layers || layer_begin >= layer_end)
+    return fail(PIC_ERR_INVALID_ARG, "pic_relocate: layer range [%d, %d) outside [0, %d)",
+                layer_begin, layer_end, geom->num_layers);
+  if (max_docs > 65535 || batch > 65535)
+    return fail(PIC_ERR_INVALID_ARG, "pic_relocate: grid too large");
+  if ((long long)max_pages * 16 >= (1LL << 31))
+    return fail(PIC_ERR_UNSUPPORTED, "pic_relocate: block table longer than 2^27 pages");
+  if (!k_pool || !v_pool || !doc_token_start || !doc_len || !doc_base_pos || !req_doc_ids ||
+      !req_num_docs || !doc_target || !block_table || !k_cache || !v_cache)
+    return fail(PIC_ERR_INVALID_ARG, "pic_relocate: NULL tensor");
+  if ((reinterpret_cast<uintptr_t>(k_pool) | reinterpret_cast<uintptr_t>(v_pool) |
+       reinterpret_cast<uintptr_t>(k_cache) | reinterpret_cast<uintptr_t>(v_cache)) & 15)
+    return fail(PIC_ERR_INVALID_ARG, "pic_relocate: K/V tensors must be 16-byte aligned");
+  int32_t *status = device_status_ptr();
+  if (!status) return fail(PIC_ERR_CUDA, "pic_relocate: no device status word");
+
+  RelocArgs a = {};
+  a.max_docs = max_docs;
+  a.hkv = geom->num_kv_heads;
+  a.layer_begin = layer_begin;
+  a.layer_end = layer_end;
+  a.pool_tokens = pool_tokens;
+  a.num_pages = num_pages;
+  a.k_pool = static_cast<const __nv_bfloat16 *>(k_pool);
+  a.v_pool = static_cast<const __nv_bfloat16 *>(v_pool);
+  a.k_cache = static_cast<__nv_bfloat16 *>(k_cache);
+  a.v_cache = static_cast<__nv_bfloat16 *>(v_cache);
+  a.status = status;
+  a.n_pool_docs = n_pool_docs;
+  a.max_pages = max_pages;
+  a.doc_start = doc_token_start;
+  a.doc_len = doc_len;
+  a.doc_base = doc_base_pos;
+  a.ids = req_doc_ids;
+  a.num_docs = req_num_docs;
+  a.target = doc_target;
+  a.block_table = block_table;
+  const bool wide = geom->num_kv_heads * geom->head_dim >= 1024;
+  // slices per document: each CTA walks every slices-th chunk of its document;
+  // few documents get more slices (up to one chunk per CTA), so that a small
+  // request still fills the GPU (CTAs past a document's last chunk exit)
+  const long long docs_total = (long long)batch * max_docs;
+  const int slices = (int)std::min<long long>(128, std::max<long long>(16, (8 * 152 + docs_total - 1) / docs_total));
+  dim3 grid(slices, max_docs, batch);
+  const dim3 block(kThreads);
+  cudaError_t e;
+  if (geom->head_dim == 128)
+    e = rp.layer_theta
+            ? (wide ? launch_dependent(relocate_docs_kernel<128, 16, true>, grid, block, 0, stream, a, rp)
+                    : launch_dependent(relocate_docs_kernel<128, 32, true>, grid, block, 0, stream, a, rp))
+            : (wide ? launch_dependent(relocate_docs_kernel<128, 16, false>, grid, block, 0, stream, a, rp)
+                    : launch_dependent(relocate_docs_kernel<128, 32, false>, grid, block, 0, stream, a, rp));
+  else
+    e = rp.layer_theta
+            ? (wide ? launch_dependent(relocate_docs_kernel<64, 16, true>, grid, block, 0, stream, a, rp)
+                    : launch_dependent(relocate_docs_kernel<64, 32, true>, grid, block, 0, stream, a, rp))
+            : (wide ? launch_dependent(relocate_docs_kernel<64, 16, false>, grid, block, 0, stream, a, rp)
+                    : launch_dependent(relocate_docs_kernel<64, 32, false>, grid, block, 0, stream, a, rp));
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pic_relocate launch");
   return PIC_OK;

@@ -10,7 +10,7 @@ import torch
 
 from . import (Geometry, pic_append_inline, pic_attend_decode, pic_attend_prefill,
                pic_attend_prefill_fused, pic_compose, pic_copy_async, pic_decode_workspace_size,
-               pic_link, pic_prefill_workspace_size, pic_relocate)
+               pic_link, pic_prefill_workspace_size, pic_relocate, pic_relocate_mapped)
 from .workloads import Workload
 
 
@@ -177,14 +177,25 @@ class CacheHitPath:
                     self.slot_mapping, self.tok_map, self.inline_pos, self.ctx_len,
                     span_len=wl.span_len)
 
-    # -- a2 + a3: per-document rotation and stitching, all layers, one launch
+    # -- a2 + a3: per-document rotation and stitching, all layers, one launch:
+    # every document from its base position to the target compose assigned
     def relocate(self, layer_begin: int = 0, layer_end: int | None = None):
         wl = self.wl
         if layer_end is None:
             layer_end = wl.spec.layers
-        pic_relocate(self.geom, wl.k_pool, wl.v_pool, self.tok_map, self.doc_delta,
-                     self.slot_mapping, wl.num_pages, self.k_cache, self.v_cache, layer_begin,
+        pic_relocate(self.geom, wl.k_pool, wl.v_pool, wl.doc_token_start, wl.doc_len,
+                     wl.doc_base_pos, wl.req_doc_ids, wl.req_num_docs, self.doc_offset,
+                     wl.block_table, wl.num_pages, self.k_cache, self.v_cache, layer_begin,
                      layer_end)
+
+    # -- the same through compose's token and slot maps
+    def relocate_mapped(self, layer_begin: int = 0, layer_end: int | None = None):
+        wl = self.wl
+        if layer_end is None:
+            layer_end = wl.spec.layers
+        pic_relocate_mapped(self.geom, wl.k_pool, wl.v_pool, self.tok_map, self.doc_delta,
+                            self.slot_mapping, wl.num_pages, self.k_cache, self.v_cache,
+                            layer_begin, layer_end)
 
     # -- a1 + a2 + a3 + a4 (first layer) in one launch
     def link(self, append_layer: int = 0):
@@ -230,8 +241,15 @@ class CacheHitPath:
                                  self.prefill_splits, self.ws_prefill)
 
     def prefill(self, layer: int):
-        self.append(layer)
-        self.attend(layer)
+        """Append and attention of one layer: one pic_attend_prefill call
+        given the layer's projections (the same launches as append then
+        attend)."""
+        wl = self.wl
+        pic_attend_prefill(self.geom, layer, self.inline_pos, wl.inline_len, self.max_ctx,
+                           wl.block_table, wl.num_pages, self.k_cache, self.v_cache,
+                           self.out[layer], None if self.lse is None else self.lse[layer],
+                           self.prefill_splits, self.ws_prefill, q=wl.q_inline[layer],
+                           k_new=wl.k_inline[layer], v_new=wl.v_inline[layer])
 
     def fused_pass(self):
         """The cache-hit path with rotate-on-load attention: layout, then per

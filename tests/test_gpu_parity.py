@@ -579,7 +579,7 @@ def test_attention_deviation_matches_oracle(cuda_lib, name, rows):
     A.compose()
     A.relocate()
     Bp.compose()
-    pic.pic_relocate(Bp.geom, wl.k_pool, wl.v_pool, Bp.tok_map, torch.zeros_like(Bp.doc_delta),
+    pic.pic_relocate_mapped(Bp.geom, wl.k_pool, wl.v_pool, Bp.tok_map, torch.zeros_like(Bp.doc_delta),
                      Bp.slot_mapping, wl.num_pages, Bp.k_cache, Bp.v_cache, 0, spec.layers)
     theta = theta_of(spec)
     if rows == "query":
