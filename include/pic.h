@@ -341,20 +341,28 @@ pic_status_t pic_attend_prefill(const pic_geom_t *geom, int32_t layer, int32_t b
 /*
  * pic_attend_prefill_fused -- pic_attend_prefill without the relocated cache:
  * the same outputs, with every document key and value read straight from the
- * pool as it was compiled (a fused rotate-on-load form of the re-rotation of
- * Eq. 3).  Because rotations are orthogonal,
- *     (R(p) q) . (R(delta_k) k) = (R(-delta_k) R(p) q) . k,
- * so per document k the 128-row query tile is rotated by -delta_k (in TMEM)
- * instead of rotating the document's keys; values are used as they are.
- * Prefix and query keys come from the paged cache: pass the layer's inline
- * projections q, k_new, v_new to append them first (as pic_attend_prefill
- * does), or NULL when pic_append_inline already ran for this layer; no
- * relocation is needed.
- * Extra inputs: k_pool, v_pool, pool_tokens (layout above), doc_token_start
- *   int64 [n_pool_docs], doc_len int32 [n_pool_docs], and, from the request,
- *   req_doc_ids, doc_offset, doc_delta [batch][max_docs] (max_docs <= 1024),
- *   req_num_docs [batch].  Other arguments as pic_attend_prefill; the
- *   workspace is the one pic_append_inline filled.
+ * pool as it was compiled and the key re-rotation of Eq. 3 applied while the
+ * keys are loaded (rotate-on-load), so pic_relocate never runs and the
+ * documents' cache slots are never written.
+ *
+ * Each 128-key tile of the attention is assembled page by page: a page whose
+ * 16 positions belong to one document is one box of the document's
+ * consecutive pool rows, a page of inline tokens one box of the cache, a page
+ * across a boundary is gathered row by row.  The document rows of the key
+ * tile are then rotated in shared memory by R(doc_delta[b][k]) with the
+ * arithmetic of pic_relocate (fp64-reduced angle, fp32 rotation, bf16 round
+ * to nearest even), so the attention reads exactly the keys pic_relocate
+ * would have stitched: outputs equal pic_attend_prefill's over that cache
+ * bit for bit (same split count).  Values are used as they are.
+ *
+ * Arguments as pic_attend_prefill, plus: k_pool, v_pool with pool_tokens
+ * rows per layer (pool layout above; pool_tokens > 16); tok_map int64
+ * [batch][max_ctx] and doc_delta int32 [batch][max_docs] as pic_compose (or
+ * pic_link) wrote them for this request layout.  Inline keys and values come
+ * from the paged cache: pass the layer's projections q, k_new, v_new to
+ * append them first, or NULL when pic_append_inline already ran for this
+ * layer.  Launches: the append when given, the attention, the merge when
+ * split.
  */
 pic_status_t pic_attend_prefill_fused(const pic_geom_t *geom, int32_t layer, int32_t batch,
                                       int32_t max_inline, const void *q, const void *k_new,
@@ -363,9 +371,7 @@ pic_status_t pic_attend_prefill_fused(const pic_geom_t *geom, int32_t layer, int
                                       const int32_t *block_table, int32_t max_pages,
                                       int64_t num_pages, void *k_cache, void *v_cache,
                                       const void *k_pool, const void *v_pool, int64_t pool_tokens,
-                                      int32_t max_docs, const int64_t *doc_token_start,
-                                      const int32_t *doc_len, const int32_t *req_doc_ids,
-                                      const int32_t *req_num_docs, const int32_t *doc_offset,
+                                      int32_t max_docs, const int64_t *tok_map,
                                       const int32_t *doc_delta, void *out, float *lse,
                                       int32_t num_splits, void *workspace, size_t workspace_bytes,
                                       pic_stream_t stream);

@@ -127,8 +127,7 @@ def load():
         "pic_attend_prefill": (I32, [G, I32, I32, I32, P, P, P, P, P, I32, P, I32, I64, P, P, P,
                                      P, I32, P, SZ, P]),
         "pic_attend_prefill_fused": (I32, [G, I32, I32, I32, P, P, P, P, P, I32, P, I32, I64, P,
-                                           P, P, P, I64, I32, P, P, P, P, P, P, P, P, I32, P, SZ,
-                                           P]),
+                                           P, P, P, I64, I32, P, P, P, P, I32, P, SZ, P]),
         "pic_decode_workspace_size": (SZ, [G, I32, I32, I32]),
         "pic_attend_decode_noalloc": (I32, [G, I32, I32, P, P, P, P, I32, P, I32, I64, P, P, P, P,
                                             I32, I32, P]),
@@ -370,26 +369,25 @@ def pic_attend_prefill(geom: Geometry, layer: int, inline_pos, inline_len, max_c
 
 def pic_attend_prefill_fused(geom: Geometry, layer: int, inline_pos, inline_len, max_ctx: int,
                              block_table, num_pages: int, k_cache, v_cache, k_pool, v_pool,
-                             doc_token_start, doc_len, req_doc_ids, req_num_docs, doc_offset,
-                             doc_delta, out, lse=None, num_splits: int = 0, workspace=None,
-                             stream=None, q=None, k_new=None, v_new=None):
-    """Rotate-on-load prefill attention (documents read from the pool); q,
+                             tok_map, doc_delta, out, lse=None, num_splits: int = 0,
+                             workspace=None, stream=None, q=None, k_new=None, v_new=None):
+    """Rotate-on-load prefill attention: documents read from the pool and
+    rotated as they are loaded (tok_map / doc_delta from pic_compose); q,
     k_new, v_new as for pic_attend_prefill."""
     lib = load()
     g = geom._c()
     B, max_inline = inline_pos.shape
-    max_docs = req_doc_ids.shape[1]
+    max_docs = doc_delta.shape[1]
+    if tuple(tok_map.shape) != (B, max_ctx):
+        raise ValueError("tok_map must be [batch][max_ctx]")
     st = lib.pic_attend_prefill_fused(
         ctypes.byref(g), layer, B, max_inline, *_projections(q, k_new, v_new),
-        _ptr(inline_pos, i32, "inline_pos"),
-        _ptr(inline_len, i32, "inline_len"), max_ctx, _ptr(block_table, i32, "block_table"),
-        block_table.shape[1], num_pages, _ptr(k_cache, bf16, "k_cache"),
-        _ptr(v_cache, bf16, "v_cache"), _ptr(k_pool, bf16, "k_pool"), _ptr(v_pool, bf16, "v_pool"),
-        k_pool.shape[1], max_docs, _ptr(doc_token_start, i64, "doc_token_start"),
-        _ptr(doc_len, i32, "doc_len"), _ptr(req_doc_ids, i32, "req_doc_ids", allow_none=True),
-        _ptr(req_num_docs, i32, "req_num_docs"), _ptr(doc_offset, i32, "doc_offset", allow_none=True),
-        _ptr(doc_delta, i32, "doc_delta", allow_none=True), _ptr(out, bf16, "out"),
-        _ptr(lse, f32, "lse", allow_none=True), num_splits,
+        _ptr(inline_pos, i32, "inline_pos"), _ptr(inline_len, i32, "inline_len"), max_ctx,
+        _ptr(block_table, i32, "block_table"), block_table.shape[1], num_pages,
+        _ptr(k_cache, bf16, "k_cache"), _ptr(v_cache, bf16, "v_cache"),
+        _ptr(k_pool, bf16, "k_pool"), _ptr(v_pool, bf16, "v_pool"), k_pool.shape[1], max_docs,
+        _ptr(tok_map, i64, "tok_map"), _ptr(doc_delta, i32, "doc_delta"),
+        _ptr_or_pinned(out, bf16, "out"), _ptr(lse, f32, "lse", allow_none=True), num_splits,
         _ptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream))
     _check(st, "pic_attend_prefill_fused")
 

@@ -173,6 +173,27 @@ pic_status_t encode_tmap_3d(CUtensorMap *map, const void *base, uint64_t inner, 
   return PIC_OK;
 }
 
+pic_status_t encode_tmap_pool128(CUtensorMap *map, const void *base, uint64_t rows, int hkv) {
+  EncodeFn enc = get_encode();
+  if (!enc) return fail(PIC_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+  if (reinterpret_cast<uintptr_t>(base) & 15)
+    return fail(PIC_ERR_INVALID_ARG, "tensor base not 16-byte aligned");
+  if (rows <= 16) return fail(PIC_ERR_INVALID_ARG, "pool has too few rows for a page box");
+  const uint64_t row_bytes = (uint64_t)hkv * 128 * 2;
+  // {column, row, panel, 8-row half, head}: a box at row R covers rows R..R+7
+  // (half 0) and R+8..R+15 (half 1); the row extent stops 8 short of the end
+  // so both halves stay inside the pool
+  cuuint64_t dims[5] = {64, rows - 8, 2, 2, (cuuint64_t)hkv};
+  cuuint64_t strides[4] = {row_bytes, 128, 8 * row_bytes, 256};
+  cuuint32_t box[5] = {64, 8, 2, 2, 1};
+  cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void *>(base), dims,
+                   strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(PIC_ERR_CUDA, "cuTensorMapEncodeTiled (pool) failed (%d)", (int)r);
+  return PIC_OK;
+}
+
 pic_status_t encode_tmap_pages128(CUtensorMap *map, const void *base, uint64_t n_page_heads) {
   EncodeFn enc = get_encode();
   if (!enc) return fail(PIC_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");

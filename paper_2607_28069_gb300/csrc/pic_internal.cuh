@@ -52,6 +52,11 @@ inline pic_status_t make_rope(const pic_geom_t *g, RopeParams *rp) {
   return s;
 }
 
+// Document pool [L * pool_tokens][Hkv][128] bf16 as a 5-D view whose box of
+// 16 consecutive rows of one head (from any row) lands like a page-head box of
+// the cache: [8-row half][64-column panel][8 rows][128 B], 128-byte swizzled.
+// Rows past rows - 8 read as zeros (a box always stays inside one document).
+pic_status_t encode_tmap_pool128(CUtensorMap *map, const void *base, uint64_t rows, int hkv);
 // cuTensorMapEncodeTiled through the runtime's driver entry point.
 pic_status_t encode_tmap_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t rows,
                             uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows);
@@ -297,6 +302,12 @@ PIC_DEV void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
                : "memory");
 }
+// Adds `bytes` to the barrier's expected transaction count without arriving
+// (the arrival comes later, e.g. after this thread's own shared-memory writes).
+PIC_DEV void mbar_expect_tx_only(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
 PIC_DEV bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -358,6 +369,14 @@ PIC_DEV void tma_load_4d(uint32_t dst, const CUtensorMap *map, int x, int y, int
       "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
       " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(w), "r"(bar)
+      : "memory");
+}
+PIC_DEV void tma_load_5d(uint32_t dst, const CUtensorMap *map, int x, int y, int z, int w, int v,
+                         uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.5d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(w), "r"(v), "r"(bar)
       : "memory");
 }
 PIC_DEV void prefetch_tmap(const CUtensorMap *map) {
@@ -497,6 +516,21 @@ PIC_DEV void mma16816(float *d, const uint32_t *a, uint32_t b0, uint32_t b1) {
       "{%8,%9}, {%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// 16-byte shared-memory load and store (generic proxy).
+PIC_DEV uint4 lds128(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
+PIC_DEV void sts128(uint32_t addr, const uint4 &v) {
+  asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y),
+               "r"(v.z), "r"(v.w)
+               : "memory");
 }
 
 // Byte offset of element (row, col) inside a [rows][64] bf16 panel written by

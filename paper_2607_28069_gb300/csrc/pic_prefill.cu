@@ -38,6 +38,17 @@ constexpr int BN = 128;  // keys per KV tile
 constexpr int NSK = 3;   // K ring stages (released after the last QK of a tile)
 constexpr int NSV = 2;   // V ring stages (released after the last PV of a tile)
 constexpr int kThreads = 128 + NQ * 128;  // K producer, MMA, NQ softmax warpgroups, V producer, relay
+// Rotate-on-load adds a warpgroup that rotates the document keys of each K
+// tile (warps 12-15); its roles are warpgroup-aligned so the registers can be
+// redistributed with setmaxnreg: the control warpgroup (K producer, MMA, V
+// producer, relay) and the rotators give registers to the softmax warpgroups.
+constexpr int kThreadsFused = 512;
+constexpr int kRegLaunchFused = 65536 / kThreadsFused;  // 128 per thread at launch
+constexpr int kRegCtl = 64, kRegRot = 96, kRegSoftmax = 176;
+static_assert(128 * kRegCtl + 128 * kRegRot + 256 * kRegSoftmax <= 128 * 4 * kRegLaunchFused,
+              "setmaxnreg split exceeds the registers the CTA is launched with");
+template <bool kFused>
+constexpr int threads_of() { return kFused ? kThreadsFused : kThreads; }
 constexpr int kWarpV = 2 + 4 * NQ;        // the V producer warp
 constexpr int kWarpRelay = kWarpV + 1;    // waits on behalf of the MMA issuer
 // Named barriers between the relay warp and the MMA warp (64 threads each);
@@ -69,7 +80,8 @@ enum {
   B_SFULL = B_VEMPTY + NSV,  // one per query tile
   B_PFULL = B_SFULL + NQ,     // one per query tile (one arrival per softmax warp)
   B_OFINAL = B_PFULL + NQ,
-  B_COUNT = B_OFINAL + 1
+  B_KROT = B_OFINAL + 1,  // rotate-on-load: K(j) rotated in place (one arrival)
+  B_COUNT = B_KROT + NSK
 };
 
 struct Params {
@@ -82,6 +94,84 @@ struct Params {
   float scale_log2;
 };
 
+// Source of one page of 16 positions (written by page_src_kernel): kind as
+// PageSrc below; for kind 1 the pool row of its first position and the
+// document's delta.
+struct alignas(16) PageSrcEntry {
+  int32_t kind, delta;
+  int64_t row;
+};
+
+// Rotate-on-load sources (attn_kernel<D, true>): every logical position's
+// source from pic_compose's token map -- a pool row of a document (moved by
+// that document's delta) or, for inline tokens, the paged cache.
+struct FusedArgs {
+  const int64_t *tok_map;    // [batch][max_ctx]: (k << 40) | pool row, -1 inline
+  const int32_t *doc_delta;  // [batch][max_docs]
+  const __nv_bfloat16 *k_pool, *v_pool;    // [L][pool_tokens][Hkv][D]
+  const __nv_bfloat16 *k_cache, *v_cache;  // [L][num_pages][Hkv][16][D]
+  long long pool_tokens;
+  int max_ctx, max_docs, layer;
+  bool pool_boxes;  // false: the pool is too small for a page box (all pages row by row)
+  const PageSrcEntry *page_src;  // [batch][n_pidx]
+  int n_pidx;
+};
+
+// Byte offset of the 16-byte piece ch (0 .. D/8-1) of row r (0..15) of a page
+// inside a K/V ring tile, as the page boxes lay it out with the 128-byte
+// swizzle: [8-row half][64-column panel][8 rows][128 B] at d = 128,
+// [16 rows][128 B] at d = 64.
+template <int D>
+PIC_DEV uint32_t page_piece(int r, int ch) {
+  const int c8 = ch & 7;
+  if constexpr (D == 128)
+    return (uint32_t)((r >> 3) * 2048 + (ch >> 3) * 1024 + (r & 7) * 128 + ((c8 ^ (r & 7)) << 4));
+  else
+    return (uint32_t)(r * 128 + ((c8 ^ (r & 7)) << 4));
+}
+
+// The source of every page of positions < max_ctx of every request, from the
+// token map: a page whose first and last positions are rows of one document
+// is that document's (documents occupy contiguous positions), a page of
+// inline tokens only is the cache's, anything else is mixed.  One warp per
+// page; runs once per call, ahead of the attention (programmatic launch).
+__global__ void __launch_bounds__(256) page_src_kernel(FusedArgs f, int batch, int32_t *status) {
+  pdl_entry();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long pidx = (long long)blockIdx.x * 8 + warp;
+  const int b = blockIdx.y;
+  if (pidx >= f.n_pidx || b >= batch) return;
+  const long long t = pidx * 16 + (lane & 15);
+  const long long tm = t < f.max_ctx ? f.tok_map[(size_t)b * f.max_ctx + t] : -1;
+  const unsigned inl = __ballot_sync(0xffffffffu, tm < 0) & 0xffffu;
+  const long long first = __shfl_sync(0xffffffffu, tm, 0), last = __shfl_sync(0xffffffffu, tm, 15);
+  if (lane != 0) return;
+  PageSrcEntry e;
+  e.kind = inl == 0xffffu ? 0 : 2;
+  e.delta = 0;
+  e.row = 0;
+  if (e.kind == 2 && f.pool_boxes && first >= 0 && last >= 0 && (first >> 40) == (last >> 40)) {
+    const int k = (int)(first >> 40);
+    const long long row = first & ((1LL << 40) - 1);
+    if (k < f.max_docs && row + 15 < f.pool_tokens) {
+      e.kind = 1;
+      e.delta = f.doc_delta[(size_t)b * f.max_docs + k];
+      e.row = row;
+    } else {
+      dev_fail(status, PIC_DEV_BAD_DOC_LEN, b);
+    }
+  }
+  const_cast<PageSrcEntry *>(f.page_src)[(size_t)b * f.n_pidx + pidx] = e;
+}
+
+// Sources of the 8 pages of a key tile (one page per lane 0..7).
+struct PageSrc {
+  int kind;   // 0: inline tokens (cache box at row y), 1: one document's rows
+              // (pool box at row y, rotated by delta), 2: mixed (row by row;
+              // y = the page's cache rows for its inline tokens)
+  int y, delta;
+};
+
 // One CTA = (pair of 128-row query tiles, key split, kv head, request).
 // TMEM: S_t at columns 128 t (P_t written over it as bf16), O_t at 256 + 128 t.
 // MMA order per KV tile j: PV_0(j-1), QK_0(j), PV_1(j-1), QK_1(j).  Because
@@ -92,10 +182,23 @@ struct Params {
 // a thread queues behind the MMAs that thread issued, so each one left the
 // tensor core idle for a while.  A relay warp waits for K(j), V(j-1) and
 // P_t(j-1) in the issuer's order and hands each over on a named barrier.
-template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
+//
+// kFused (rotate-on-load, pic_attend_prefill_fused): the key and value tiles
+// are assembled from the document pool and the cache instead of the stitched
+// cache alone.  A page whose 16 positions are all one document's comes from
+// the pool as one box (the document's rows are consecutive there); a page of
+// inline tokens from the cache as before; a page across a boundary is filled
+// row by row by the producer warp.  The K producer warp then rotates every
+// document row of the tile in shared memory by its document's delta -- the
+// same fp32 arithmetic and bf16 rounding as the relocation, so the tile holds
+// exactly the keys pic_relocate would have stitched -- and signals K(j) on
+// B_KROT instead of the TMA barrier.  Everything downstream (MMAs, softmax,
+// merge) is the materialised kernel's.
+template <int D, bool kFused>
+__global__ void __launch_bounds__(threads_of<kFused>(), 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                const __grid_constant__ CUtensorMap tm_v, Params p) {
+                const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_kp,
+                const __grid_constant__ CUtensorMap tm_vp, Params p, FusedArgs f, RopeParams rp) {
   using L = Layout<D>;
   constexpr int PANELS = D / 64;
   constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
@@ -118,6 +221,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::kBar + 8 * B_COUNT + 8);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // Warp roles: 0 K producer, 1 MMA issuer, then either 2-9 softmax, 10 V
+  // producer, 11 relay, or (rotate-on-load) 2 V producer, 3 relay, 4-11
+  // softmax, 12-15 rotators.
+  constexpr int W_V = kFused ? 2 : kWarpV;
+  constexpr int W_RELAY = kFused ? 3 : kWarpRelay;
+  constexpr int W_SM = kFused ? 4 : 2;  // first softmax warp
+  constexpr int W_ROT = 12;             // first rotator warp (rotate-on-load)
   // Grid (split + splits * pair, kv head, request), pairs in reverse order.
   // CTAs start in linear block order, so all CTAs of one (request, kv head)
   // start together and its K/V, read by every pair, is reused from L2; within
@@ -133,12 +243,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   // the programmatic-launch wait, while that kernel may still be finishing
   if (threadIdx.x == 0) {
     for (int i = 0; i < B_COUNT; ++i)
-      mbar_init(bar(i), (i >= B_PFULL && i < B_PFULL + NQ) ? 4 : 1);
+      mbar_init(bar(i), ((i >= B_PFULL && i < B_PFULL + NQ) || (i >= B_KROT && i < B_KROT + NSK))
+                            ? 4 : 1);
     *abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tm_q);
     prefetch_tmap(&tm_k);
     prefetch_tmap(&tm_v);
+    if constexpr (kFused) {
+      prefetch_tmap(&tm_kp);
+      prefetch_tmap(&tm_vp);
+    }
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
@@ -202,7 +317,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     return;
   }
 
-  if (warp == 0 || warp == kWarpV) {
+  // ---- the roles, each a lambda called by the warps that take it
+  auto role_producer = [&]() {
     // ===================================================== TMA producers
     // Warp 0 streams K tiles into a 3-deep ring, warp kWarpV V tiles into a
     // 2-deep ring.  Lane l < 8 moves page l of the tile as one box (a whole
@@ -240,33 +356,120 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     if (!is_k && lane == 0) prefetch_tmap(&tm_v);
-    int y_next = page_row(kv_begin);
-    int issued = 0;
-    for (int j = 0; j < n; ++j) {
-      const int st = j % nst;
-      const int y_mine = y_next;
-      if (j + 1 < n) y_next = page_row(kv_begin + j + 1);
-      if (j >= nst) {
-        const bool ok = mbar_wait(bar(b_empty + st), ((j / nst) - 1) & 1, abort_flag, p.status, detail);
-        if (!__all_sync(0xffffffffu, ok)) break;
+    if constexpr (!kFused) {
+      int y_next = page_row(kv_begin);
+      int issued = 0;
+      for (int j = 0; j < n; ++j) {
+        const int st = j % nst;
+        const int y_mine = y_next;
+        if (j + 1 < n) y_next = page_row(kv_begin + j + 1);
+        if (j >= nst) {
+          const bool ok = mbar_wait(bar(b_empty + st), ((j / nst) - 1) & 1, abort_flag, p.status, detail);
+          if (!__all_sync(0xffffffffu, ok)) break;
+        }
+        if (lane == 0) mbar_expect_tx(bar(b_full + st), L::kTile);
+        __syncwarp();
+        if (lane < 8) {  // one box per page-head
+          const uint32_t dst = ring + st * L::kTile + lane * kPageBytes;
+          if constexpr (PANELS == 2)
+            tma_load_4d(dst, tmap, 0, 0, 0, y_mine >> 3, bar(b_full + st));
+          else
+            tma_load_2d(dst, tmap, 0, y_mine, bar(b_full + st));
+        }
+        issued = j + 1;
       }
-      if (lane == 0) mbar_expect_tx(bar(b_full + st), L::kTile);
-      __syncwarp();
-      if (lane < 8) {  // one box per page-head
-        const uint32_t dst = ring + st * L::kTile + lane * kPageBytes;
-        if constexpr (PANELS == 2)
-          tma_load_4d(dst, tmap, 0, 0, 0, y_mine >> 3, bar(b_full + st));
-        else
-          tma_load_2d(dst, tmap, 0, y_mine, bar(b_full + st));
+      if (lane == 0 && *abort_flag) {
+        // Let the copies already issued land before the CTA exits.
+        for (int j = max(0, issued - nst); j < issued; ++j)
+          mbar_wait(bar(b_full + j % nst), (j / nst) & 1, abort_flag, p.status, detail);
       }
-      issued = j + 1;
+    } else {
+      // ---- rotate-on-load producers: pages from the pool or the cache as the
+      // page-source table says; mixed pages row by row.  The rotators (warps
+      // 12-15) then rotate the K tile's document rows.
+      const CUtensorMap *pmap = is_k ? &tm_kp : &tm_vp;
+      if (lane == 0) prefetch_tmap(pmap);
+      const int64_t *tmr = f.tok_map + (size_t)b * f.max_ctx;
+      const __nv_bfloat16 *pool = is_k ? f.k_pool : f.v_pool;
+      const __nv_bfloat16 *cache = is_k ? f.k_cache : f.v_cache;
+      const PageSrcEntry *ps = f.page_src + (size_t)b * f.n_pidx;
+      // lanes 0..7: the source of page `lane` of tile kt (kind 0 and 2 carry
+      // the page's cache row, kind 1 the pool row)
+      auto source = [&](int kt) -> PageSrc {
+        PageSrc src{0, page_row(kt), 0};
+        const int pidx = kt * 8 + lane;
+        if (lane < 8 && pidx < f.n_pidx) {
+          const PageSrcEntry e = ps[pidx];
+          src.kind = e.kind;
+          if (e.kind == 1) src.y = (int)((long long)f.layer * f.pool_tokens + e.row);
+        }
+        return src;
+      };
+      auto issue = [&](int st, int kt, const PageSrc &src) {
+        const uint32_t stage = ring + st * L::kTile;
+        const unsigned box_mask = __ballot_sync(0xffffffffu, lane < 8 && src.kind != 2);
+        unsigned mixed = __ballot_sync(0xffffffffu, lane < 8 && src.kind == 2);
+        if (lane == 0) mbar_expect_tx_only(bar(b_full + st), __popc(box_mask) * kPageBytes);
+        __syncwarp();
+        if (lane < 8 && src.kind != 2) {
+          const uint32_t dst = stage + lane * kPageBytes;
+          if (src.kind == 0) {
+            if constexpr (PANELS == 2)
+              tma_load_4d(dst, tmap, 0, 0, 0, src.y >> 3, bar(b_full + st));
+            else
+              tma_load_2d(dst, tmap, 0, src.y, bar(b_full + st));
+          } else {
+            if constexpr (PANELS == 2)
+              tma_load_5d(dst, pmap, 0, src.y, 0, 0, hk, bar(b_full + st));
+            else
+              tma_load_3d(dst, pmap, 0, hk, src.y, bar(b_full + st));
+          }
+        }
+        while (mixed) {  // row by row: 16-byte loads, swizzled 16-byte stores
+          const int q = __ffs(mixed) - 1;
+          mixed &= mixed - 1;
+          const int yq = __shfl_sync(0xffffffffu, src.y, q);
+          constexpr int CH = D / 8;
+          for (int e = lane; e < 16 * CH; e += 32) {
+            const int r = e / CH, ch = e % CH;
+            const long long t = (long long)kt * BN + q * 16 + r;
+            const long long tv = t < f.max_ctx ? tmr[t] : -1;
+            uint4 v = make_uint4(0, 0, 0, 0);
+            if (tv >= 0) {
+              const long long row = tv & ((1LL << 40) - 1);
+              if (row < f.pool_tokens)
+                v = ld_stream(pool + (((size_t)f.layer * f.pool_tokens + row) * p.Hkv + hk) * D + ch * 8);
+            } else if (yq != p.oob_row) {
+              v = ld_stream(cache + (size_t)(yq + r) * D + ch * 8);
+            }
+            sts128(stage + q * kPageBytes + page_piece<D>(r, ch), v);
+          }
+        }
+        fence_proxy_async();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(b_full + st));
+      };
+      PageSrc s_next = source(kv_begin);
+      int issued = 0;
+      for (int j = 0; j < n; ++j) {
+        const int st = j % nst;
+        const PageSrc s_cur = s_next;
+        if (j + 1 < n) s_next = source(kv_begin + j + 1);
+        if (j >= nst) {
+          const bool ok = mbar_wait(bar(b_empty + st), ((j / nst) - 1) & 1, abort_flag, p.status, detail);
+          if (!__all_sync(0xffffffffu, ok)) break;
+        }
+        issue(st, kv_begin + j, s_cur);
+        issued = j + 1;
+      }
+      if (lane == 0 && *abort_flag) {
+        // Let the copies already issued land before the CTA exits.
+        for (int j = max(0, issued - nst); j < issued; ++j)
+          mbar_wait(bar(b_full + j % nst), (j / nst) & 1, abort_flag, p.status, detail);
+      }
     }
-    if (lane == 0 && *abort_flag) {
-      // Let the copies already issued land before the CTA exits.
-      for (int j = max(0, issued - nst); j < issued; ++j)
-        mbar_wait(bar(b_full + j % nst), (j / nst) & 1, abort_flag, p.status, detail);
-    }
-  } else if (warp == 1) {
+  };
+  auto role_issuer = [&]() {
     // ===================================================== MMA issuer
     // The whole warp takes part in the named barriers; lane 0 issues.  After
     // an abort both this loop and the relay's run to the end (skipping their
@@ -324,7 +527,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     if (leader) mma_commit(bar(B_OFINAL));
-  } else if (warp == kWarpRelay) {
+  };
+  auto role_relay = [&]() {
     // ===================================================== relay for the issuer
     // Mirrors the issuer's loop: the same conditions, the same order.  Its
     // arrival on a barrier in iteration j + 1 depends on an MMA the issuer
@@ -345,16 +549,115 @@ __global__ void __launch_bounds__(kThreads, 1)
           named_bar_arrive(kNbPv + t, 64);
         }
         if (j < nt[t] && !k_ready) {
-          mbar_wait(bar(B_KFULL + j % NSK), (j / NSK) & 1, abort_flag, p.status, detail);
+          mbar_wait(bar((kFused ? B_KROT : B_KFULL) + j % NSK), (j / NSK) & 1, abort_flag, p.status,
+                    detail);
           named_bar_arrive(kNbK, 64);
           k_ready = true;
         }
       }
     }
-  } else {
+  };
+  auto role_rotator = [&]() {
+    // ===================================================== rotators (rotate-on-load)
+    // For every K tile: wait for its pages, rotate each document row by its
+    // document's delta exactly as pic_relocate does (cos/sin of the
+    // fp64-reduced angle, fp32 rotation, bf16 round to nearest even), then
+    // release the tile to the MMA issuer on B_KROT (one arrival per warp).
+    // Thread rt takes the 8-pair chunk rt % KC of one row of KC of the
+    // tile's pages; its cos/sin are recomputed only when its rows' document
+    // changes.
+    if constexpr (kFused) {
+      constexpr int KC = D / 16;
+      const int rt = threadIdx.x - W_ROT * 32;
+      const int my_c = rt % KC;
+      const PairChunk pc = pair_chunk(my_c, D / 2, rp.style);
+      const int64_t *tmr = f.tok_map + (size_t)b * f.max_ctx;
+      const PageSrcEntry *ps = f.page_src + (size_t)b * f.n_pidx;
+      float2 cs[8];
+      int cs_delta = 0;
+      bool cs_ok = false;
+      auto ensure_cs = [&](int delta) {
+        if (cs_ok && delta == cs_delta) return;
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          cs[q] = rp.layer_theta ? rope_cos_sin_fast(delta, rope_theta(rp, f.layer, 8 * my_c + q))
+                                 : rope_cos_sin(delta, rope_theta(rp, f.layer, 8 * my_c + q));
+        cs_delta = delta;
+        cs_ok = true;
+      };
+      for (int j = 0; j < n; ++j) {
+        const int st = j % NSK, kt = kv_begin + j;
+        // this tile's page sources (L2), then its pages
+        int kind[KC], delta[KC];
+#pragma unroll
+        for (int u = 0; u < KC; ++u) {
+          const int i = rt + 128 * u, q = i / (16 * KC);
+          const int pidx = kt * 8 + q;
+          kind[u] = 0;
+          delta[u] = 0;
+          if (pidx < f.n_pidx) {
+            const PageSrcEntry e = ps[pidx];
+            kind[u] = e.kind;
+            delta[u] = e.delta;
+          }
+        }
+        const bool ok = mbar_wait(bar(B_KFULL + st), (j / NSK) & 1, abort_flag, p.status, detail);
+        if (!__all_sync(0xffffffffu, ok)) break;
+        const uint32_t stage = sbase + L::kK + st * L::kTile;
+        // not unrolled: one copy of the (rare) cos/sin recomputation; the
+        // rotators have ample time per tile
+#pragma unroll 1
+        for (int u = 0; u < KC; ++u) {
+          if (kind[u] == 0) continue;
+          const int i = rt + 128 * u, q = i / (16 * KC), r = (i % (16 * KC)) / KC;
+          int dl = delta[u];
+          if (kind[u] == 2) {  // mixed page: this row's own document, if any
+            const long long t = (long long)kt * BN + q * 16 + r;
+            const long long tv = t < f.max_ctx ? tmr[t] : -1;
+            if (tv < 0 || (tv >> 40) >= f.max_docs) continue;
+            dl = f.doc_delta[(size_t)b * f.max_docs + (int)(tv >> 40)];
+          }
+          ensure_cs(dl);
+          const uint32_t a0 = stage + q * kPageBytes + page_piece<D>(r, pc.off_a / 8);
+          const uint32_t a1 = stage + q * kPageBytes + page_piece<D>(r, pc.off_b / 8);
+          uint4 va = lds128(a0), vb = lds128(a1);
+          float x[8], y[8], uu[8], ww[8];
+          unpack8(va, x);
+          unpack8(vb, y);
+          if (rp.style == PIC_ROPE_HALF) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) { uu[e] = x[e]; ww[e] = y[e]; }
+          } else {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              uu[e] = x[2 * e]; ww[e] = x[2 * e + 1];
+              uu[4 + e] = y[2 * e]; ww[4 + e] = y[2 * e + 1];
+            }
+          }
+          rotate8(uu, ww, cs);
+          if (rp.style == PIC_ROPE_HALF) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) { x[e] = uu[e]; y[e] = ww[e]; }
+          } else {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              x[2 * e] = uu[e]; x[2 * e + 1] = ww[e];
+              y[2 * e] = uu[4 + e]; y[2 * e + 1] = ww[4 + e];
+            }
+          }
+          sts128(a0, pack8(x));
+          sts128(a1, pack8(y));
+        }
+        fence_proxy_async();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(B_KROT + st));
+      }
+    }
+  };
+  auto role_softmax = [&]() {
     // ===================================================== softmax warpgroups
     static_assert(NQ == 2, "softmax warpgroup selection assumes two query tiles");
-    const int t = (warp - 2) >> 2;  // query tile of this warpgroup
+    const int t = (warp - W_SM) >> 2;  // query tile of this warpgroup
     const int wq = warp & 3;        // TMEM lane quarter
     const int row = wq * 32 + lane;
     // constant-index selects keep the per-tile values in registers
@@ -506,6 +809,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+  };
+  if constexpr (kFused) {
+    // Registers move from the control and rotator warpgroups to the softmax
+    // ones: each warpgroup runs one setmaxnreg at one place, and its roles'
+    // code follows it.
+    if (warp < 4) {
+      asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegCtl));
+      if (warp == 0 || warp == W_V) role_producer();
+      else if (warp == 1) role_issuer();
+      else role_relay();
+    } else if (warp >= W_ROT) {
+      asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegRot));
+      role_rotator();
+    } else {
+      asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegSoftmax));
+      role_softmax();
+    }
+  } else {
+    if (warp == 0 || warp == W_V) role_producer();
+    else if (warp == 1) role_issuer();
+    else if (warp == W_RELAY) role_relay();
+    else role_softmax();
   }
   // Release the dependent launch (the split merge, or the next layer's
   // append) only now: released at the start, it made the pass slower.
@@ -524,565 +849,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// ===========================================================================
-// Fused rotate-on-load prefill attention (documents read from the pool).
-//
-// Instead of reading relocated keys R(delta_k) k from the stitched cache, the
-// kernel reads the documents' keys and values straight from the pool (as they
-// were compiled) and rotates the *queries* the other way:
-//     (R(p) q) . (R(delta_k) k) = (R(-delta_k) R(p) q) . k,
-// since rotations are orthogonal.  Per document the query tile is turned into
-// Q'_k = R(-delta_k) Q in TMEM by the softmax threads (each owns one TMEM lane,
-// i.e. one query row) and the QK^T MMA takes its A operand from TMEM.  Prefix
-// and query keys (written by pic_append_inline) still come from the paged
-// cache.  A pool tile is 128 consecutive rows of one document: two 16 KB TMA
-// boxes per operand instead of 16 page boxes.
-//
-// Key tiles are segment aligned: the prefix [0, P) and the query span [Q0, Q1)
-// in 128-key tiles of the absolute position grid (keys outside the segment
-// masked), each document in 128-key tiles from its first token (keys past its
-// end masked).  Everything else (splits, pipeline, epilogue) is as in
-// attn_kernel's single-tile form.
-// TMEM: S_0 [0,128), S_1 [128,256), O [256,256+D), Q'_0 [384,384+D/2),
-// Q'_1 [448,448+D/2) (bf16 pairs).
-namespace fused {
-
-constexpr int BN = 128, NST = 2, kThreads = 192, kMaxDocs = 1024;
-
-template <int D>
-struct Layout {
-  static constexpr int kTile = BN * D * 2;
-  static constexpr int kQ = 0;
-  static constexpr int kK = kQ + BM * D * 2;
-  static constexpr int kV = kK + NST * kTile;
-  static constexpr int kMeta = kV + NST * kTile;
-  // seg_first[2 kMaxDocs + 2] int32, off/len/delta [kMaxDocs] int32, start [kMaxDocs] int64
-  static constexpr int kSegFirst = kMeta;
-  static constexpr int kOff = kSegFirst + (2 * kMaxDocs + 4) * 4;
-  static constexpr int kLen = kOff + kMaxDocs * 4;
-  static constexpr int kDelta = kLen + kMaxDocs * 4;
-  static constexpr int kStart = kDelta + kMaxDocs * 4;
-  static constexpr int kCS = kStart + kMaxDocs * 8;  // 64 float2
-  static constexpr int kBar = kCS + 64 * 8;
-  static constexpr int kBytes = kBar + 256;
-  static constexpr int kAlloc = kBytes + 1024;
-};
-
-enum {
-  F_Q = 0,
-  F_KFULL = 1,
-  F_VFULL = F_KFULL + NST,
-  F_KVEMPTY = F_VFULL + NST,
-  F_SFULL = F_KVEMPTY + NST,
-  F_PFULL = F_SFULL + 2,
-  F_PFREE = F_PFULL + 2,
-  F_QREADY = F_PFREE + 2,
-  F_OFINAL = F_QREADY + 2,
-  F_COUNT = F_OFINAL + 1
-};
-
-struct FParams {
-  Params base;
-  RopeParams rp;
-  long long pool_tokens;
-  int max_docs, layer;
-  const int32_t *num_docs, *doc_offset, *doc_delta, *ids, *doc_len;
-  const int64_t *doc_start;
-};
-
-// The tile sequence seen by every role.  Segment s: 0 = prefix, 1..m = doc
-// s-1, m+1 = query.  seg_first[s] = index of the segment's first tile.
-struct TileInfo {
-  int doc;         // document index, -1 for a cache tile
-  int key_base;    // logical position of smem row 0
-  int vlo, vhi;    // valid logical key range of this tile
-  int cache_kt;    // absolute 128-key tile index (cache tiles)
-  long long prow;  // pool row of smem row 0 (document tiles)
-  bool doc_first;  // first tile of its document
-};
-
-// Segments of a query tile's visible keys in logical order: cache segment
-// C_0 (the prefix), document D_0, C_1 (the inline span after D_0), D_1, ...,
-// D_{m-1}, C_m (the last span and the query).  Segment 2c is C_c, 2k+1 is
-// D_k; every range is clipped to the keys below kend.
-struct Seq {
-  const int32_t *seg_first, *off, *len, *delta;
-  const long long *start;
-  int m, kend;
-  __device__ int cache_lo(int c) const { return c == 0 ? 0 : min(off[c - 1] + len[c - 1], kend); }
-  __device__ int cache_hi(int c) const { return c < m ? min(off[c], kend) : kend; }
-  __device__ TileInfo at(int t) const {
-    // segment containing global tile t (binary search over seg_first[0..2m+1))
-    int lo = 0, hi = 2 * m;
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (seg_first[mid] <= t) lo = mid;
-      else hi = mid - 1;
-    }
-    const int j = t - seg_first[lo];
-    TileInfo ti;
-    if ((lo & 1) == 0) {
-      const int a = cache_lo(lo >> 1), e = cache_hi(lo >> 1);
-      ti.doc = -1;
-      ti.cache_kt = a / BN + j;
-      ti.key_base = ti.cache_kt * BN;
-      ti.vlo = max(a, ti.key_base);
-      ti.vhi = min(e, ti.key_base + BN);
-      ti.prow = 0;
-      ti.doc_first = false;
-    } else {
-      const int k = lo >> 1;
-      ti.doc = k;
-      ti.cache_kt = -1;
-      ti.key_base = off[k] + j * BN;
-      ti.vlo = ti.key_base;
-      ti.vhi = min(off[k] + len[k], ti.key_base + BN);
-      ti.prow = start[k] + (long long)j * BN;
-      ti.doc_first = j == 0;
-    }
-    return ti;
-  }
-};
-
-template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
-    attn_fused_kernel(const __grid_constant__ CUtensorMap tm_q,
-                      const __grid_constant__ CUtensorMap tm_k,
-                      const __grid_constant__ CUtensorMap tm_v,
-                      const __grid_constant__ CUtensorMap tm_kp,
-                      const __grid_constant__ CUtensorMap tm_vp, FParams fp) {
-  // programmatic dependent launch: the kernel before (the append) has finished
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  using L = Layout<D>;
-  const Params &p = fp.base;
-  constexpr int PANELS = D / 64;
-  constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
-  constexpr uint32_t IDESC_PV = idesc_bf16(BM, D, false, true);
-
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                              ~(uintptr_t)1023);
-  const uint32_t sbase = smem_u32(smem);
-  const uint32_t bar0 = sbase + L::kBar;
-  auto bar = [&](int i) { return bar0 + 8u * (uint32_t)i; };
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + L::kBar + 8 * F_COUNT);
-  volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::kBar + 8 * F_COUNT + 8);
-  int32_t *s_seg = reinterpret_cast<int32_t *>(smem + L::kSegFirst);
-  int32_t *s_off = reinterpret_cast<int32_t *>(smem + L::kOff);
-  int32_t *s_len = reinterpret_cast<int32_t *>(smem + L::kLen);
-  int32_t *s_delta = reinterpret_cast<int32_t *>(smem + L::kDelta);
-  long long *s_start = reinterpret_cast<long long *>(smem + L::kStart);
-  float2 *s_cs = reinterpret_cast<float2 *>(smem + L::kCS);
-
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int mt = blockIdx.x / p.num_splits, split = blockIdx.x % p.num_splits;
-  const int hk = blockIdx.y, b = blockIdx.z;
-  const int detail = b;
-
-  const int tin = min(max(p.inline_len[b], 0), p.max_inline);
-  const int rows = tin * p.G;
-  const int r0 = mt * BM;
-  if (r0 >= rows) return;
-  const int r_last = min(r0 + BM, rows) - 1;
-  const int32_t *ipos = p.inline_pos + (size_t)b * p.max_inline;
-  const int kmax = ipos[r_last / p.G];
-
-  // ---- per-document metadata into shared memory (all threads)
-  const int m = min(max(fp.num_docs[b], 0), fp.max_docs);
-  for (int k = threadIdx.x; k < m; k += kThreads) {
-    const size_t i = (size_t)b * fp.max_docs + k;
-    const int id = fp.ids[i];
-    s_off[k] = fp.doc_offset[i];
-    s_delta[k] = fp.doc_delta[i];
-    s_len[k] = (id >= 0) ? fp.doc_len[id] : 0;
-    s_start[k] = (id >= 0) ? fp.doc_start[id] : 0;
-  }
-  __syncthreads();
-  Seq sq;
-  sq.seg_first = s_seg;
-  sq.off = s_off;
-  sq.len = s_len;
-  sq.delta = s_delta;
-  sq.start = s_start;
-  sq.m = m;
-  sq.kend = kmax + 1;  // keys at or beyond kend are never visible here
-  if (threadIdx.x == 0) {  // tiles per segment, prefix sums (m <= kMaxDocs, serial is fine)
-    int t = 0;
-    auto cache_tiles = [&](int a, int e) { return e > a ? (e - 1) / BN - a / BN + 1 : 0; };
-    for (int c = 0; c <= m; ++c) {
-      s_seg[2 * c] = t;
-      t += cache_tiles(sq.cache_lo(c), sq.cache_hi(c));
-      if (c == m) break;
-      s_seg[2 * c + 1] = t;
-      const int e = min(s_off[c] + s_len[c], sq.kend);
-      t += e > s_off[c] ? (e - s_off[c] + BN - 1) / BN : 0;
-    }
-    s_seg[2 * m + 1] = t;
-  }
-  __syncthreads();
-  const int n_all = s_seg[2 * m + 1];
-  const int per = (n_all + p.num_splits - 1) / p.num_splits;
-  const int kv_begin = split * per;
-  const int n = max(0, min(per, n_all - kv_begin));
-  const size_t part_row0 =
-      ((((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * p.num_splits + split) * BM;
-  if (n == 0) {
-    if (p.num_splits > 1 && threadIdx.x < BM) {
-      p.part_ml[(part_row0 + threadIdx.x) * 2] = -INFINITY;
-      p.part_ml[(part_row0 + threadIdx.x) * 2 + 1] = 0.f;
-    }
-    return;
-  }
-
-  if (threadIdx.x == 0) {
-    for (int i = 0; i < F_COUNT; ++i)
-      mbar_init(bar(i), (i == F_PFULL || i == F_PFULL + 1 || i == F_QREADY || i == F_QREADY + 1)
-                            ? 128 : 1);
-    *abort_flag = 0;
-    fence_mbar_init();
-  }
-  if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
-    tmem_relinquish();
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tbase = *tmem_slot;
-
-  if (warp == 0) {
-    // ===================================================== TMA producer
-    const int32_t *bt = p.block_table + (size_t)b * p.max_pages;
-    if (lane == 0) {
-      prefetch_tmap(&tm_q);
-      prefetch_tmap(&tm_k);
-      prefetch_tmap(&tm_v);
-      prefetch_tmap(&tm_kp);
-      prefetch_tmap(&tm_vp);
-      mbar_expect_tx(bar(F_Q), BM * D * 2);
-      const int qrow = (b * p.Hkv + hk) * p.R_pad + r0;
-      for (int pn = 0; pn < PANELS; ++pn)
-        tma_load_2d(sbase + L::kQ + pn * BM * 128, &tm_q, pn * 64, qrow, bar(F_Q));
-    }
-    int issued = 0;
-    for (int j = 0; j < n; ++j) {
-      const int st = j % NST;
-      const TileInfo ti = sq.at(kv_begin + j);
-      int y = p.oob_row;  // cache tile: lanes 0..7 look up their page
-      if (ti.doc < 0 && lane < 8) {
-        const int pidx = ti.cache_kt * 8 + lane;
-        if (pidx * 16 < ti.vhi && pidx < p.max_pages) {
-          const int page = bt[pidx];
-          if (page >= 0 && page < p.num_pages)
-            y = (int)(p.layer_row0 + ((long long)page * p.Hkv + hk) * 16);
-          else
-            dev_fail(p.status, PIC_DEV_BAD_PAGE, detail);
-        }
-      }
-      if (j >= NST) {
-        const bool ok = mbar_wait(bar(F_KVEMPTY + st), ((j / NST) - 1) & 1, abort_flag, p.status, detail);
-        if (!__all_sync(0xffffffffu, ok)) break;
-      }
-      if (lane == 0) mbar_expect_tx(bar(F_KFULL + st), L::kTile);
-      if (lane == 16) mbar_expect_tx(bar(F_VFULL + st), L::kTile);
-      __syncwarp();
-      if (ti.doc < 0) {
-        const int box = lane & 15, bpage = box / PANELS, bpanel = box % PANELS;
-        const int yb = __shfl_sync(0xffffffffu, y, bpage);
-        if (box < 8 * PANELS) {
-          const uint32_t off = st * L::kTile + bpanel * BN * 128 + bpage * 16 * 128;
-          if (lane < 16)
-            tma_load_2d(sbase + L::kK + off, &tm_k, bpanel * 64, yb, bar(F_KFULL + st));
-          else
-            tma_load_2d(sbase + L::kV + off, &tm_v, bpanel * 64, yb, bar(F_VFULL + st));
-        }
-      } else {
-        // two 128-row boxes per operand, straight from the pool rows of the document
-        const int z = (int)((long long)fp.layer * fp.pool_tokens + ti.prow);
-        if (lane < PANELS)
-          tma_load_3d(sbase + L::kK + st * L::kTile + lane * BN * 128, &tm_kp, lane * 64, hk, z,
-                      bar(F_KFULL + st));
-        else if (lane >= 16 && lane < 16 + PANELS)
-          tma_load_3d(sbase + L::kV + st * L::kTile + (lane - 16) * BN * 128, &tm_vp,
-                      (lane - 16) * 64, hk, z, bar(F_VFULL + st));
-      }
-      issued = j + 1;
-    }
-    if (lane == 0 && *abort_flag) {
-      for (int j = max(0, issued - NST); j < issued; ++j) {
-        mbar_wait(bar(F_KFULL + j % NST), (j / NST) & 1, abort_flag, p.status, detail);
-        mbar_wait(bar(F_VFULL + j % NST), (j / NST) & 1, abort_flag, p.status, detail);
-      }
-    }
-  } else if (warp == 1) {
-    // ===================================================== MMA issuer
-    if (lane == 0) {
-      const uint32_t tS0 = tbase, tO = tbase + 256, tQd = tbase + 384;
-      bool ok = mbar_wait(bar(F_Q), 0, abort_flag, p.status, detail);
-      tc_fence_after();
-      // base descriptors; stages and k-steps add (offset >> 4) to the address field
-      const uint64_t dQ = sdesc_sw128(sbase + L::kQ, 16, 1024);
-      const uint64_t dK = sdesc_sw128(sbase + L::kK, 16, 1024);
-      const uint64_t dV = sdesc_sw128(sbase + L::kV, BN * 128, 1024);
-      int dcount = -1;  // documents entered so far in this split
-      for (int j = 0; ok && j <= n; ++j) {
-        if (j < n) {
-          const int st = j % NST, sb = j & 1;
-          const TileInfo ti = sq.at(kv_begin + j);
-          if (ti.doc >= 0 && (ti.doc_first || j == 0)) {  // entering a document
-            ++dcount;
-            if (!mbar_wait(bar(F_QREADY + (dcount & 1)), (dcount >> 1) & 1, abort_flag, p.status, detail)) break;
-          }
-          if (!mbar_wait(bar(F_KFULL + st), (j / NST) & 1, abort_flag, p.status, detail)) break;
-          tc_fence_after();
-          const uint64_t dk = dK + (uint64_t)((st * L::kTile) >> 4);
-          if (ti.doc < 0) {
-#pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk)
-              mma_ss(tS0 + sb * 128, dQ + ((kk >> 2) * (BM * 128) + (kk & 3) * 32) / 16,
-                     dk + ((kk >> 2) * (BN * 128) + (kk & 3) * 32) / 16, IDESC_QK, kk > 0);
-          } else {
-            const uint32_t qa = tQd + (dcount & 1) * 64;
-#pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk)
-              mma_ts(tS0 + sb * 128, qa + kk * 8, dk + ((kk >> 2) * (BN * 128) + (kk & 3) * 32) / 16,
-                     IDESC_QK, kk > 0);
-          }
-          mma_commit(bar(F_SFULL + sb));
-        }
-        if (j >= 1) {
-          const int pj = j - 1, pst = pj % NST, pb = pj & 1;
-          if (!mbar_wait(bar(F_PFULL + pb), (pj >> 1) & 1, abort_flag, p.status, detail)) break;
-          if (!mbar_wait(bar(F_VFULL + pst), (pj / NST) & 1, abort_flag, p.status, detail)) break;
-          tc_fence_after();
-          const uint64_t dv = dV + (uint64_t)((pst * L::kTile) >> 4);
-#pragma unroll
-          for (int kk = 0; kk < BN / 16; ++kk)
-            mma_ts(tO, tS0 + pb * 128 + kk * 8, dv + (kk * 16 * 128) / 16, IDESC_PV,
-                   (pj > 0 || kk > 0));
-          mma_commit(bar(F_KVEMPTY + pst));
-          mma_commit(bar(F_PFREE + pb));
-        }
-      }
-      mma_commit(bar(F_OFINAL));
-    }
-  } else {
-    // ===================================================== softmax warps
-    const int wq = warp & 3;
-    const int row = wq * 32 + lane;
-    const int rg = r0 + row;
-    const bool valid = rg < rows;
-    const int tok = rg / p.G, g = rg % p.G;
-    const int pos = valid ? ipos[tok] : -1;
-    const uint32_t tl = tbase + ((uint32_t)(wq * 32) << 16);
-    const uint32_t tQd = tl + 384;
-    const int tid128 = threadIdx.x - 64;
-    bool ok = true;
-
-    float m_used = -INFINITY, l = 0.f;
-    int dcount = -1;
-    // Q'_k = R(-delta_k) Q for this thread's row, into TMEM buffer `buf`.
-    auto make_qd = [&](int k, int buf) {
-      asm volatile("bar.sync 1, 128;" ::: "memory");  // previous table no longer read
-      if (tid128 < D / 2) {
-        const float2 cs = rope_cos_sin(s_delta[k], rope_theta(fp.rp, fp.layer, tid128));
-        s_cs[tid128] = make_float2(cs.x, -cs.y);  // R(-delta): sin changes sign
-      }
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      // my row of Q from shared memory (128-byte swizzled panels), rotate, pack
-      float x[D];
-      const uint8_t *qs = smem + L::kQ;
-#pragma unroll
-      for (int c = 0; c < D / 8; ++c) {
-        const int pn = c >> 3, ch = c & 7;
-        const uint4 v = *reinterpret_cast<const uint4 *>(
-            qs + pn * BM * 128 + row * 128 + ((ch ^ (row & 7)) << 4));
-        unpack8(v, x + 8 * c);
-      }
-      uint32_t pk[D / 2];
-      if (fp.rp.style == PIC_ROPE_HALF) {
-#pragma unroll
-        for (int i = 0; i < D / 2; ++i) {
-          const float2 cs = s_cs[i];
-          const float u = x[i], w = x[i + D / 2];
-          x[i] = fmaf(u, cs.x, -w * cs.y);
-          x[i + D / 2] = fmaf(u, cs.y, w * cs.x);
-        }
-      } else {
-#pragma unroll
-        for (int i = 0; i < D / 2; ++i) {
-          const float2 cs = s_cs[i];
-          const float u = x[2 * i], w = x[2 * i + 1];
-          x[2 * i] = fmaf(u, cs.x, -w * cs.y);
-          x[2 * i + 1] = fmaf(u, cs.y, w * cs.x);
-        }
-      }
-#pragma unroll
-      for (int i = 0; i < D / 2; ++i) pk[i] = pack2(x[2 * i], x[2 * i + 1]);
-#pragma unroll
-      for (int c = 0; c < D / 64; ++c) tmem_st32(tQd + buf * 64 + c * 32, pk + c * 32);
-      tmem_wait_st();
-      tc_fence_before();
-      mbar_arrive(bar(F_QREADY + buf));
-    };
-
-    if (!__all_sync(0xffffffffu, mbar_wait(bar(F_Q), 0, abort_flag, p.status, detail))) ok = false;
-    // documents of this split, in order: first one prepared up front
-    int next_doc = -1;  // next document whose Q' is still to be prepared
-    if (ok) {
-      for (int j = 0; j < n; ++j) {
-        const TileInfo ti = sq.at(kv_begin + j);
-        if (ti.doc >= 0) {
-          next_doc = ti.doc;
-          break;
-        }
-      }
-      if (next_doc >= 0) {
-        make_qd(next_doc, 0);
-        ++next_doc;
-      }
-    }
-    int last_tile_doc = -1;  // last document with a tile in this split
-    for (int j = n - 1; ok && j >= 0; --j) {
-      const int dj = sq.at(kv_begin + j).doc;
-      if (dj >= 0) {
-        last_tile_doc = dj;
-        break;
-      }
-    }
-    for (int j = 0; ok && j < n; ++j) {
-      const int sb = j & 1;
-      const TileInfo ti = sq.at(kv_begin + j);
-      if (!__all_sync(0xffffffffu, mbar_wait(bar(F_SFULL + sb), (j >> 1) & 1, abort_flag, p.status, detail))) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      if (ti.doc >= 0 && (ti.doc_first || j == 0)) {
-        ++dcount;
-        // S of this document's first tile is ready, so every QK of the
-        // document before it has finished: its Q' buffer may be reused.
-        if (next_doc >= 0 && next_doc <= last_tile_doc) {
-          make_qd(next_doc, (dcount + 1) & 1);
-          ++next_doc;
-        }
-      }
-      float s[BN];
-#pragma unroll
-      for (int c = 0; c < BN / 32; ++c)
-        tmem_ld32(tl + sb * 128 + c * 32, reinterpret_cast<uint32_t *>(s + c * 32));
-      tmem_wait_ld();
-      {
-        const int lo = ti.vlo - ti.key_base, hi = min(ti.vhi, pos + 1) - ti.key_base;
-        if (lo > 0 || hi < BN) {
-#pragma unroll
-          for (int c = 0; c < BN; ++c)
-            if (c < lo || c >= hi) s[c] = -INFINITY;
-        }
-      }
-      float mx8[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) mx8[i] = s[i];
-#pragma unroll
-      for (int c = 8; c < BN; c += 8)
-#pragma unroll
-        for (int i = 0; i < 8; ++i) mx8[i] = fmaxf(mx8[i], s[c + i]);
-#pragma unroll
-      for (int w = 4; w; w >>= 1)
-#pragma unroll
-        for (int i = 0; i < w; ++i) mx8[i] = fmaxf(mx8[i], mx8[i + w]);
-      const float m_new = fmaxf(m_used, mx8[0] * p.scale_log2);
-      float alpha = 1.f;
-      const bool resc = m_new > m_used + 8.f;
-      if (resc) {
-        alpha = ex2(m_used - m_new);
-        m_used = m_new;
-      }
-      const float mref = (m_used == -INFINITY) ? 0.f : m_used;
-      float ls8[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) ls8[i] = 0.f;
-      uint32_t pk[BN / 2];
-#pragma unroll
-      for (int c = 0; c < BN; c += 2) {
-        const float p0 = ex2(fmaf(s[c], p.scale_log2, -mref));
-        const float p1 = ex2(fmaf(s[c + 1], p.scale_log2, -mref));
-        ls8[(c >> 1) & 7] += p0 + p1;
-        pk[c / 2] = pack2(p0, p1);
-      }
-#pragma unroll
-      for (int w = 4; w; w >>= 1)
-#pragma unroll
-        for (int i = 0; i < w; ++i) ls8[i] += ls8[i + w];
-      l = fmaf(l, alpha, ls8[0]);
-      if (j > 0 && __any_sync(0xffffffffu, resc)) {
-        const int pj = j - 1;
-        if (!__all_sync(0xffffffffu, mbar_wait(bar(F_PFREE + (pj & 1)), (pj >> 1) & 1, abort_flag, p.status, detail))) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-#pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
-          float o[32];
-          tmem_ld32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o));
-          tmem_wait_ld();
-#pragma unroll
-          for (int q = 0; q < 32; ++q) o[q] *= alpha;
-          tmem_st32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o));
-        }
-      }
-      tmem_st32(tl + sb * 128, pk);
-      tmem_st32(tl + sb * 128 + 32, pk + 32);
-      tmem_wait_st();
-      tc_fence_before();
-      mbar_arrive(bar(F_PFULL + sb));
-    }
-    // ---- epilogue
-    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(F_OFINAL), 0, abort_flag, p.status, detail));
-    tc_fence_after();
-    if (ok) {
-      float o[D];
-#pragma unroll
-      for (int c = 0; c < D / 32; ++c) tmem_ld32(tl + 256 + c * 32, reinterpret_cast<uint32_t *>(o + c * 32));
-      tmem_wait_ld();
-      if (p.num_splits == 1) {
-        const float inv = l > 0.f ? 1.f / l : 0.f;
-        __nv_bfloat16 *dst = p.out + (((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g) * D;
-        if (valid) {
-#pragma unroll
-          for (int q = 0; q < D; ++q) o[q] *= inv;
-#pragma unroll
-          for (int q = 0; q < D / 8; ++q) st_global16(dst + q * 8, pack8(o + q * 8));
-        }
-        if (valid && p.lse)
-          p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
-              l > 0.f ? (m_used + __log2f(l)) * 0.69314718055994531f : -INFINITY;
-      } else {
-        float *dst = p.part_o + (part_row0 + row) * D;
-        if (valid) {
-#pragma unroll
-          for (int q = 0; q < D / 4; ++q)
-            reinterpret_cast<float4 *>(dst)[q] =
-                make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
-        }
-        p.part_ml[(part_row0 + row) * 2] = (l > 0.f) ? m_used : -INFINITY;
-        p.part_ml[(part_row0 + row) * 2 + 1] = l;
-      }
-    }
-  }
-
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    if (*abort_flag && lane == 0) mbar_wait(bar(F_OFINAL), 0, abort_flag, p.status, detail);
-    __syncwarp();
-    tmem_dealloc(tbase, kTmemCols);
-  }
-}
-
-}  // namespace fused
 
 // Merge the split partials (O unnormalised, m in log2 units, l) of every
 // query row by log-sum-exp, lanes over the d columns.  A warp takes R rows
@@ -1317,8 +1083,8 @@ __global__ void __launch_bounds__(256) append_kernel(AppendArgs a, RopeParams rp
 }
 
 struct Plan {
-  int G, m_tiles, R_pad, splits;
-  size_t q_bytes, po_bytes, pml_bytes, total;
+  int G, m_tiles, R_pad, splits, n_pidx;
+  size_t q_bytes, po_bytes, pml_bytes, ps_bytes, total;
 };
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -1352,7 +1118,10 @@ inline Plan plan(const pic_geom_t *g, int batch, int max_inline, int max_ctx, in
   } else {
     pl.po_bytes = pl.pml_bytes = 0;
   }
-  pl.total = pl.q_bytes + pl.po_bytes + pl.pml_bytes;
+  // rotate-on-load: the source of every page of positions < max_ctx
+  pl.n_pidx = (max_ctx + 15) / 16;
+  pl.ps_bytes = align256((size_t)batch * pl.n_pidx * sizeof(PageSrcEntry));
+  pl.total = pl.q_bytes + pl.po_bytes + pl.pml_bytes + pl.ps_bytes;
   return pl;
 }
 
@@ -1524,6 +1293,47 @@ extern "C" pic_status_t pic_append_inline(
                        num_pages, k_cache, v_cache, workspace, stream);
 }
 
+namespace pic {
+namespace prefill {
+
+// The attention launch (and the merge launch when the key range is split).
+template <int D, bool kFused>
+static cudaError_t launch_attention(const Plan &pl, const Params &pp, const FusedArgs &fa,
+                                    const RopeParams &rp, const CUtensorMap &tq,
+                                    const CUtensorMap &tk, const CUtensorMap &tv,
+                                    const CUtensorMap &tkp, const CUtensorMap &tvp,
+                                    cudaStream_t stream) {
+  const int smem = Layout<D>::kAlloc;
+  cudaError_t e = cudaFuncSetAttribute(attn_kernel<D, kFused>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  if constexpr (kFused) {
+    // setmaxnreg.inc waits for registers the CTA was launched with: refuse to
+    // launch a build whose register count at launch would not cover the split
+    cudaFuncAttributes fa_attr;
+    e = cudaFuncGetAttributes(&fa_attr, attn_kernel<D, kFused>);
+    if (e != cudaSuccess) return e;
+    if (fa_attr.numRegs < kRegLaunchFused) return cudaErrorInvalidConfiguration;
+    // page sources of the call, ahead of the attention
+    const dim3 pgrid((fa.n_pidx + 7) / 8, pp.batch);
+    e = launch_dependent(page_src_kernel, pgrid, dim3(256), 0, stream, fa, pp.batch, pp.status);
+    if (e != cudaSuccess) return e;
+  }
+  dim3 grid(((pl.m_tiles + NQ - 1) / NQ) * pl.splits, pp.Hkv, pp.batch);
+  e = launch_dependent(attn_kernel<D, kFused>, grid, dim3(threads_of<kFused>()), smem, stream, tq,
+                       tk, tv, tkp, tvp, pp, fa, rp);
+  if (e != cudaSuccess) return e;
+  if (pl.splits > 1) {
+    const long long rows = (long long)pp.batch * pp.Hkv * pl.m_tiles * BM;
+    e = launch_combine<D>(rows, pp, stream);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace prefill
+}  // namespace pic
+
 extern "C" pic_status_t pic_attend_prefill(
     const pic_geom_t *geom, int32_t layer, int32_t batch, int32_t max_inline, const void *q,
     const void *k_new, const void *v_new, const int32_t *inline_pos, const int32_t *inline_len,
@@ -1595,27 +1405,8 @@ extern "C" pic_status_t pic_attend_prefill(
   pp.status = status;
   pp.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
 
-  dim3 grid(((pl.m_tiles + NQ - 1) / NQ) * pl.splits, Hkv, batch);
-  cudaError_t e;
-  if (D == 128) {
-    const int smem = Layout<128>::kAlloc;
-    e = cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill smem attribute");
-    e = launch_dependent(attn_kernel<128>, grid, dim3(kThreads), smem, stream, tq, tk, tv, pp);
-    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill launch");
-  } else {
-    const int smem = Layout<64>::kAlloc;
-    e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill smem attribute");
-    e = launch_dependent(attn_kernel<64>, grid, dim3(kThreads), smem, stream, tq, tk, tv, pp);
-    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill launch");
-  }
-  if (pl.splits > 1) {
-    const long long rows = (long long)batch * Hkv * pl.m_tiles * BM;
-    e = D == 128 ? launch_combine<128>(rows, pp, stream) : launch_combine<64>(rows, pp, stream);
-    if (e != cudaSuccess) return cuda_fail(e, "merge launch");
-  }
-  e = cudaGetLastError();
+  cudaError_t e = D == 128 ? launch_attention<128, false>(pl, pp, FusedArgs{}, rp, tq, tk, tv, tk, tv, stream)
+                           : launch_attention<64, false>(pl, pp, FusedArgs{}, rp, tq, tk, tv, tk, tv, stream);
   if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill launch");
   return PIC_OK;
 }
@@ -1625,62 +1416,67 @@ extern "C" pic_status_t pic_attend_prefill_fused(
     const void *k_new, const void *v_new, const int32_t *inline_pos, const int32_t *inline_len,
     int32_t max_ctx, const int32_t *block_table, int32_t max_pages, int64_t num_pages,
     void *k_cache, void *v_cache, const void *k_pool, const void *v_pool, int64_t pool_tokens,
-    int32_t max_docs, const int64_t *doc_token_start, const int32_t *doc_len,
-    const int32_t *req_doc_ids, const int32_t *req_num_docs, const int32_t *doc_offset,
-    const int32_t *doc_delta, void *out, float *lse, int32_t num_splits, void *workspace,
-    size_t workspace_bytes, pic_stream_t stream) {
+    int32_t max_docs, const int64_t *tok_map, const int32_t *doc_delta, void *out, float *lse,
+    int32_t num_splits, void *workspace, size_t workspace_bytes, pic_stream_t stream) {
   using namespace pic;
   using namespace pic::prefill;
+  static const char *who = "pic_attend_prefill_fused";
   RopeParams rp;
   Plan pl;
-  pic_status_t st = check_common("pic_attend_prefill_fused", geom, layer, batch, max_inline,
-                                 max_ctx, num_pages, num_splits, workspace, workspace_bytes, &rp,
-                                 &pl);
+  pic_status_t st = check_common(who, geom, layer, batch, max_inline, max_ctx, num_pages,
+                                 num_splits, workspace, workspace_bytes, &rp, &pl);
   if (st != PIC_OK) return st;
   if (max_pages <= 0 || pool_tokens <= 0 || max_docs < 0)
-    return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill_fused: sizes must be positive");
-  if (max_docs > fused::kMaxDocs)
-    return fail(PIC_ERR_UNSUPPORTED, "pic_attend_prefill_fused: max_docs %d > %d", max_docs,
-                fused::kMaxDocs);
+    return fail(PIC_ERR_INVALID_ARG, "%s: sizes must be positive", who);
   if ((long long)geom->num_layers * pool_tokens >= (long long)INT32_MAX)
-    return fail(PIC_ERR_UNSUPPORTED, "pic_attend_prefill_fused: pool has more than 2^31 rows");
+    return fail(PIC_ERR_UNSUPPORTED, "%s: pool has more than 2^31 rows", who);
   if (!inline_pos || !inline_len || !block_table || !k_cache || !v_cache || !k_pool || !v_pool ||
-      !out || (max_docs > 0 && (!doc_token_start || !doc_len || !req_doc_ids || !doc_offset ||
-                                !doc_delta)) || !req_num_docs)
-    return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill_fused: NULL tensor");
+      !out || !tok_map || (max_docs > 0 && !doc_delta))
+    return fail(PIC_ERR_INVALID_ARG, "%s: NULL tensor", who);
+  st = check_projections(who, q, k_new, v_new);
+  if (st != PIC_OK) return st;
+  out = device_address(out);
+  if (!out)
+    return fail(PIC_ERR_INVALID_ARG,
+                "%s: out is neither memory of the current device nor page-locked host memory", who);
   if ((reinterpret_cast<uintptr_t>(k_cache) | reinterpret_cast<uintptr_t>(v_cache) |
        reinterpret_cast<uintptr_t>(k_pool) | reinterpret_cast<uintptr_t>(v_pool) |
        reinterpret_cast<uintptr_t>(out)) & 15)
-    return fail(PIC_ERR_INVALID_ARG, "pic_attend_prefill_fused: bf16 tensors must be 16-byte aligned");
-  st = check_projections("pic_attend_prefill_fused", q, k_new, v_new);
-  if (st != PIC_OK) return st;
+    return fail(PIC_ERR_INVALID_ARG, "%s: bf16 tensors must be 16-byte aligned", who);
   int32_t *status = device_status_ptr();
-  if (!status) return fail(PIC_ERR_CUDA, "pic_attend_prefill_fused: no device status word");
+  if (!status) return fail(PIC_ERR_CUDA, "%s: no device status word", who);
   if (q) {  // the inline tokens' RoPE and append first (slots from the block table)
-    st = launch_append("pic_attend_prefill_fused", geom, rp, pl, layer, batch, max_inline, q,
-                       k_new, v_new, inline_pos, inline_len, nullptr, block_table, max_pages,
-                       max_ctx, num_pages, k_cache, v_cache, workspace, stream);
+    st = launch_append(who, geom, rp, pl, layer, batch, max_inline, q, k_new, v_new, inline_pos,
+                       inline_len, nullptr, block_table, max_pages, max_ctx, num_pages, k_cache,
+                       v_cache, workspace, stream);
     if (st != PIC_OK) return st;
   }
   const int D = geom->head_dim, Hkv = geom->num_kv_heads;
   const long long rows_total = (long long)geom->num_layers * num_pages * Hkv * 16;
+  const uint64_t pool_rows = (uint64_t)geom->num_layers * pool_tokens;
   uint8_t *ws = static_cast<uint8_t *>(workspace);
 
   CUtensorMap tq, tk, tv, tkp, tvp;
   st = encode_tmap_2d(&tq, ws, D, (uint64_t)batch * Hkv * pl.R_pad, (uint64_t)D * 2, 64, BM);
-  if (st == PIC_OK) st = encode_tmap_2d(&tk, k_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
-  if (st == PIC_OK) st = encode_tmap_2d(&tv, v_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
-  const uint64_t pool_rows = (uint64_t)geom->num_layers * pool_tokens;
-  if (st == PIC_OK)
-    st = encode_tmap_3d(&tkp, k_pool, D, Hkv, pool_rows, (uint64_t)D * 2, (uint64_t)Hkv * D * 2,
-                        64, 1, fused::BN);
-  if (st == PIC_OK)
-    st = encode_tmap_3d(&tvp, v_pool, D, Hkv, pool_rows, (uint64_t)D * 2, (uint64_t)Hkv * D * 2,
-                        64, 1, fused::BN);
+  const bool pool_boxes = pool_rows > 16;  // else the maps below are placeholders, never used
+  if (D == 128) {
+    if (st == PIC_OK) st = encode_tmap_pages128(&tk, k_cache, (uint64_t)rows_total / 16);
+    if (st == PIC_OK) st = encode_tmap_pages128(&tv, v_cache, (uint64_t)rows_total / 16);
+    if (st == PIC_OK) st = encode_tmap_pool128(&tkp, k_pool, pool_boxes ? pool_rows : 17, Hkv);
+    if (st == PIC_OK) st = encode_tmap_pool128(&tvp, v_pool, pool_boxes ? pool_rows : 17, Hkv);
+  } else {
+    if (st == PIC_OK) st = encode_tmap_2d(&tk, k_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
+    if (st == PIC_OK) st = encode_tmap_2d(&tv, v_cache, D, rows_total, (uint64_t)D * 2, 64, 16);
+    if (st == PIC_OK)
+      st = encode_tmap_3d(&tkp, k_pool, D, Hkv, pool_boxes ? pool_rows : 16, (uint64_t)D * 2,
+                          (uint64_t)Hkv * D * 2, 64, 1, 16);
+    if (st == PIC_OK)
+      st = encode_tmap_3d(&tvp, v_pool, D, Hkv, pool_boxes ? pool_rows : 16, (uint64_t)D * 2,
+                          (uint64_t)Hkv * D * 2, 64, 1, 16);
+  }
   if (st != PIC_OK) return st;
 
-  fused::FParams fp;
-  Params &pp = fp.base;
+  Params pp;
   pp.batch = batch;
   pp.Hq = geom->num_q_heads;
   pp.Hkv = Hkv;
@@ -1702,40 +1498,22 @@ extern "C" pic_status_t pic_attend_prefill_fused(
   pp.part_ml = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes + pl.po_bytes) : nullptr;
   pp.status = status;
   pp.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
-  fp.rp = rp;
-  fp.pool_tokens = pool_tokens;
-  fp.max_docs = max_docs;
-  fp.layer = layer;
-  fp.num_docs = req_num_docs;
-  fp.doc_offset = doc_offset;
-  fp.doc_delta = doc_delta;
-  fp.ids = req_doc_ids;
-  fp.doc_len = doc_len;
-  fp.doc_start = doc_token_start;
-
-  dim3 grid(pl.m_tiles * pl.splits, Hkv, batch);
-  cudaError_t e;
-  if (D == 128) {
-    const int smem = fused::Layout<128>::kAlloc;
-    e = cudaFuncSetAttribute(fused::attn_fused_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused smem attribute");
-    e = launch_dependent(fused::attn_fused_kernel<128>, grid, dim3(fused::kThreads), smem, stream,
-                         tq, tk, tv, tkp, tvp, fp);
-    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused launch");
-  } else {
-    const int smem = fused::Layout<64>::kAlloc;
-    e = cudaFuncSetAttribute(fused::attn_fused_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused smem attribute");
-    e = launch_dependent(fused::attn_fused_kernel<64>, grid, dim3(fused::kThreads), smem, stream,
-                         tq, tk, tv, tkp, tvp, fp);
-    if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused launch");
-  }
-  if (pl.splits > 1) {
-    const long long crows = (long long)batch * Hkv * pl.m_tiles * BM;
-    e = D == 128 ? launch_combine<128>(crows, pp, stream) : launch_combine<64>(crows, pp, stream);
-    if (e != cudaSuccess) return cuda_fail(e, "merge launch");
-  }
-  e = cudaGetLastError();
+  FusedArgs fa;
+  fa.tok_map = tok_map;
+  fa.doc_delta = doc_delta;
+  fa.k_pool = static_cast<const __nv_bfloat16 *>(k_pool);
+  fa.v_pool = static_cast<const __nv_bfloat16 *>(v_pool);
+  fa.k_cache = static_cast<const __nv_bfloat16 *>(k_cache);
+  fa.v_cache = static_cast<const __nv_bfloat16 *>(v_cache);
+  fa.pool_tokens = pool_tokens;
+  fa.max_ctx = max_ctx;
+  fa.max_docs = max_docs;
+  fa.layer = layer;
+  fa.pool_boxes = pool_boxes;
+  fa.page_src = reinterpret_cast<const PageSrcEntry *>(ws + pl.q_bytes + pl.po_bytes + pl.pml_bytes);
+  fa.n_pidx = pl.n_pidx;
+  cudaError_t e = D == 128 ? launch_attention<128, true>(pl, pp, fa, rp, tq, tk, tv, tkp, tvp, stream)
+                           : launch_attention<64, true>(pl, pp, fa, rp, tq, tk, tv, tkp, tvp, stream);
   if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused launch");
   return PIC_OK;
 }

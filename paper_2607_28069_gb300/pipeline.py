@@ -231,13 +231,15 @@ class CacheHitPath:
                            self.prefill_splits, self.ws_prefill)
 
     # -- a7: prefill attention reading the documents from the pool (no relocate)
-    def attend_fused(self, layer: int):
+    def attend_fused(self, layer: int, out: torch.Tensor | None = None):
+        """Rotate-on-load attention of one layer (the workspace holds the
+        layer's append); `out` as for attend."""
         wl = self.wl
         pic_attend_prefill_fused(self.geom, layer, self.inline_pos, wl.inline_len, self.max_ctx,
                                  wl.block_table, wl.num_pages, self.k_cache, self.v_cache,
-                                 wl.k_pool, wl.v_pool, wl.doc_token_start, wl.doc_len,
-                                 wl.req_doc_ids, wl.req_num_docs, self.doc_offset, self.doc_delta,
-                                 self.out[layer], None if self.lse is None else self.lse[layer],
+                                 wl.k_pool, wl.v_pool, self.tok_map, self.doc_delta,
+                                 self.out[layer] if out is None else out,
+                                 None if self.lse is None else self.lse[layer],
                                  self.prefill_splits, self.ws_prefill)
 
     def prefill(self, layer: int):
