@@ -356,14 +356,23 @@ pic_status_t pic_attend_prefill(const pic_geom_t *geom, int32_t layer, int32_t b
  * bit for bit (same split count).  Values are used as they are.
  *
  * Arguments as pic_attend_prefill, plus: k_pool, v_pool with pool_tokens
- * rows per layer (pool layout above; pool_tokens > 16); tok_map int64
+ * rows per layer (pool layout above); tok_map int64
  * [batch][max_ctx] and doc_delta int32 [batch][max_docs] as pic_compose (or
  * pic_link) wrote them for this request layout.  Inline keys and values come
  * from the paged cache: pass the layer's projections q, k_new, v_new to
  * append them first, or NULL when pic_append_inline already ran for this
- * layer.  Launches: the append when given, the attention, the merge when
- * split.
+ * layer.  workspace: >= pic_prefill_fused_workspace_size(...) bytes, the
+ * same buffer pic_append_inline filled.  Launches: the append when given, a
+ * set-up kernel (page sources, document cos/sin), the attention, the merge
+ * when split.
  */
+/* Workspace of pic_attend_prefill_fused (>= pic_prefill_workspace_size of the
+ * same sizes: after the packed queries and split partials, the source of
+ * every page of positions < max_ctx and the cos/sin of every listed
+ * document).  0 on bad arguments. */
+size_t pic_prefill_fused_workspace_size(const pic_geom_t *geom, int32_t batch, int32_t max_inline,
+                                        int32_t max_ctx, int32_t max_docs, int32_t num_splits);
+
 pic_status_t pic_attend_prefill_fused(const pic_geom_t *geom, int32_t layer, int32_t batch,
                                       int32_t max_inline, const void *q, const void *k_new,
                                       const void *v_new, const int32_t *inline_pos,

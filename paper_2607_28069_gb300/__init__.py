@@ -20,7 +20,7 @@ __all__ = [
     "pic_relocate_mapped", "pic_link",
     "pic_attention_deviation", "pic_copy_async",
     "pic_append_inline", "pic_attend_prefill", "pic_attend_prefill_fused",
-    "pic_prefill_workspace_size",
+    "pic_prefill_workspace_size", "pic_prefill_fused_workspace_size",
     "pic_prefill_num_splits", "pic_decode_num_splits", "pic_attend_decode_noalloc",
     "pic_attend_decode", "pic_decode_workspace_size", "pic_device_status", "PicError",
     "EXPORTED_SYMBOLS", "ROPE_HALF", "ROPE_INTERLEAVED",
@@ -36,7 +36,8 @@ ROPE_INTERLEAVED = 1
 # Every symbol include/pic.h declares.
 EXPORTED_SYMBOLS = (
     "pic_abi_version", "pic_last_error", "pic_device_status", "pic_compose", "pic_relocate",
-    "pic_relocate_mapped", "pic_link", "pic_attention_deviation", "pic_prefill_workspace_size", "pic_prefill_num_splits",
+    "pic_relocate_mapped", "pic_link", "pic_attention_deviation", "pic_prefill_workspace_size",
+    "pic_prefill_fused_workspace_size", "pic_prefill_num_splits",
     "pic_append_inline",
     "pic_attend_prefill", "pic_attend_prefill_fused", "pic_decode_workspace_size", "pic_decode_num_splits",
     "pic_attend_decode", "pic_attend_decode_noalloc", "pic_copy_async",
@@ -120,6 +121,7 @@ def load():
         "pic_link": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, P, I32, I64, I32, I32, P, P, I64,
                            I32, I32, I32, P, P, P, P, P, P, P, P, P, P, P, P, P, SZ, P]),
         "pic_prefill_workspace_size": (SZ, [G, I32, I32, I32, I32]),
+        "pic_prefill_fused_workspace_size": (SZ, [G, I32, I32, I32, I32, I32]),
         "pic_attention_deviation": (I32, [G, I32, I32, I32, I32, I32, I64, P, P, P, I32, P, P, P,
                                           P, P, P, P, P, P, I32, P, SZ, P, P, P]),
         "pic_append_inline": (I32, [G, I32, I32, I32, P, P, P, P, P, P, I32, I64, P, P, P, SZ,
@@ -309,6 +311,13 @@ def pic_prefill_workspace_size(geom: Geometry, batch: int, max_inline: int, max_
     g = geom._c()
     return load().pic_prefill_workspace_size(ctypes.byref(g), batch, max_inline, max_ctx,
                                              num_splits)
+
+
+def pic_prefill_fused_workspace_size(geom: Geometry, batch: int, max_inline: int, max_ctx: int,
+                                     max_docs: int, num_splits: int = 0) -> int:
+    g = geom._c()
+    return load().pic_prefill_fused_workspace_size(ctypes.byref(g), batch, max_inline, max_ctx,
+                                                   max_docs, num_splits)
 
 
 def pic_prefill_num_splits(geom: Geometry, batch: int, max_inline: int, max_ctx: int,

@@ -66,7 +66,9 @@ struct Layout {
   static constexpr int kK = kQ + NQ * kQTile;
   static constexpr int kV = kK + NSK * kTile;
   static constexpr int kBar = kV + NSV * kTile;
-  static constexpr int kBytes = kBar + 256;
+  // rotate-on-load: per K stage the sources of its 8 pages ({kind, delta})
+  static constexpr int kInfo = kBar + 256;
+  static constexpr int kBytes = kInfo + NSK * 8 * 8;
   static constexpr int kAlloc = kBytes + 1024;  // slack for 1024-byte alignment
 };
 
@@ -94,9 +96,9 @@ struct Params {
   float scale_log2;
 };
 
-// Source of one page of 16 positions (written by page_src_kernel): kind as
+// Source of one page of 16 positions (written by fused_setup_kernel): kind as
 // PageSrc below; for kind 1 the pool row of its first position and the
-// document's delta.
+// document's index k in the request (field `delta`).
 struct alignas(16) PageSrcEntry {
   int32_t kind, delta;
   int64_t row;
@@ -114,7 +116,8 @@ struct FusedArgs {
   int max_ctx, max_docs, layer;
   bool pool_boxes;  // false: the pool is too small for a page box (all pages row by row)
   const PageSrcEntry *page_src;  // [batch][n_pidx]
-  int n_pidx;
+  const float2 *doc_cs;          // [batch][max_docs][D/2]: cos/sin of each document's delta
+  int n_pidx, half;
 };
 
 // Byte offset of the 16-byte piece ch (0 .. D/8-1) of row r (0..15) of a page
@@ -130,17 +133,33 @@ PIC_DEV uint32_t page_piece(int r, int ch) {
     return (uint32_t)(r * 128 + ((c8 ^ (r & 7)) << 4));
 }
 
-// The source of every page of positions < max_ctx of every request, from the
-// token map: a page whose first and last positions are rows of one document
-// is that document's (documents occupy contiguous positions), a page of
-// inline tokens only is the cache's, anything else is mixed.  One warp per
-// page; runs once per call, ahead of the attention (programmatic launch).
-__global__ void __launch_bounds__(256) page_src_kernel(FusedArgs f, int batch, int32_t *status) {
+// Set-up of a rotate-on-load call (one launch, ahead of the attention):
+// blocks [0, page_blocks) write the source of every page of positions
+// < max_ctx of every request, from the token map -- a page whose first and
+// last positions are rows of one document is that document's (documents
+// occupy contiguous positions), a page of inline tokens only is the cache's,
+// anything else is mixed -- one warp per page; blocks from page_blocks on
+// write cos/sin of delta_k * theta_i for every listed document k, as
+// pic_relocate forms them (fp64-reduced angle; the fast sine and cosine with
+// per-layer tables, as pic_relocate's per-layer instantiation).
+__global__ void __launch_bounds__(256) fused_setup_kernel(FusedArgs f, RopeParams rp, int batch,
+                                                          int page_blocks, int32_t *status) {
   pdl_entry();
+  const int b = blockIdx.y;
+  if (b >= batch) return;
+  if ((int)blockIdx.x >= page_blocks) {
+    const int k0 = ((int)blockIdx.x - page_blocks) * (256 / f.half);
+    const int k = k0 + (int)threadIdx.x / f.half, i = (int)threadIdx.x % f.half;
+    if (k >= f.max_docs || (int)threadIdx.x >= (256 / f.half) * f.half) return;
+    const int delta = f.doc_delta[(size_t)b * f.max_docs + k];
+    const double th = rope_theta(rp, f.layer, i);
+    const_cast<float2 *>(f.doc_cs)[((size_t)b * f.max_docs + k) * f.half + i] =
+        rp.layer_theta ? rope_cos_sin_fast(delta, th) : rope_cos_sin(delta, th);
+    return;
+  }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const long long pidx = (long long)blockIdx.x * 8 + warp;
-  const int b = blockIdx.y;
-  if (pidx >= f.n_pidx || b >= batch) return;
+  if (pidx >= f.n_pidx) return;
   const long long t = pidx * 16 + (lane & 15);
   const long long tm = t < f.max_ctx ? f.tok_map[(size_t)b * f.max_ctx + t] : -1;
   const unsigned inl = __ballot_sync(0xffffffffu, tm < 0) & 0xffffu;
@@ -155,7 +174,7 @@ __global__ void __launch_bounds__(256) page_src_kernel(FusedArgs f, int batch, i
     const long long row = first & ((1LL << 40) - 1);
     if (k < f.max_docs && row + 15 < f.pool_tokens) {
       e.kind = 1;
-      e.delta = f.doc_delta[(size_t)b * f.max_docs + k];
+      e.delta = k;  // the document index: its cos/sin are row k of doc_cs
       e.row = row;
     } else {
       dev_fail(status, PIC_DEV_BAD_DOC_LEN, b);
@@ -401,6 +420,7 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
         if (lane < 8 && pidx < f.n_pidx) {
           const PageSrcEntry e = ps[pidx];
           src.kind = e.kind;
+          src.delta = e.delta;
           if (e.kind == 1) src.y = (int)((long long)f.layer * f.pool_tokens + e.row);
         }
         return src;
@@ -445,6 +465,8 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
             sts128(stage + q * kPageBytes + page_piece<D>(r, ch), v);
           }
         }
+        if (is_k && lane < 8)  // for the rotators: this stage's page sources
+          reinterpret_cast<int2 *>(smem + L::kInfo)[st * 8 + lane] = make_int2(src.kind, src.delta);
         fence_proxy_async();
         __syncwarp();
         if (lane == 0) mbar_arrive(bar(b_full + st));
@@ -567,86 +589,102 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
     // tile's pages; its cos/sin are recomputed only when its rows' document
     // changes.
     if constexpr (kFused) {
-      constexpr int KC = D / 16;
-      const int rt = threadIdx.x - W_ROT * 32;
-      const int my_c = rt % KC;
+      // Warp w of the rotators takes pages 2w and 2w+1 of each tile; lane l
+      // the 8-pair chunk l % KC of rows l / KC + RG i of those pages, RPL
+      // rows per page at once.
+      constexpr int KC = D / 16, RG = 32 / KC, RPL = 16 / RG;
+      const int wr = warp - W_ROT;
+      const int my_c = lane % KC, my_rg = lane / KC;
       const PairChunk pc = pair_chunk(my_c, D / 2, rp.style);
       const int64_t *tmr = f.tok_map + (size_t)b * f.max_ctx;
-      const PageSrcEntry *ps = f.page_src + (size_t)b * f.n_pidx;
+      const int2 *info = reinterpret_cast<const int2 *>(smem + L::kInfo);
+      // cos/sin of this lane's 8 pairs for document k: 64 bytes of the
+      // set-up kernel's table (reloaded only when the document changes)
       float2 cs[8];
-      int cs_delta = 0;
-      bool cs_ok = false;
-      auto ensure_cs = [&](int delta) {
-        if (cs_ok && delta == cs_delta) return;
+      int cs_doc = -1;
+      auto ensure_cs = [&](int k) {
+        if (k == cs_doc) return;
+        const float4 *src = reinterpret_cast<const float4 *>(
+            f.doc_cs + ((size_t)b * f.max_docs + k) * (D / 2) + 8 * my_c);
 #pragma unroll
-        for (int q = 0; q < 8; ++q)
-          cs[q] = rp.layer_theta ? rope_cos_sin_fast(delta, rope_theta(rp, f.layer, 8 * my_c + q))
-                                 : rope_cos_sin(delta, rope_theta(rp, f.layer, 8 * my_c + q));
-        cs_delta = delta;
-        cs_ok = true;
+        for (int q = 0; q < 4; ++q) {
+          const float4 v = src[q];
+          cs[2 * q] = make_float2(v.x, v.y);
+          cs[2 * q + 1] = make_float2(v.z, v.w);
+        }
+        cs_doc = k;
+      };
+      auto rot = [&](uint4 &va, uint4 &vb) {
+        float x[8], y[8], uu[8], ww[8];
+        unpack8(va, x);
+        unpack8(vb, y);
+        if (rp.style == PIC_ROPE_HALF) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) { uu[e] = x[e]; ww[e] = y[e]; }
+        } else {
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            uu[e] = x[2 * e]; ww[e] = x[2 * e + 1];
+            uu[4 + e] = y[2 * e]; ww[4 + e] = y[2 * e + 1];
+          }
+        }
+        rotate8(uu, ww, cs);
+        if (rp.style == PIC_ROPE_HALF) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) { x[e] = uu[e]; y[e] = ww[e]; }
+        } else {
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            x[2 * e] = uu[e]; x[2 * e + 1] = ww[e];
+            y[2 * e] = uu[4 + e]; y[2 * e + 1] = ww[4 + e];
+          }
+        }
+        va = pack8(x);
+        vb = pack8(y);
       };
       for (int j = 0; j < n; ++j) {
         const int st = j % NSK, kt = kv_begin + j;
-        // this tile's page sources (L2), then its pages
-        int kind[KC], delta[KC];
-#pragma unroll
-        for (int u = 0; u < KC; ++u) {
-          const int i = rt + 128 * u, q = i / (16 * KC);
-          const int pidx = kt * 8 + q;
-          kind[u] = 0;
-          delta[u] = 0;
-          if (pidx < f.n_pidx) {
-            const PageSrcEntry e = ps[pidx];
-            kind[u] = e.kind;
-            delta[u] = e.delta;
-          }
-        }
         const bool ok = mbar_wait(bar(B_KFULL + st), (j / NSK) & 1, abort_flag, p.status, detail);
         if (!__all_sync(0xffffffffu, ok)) break;
         const uint32_t stage = sbase + L::kK + st * L::kTile;
-        // not unrolled: one copy of the (rare) cos/sin recomputation; the
-        // rotators have ample time per tile
 #pragma unroll 1
-        for (int u = 0; u < KC; ++u) {
-          if (kind[u] == 0) continue;
-          const int i = rt + 128 * u, q = i / (16 * KC), r = (i % (16 * KC)) / KC;
-          int dl = delta[u];
-          if (kind[u] == 2) {  // mixed page: this row's own document, if any
-            const long long t = (long long)kt * BN + q * 16 + r;
-            const long long tv = t < f.max_ctx ? tmr[t] : -1;
-            if (tv < 0 || (tv >> 40) >= f.max_docs) continue;
-            dl = f.doc_delta[(size_t)b * f.max_docs + (int)(tv >> 40)];
-          }
-          ensure_cs(dl);
-          const uint32_t a0 = stage + q * kPageBytes + page_piece<D>(r, pc.off_a / 8);
-          const uint32_t a1 = stage + q * kPageBytes + page_piece<D>(r, pc.off_b / 8);
-          uint4 va = lds128(a0), vb = lds128(a1);
-          float x[8], y[8], uu[8], ww[8];
-          unpack8(va, x);
-          unpack8(vb, y);
-          if (rp.style == PIC_ROPE_HALF) {
+        for (int h = 0; h < 2; ++h) {
+          const int q = 2 * wr + h;
+          const int2 pi = info[st * 8 + q];
+          if (pi.x == 0) continue;
+          const uint32_t pbase = stage + q * kPageBytes;
+          if (pi.x == 1) {  // one document: RPL rows at once
+            ensure_cs(pi.y);
+            uint4 va[RPL], vb[RPL];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) { uu[e] = x[e]; ww[e] = y[e]; }
-          } else {
+            for (int i = 0; i < RPL; ++i) {
+              const int r = my_rg + RG * i;
+              va[i] = lds128(pbase + page_piece<D>(r, pc.off_a / 8));
+              vb[i] = lds128(pbase + page_piece<D>(r, pc.off_b / 8));
+            }
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              uu[e] = x[2 * e]; ww[e] = x[2 * e + 1];
-              uu[4 + e] = y[2 * e]; ww[4 + e] = y[2 * e + 1];
+            for (int i = 0; i < RPL; ++i) {
+              const int r = my_rg + RG * i;
+              rot(va[i], vb[i]);
+              sts128(pbase + page_piece<D>(r, pc.off_a / 8), va[i]);
+              sts128(pbase + page_piece<D>(r, pc.off_b / 8), vb[i]);
+            }
+          } else {  // mixed page: each row's own document, inline rows as they are
+#pragma unroll 1
+            for (int i = 0; i < RPL; ++i) {
+              const int r = my_rg + RG * i;
+              const long long t = (long long)kt * BN + q * 16 + r;
+              const long long tv = t < f.max_ctx ? tmr[t] : -1;
+              if (tv < 0 || (tv >> 40) >= f.max_docs) continue;
+              ensure_cs((int)(tv >> 40));
+              const uint32_t a0 = pbase + page_piece<D>(r, pc.off_a / 8);
+              const uint32_t a1 = pbase + page_piece<D>(r, pc.off_b / 8);
+              uint4 va = lds128(a0), vb = lds128(a1);
+              rot(va, vb);
+              sts128(a0, va);
+              sts128(a1, vb);
             }
           }
-          rotate8(uu, ww, cs);
-          if (rp.style == PIC_ROPE_HALF) {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) { x[e] = uu[e]; y[e] = ww[e]; }
-          } else {
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              x[2 * e] = uu[e]; x[2 * e + 1] = ww[e];
-              y[2 * e] = uu[4 + e]; y[2 * e + 1] = ww[4 + e];
-            }
-          }
-          sts128(a0, pack8(x));
-          sts128(a1, pack8(y));
         }
         fence_proxy_async();
         __syncwarp();
@@ -1084,7 +1122,7 @@ __global__ void __launch_bounds__(256) append_kernel(AppendArgs a, RopeParams rp
 
 struct Plan {
   int G, m_tiles, R_pad, splits, n_pidx;
-  size_t q_bytes, po_bytes, pml_bytes, ps_bytes, total;
+  size_t q_bytes, po_bytes, pml_bytes, total;
 };
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -1118,11 +1156,18 @@ inline Plan plan(const pic_geom_t *g, int batch, int max_inline, int max_ctx, in
   } else {
     pl.po_bytes = pl.pml_bytes = 0;
   }
-  // rotate-on-load: the source of every page of positions < max_ctx
   pl.n_pidx = (max_ctx + 15) / 16;
-  pl.ps_bytes = align256((size_t)batch * pl.n_pidx * sizeof(PageSrcEntry));
-  pl.total = pl.q_bytes + pl.po_bytes + pl.pml_bytes + pl.ps_bytes;
+  pl.total = pl.q_bytes + pl.po_bytes + pl.pml_bytes;
   return pl;
+}
+
+// Rotate-on-load's extra workspace, after the plan's: the source of every
+// page of positions < max_ctx, then the cos/sin of every listed document.
+inline size_t fused_page_bytes(const Plan &pl, int batch) {
+  return align256((size_t)batch * pl.n_pidx * sizeof(PageSrcEntry));
+}
+inline size_t fused_cs_bytes(const pic_geom_t *g, int batch, int max_docs) {
+  return align256((size_t)batch * std::max(max_docs, 1) * (g->head_dim / 2) * sizeof(float2));
 }
 
 }  // namespace prefill
@@ -1152,6 +1197,17 @@ static cudaError_t launch_combine(long long rows, const Params &pp, cudaStream_t
 }
 }  // namespace prefill
 }  // namespace pic
+
+extern "C" size_t pic_prefill_fused_workspace_size(const pic_geom_t *geom, int32_t batch,
+                                                   int32_t max_inline, int32_t max_ctx,
+                                                   int32_t max_docs, int32_t num_splits) {
+  if (!geom || batch <= 0 || max_inline <= 0 || max_ctx <= 0 || max_docs < 0 ||
+      geom->num_kv_heads <= 0 || geom->num_q_heads % geom->num_kv_heads)
+    return 0;
+  const pic::prefill::Plan pl = pic::prefill::plan(geom, batch, max_inline, max_ctx, num_splits);
+  return pl.total + pic::prefill::fused_page_bytes(pl, batch) +
+         pic::prefill::fused_cs_bytes(geom, batch, max_docs);
+}
 
 extern "C" size_t pic_prefill_workspace_size(const pic_geom_t *geom, int32_t batch,
                                              int32_t max_inline, int32_t max_ctx,
@@ -1314,9 +1370,11 @@ static cudaError_t launch_attention(const Plan &pl, const Params &pp, const Fuse
     e = cudaFuncGetAttributes(&fa_attr, attn_kernel<D, kFused>);
     if (e != cudaSuccess) return e;
     if (fa_attr.numRegs < kRegLaunchFused) return cudaErrorInvalidConfiguration;
-    // page sources of the call, ahead of the attention
-    const dim3 pgrid((fa.n_pidx + 7) / 8, pp.batch);
-    e = launch_dependent(page_src_kernel, pgrid, dim3(256), 0, stream, fa, pp.batch, pp.status);
+    // page sources and document cos/sin of the call, ahead of the attention
+    const int page_blocks = (fa.n_pidx + 7) / 8;
+    const int doc_blocks = (fa.max_docs + 256 / fa.half - 1) / (256 / fa.half);
+    e = launch_dependent(fused_setup_kernel, dim3(page_blocks + doc_blocks, pp.batch), dim3(256), 0,
+                         stream, fa, rp, pp.batch, page_blocks, pp.status);
     if (e != cudaSuccess) return e;
   }
   dim3 grid(((pl.m_tiles + NQ - 1) / NQ) * pl.splits, pp.Hkv, pp.batch);
@@ -1428,6 +1486,12 @@ extern "C" pic_status_t pic_attend_prefill_fused(
   if (st != PIC_OK) return st;
   if (max_pages <= 0 || pool_tokens <= 0 || max_docs < 0)
     return fail(PIC_ERR_INVALID_ARG, "%s: sizes must be positive", who);
+  if (max_docs > 65535 * 256)
+    return fail(PIC_ERR_UNSUPPORTED, "%s: max_docs too large", who);
+  const size_t ws_need = pl.total + fused_page_bytes(pl, batch) + fused_cs_bytes(geom, batch, max_docs);
+  if (workspace_bytes < ws_need)
+    return fail(PIC_ERR_WORKSPACE, "%s: workspace needs %zu bytes (pic_prefill_fused_workspace_size)",
+                who, ws_need);
   if ((long long)geom->num_layers * pool_tokens >= (long long)INT32_MAX)
     return fail(PIC_ERR_UNSUPPORTED, "%s: pool has more than 2^31 rows", who);
   if (!inline_pos || !inline_len || !block_table || !k_cache || !v_cache || !k_pool || !v_pool ||
@@ -1510,8 +1574,10 @@ extern "C" pic_status_t pic_attend_prefill_fused(
   fa.max_docs = max_docs;
   fa.layer = layer;
   fa.pool_boxes = pool_boxes;
-  fa.page_src = reinterpret_cast<const PageSrcEntry *>(ws + pl.q_bytes + pl.po_bytes + pl.pml_bytes);
+  fa.page_src = reinterpret_cast<const PageSrcEntry *>(ws + pl.total);
+  fa.doc_cs = reinterpret_cast<const float2 *>(ws + pl.total + fused_page_bytes(pl, batch));
   fa.n_pidx = pl.n_pidx;
+  fa.half = D / 2;
   cudaError_t e = D == 128 ? launch_attention<128, true>(pl, pp, fa, rp, tq, tk, tv, tkp, tvp, stream)
                            : launch_attention<64, true>(pl, pp, fa, rp, tq, tk, tv, tkp, tvp, stream);
   if (e != cudaSuccess) return cuda_fail(e, "pic_attend_prefill_fused launch");

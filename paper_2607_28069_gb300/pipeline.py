@@ -10,7 +10,7 @@ import torch
 
 from . import (Geometry, pic_append_inline, pic_attend_decode, pic_attend_prefill,
                pic_attend_prefill_fused, pic_compose, pic_copy_async, pic_decode_workspace_size,
-               pic_link, pic_prefill_workspace_size, pic_relocate, pic_relocate_mapped)
+               pic_link, pic_prefill_fused_workspace_size, pic_relocate, pic_relocate_mapped)
 from .workloads import Workload
 
 
@@ -42,8 +42,11 @@ class CacheHitPath:
         self.k_cache = torch.zeros(shape, dtype=bf16, device=dev)
         self.v_cache = torch.zeros(shape, dtype=bf16, device=dev)
         u8 = torch.uint8
+        # one prefill workspace for the materialised and the rotate-on-load
+        # calls (the latter's is the larger)
         self.ws_prefill = torch.empty(
-            pic_prefill_workspace_size(self.geom, B, self.max_inline, self.max_ctx, prefill_splits),
+            pic_prefill_fused_workspace_size(self.geom, B, self.max_inline, self.max_ctx, md,
+                                             prefill_splits),
             dtype=u8, device=dev)
         self.out = torch.empty((L, B, self.max_inline, Hq, d), dtype=bf16, device=dev)
         self.lse = torch.empty((L, B, self.max_inline, Hq), dtype=torch.float32,

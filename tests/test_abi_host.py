@@ -48,10 +48,13 @@ def _geom(**kw):
 
 def test_workspace_sizes_are_host_arithmetic(lib):
     g = _geom()
-    # packed Q: B * Hkv * ceil(Tin*G/128)*128 rows of d bf16, then (for the
-    # rotate-on-load call) one 16-byte source entry per page of max_ctx
+    # packed Q: B * Hkv * ceil(Tin*G/128)*128 rows of d bf16
     ws1 = pic.pic_prefill_workspace_size(g, 1, 192, 4288, 1)
-    assert ws1 == 1 * 8 * 768 * 128 * 2 + ((1 * 268 * 16 + 255) // 256) * 256
+    assert ws1 == 1 * 8 * 768 * 128 * 2
+    # rotate-on-load adds a 16-byte source per page of max_ctx and d/2 cos/sin
+    # pairs per listed document
+    wf = pic.pic_prefill_fused_workspace_size(g, 1, 192, 4288, 8, 1)
+    assert wf == ws1 + ((268 * 16 + 255) // 256) * 256 + 8 * 64 * 8
     ws3 = pic.pic_prefill_workspace_size(g, 1, 192, 4288, 3)
     assert ws3 > ws1
     assert pic.pic_decode_workspace_size(g, 16, 33000, 1) == ((16 * 32 * 128 * 2 + 255) // 256) * 256
