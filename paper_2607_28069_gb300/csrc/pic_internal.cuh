@@ -154,6 +154,30 @@ PIC_DEV uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
   asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
   return r;
 }
+PIC_DEV uint64_t mul2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+// A bf16 pair (one 32-bit word, low element first) as a packed fp32 pair (exact).
+PIC_DEV uint64_t bf2_to_f2(uint32_t w) {
+  uint64_t r;
+  asm("{\n\t.reg .b32 lo, hi;\n\tshl.b32 lo, %1, 16;\n\tand.b32 hi, %1, 0xffff0000;\n\t"
+      "mov.b64 %0, {lo, hi};\n\t}" : "=l"(r) : "r"(w));
+  return r;
+}
+// A packed fp32 pair as a bf16 pair, each rounded to nearest even.
+PIC_DEV uint32_t f2_to_bf2(uint64_t v) {
+  uint32_t r;
+  asm("{\n\t.reg .f32 lo, hi;\n\tmov.b64 {lo, hi}, %1;\n\tcvt.rn.bf16x2.f32 %0, hi, lo;\n\t}"
+      : "=r"(r) : "l"(v));
+  return r;
+}
+// The two halves of a packed pair, each duplicated: (lo, lo) and (hi, hi).
+PIC_DEV void f2_split_dup(uint64_t v, uint64_t &lo2, uint64_t &hi2) {
+  asm("{\n\t.reg .b32 lo, hi;\n\tmov.b64 {lo, hi}, %2;\n\tmov.b64 %0, {lo, lo};\n\t"
+      "mov.b64 %1, {hi, hi};\n\t}" : "=l"(lo2), "=l"(hi2) : "l"(v));
+}
 PIC_DEV uint64_t add2(uint64_t a, uint64_t b) {
   uint64_t r;
   asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));

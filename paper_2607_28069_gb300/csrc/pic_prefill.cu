@@ -44,7 +44,7 @@ constexpr int kThreads = 128 + NQ * 128;  // K producer, MMA, NQ softmax warpgro
 // producer, relay) and the rotators give registers to the softmax warpgroups.
 constexpr int kThreadsFused = 512;
 constexpr int kRegLaunchFused = 65536 / kThreadsFused;  // 128 per thread at launch
-constexpr int kRegCtl = 64, kRegRot = 96, kRegSoftmax = 176;
+constexpr int kRegCtl = 72, kRegRot = 88, kRegSoftmax = 176;
 static_assert(128 * kRegCtl + 128 * kRegRot + 256 * kRegSoftmax <= 128 * 4 * kRegLaunchFused,
               "setmaxnreg split exceeds the registers the CTA is launched with");
 template <bool kFused>
@@ -598,49 +598,68 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
       const PairChunk pc = pair_chunk(my_c, D / 2, rp.style);
       const int64_t *tmr = f.tok_map + (size_t)b * f.max_ctx;
       const int2 *info = reinterpret_cast<const int2 *>(smem + L::kInfo);
-      // cos/sin of this lane's 8 pairs for document k: 64 bytes of the
-      // set-up kernel's table (reloaded only when the document changes)
-      float2 cs[8];
+      // cos/sin of this lane's 8 pairs for document k (64 bytes of the set-up
+      // kernel's table, reloaded only when the document changes), kept as the
+      // packed fp32 pairs the rotation multiplies by:
+      //   half-split:  A[j] = (c_2j, c_2j+1), A[4+j] = (s_2j, s_2j+1),
+      //                N[j] = (-s_2j, -s_2j+1)                      (j < 4)
+      //   interleaved: A[q] = (c_q, s_q), N[q] = (-s_q, c_q)        (q < 8)
+      uint64_t A[8], N[8];
       int cs_doc = -1;
+      const bool half_style = rp.style == PIC_ROPE_HALF;
       auto ensure_cs = [&](int k) {
         if (k == cs_doc) return;
         const float4 *src = reinterpret_cast<const float4 *>(
             f.doc_cs + ((size_t)b * f.max_docs + k) * (D / 2) + 8 * my_c);
+        float c[8], sn[8];
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
           const float4 v = src[q];
-          cs[2 * q] = make_float2(v.x, v.y);
-          cs[2 * q + 1] = make_float2(v.z, v.w);
+          c[2 * q] = v.x;
+          sn[2 * q] = v.y;
+          c[2 * q + 1] = v.z;
+          sn[2 * q + 1] = v.w;
+        }
+        if (half_style) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            A[j] = f2pack(c[2 * j], c[2 * j + 1]);
+            A[4 + j] = f2pack(sn[2 * j], sn[2 * j + 1]);
+            N[j] = f2pack(-sn[2 * j], -sn[2 * j + 1]);
+          }
+        } else {
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            A[q] = f2pack(c[q], sn[q]);
+            N[q] = f2pack(-sn[q], c[q]);
+          }
         }
         cs_doc = k;
       };
+      // Rotates the 8 pairs of one chunk in place, on packed fp32 pairs:
+      //   u' = fma(u, c, w * -s),  w' = fma(u, s, w * c)
+      // -- per element exactly the operations of the relocation kernel's
+      // scalar rotation, so the rounded keys are identical.
       auto rot = [&](uint4 &va, uint4 &vb) {
-        float x[8], y[8], uu[8], ww[8];
-        unpack8(va, x);
-        unpack8(vb, y);
-        if (rp.style == PIC_ROPE_HALF) {
+        uint32_t *wa = reinterpret_cast<uint32_t *>(&va), *wb = reinterpret_cast<uint32_t *>(&vb);
+        if (half_style) {  // va: u of pairs 0..7, vb: w of the same pairs
 #pragma unroll
-          for (int e = 0; e < 8; ++e) { uu[e] = x[e]; ww[e] = y[e]; }
-        } else {
+          for (int j = 0; j < 4; ++j) {
+            const uint64_t u2 = bf2_to_f2(wa[j]), w2 = bf2_to_f2(wb[j]);
+            const uint64_t nu = fma2(u2, A[j], mul2(w2, N[j]));
+            const uint64_t nw = fma2(u2, A[4 + j], mul2(w2, A[j]));
+            wa[j] = f2_to_bf2(nu);
+            wb[j] = f2_to_bf2(nw);
+          }
+        } else {  // each word one pair (u, w): pairs 0..3 in va, 4..7 in vb
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            uu[e] = x[2 * e]; ww[e] = x[2 * e + 1];
-            uu[4 + e] = y[2 * e]; ww[4 + e] = y[2 * e + 1];
+          for (int q = 0; q < 8; ++q) {
+            uint32_t &wq = q < 4 ? wa[q] : wb[q - 4];
+            uint64_t uu, ww;
+            f2_split_dup(bf2_to_f2(wq), uu, ww);
+            wq = f2_to_bf2(fma2(uu, A[q], mul2(ww, N[q])));
           }
         }
-        rotate8(uu, ww, cs);
-        if (rp.style == PIC_ROPE_HALF) {
-#pragma unroll
-          for (int e = 0; e < 8; ++e) { x[e] = uu[e]; y[e] = ww[e]; }
-        } else {
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            x[2 * e] = uu[e]; x[2 * e + 1] = ww[e];
-            y[2 * e] = uu[4 + e]; y[2 * e + 1] = ww[4 + e];
-          }
-        }
-        va = pack8(x);
-        vb = pack8(y);
       };
       for (int j = 0; j < n; ++j) {
         const int st = j % NSK, kt = kv_begin + j;
