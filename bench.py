@@ -53,6 +53,8 @@ def parse_args(argv=None):
                     help="also time the attention-deviation diagnostic on layer 0")
     ap.add_argument("--fused", action="store_true",
                     help="also time the rotate-on-load pass (default for stress_128k_b4)")
+    ap.add_argument("--floor", action="store_true",
+                    help="also time empty kernels with the pass's launch shapes (launch floor)")
     ap.add_argument("--oracle-sample", default=None, help=argparse.SUPPRESS)
     ap.add_argument("--oracle-seconds", type=float, default=10.0, help=argparse.SUPPRESS)
     ap.add_argument("--oracle-passes", type=int, default=0, help=argparse.SUPPRESS)
@@ -624,6 +626,47 @@ def main_gpu(args, rank, world):
             "frac_bf16": work["attend_flops"] / (fatt * 1e9) / peaks["bf16_tflops"],
             "query_tok_s": work["query_tokens"] / (fms / 1e3),
             "speedup_vs_materialised": ms_per_step / fms}
+
+    # launch floor of the pass: empty programmatic-dependent kernels with the
+    # pass's launch shapes (link, then per layer the attention and its merge,
+    # and for later layers the append first), timed like the pass
+    if args.floor:
+        B, Hkv, d = spec.batch, spec.kv_heads, spec.head_dim
+        G = spec.q_heads // Hkv
+        m_tiles = -(-path.max_inline * G // 128)
+        pairs = -(-m_tiles // 2)
+        tile = 128 * d * 2
+        attn_smem = 2 * tile + 3 * tile + 2 * tile + 256 + 3 * 8 * 8 + 1024
+        tok = 16 if Hkv * d >= 1024 else 32
+        shapes = [((-(-path.max_ctx // tok), B, 1), 256, 0)]
+        for layer in range(L):
+            if layer > 0:
+                shapes.append(((max(path.max_inline, -(-m_tiles * 128 // G)), B, 1), 256, 0))
+            shapes.append(((pairs * psplits, Hkv, B), 384, attn_smem))
+            if psplits > 1:
+                u = 2 if psplits <= 2 else (4 if psplits <= 4 else 8)
+                rows_m = B * Hkv * m_tiles * 128
+                shapes.append(((-(-rows_m // (8 * (8 // u))), 1, 1), 256, 0))
+        fe = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
+        gf = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gf):
+            fe[0].record()
+            pic.pic_launch_probe(shapes)
+            fe[1].record()
+        torch.cuda.synchronize()
+        fts = []
+        for k in range(W + max(3, K)):
+            flush.zero_()
+            torch.cuda._sleep(sleep_cycles)
+            gf.replay()
+            torch.cuda.synchronize()
+            if k >= W:
+                fts.append(fe[0].elapsed_time(fe[1]))
+        fl_ms = sum(fts) / len(fts)
+        rows["floor"] = {"ms": fl_ms, "launches": len(shapes), "frac_of_pass": fl_ms / ms_per_step,
+                         "note": "empty programmatic-dependent kernels with the pass's launch "
+                                 "shapes (grid, block, dynamic shared memory), one graph, "
+                                 "timed like the pass"}
 
     # attention-deviation diagnostic (off the serving path): D_r between the
     # relocated cache and the documents copied without re-rotation, layer 0

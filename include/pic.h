@@ -126,6 +126,19 @@ pic_status_t pic_device_status(pic_stream_t stream, int32_t *code, int32_t *deta
 pic_status_t pic_copy_async(void *dst, const void *src, size_t bytes, pic_stream_t stream);
 
 /*
+ * pic_launch_probe -- a measurement aid, not an operation of the paper: n
+ * empty kernels launched in order on `stream`, each a programmatic dependent
+ * of the one before (as every kernel of the path is), with grid
+ * grid[3i .. 3i+2], block[i] threads and smem[i] bytes of dynamic shared
+ * memory.  Timing a chain with the launch shapes of a pass gives the part of
+ * that pass no kernel work can remove: launch, dependency and CTA
+ * scheduling.  PIC_ERR_INVALID_ARG for sizes out of range (block > 1024,
+ * shared memory above the device's opt-in limit).
+ */
+pic_status_t pic_launch_probe(int32_t n, const int32_t *grid, const int32_t *block,
+                              const int32_t *smem, pic_stream_t stream);
+
+/*
  * pic_compose -- link operator R: logical layout of each request and its
  * token-level maps (Eqs. 1-2, "Background: Position-Independent Caching";
  * appendix "Logical Layout and Re-Rotation").

@@ -18,7 +18,7 @@ import torch
 __all__ = [
     "Geometry", "load", "lib_path", "pic_abi_version", "pic_compose", "pic_relocate",
     "pic_relocate_mapped", "pic_link",
-    "pic_attention_deviation", "pic_copy_async",
+    "pic_attention_deviation", "pic_copy_async", "pic_launch_probe",
     "pic_append_inline", "pic_attend_prefill", "pic_attend_prefill_fused",
     "pic_prefill_workspace_size", "pic_prefill_fused_workspace_size",
     "pic_prefill_num_splits", "pic_decode_num_splits", "pic_attend_decode_noalloc",
@@ -40,7 +40,7 @@ EXPORTED_SYMBOLS = (
     "pic_prefill_fused_workspace_size", "pic_prefill_num_splits",
     "pic_append_inline",
     "pic_attend_prefill", "pic_attend_prefill_fused", "pic_decode_workspace_size", "pic_decode_num_splits",
-    "pic_attend_decode", "pic_attend_decode_noalloc", "pic_copy_async",
+    "pic_attend_decode", "pic_attend_decode_noalloc", "pic_copy_async", "pic_launch_probe",
 )
 
 DEVICE_CODES = {
@@ -112,6 +112,7 @@ def load():
         "pic_last_error": (ctypes.c_char_p, []),
         "pic_device_status": (I32, [P, P, P]),
         "pic_copy_async": (I32, [P, P, SZ, P]),
+        "pic_launch_probe": (I32, [I32, P, P, P, P]),
         "pic_compose": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, P, I32, I64, I32, I32,
                               P, P, P, P, P, P, P]),
         "pic_relocate": (I32, [G, I32, I32, I32, P, P, I64, P, P, P, P, P, P, P, I32, I64, P, P,
@@ -214,6 +215,17 @@ def pic_copy_async(dst: torch.Tensor, src: torch.Tensor, stream=None):
     st = load().pic_copy_async(ctypes.c_void_p(dst.data_ptr()), ctypes.c_void_p(src.data_ptr()),
                                nbytes, _stream(stream))
     _check(st, "pic_copy_async")
+
+
+def pic_launch_probe(shapes, stream=None):
+    """Launch empty programmatic-dependent kernels with the given shapes, a
+    list of (grid (x, y, z), block threads, dynamic shared bytes)."""
+    n = len(shapes)
+    grid = (ctypes.c_int32 * (3 * n))(*[int(g) for s in shapes for g in s[0]])
+    block = (ctypes.c_int32 * n)(*[int(s[1]) for s in shapes])
+    smem = (ctypes.c_int32 * n)(*[int(s[2]) for s in shapes])
+    st = load().pic_launch_probe(n, grid, block, smem, _stream(stream))
+    _check(st, "pic_launch_probe")
 
 
 def pic_compose(geom: Geometry, doc_len, doc_base_pos, doc_token_start, req_doc_ids,

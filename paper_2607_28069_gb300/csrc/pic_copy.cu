@@ -7,6 +7,8 @@
 // page-locked host memory (cudaHostAlloc / cudaHostRegister, e.g. a pinned
 // torch tensor); the kernel addresses host memory through its device
 // pointer.
+#include <algorithm>
+
 #include "pic_internal.cuh"
 
 namespace pic {
@@ -39,8 +41,38 @@ __global__ void __launch_bounds__(kCopyThreads) copy_kernel(uint4 *__restrict__ 
   if (blockIdx.x == 0 && (int)threadIdx.x < tail) dst_tail[threadIdx.x] = src_tail[threadIdx.x];
 }
 
+// An empty programmatic dependent: waits for the kernel before, lets the
+// next one launch, and does nothing else (pic_launch_probe).
+__global__ void probe_kernel() { pdl_entry(); }
+
 }  // namespace
 }  // namespace pic
+
+extern "C" pic_status_t pic_launch_probe(int32_t n, const int32_t *grid, const int32_t *block,
+                                         const int32_t *smem, pic_stream_t stream) {
+  using namespace pic;
+  if (n <= 0 || !grid || !block || !smem)
+    return fail(PIC_ERR_INVALID_ARG, "pic_launch_probe: n > 0 and all arrays required");
+  int dev = 0, max_smem = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&max_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (e != cudaSuccess) return cuda_fail(e, "pic_launch_probe: device query");
+  int top = 0;
+  for (int i = 0; i < n; ++i) {
+    if (grid[3 * i] <= 0 || grid[3 * i + 1] <= 0 || grid[3 * i + 2] <= 0 || block[i] <= 0 ||
+        block[i] > 1024 || smem[i] < 0 || smem[i] > max_smem)
+      return fail(PIC_ERR_INVALID_ARG, "pic_launch_probe: launch %d out of range", i);
+    top = std::max(top, (int)smem[i]);
+  }
+  e = cudaFuncSetAttribute(probe_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, top);
+  if (e != cudaSuccess) return cuda_fail(e, "pic_launch_probe smem attribute");
+  for (int i = 0; i < n; ++i) {
+    e = launch_dependent(probe_kernel, dim3(grid[3 * i], grid[3 * i + 1], grid[3 * i + 2]),
+                         dim3(block[i]), (size_t)smem[i], stream);
+    if (e != cudaSuccess) return cuda_fail(e, "pic_launch_probe launch");
+  }
+  return PIC_OK;
+}
 
 extern "C" pic_status_t pic_copy_async(void *dst, const void *src, size_t bytes, pic_stream_t stream) {
   using namespace pic;

@@ -155,3 +155,12 @@ def test_copy_binding_refuses_pageable_and_mismatched_tensors():
         pic.pic_copy_async(a, torch.zeros(64, dtype=torch.uint8))
     with pytest.raises(ValueError):
         pic.pic_copy_async(a[::2], a[1::2])            # not contiguous
+
+
+def test_launch_probe_rejects_bad_shapes_before_any_launch(lib):
+    import ctypes as C
+    g = (C.c_int32 * 3)(1, 1, 1)
+    b = (C.c_int32 * 1)(32)
+    m = (C.c_int32 * 1)(0)
+    assert pic.load().pic_launch_probe(0, g, b, m, None) == 1      # n must be positive
+    assert pic.load().pic_launch_probe(1, None, b, m, None) == 1   # arrays required

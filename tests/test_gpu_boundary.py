@@ -182,3 +182,15 @@ def test_relocate_reports_overlapping_targets(cuda_lib):
                      bt[:, :max(1, -(-int(lens[0]) // 16))], pages, kc, vc, 0, spec.layers)
     code, _ = pic.pic_device_status()
     assert code == 5
+
+
+def test_launch_probe_runs_a_dependent_chain(cuda_lib):
+    """The measurement aid launches a chain of empty dependent kernels with
+    the attention's shape (384 threads, 230 KB of shared memory) and rejects
+    a block above 1024 threads."""
+    import paper_2607_28069_gb300 as pic
+    shapes = [((268, 1, 1), 256, 0), ((144, 1, 1), 384, 230912), ((768, 1, 1), 256, 0)]
+    pic.pic_launch_probe(shapes)
+    torch.cuda.synchronize()
+    with pytest.raises(pic.PicError):
+        pic.pic_launch_probe([((1, 1, 1), 2048, 0)])
