@@ -66,9 +66,11 @@ struct Layout {
   static constexpr int kK = kQ + NQ * kQTile;
   static constexpr int kV = kK + NSK * kTile;
   static constexpr int kBar = kV + NSV * kTile;
-  // rotate-on-load: per K stage the sources of its 8 pages ({kind, delta})
+  // rotate-on-load: per K stage the sources of its 8 pages ({kind, delta}),
+  // and for pages across a boundary each row's document (-1: inline)
   static constexpr int kInfo = kBar + 256;
-  static constexpr int kBytes = kInfo + NSK * 8 * 8;
+  static constexpr int kRowDoc = kInfo + NSK * 8 * 8;
+  static constexpr int kBytes = kRowDoc + NSK * 8 * 16 * 2;
   static constexpr int kAlloc = kBytes + 1024;  // slack for 1024-byte alignment
 };
 
@@ -452,20 +454,35 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
           const int q = __ffs(mixed) - 1;
           mixed &= mixed - 1;
           const int yq = __shfl_sync(0xffffffffu, src.y, q);
-          constexpr int CH = D / 8;
-          for (int e = lane; e < 16 * CH; e += 32) {
-            const int r = e / CH, ch = e % CH;
-            const long long t = (long long)kt * BN + q * 16 + r;
-            const long long tv = t < f.max_ctx ? tmr[t] : -1;
-            uint4 v = make_uint4(0, 0, 0, 0);
-            if (tv >= 0) {
-              const long long row = tv & ((1LL << 40) - 1);
-              if (row < f.pool_tokens)
-                v = ld_stream(pool + (((size_t)f.layer * f.pool_tokens + row) * p.Hkv + hk) * D + ch * 8);
-            } else if (yq != p.oob_row) {
-              v = ld_stream(cache + (size_t)(yq + r) * D + ch * 8);
+          // the page's 16 token-map entries (lane r < 16 holds row r's), then
+          // every 16-byte piece of the page loaded at once, then stored
+          const long long t_l = (long long)kt * BN + q * 16 + (lane & 15);
+          const long long tv_l = t_l < f.max_ctx ? tmr[t_l] : -1;
+          if (is_k && lane < 16)  // each row's document for the rotators (-1: inline)
+            reinterpret_cast<int16_t *>(smem + L::kRowDoc)[(st * 8 + q) * 16 + lane] =
+                (tv_l >= 0 && (tv_l >> 40) < f.max_docs) ? (int16_t)(tv_l >> 40) : (int16_t)-1;
+          constexpr int CH = D / 8, PER = 16 * CH / 32, GRP = 4;  // GRP loads in flight per lane
+#pragma unroll
+          for (int i0 = 0; i0 < PER; i0 += GRP) {
+            uint4 v[GRP];
+#pragma unroll
+            for (int i = 0; i < GRP; ++i) {
+              const int e = lane + 32 * (i0 + i), r = e / CH, ch = e % CH;
+              const long long tv = __shfl_sync(0xffffffffu, tv_l, r);
+              v[i] = make_uint4(0, 0, 0, 0);
+              if (tv >= 0) {
+                const long long row = tv & ((1LL << 40) - 1);
+                if (row < f.pool_tokens)
+                  v[i] = ld_stream(pool + (((size_t)f.layer * f.pool_tokens + row) * p.Hkv + hk) * D + ch * 8);
+              } else if (yq != p.oob_row) {
+                v[i] = ld_stream(cache + (size_t)(yq + r) * D + ch * 8);
+              }
             }
-            sts128(stage + q * kPageBytes + page_piece<D>(r, ch), v);
+#pragma unroll
+            for (int i = 0; i < GRP; ++i) {
+              const int e = lane + 32 * (i0 + i), r = e / CH, ch = e % CH;
+              sts128(stage + q * kPageBytes + page_piece<D>(r, ch), v[i]);
+            }
           }
         }
         if (is_k && lane < 8)  // for the rotators: this stage's page sources
@@ -692,13 +709,13 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
               sts128(pbase + page_piece<D>(r, pc.off_b / 8), vb[i]);
             }
           } else {  // mixed page: each row's own document, inline rows as they are
+            const int16_t *rd = reinterpret_cast<const int16_t *>(smem + L::kRowDoc) + (st * 8 + q) * 16;
 #pragma unroll 1
             for (int i = 0; i < RPL; ++i) {
               const int r = my_rg + RG * i;
-              const long long t = (long long)kt * BN + q * 16 + r;
-              const long long tv = t < f.max_ctx ? tmr[t] : -1;
-              if (tv < 0 || (tv >> 40) >= f.max_docs) continue;
-              ensure_cs((int)(tv >> 40));
+              const int kd = rd[r];
+              if (kd < 0) continue;
+              ensure_cs(kd);
               const uint32_t a0 = pbase + page_piece<D>(r, pc.off_a / 8);
               const uint32_t a1 = pbase + page_piece<D>(r, pc.off_b / 8);
               uint4 va = lds128(a0), vb = lds128(a1);
