@@ -616,7 +616,6 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
       const int wr = warp - W_ROT;
       const int my_c = lane % KC, my_rg = lane / KC;
       const PairChunk pc = pair_chunk(my_c, D / 2, rp.style);
-      const int64_t *tmr = f.tok_map + (size_t)b * f.max_ctx;
       const int2 *info = reinterpret_cast<const int2 *>(smem + L::kInfo);
       // cos/sin of this lane's 8 pairs for document k (64 bytes of the set-up
       // kernel's table, reloaded only when the document changes), kept as the
@@ -659,76 +658,84 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
       // Rotates the 8 pairs of one chunk in place, on packed fp32 pairs:
       //   u' = fma(u, c, w * -s),  w' = fma(u, s, w * c)
       // -- per element exactly the operations of the relocation kernel's
-      // scalar rotation, so the rounded keys are identical.
-      auto rot = [&](uint4 &va, uint4 &vb) {
-        uint32_t *wa = reinterpret_cast<uint32_t *>(&va), *wb = reinterpret_cast<uint32_t *>(&vb);
-        if (half_style) {  // va: u of pairs 0..7, vb: w of the same pairs
+      // scalar rotation, so the rounded keys are identical.  The tile loop
+      // below is instantiated once per RoPE style, so the warps execute only
+      // their style's code (the loop shares the SMSPs' instruction caches
+      // with the softmax).
+      auto rotate_tiles = [&](auto half_c) {
+        constexpr bool kHalf = decltype(half_c)::value;
+        auto rot = [&](uint4 &va, uint4 &vb) {
+          uint32_t *wa = reinterpret_cast<uint32_t *>(&va), *wb = reinterpret_cast<uint32_t *>(&vb);
+          if constexpr (kHalf) {  // va: u of pairs 0..7, vb: w of the same pairs
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const uint64_t u2 = bf2_to_f2(wa[j]), w2 = bf2_to_f2(wb[j]);
-            const uint64_t nu = fma2(u2, A[j], mul2(w2, N[j]));
-            const uint64_t nw = fma2(u2, A[4 + j], mul2(w2, A[j]));
-            wa[j] = f2_to_bf2(nu);
-            wb[j] = f2_to_bf2(nw);
-          }
-        } else {  // each word one pair (u, w): pairs 0..3 in va, 4..7 in vb
+            for (int j = 0; j < 4; ++j) {
+              const uint64_t u2 = bf2_to_f2(wa[j]), w2 = bf2_to_f2(wb[j]);
+              const uint64_t nu = fma2(u2, A[j], mul2(w2, N[j]));
+              const uint64_t nw = fma2(u2, A[4 + j], mul2(w2, A[j]));
+              wa[j] = f2_to_bf2(nu);
+              wb[j] = f2_to_bf2(nw);
+            }
+          } else {  // each word one pair (u, w): pairs 0..3 in va, 4..7 in vb
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            uint32_t &wq = q < 4 ? wa[q] : wb[q - 4];
-            uint64_t uu, ww;
-            f2_split_dup(bf2_to_f2(wq), uu, ww);
-            wq = f2_to_bf2(fma2(uu, A[q], mul2(ww, N[q])));
+            for (int q = 0; q < 8; ++q) {
+              uint32_t &wq = q < 4 ? wa[q] : wb[q - 4];
+              uint64_t uu, ww;
+              f2_split_dup(bf2_to_f2(wq), uu, ww);
+              wq = f2_to_bf2(fma2(uu, A[q], mul2(ww, N[q])));
+            }
           }
+        };
+        for (int j = 0; j < n; ++j) {
+          const int st = j % NSK, kt = kv_begin + j;
+          const bool ok = mbar_wait(bar(B_KFULL + st), (j / NSK) & 1, abort_flag, p.status, detail);
+          if (!__all_sync(0xffffffffu, ok)) break;
+          const uint32_t stage = sbase + L::kK + st * L::kTile;
+#pragma unroll 1
+          for (int h = 0; h < 2; ++h) {
+            const int q = 2 * wr + h;
+            const int2 pi = info[st * 8 + q];
+            if (pi.x == 0) continue;
+            const uint32_t pbase = stage + q * kPageBytes;
+            if (pi.x == 1) {  // one document: RPL rows at once
+              ensure_cs(pi.y);
+              uint4 va[RPL], vb[RPL];
+#pragma unroll
+              for (int i = 0; i < RPL; ++i) {
+                const int r = my_rg + RG * i;
+                va[i] = lds128(pbase + page_piece<D>(r, pc.off_a / 8));
+                vb[i] = lds128(pbase + page_piece<D>(r, pc.off_b / 8));
+              }
+#pragma unroll
+              for (int i = 0; i < RPL; ++i) {
+                const int r = my_rg + RG * i;
+                rot(va[i], vb[i]);
+                sts128(pbase + page_piece<D>(r, pc.off_a / 8), va[i]);
+                sts128(pbase + page_piece<D>(r, pc.off_b / 8), vb[i]);
+              }
+            } else {  // mixed page: each row's own document, inline rows as they are
+              const int16_t *rd = reinterpret_cast<const int16_t *>(smem + L::kRowDoc) + (st * 8 + q) * 16;
+#pragma unroll 1
+              for (int i = 0; i < RPL; ++i) {
+                const int r = my_rg + RG * i;
+                const int kd = rd[r];
+                if (kd < 0) continue;
+                ensure_cs(kd);
+                const uint32_t a0 = pbase + page_piece<D>(r, pc.off_a / 8);
+                const uint32_t a1 = pbase + page_piece<D>(r, pc.off_b / 8);
+                uint4 va = lds128(a0), vb = lds128(a1);
+                rot(va, vb);
+                sts128(a0, va);
+                sts128(a1, vb);
+              }
+            }
+          }
+          fence_proxy_async();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar(B_KROT + st));
         }
       };
-      for (int j = 0; j < n; ++j) {
-        const int st = j % NSK, kt = kv_begin + j;
-        const bool ok = mbar_wait(bar(B_KFULL + st), (j / NSK) & 1, abort_flag, p.status, detail);
-        if (!__all_sync(0xffffffffu, ok)) break;
-        const uint32_t stage = sbase + L::kK + st * L::kTile;
-#pragma unroll 1
-        for (int h = 0; h < 2; ++h) {
-          const int q = 2 * wr + h;
-          const int2 pi = info[st * 8 + q];
-          if (pi.x == 0) continue;
-          const uint32_t pbase = stage + q * kPageBytes;
-          if (pi.x == 1) {  // one document: RPL rows at once
-            ensure_cs(pi.y);
-            uint4 va[RPL], vb[RPL];
-#pragma unroll
-            for (int i = 0; i < RPL; ++i) {
-              const int r = my_rg + RG * i;
-              va[i] = lds128(pbase + page_piece<D>(r, pc.off_a / 8));
-              vb[i] = lds128(pbase + page_piece<D>(r, pc.off_b / 8));
-            }
-#pragma unroll
-            for (int i = 0; i < RPL; ++i) {
-              const int r = my_rg + RG * i;
-              rot(va[i], vb[i]);
-              sts128(pbase + page_piece<D>(r, pc.off_a / 8), va[i]);
-              sts128(pbase + page_piece<D>(r, pc.off_b / 8), vb[i]);
-            }
-          } else {  // mixed page: each row's own document, inline rows as they are
-            const int16_t *rd = reinterpret_cast<const int16_t *>(smem + L::kRowDoc) + (st * 8 + q) * 16;
-#pragma unroll 1
-            for (int i = 0; i < RPL; ++i) {
-              const int r = my_rg + RG * i;
-              const int kd = rd[r];
-              if (kd < 0) continue;
-              ensure_cs(kd);
-              const uint32_t a0 = pbase + page_piece<D>(r, pc.off_a / 8);
-              const uint32_t a1 = pbase + page_piece<D>(r, pc.off_b / 8);
-              uint4 va = lds128(a0), vb = lds128(a1);
-              rot(va, vb);
-              sts128(a0, va);
-              sts128(a1, vb);
-            }
-          }
-        }
-        fence_proxy_async();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar(B_KROT + st));
-      }
+      if (half_style) rotate_tiles(std::true_type{});
+      else rotate_tiles(std::false_type{});
     }
   };
   auto role_softmax = [&]() {
