@@ -249,17 +249,17 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
   constexpr int W_RELAY = kFused ? 3 : kWarpRelay;
   constexpr int W_SM = kFused ? 4 : 2;  // first softmax warp
   constexpr int W_ROT = 12;             // first rotator warp (rotate-on-load)
-  // Grid (pair + npairs * split, kv head, request), pairs in reverse order.
-  // CTAs start in linear block order: the query pairs that read one key
-  // split of one (request, kv head) are adjacent, so they start in the same
-  // wave and read each K/V tile within a short window (from DRAM once, then
-  // from L2); a split-minor order let waves cut through those sets and the
-  // late readers of a range found it evicted (1.48x the algorithmic K/V
-  // read on the 4 x 139k workload, 1.05x in this order).  Within a set the
-  // pairs of the last query rows, which see the most keys, go first.
+  // Grid (pair + npairs * split, kv head, request).  CTAs start in linear
+  // block order: the query pairs that read one key split of one (request,
+  // kv head) are adjacent, so they start in the same wave and read each K/V
+  // tile within a short window (from DRAM once, then from L2); a split-minor
+  // order let waves cut through those sets and the late readers of a range
+  // found it evicted (1.48x the algorithmic K/V read on the 4 x 139k
+  // workload, 1.05x in this order).  Query tiles are counted from a
+  // request's last row, so pair 0, which sees the most keys, goes first.
   const int npairs = (int)gridDim.x / p.num_splits;
   const int split = (int)blockIdx.x / npairs;
-  const int pair = npairs - 1 - (int)blockIdx.x % npairs;
+  const int pair = (int)blockIdx.x % npairs;
   const int hk = blockIdx.y, b = blockIdx.z;
   const int detail = b;
 
@@ -301,14 +301,22 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
   const int tin = min(max(p.inline_len[b], 0), p.max_inline);
   const int rows = tin * p.G;
   const int32_t *ipos = p.inline_pos + (size_t)b * p.max_inline;
+  // Query tile mt of a request holds its packed rows [rows - 128 (mt + 1),
+  // rows - 128 mt): the tiles are aligned to the request's last row, so a
+  // query chunk whose rows are a multiple of 128 fills whole tiles and never
+  // shares one with the prefix rows, which see only the prefix keys.  The
+  // lowest tile may start below row 0 (those rows are padding: loaded from
+  // outside the request, fully masked, never written).  Tile t of the pair is
+  // mt = NQ pair + t, so tile 0 has the most keys and tile 1 at most as many.
   int r0[NQ], kmin[NQ], kmax[NQ], ntile = 0;
 #pragma unroll
   for (int t = 0; t < NQ; ++t) {
-    r0[t] = (pair * NQ + t) * BM;
+    const int mt = pair * NQ + t;
+    r0[t] = rows - (mt + 1) * BM;
     kmin[t] = kmax[t] = -1;
-    if (r0[t] < rows && t < p.m_tiles - pair * NQ) {
-      kmin[t] = ipos[r0[t] / p.G];
-      kmax[t] = ipos[(min(r0[t] + BM, rows) - 1) / p.G];
+    if (mt < p.m_tiles && r0[t] + BM > 0) {
+      kmin[t] = ipos[max(r0[t], 0) / p.G];
+      kmax[t] = ipos[(r0[t] + BM - 1) / p.G];
       ntile = t + 1;
     }
   }
@@ -316,7 +324,7 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
     release_and_exit();
     return;
   }
-  const int kmax_all = ntile == 2 ? kmax[1] : kmax[0];
+  const int kmax_all = kmax[0];
   const int n_kv_all = kmax_all >= 0 ? kmax_all / BN + 1 : 0;
   const int per = (n_kv_all + p.num_splits - 1) / p.num_splits;
   const int kv_begin = split * per;
@@ -544,7 +552,8 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
 #pragma unroll
             for (int kk = 0; kk < BN / 16; ++kk)  // one page of 16 keys per MMA
               mma_ts(tO, tS + kk * 8, dv + (kk * kPageBytes) / 16, IDESC_PV, (pj > 0 || kk > 0));
-            if (t == ntile - 1) mma_commit(bar(B_VEMPTY + pst));  // last reader of V(j-1)
+            // the last tile that reads V(j-1) releases it (tile 1 reads a prefix of tile 0's range)
+            if (t == ntile - 1 || pj >= nt[1]) mma_commit(bar(B_VEMPTY + pst));
           }
         }
         // S_t = Q_t K(j)^T
@@ -563,7 +572,7 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
               mma_ss(tS, dq + ((kk >> 2) * (BM * 128) + (kk & 3) * 32) / 16,
                      dk + ((kk >> 2) * kPanelOff + (kk & 3) * 32) / 16, IDESC_QK, kk > 0);
             mma_commit(bar(B_SFULL + t));
-            if (t == ntile - 1) mma_commit(bar(B_KEMPTY + st));  // last reader of K(j)
+            if (t == ntile - 1 || j >= nt[1]) mma_commit(bar(B_KEMPTY + st));  // last reader of K(j)
           }
         }
       }
@@ -750,8 +759,8 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
     const int my_n = t < ntile ? (t == 0 ? nt[0] : nt[1]) : 0;
     const size_t my_part0 = part_row0(t);
     const int rg = my_r0 + row;
-    const bool valid = t < ntile && rg < rows;
-    const int tok = rg / p.G, g = rg % p.G;
+    const bool valid = t < ntile && rg >= 0 && rg < rows;
+    const int tok = valid ? rg / p.G : 0, g = valid ? rg % p.G : 0;
     const int pos = valid ? ipos[tok] : -1;
     const uint32_t tl = tbase + ((uint32_t)(wq * 32) << 16);
     const uint32_t tS = tl + t * 128, tO = tl + 256 + t * 128;
@@ -870,11 +879,12 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
       }
       asm volatile("bar.sync %0, 128;" ::"r"(1 + t) : "memory");
       if (ok) {
-        const int nrows = min(BM, rows - my_r0);  // valid rows of this tile
+        const int rlo = max(0, -my_r0);  // the tile's rows from rlo on exist
         if (single) {
           // 16 lanes per 256-byte row (D = 128) or 8 per 128-byte row (D = 64)
           constexpr int LPR = D / 8, RPI = 32 / LPR;
-          for (int r = wq * RPI + lane / LPR; r < nrows; r += 4 * RPI) {
+          for (int r = wq * RPI + lane / LPR; r < BM; r += 4 * RPI) {
+            if (r < rlo) continue;
             const int rg2 = my_r0 + r, tk = rg2 / p.G, gg = rg2 % p.G;
             const uint4 v = *reinterpret_cast<const uint4 *>(stage + r * kRowOut + (lane % LPR) * 16);
             st_global16(p.out + (((size_t)b * p.max_inline + tk) * p.Hq + hk * p.G + gg) * D +
@@ -884,9 +894,10 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
           // fp32 rows are contiguous in the partial buffer: one row per warp pass
           constexpr int LPR = D / 4;  // 16-byte pieces per row
           constexpr int RPI = 32 / LPR > 0 ? 32 / LPR : 1;
-          for (int r = wq * RPI + lane / LPR; r < nrows; r += 4 * RPI)
+          for (int r = wq * RPI + lane / LPR; r < BM; r += 4 * RPI)
 #pragma unroll
             for (int c = lane % LPR; c < D / 4; c += (LPR < 32 ? LPR : 32)) {
+              if (r < rlo) continue;
               const float4 v = *reinterpret_cast<const float4 *>(stage + r * kRowPart + c * 16);
               reinterpret_cast<float4 *>(p.part_o + (my_part0 + r) * D)[c] = v;
             }
@@ -958,8 +969,10 @@ __global__ void __launch_bounds__(256) combine_kernel(Params p) {
   const int hk = (int)(rem / ((long long)p.m_tiles * BM));
   const int mt = (int)((rem / BM) % p.m_tiles), row0 = (int)(rem % BM);
   const int tin = min(max(p.inline_len[b], 0), p.max_inline);
-  const int valid_rows = tin * p.G - (mt * BM + row0);  // rows of this warp that exist
-  if (valid_rows <= 0) return;
+  // the warp's rows are rg0 .. rg0 + R - 1 of the request (tiles counted
+  // from its last row); those below row 0 are padding
+  const int rg0 = tin * p.G - (mt + 1) * BM + row0;
+  if (rg0 + R <= 0) return;
   const int S = p.num_splits;
   const size_t base = (((size_t)b * p.Hkv + hk) * p.m_tiles + mt) * S;
   float ms[R], ls[R];
@@ -1019,8 +1032,8 @@ __global__ void __launch_bounds__(256) combine_kernel(Params p) {
   }
 #pragma unroll
   for (int r = 0; r < R; ++r) {
-    if (r >= valid_rows) break;
-    const int rg = mt * BM + row0 + r;
+    const int rg = rg0 + r;
+    if (rg < 0) continue;
     const float inv = Lsum[r] > 0.f ? 1.f / Lsum[r] : 0.f;
     const int tok = rg / p.G, g = rg % p.G;
     __nv_bfloat16 *dst =
