@@ -44,7 +44,7 @@ constexpr int kThreads = 128 + NQ * 128;  // K producer, MMA, NQ softmax warpgro
 // producer, relay) and the rotators give registers to the softmax warpgroups.
 constexpr int kThreadsFused = 512;
 constexpr int kRegLaunchFused = 65536 / kThreadsFused;  // 128 per thread at launch
-constexpr int kRegCtl = 72, kRegRot = 88, kRegSoftmax = 176;
+constexpr int kRegCtl = 88, kRegRot = 88, kRegSoftmax = 168;
 static_assert(128 * kRegCtl + 128 * kRegRot + 256 * kRegSoftmax <= 128 * 4 * kRegLaunchFused,
               "setmaxnreg split exceeds the registers the CTA is launched with");
 template <bool kFused>
@@ -209,17 +209,23 @@ struct PageSrc {
 // cache alone.  A page whose 16 positions are all one document's comes from
 // the pool as one box (the document's rows are consecutive there); a page of
 // inline tokens from the cache as before; a page across a boundary is filled
-// row by row by the producer warp.  The K producer warp then rotates every
+// row by row by the producer warp.  A rotator warpgroup then rotates every
 // document row of the tile in shared memory by its document's delta -- the
 // same fp32 arithmetic and bf16 rounding as the relocation, so the tile holds
 // exactly the keys pic_relocate would have stitched -- and signals K(j) on
 // B_KROT instead of the TMA barrier.  Everything downstream (MMAs, softmax,
 // merge) is the materialised kernel's.
-template <int D, bool kFused>
-__global__ void __launch_bounds__(threads_of<kFused>(), 1)
-    attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_kp,
-                const __grid_constant__ CUtensorMap tm_vp, Params p, FusedArgs f, RopeParams rp) {
+//
+// The body is one function per group of warps (kGroup: 0 the control
+// warpgroup, 1 the rotators, 2 the softmax warpgroups; -1 all warps of the
+// materialised kernel), entered right after the group's setmaxnreg, so no
+// value is live across the register reallocation (values live across it
+// were spilled and reloaded in the control warps' loops).
+template <int D, bool kFused, int kGroup>
+__device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtensorMap &tm_k,
+                                          const CUtensorMap &tm_v, const CUtensorMap &tm_kp,
+                                          const CUtensorMap &tm_vp, Params p, FusedArgs f,
+                                          RopeParams rp) {
   using L = Layout<D>;
   constexpr int PANELS = D / 64;
   constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
@@ -906,19 +912,13 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
     }
   };
   if constexpr (kFused) {
-    // Registers move from the control and rotator warpgroups to the softmax
-    // ones: each warpgroup runs one setmaxnreg at one place, and its roles'
-    // code follows it.
-    if (warp < 4) {
-      asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegCtl));
+    if constexpr (kGroup == 0) {
       if (warp == 0 || warp == W_V) role_producer();
       else if (warp == 1) role_issuer();
       else role_relay();
-    } else if (warp >= W_ROT) {
-      asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegRot));
+    } else if constexpr (kGroup == 1) {
       role_rotator();
     } else {
-      asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegSoftmax));
       role_softmax();
     }
   } else {
@@ -941,6 +941,31 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
     }
     __syncwarp();
     tmem_dealloc(tbase, kTmemCols);
+  }
+}
+
+template <int D, bool kFused>
+__global__ void __launch_bounds__(threads_of<kFused>(), 1)
+    attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_kp,
+                const __grid_constant__ CUtensorMap tm_vp, Params p, FusedArgs f, RopeParams rp) {
+  if constexpr (kFused) {
+    // Registers move from the control and rotator warpgroups to the softmax
+    // ones: each warpgroup runs one setmaxnreg, first thing, and then its
+    // own copy of the body.
+    const int wg = threadIdx.x >> 7;
+    if (wg == 0) {
+      asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegCtl));
+      attn_body<D, true, 0>(tm_q, tm_k, tm_v, tm_kp, tm_vp, p, f, rp);
+    } else if (wg == 3) {
+      asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegRot));
+      attn_body<D, true, 1>(tm_q, tm_k, tm_v, tm_kp, tm_vp, p, f, rp);
+    } else {
+      asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegSoftmax));
+      attn_body<D, true, 2>(tm_q, tm_k, tm_v, tm_kp, tm_vp, p, f, rp);
+    }
+  } else {
+    attn_body<D, false, -1>(tm_q, tm_k, tm_v, tm_kp, tm_vp, p, f, rp);
   }
 }
 
