@@ -55,6 +55,7 @@ constexpr int kWarpRelay = kWarpV + 1;    // waits on behalf of the MMA issuer
 // 0 is __syncthreads, 1 and 2 belong to the softmax warpgroups' epilogue.
 constexpr int kNbPv = 3;  // + t: P_t(j-1) and V(j-1) are ready
 constexpr int kNbK = 5;   // K(j) is ready
+constexpr int kNbRot = 6; // rotate-on-load: the rotator warps have rotated their pages
 constexpr int kMaxSplits = 32;
 constexpr uint32_t kTmemCols = 512;
 
@@ -84,8 +85,10 @@ enum {
   B_SFULL = B_VEMPTY + NSV,  // one per query tile
   B_PFULL = B_SFULL + NQ,     // one per query tile (one arrival per softmax warp)
   B_OFINAL = B_PFULL + NQ,
-  B_KROT = B_OFINAL + 1,  // rotate-on-load: K(j) rotated in place (one arrival)
-  B_COUNT = B_KROT + NSK
+  B_KROT = B_OFINAL + 1,  // rotate-on-load: this CTA's half of K(j) rotated (one arrival per rotator warp)
+  B_KPEER = B_KROT + NSK,  // rotate-on-load: the cluster peer's rotated half of K(j) has landed
+  B_EXIT = B_KPEER + NSK,  // rotate-on-load: the peer is done with this CTA's shared memory
+  B_COUNT = B_EXIT + 1
 };
 
 struct Params {
@@ -274,7 +277,9 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
   if (threadIdx.x == 0) {
     for (int i = 0; i < B_COUNT; ++i)
       mbar_init(bar(i), ((i >= B_PFULL && i < B_PFULL + NQ) || (i >= B_KROT && i < B_KROT + NSK))
-                            ? 4 : 1);
+                            ? 4
+                        : (kFused && i >= B_KEMPTY && i < B_KEMPTY + NSK) ? 2  // both CTAs' QK
+                                                                          : 1);
     *abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tm_q);
@@ -292,6 +297,12 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // rotate-on-load runs in clusters of two CTAs (consecutive query pairs of
+  // one key split): each loads and rotates half of every key tile and copies
+  // it into the other's ring, so the barriers must be initialised in both
+  // before either touches the other's
+  const uint32_t crank = kFused ? cluster_rank() : 0u, cpeer = crank ^ 1u;
+  if constexpr (kFused) cluster_sync_all();
   const uint32_t tbase = *tmem_slot;
   asm volatile("griddepcontrol.wait;" ::: "memory");  // the kernel before has finished
   auto release_and_exit = [&]() {  // a CTA without work frees its TMEM
@@ -326,11 +337,21 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
       ntile = t + 1;
     }
   }
-  if (ntile == 0) {  // no query row in this pair
+  int kmax_all = kmax[0];
+  if constexpr (kFused) {
+    // Both CTAs of a cluster stream the key tiles of its upper pair, whose
+    // first tile sees the most keys; the lower pair may have no rows and then
+    // only loads, rotates and passes on its half of every key tile.
+    const int mt_top = (pair & ~1) * NQ, r_top = rows - (mt_top + 1) * BM;
+    kmax_all = (mt_top < p.m_tiles && r_top + BM > 0) ? ipos[(r_top + BM - 1) / p.G] : -1;
+    if (kmax_all < 0) {  // neither pair of the cluster has a query row
+      release_and_exit();
+      return;
+    }
+  } else if (ntile == 0) {  // no query row in this pair
     release_and_exit();
     return;
   }
-  const int kmax_all = kmax[0];
   const int n_kv_all = kmax_all >= 0 ? kmax_all / BN + 1 : 0;
   const int per = (n_kv_all + p.num_splits - 1) / p.num_splits;
   const int kv_begin = split * per;
@@ -444,13 +465,20 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
         }
         return src;
       };
+      // The K producer fills its CTA's half of every key tile (pages
+      // 4 crank .. 4 crank + 3; the cluster peer sends the rotated other
+      // half), the V producer whole tiles.
+      const bool mine = lane < 8 && (!is_k || (uint32_t)(lane >> 2) == crank);
       auto issue = [&](int st, int kt, const PageSrc &src) {
         const uint32_t stage = ring + st * L::kTile;
-        const unsigned box_mask = __ballot_sync(0xffffffffu, lane < 8 && src.kind != 2);
-        unsigned mixed = __ballot_sync(0xffffffffu, lane < 8 && src.kind == 2);
-        if (lane == 0) mbar_expect_tx_only(bar(b_full + st), __popc(box_mask) * kPageBytes);
+        const unsigned box_mask = __ballot_sync(0xffffffffu, mine && src.kind != 2);
+        unsigned mixed = __ballot_sync(0xffffffffu, mine && src.kind == 2);
+        if (lane == 0) {
+          mbar_expect_tx_only(bar(b_full + st), __popc(box_mask) * kPageBytes);
+          if (is_k) mbar_expect_tx(bar(B_KPEER + st), 4 * kPageBytes);
+        }
         __syncwarp();
-        if (lane < 8 && src.kind != 2) {
+        if (mine && src.kind != 2) {
           const uint32_t dst = stage + lane * kPageBytes;
           if (src.kind == 0) {
             if constexpr (PANELS == 2)
@@ -505,12 +533,15 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
         __syncwarp();
         if (lane == 0) mbar_arrive(bar(b_full + st));
       };
+      // every key tile of the cluster's range; the value tiles this CTA's
+      // first query tile needs
+      const int n_mine = is_k ? n : nt[0];
       PageSrc s_next = source(kv_begin);
       int issued = 0;
-      for (int j = 0; j < n; ++j) {
+      for (int j = 0; j < n_mine; ++j) {
         const int st = j % nst;
         const PageSrc s_cur = s_next;
-        if (j + 1 < n) s_next = source(kv_begin + j + 1);
+        if (j + 1 < n_mine) s_next = source(kv_begin + j + 1);
         if (j >= nst) {
           const bool ok = mbar_wait(bar(b_empty + st), ((j / nst) - 1) & 1, abort_flag, p.status, detail);
           if (!__all_sync(0xffffffffu, ok)) break;
@@ -534,6 +565,12 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
     if (leader) mbar_wait(bar(B_Q), 0, abort_flag, p.status, detail);
     __syncwarp();
     tc_fence_after();
+    // K(j)'s ring slot is free once every QK reading it has completed -- in
+    // rotate-on-load, in both CTAs of the cluster (the peer writes half of it)
+    auto release_k = [&](int st) {
+      if constexpr (kFused) mma_commit_mc(bar(B_KEMPTY + st), 0x3);
+      else mma_commit(bar(B_KEMPTY + st));
+    };
     // Matrix descriptors: one base per operand region.  A ring stage, a query
     // tile or a k-step only moves the start address, which sits in the low 14
     // bits as address >> 4; shared addresses stay below 256 KB, so adding
@@ -578,9 +615,22 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
               mma_ss(tS, dq + ((kk >> 2) * (BM * 128) + (kk & 3) * 32) / 16,
                      dk + ((kk >> 2) * kPanelOff + (kk & 3) * 32) / 16, IDESC_QK, kk > 0);
             mma_commit(bar(B_SFULL + t));
-            if (t == ntile - 1 || j >= nt[1]) mma_commit(bar(B_KEMPTY + st));  // last reader of K(j)
+            if (t == ntile - 1 || j >= nt[1]) release_k(st);  // last reader of K(j)
           }
         }
+      }
+      if (kFused && j < n && !k_ready) {
+        // A key tile only the cluster peer uses: released once both halves
+        // are in this CTA's ring (its rotators are done with it, the peer's
+        // copy has landed).  The issuer waits itself rather than through the
+        // relay, whose arrivals here would depend on nothing the issuer
+        // does and could run a phase ahead of its syncs.
+        if (leader) {
+          mbar_wait(bar(B_KROT + j % NSK), (j / NSK) & 1, abort_flag, p.status, detail);
+          mbar_wait(bar(B_KPEER + j % NSK), (j / NSK) & 1, abort_flag, p.status, detail);
+          release_k(j % NSK);
+        }
+        __syncwarp();
       }
     }
     if (leader) mma_commit(bar(B_OFINAL));
@@ -591,6 +641,15 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
     // arrival on a barrier in iteration j + 1 depends on an MMA the issuer
     // issues only after its sync on that barrier in iteration j, so the two
     // never get a phase apart.
+    auto wait_k = [&](int j) {  // K(j) complete in this CTA's ring
+      const uint32_t par = (j / NSK) & 1;
+      if constexpr (kFused) {
+        mbar_wait(bar(B_KROT + j % NSK), par, abort_flag, p.status, detail);
+        mbar_wait(bar(B_KPEER + j % NSK), par, abort_flag, p.status, detail);
+      } else {
+        mbar_wait(bar(B_KFULL + j % NSK), par, abort_flag, p.status, detail);
+      }
+    };
     for (int j = 0; j <= n; ++j) {
       bool k_ready = false, v_ready = false;
 #pragma unroll
@@ -606,8 +665,7 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
           named_bar_arrive(kNbPv + t, 64);
         }
         if (j < nt[t] && !k_ready) {
-          mbar_wait(bar((kFused ? B_KROT : B_KFULL) + j % NSK), (j / NSK) & 1, abort_flag, p.status,
-                    detail);
+          wait_k(j);
           named_bar_arrive(kNbK, 64);
           k_ready = true;
         }
@@ -624,9 +682,9 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
     // tile's pages; its cos/sin are recomputed only when its rows' document
     // changes.
     if constexpr (kFused) {
-      // Warp w of the rotators takes pages 2w and 2w+1 of each tile; lane l
-      // the 8-pair chunk l % KC of rows l / KC + RG i of those pages, RPL
-      // rows per page at once.
+      // Warp w of the rotators takes page 4 crank + w of each tile (the CTA's
+      // half; the cluster peer rotates the other); lane l the 8-pair chunk
+      // l % KC of rows l / KC + RG i of the page, RPL rows at once.
       constexpr int KC = D / 16, RG = 32 / KC, RPL = 16 / RG;
       const int wr = warp - W_ROT;
       const int my_c = lane % KC, my_rg = lane / KC;
@@ -701,15 +759,15 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
           }
         };
         for (int j = 0; j < n; ++j) {
-          const int st = j % NSK, kt = kv_begin + j;
-          const bool ok = mbar_wait(bar(B_KFULL + st), (j / NSK) & 1, abort_flag, p.status, detail);
-          if (!__all_sync(0xffffffffu, ok)) break;
+          const int st = j % NSK;
+          // After an abort the loop runs on without waiting or rotating, so
+          // the four warps still meet at every named barrier.
+          const bool ok = __all_sync(0xffffffffu, mbar_wait(bar(B_KFULL + st), (j / NSK) & 1,
+                                                             abort_flag, p.status, detail));
           const uint32_t stage = sbase + L::kK + st * L::kTile;
-#pragma unroll 1
-          for (int h = 0; h < 2; ++h) {
-            const int q = 2 * wr + h;
-            const int2 pi = info[st * 8 + q];
-            if (pi.x == 0) continue;
+          const int q = 4 * (int)crank + wr;  // this warp's page: one of the CTA's half
+          const int2 pi = info[st * 8 + q];
+          if (ok && pi.x != 0) {
             const uint32_t pbase = stage + q * kPageBytes;
             if (pi.x == 1) {  // one document: RPL rows at once
               ensure_cs(pi.y);
@@ -745,6 +803,14 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
             }
           }
           fence_proxy_async();
+          // the CTA's half rotated: one bulk copy into the same slot of the
+          // peer, whose K(j) is complete when these bytes and its own half are
+          named_bar_sync(kNbRot, 128);
+          if (wr == 0 && lane == 0 && !*abort_flag) {
+            const uint32_t half = stage + 4 * crank * kPageBytes;
+            bulk_copy_to_peer(map_to_rank(half, cpeer), half, 4 * kPageBytes,
+                              map_to_rank(bar(B_KPEER + st), cpeer));
+          }
           __syncwarp();
           if (lane == 0) mbar_arrive(bar(B_KROT + st));
         }
@@ -933,6 +999,17 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
 
   tc_fence_before();
   __syncthreads();
+  if constexpr (kFused) {
+    // Leave only when the cluster peer is done too: its last copies into this
+    // CTA's ring have landed (the relay waited for them) and it no longer
+    // reads the copies this CTA sent.  The wait is bounded even after an abort.
+    if (threadIdx.x == 0) {
+      mbar_arrive_remote(map_to_rank(bar(B_EXIT), cpeer));
+      volatile int keep_waiting = 0;
+      mbar_wait(bar(B_EXIT), 0, &keep_waiting, p.status, detail);
+    }
+    __syncthreads();
+  }
   if (warp == 1) {
     tc_fence_after();
     if (*abort_flag && lane == 0) {
@@ -1461,9 +1538,17 @@ static cudaError_t launch_attention(const Plan &pl, const Params &pp, const Fuse
                          stream, fa, rp, pp.batch, page_blocks, pp.status);
     if (e != cudaSuccess) return e;
   }
-  dim3 grid(((pl.m_tiles + NQ - 1) / NQ) * pl.splits, pp.Hkv, pp.batch);
-  e = launch_dependent(attn_kernel<D, kFused>, grid, dim3(threads_of<kFused>()), smem, stream, tq,
-                       tk, tv, tkp, tvp, pp, fa, rp);
+  const int npairs = (pl.m_tiles + NQ - 1) / NQ;
+  if constexpr (kFused) {
+    // clusters of two consecutive query pairs: an even count per key split
+    dim3 grid(((npairs + 1) & ~1) * pl.splits, pp.Hkv, pp.batch);
+    e = launch_dependent_cluster(attn_kernel<D, kFused>, grid, dim3(threads_of<kFused>()), smem,
+                                 stream, 2, tq, tk, tv, tkp, tvp, pp, fa, rp);
+  } else {
+    dim3 grid(npairs * pl.splits, pp.Hkv, pp.batch);
+    e = launch_dependent(attn_kernel<D, kFused>, grid, dim3(threads_of<kFused>()), smem, stream,
+                         tq, tk, tv, tkp, tvp, pp, fa, rp);
+  }
   if (e != cudaSuccess) return e;
   if (pl.splits > 1) {
     const long long rows = (long long)pp.batch * pp.Hkv * pl.m_tiles * BM;
