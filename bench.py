@@ -408,7 +408,7 @@ def main_gpu(args, rank, world):
     L = spec.layers
     geom = path.geom
     psplits = pic.pic_prefill_num_splits(geom, spec.batch, path.max_inline, path.max_ctx,
-                                         args.prefill_splits)
+                                         path.prefill_splits)
 
     # warm-up run and device-side status
     path.ttft_pass()
@@ -684,7 +684,7 @@ def main_gpu(args, rank, world):
             pth.append(0)
             pic.pic_attend_prefill(pth.geom, 0, pth.inline_pos, wl.inline_len, pth.max_ctx,
                                    wl.block_table, wl.num_pages, pth.k_cache, pth.v_cache,
-                                   pth.out[0], pth.lse[0], args.prefill_splits, pth.ws_prefill)
+                                   pth.out[0], pth.lse[0], pth.prefill_splits, pth.ws_prefill)
         qlen = torch.full((spec.batch,), spec.query_len, dtype=torch.int32, device=dev)
         dsum = torch.empty((spec.batch, 2), dtype=torch.float64, device=dev)
         dcnt = torch.empty((spec.batch, 2), dtype=torch.int64, device=dev)

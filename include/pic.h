@@ -48,7 +48,7 @@
 extern "C" {
 #endif
 
-#define PIC_ABI_VERSION 3
+#define PIC_ABI_VERSION 4
 
 typedef struct CUstream_st *pic_stream_t; /* identical to cudaStream_t */
 
@@ -334,6 +334,19 @@ size_t pic_prefill_workspace_size(const pic_geom_t *geom, int32_t batch, int32_t
  * automatic choice); > 1 means a second (merge) launch.  0 on bad arguments. */
 int32_t pic_prefill_num_splits(const pic_geom_t *geom, int32_t batch, int32_t max_inline,
                                int32_t max_ctx, int32_t num_splits);
+
+/* A key-split count for pic_attend_prefill / pic_attend_prefill_fused chosen
+ * from the requests' actual inline positions (the layout of Sec. 3.3 /
+ * Eq. 2: prefix, documents, spans, query), which decide how many key tiles
+ * each pair of query tiles reads: the call simulates the attention grid's
+ * CTAs, in launch order, on the GPU's SMs for every candidate count and
+ * returns the one with the least estimated makespan.  Host work only.
+ * inline_len: host int32 [batch]; inline_pos: host int32 [batch][max_inline]
+ *   (row b's first inline_len[b] entries used), the positions compose writes.
+ * Returns 0 on bad arguments (as pic_prefill_num_splits). */
+int32_t pic_prefill_plan_splits(const pic_geom_t *geom, int32_t batch, int32_t max_inline,
+                                int32_t max_ctx, const int32_t *inline_len,
+                                const int32_t *inline_pos);
 
 pic_status_t pic_append_inline(const pic_geom_t *geom, int32_t layer, int32_t batch,
                                int32_t max_inline, const void *q, const void *k_new,

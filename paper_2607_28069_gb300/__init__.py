@@ -21,7 +21,8 @@ __all__ = [
     "pic_attention_deviation", "pic_copy_async", "pic_launch_probe",
     "pic_append_inline", "pic_attend_prefill", "pic_attend_prefill_fused",
     "pic_prefill_workspace_size", "pic_prefill_fused_workspace_size",
-    "pic_prefill_num_splits", "pic_decode_num_splits", "pic_attend_decode_noalloc",
+    "pic_prefill_num_splits", "pic_prefill_plan_splits", "pic_decode_num_splits",
+    "pic_attend_decode_noalloc",
     "pic_attend_decode", "pic_decode_workspace_size", "pic_device_status", "PicError",
     "EXPORTED_SYMBOLS", "ROPE_HALF", "ROPE_INTERLEAVED",
 ]
@@ -37,7 +38,7 @@ ROPE_INTERLEAVED = 1
 EXPORTED_SYMBOLS = (
     "pic_abi_version", "pic_last_error", "pic_device_status", "pic_compose", "pic_relocate",
     "pic_relocate_mapped", "pic_link", "pic_attention_deviation", "pic_prefill_workspace_size",
-    "pic_prefill_fused_workspace_size", "pic_prefill_num_splits",
+    "pic_prefill_fused_workspace_size", "pic_prefill_num_splits", "pic_prefill_plan_splits",
     "pic_append_inline",
     "pic_attend_prefill", "pic_attend_prefill_fused", "pic_decode_workspace_size", "pic_decode_num_splits",
     "pic_attend_decode", "pic_attend_decode_noalloc", "pic_copy_async", "pic_launch_probe",
@@ -135,6 +136,7 @@ def load():
         "pic_attend_decode_noalloc": (I32, [G, I32, I32, P, P, P, P, I32, P, I32, I64, P, P, P, P,
                                             I32, I32, P]),
         "pic_prefill_num_splits": (I32, [G, I32, I32, I32, I32]),
+        "pic_prefill_plan_splits": (I32, [G, I32, I32, I32, P, P]),
         "pic_decode_num_splits": (I32, [G, I32, I32, I32]),
         "pic_attend_decode": (I32, [G, I32, I32, P, P, P, P, I32, P, I32, I64, P, P, P, P, I32, I32,
                                     P, SZ, P]),
@@ -336,6 +338,20 @@ def pic_prefill_num_splits(geom: Geometry, batch: int, max_inline: int, max_ctx:
                            num_splits: int = 0) -> int:
     g = geom._c()
     return load().pic_prefill_num_splits(ctypes.byref(g), batch, max_inline, max_ctx, num_splits)
+
+
+def pic_prefill_plan_splits(geom: Geometry, max_ctx: int, inline_len, inline_pos) -> int:
+    """Key-split count planned from the requests' inline positions (host int32
+    tensors [B] and [B][max_inline]); 0 on bad arguments."""
+    import torch
+    lens = inline_len.to(torch.int32).contiguous()
+    pos = inline_pos.to(torch.int32).contiguous()
+    if lens.is_cuda or pos.is_cuda or pos.dim() != 2 or lens.numel() != pos.shape[0]:
+        raise ValueError("pic_prefill_plan_splits: host int32 inline_len [B] and inline_pos [B][T]")
+    g = geom._c()
+    return load().pic_prefill_plan_splits(ctypes.byref(g), pos.shape[0], pos.shape[1], max_ctx,
+                                          ctypes.c_void_p(lens.data_ptr()),
+                                          ctypes.c_void_p(pos.data_ptr()))
 
 
 def pic_decode_num_splits(geom: Geometry, batch: int, max_ctx: int, num_splits: int = 0) -> int:

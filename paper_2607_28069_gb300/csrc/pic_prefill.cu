@@ -27,6 +27,10 @@
 //  2. combine_kernel (only when the key range of a tile is split over several
 //     CTAs): log-sum-exp merge of the per-split partials (O, m, l), one warp
 //     per query row.
+#include <algorithm>
+#include <functional>
+#include <vector>
+
 #include "pic_internal.cuh"
 
 namespace pic {
@@ -1419,6 +1423,68 @@ extern "C" int32_t pic_prefill_num_splits(const pic_geom_t *geom, int32_t batch,
       num_splits > pic::prefill::kMaxSplits)
     return 0;
   return pic::prefill::plan(geom, batch, max_inline, max_ctx, num_splits).splits;
+}
+
+// Key-split count for the requests' actual inline positions: for every
+// candidate count, the attention grid's CTAs in launch order (one per query
+// pair, key split, kv head and request, a pair's tiles counted from the
+// request's last packed row as the kernel does) are dealt greedily to the
+// SMs, each costing its key tiles plus a fixed per-CTA cost, and the count
+// with the least makespan (plus a merge cost when split) wins; a grid that
+// fits in one wave with the library's count is not split further.
+extern "C" int32_t pic_prefill_plan_splits(const pic_geom_t *geom, int32_t batch,
+                                           int32_t max_inline, int32_t max_ctx,
+                                           const int32_t *inline_len, const int32_t *inline_pos) {
+  using namespace pic::prefill;
+  if (!inline_len || !inline_pos) return 0;
+  const int32_t fallback = pic_prefill_num_splits(geom, batch, max_inline, max_ctx, 0);
+  if (fallback <= 0) return 0;
+  const int G = geom->num_q_heads / geom->num_kv_heads, Hkv = geom->num_kv_heads;
+  const int m_tiles = (int)(((long long)max_inline * G + BM - 1) / BM), npairs = (m_tiles + NQ - 1) / NQ;
+  const int kv_tiles = (max_ctx + BN - 1) / BN;
+  // key tiles of each (request, pair): 0 for a pair without rows
+  std::vector<int> pair_tiles((size_t)batch * npairs, 0);
+  for (int b = 0; b < batch; ++b) {
+    const int tin = std::min(std::max(inline_len[b], 0), max_inline);
+    const int rows = tin * G;
+    for (int pr = 0; pr < npairs; ++pr) {
+      const int r0 = rows - (pr * NQ + 1) * BM;
+      if (pr * NQ < m_tiles && r0 + BM > 0) {
+        const int kmax = inline_pos[(size_t)b * max_inline + (r0 + BM - 1) / G];
+        pair_tiles[(size_t)b * npairs + pr] = kmax >= 0 ? std::min(kmax / BN + 1, kv_tiles) : 0;
+      }
+    }
+  }
+  constexpr double kCtaFixed = 2.0, kCtaEmpty = 0.3, kMerge = 1.0;  // in key-tile times
+  constexpr int kSms = 152;
+  double best = 1e300;
+  int best_s = fallback;
+  std::vector<double> sm(kSms);
+  // A grid the library's count already fits in one wave is latency-bound:
+  // more splits there only add merge traffic the estimate leaves out.
+  int max_s = std::min(kMaxSplits, std::max(1, kv_tiles));
+  if ((long long)batch * Hkv * npairs * fallback <= kSms) max_s = std::min(max_s, fallback);
+  for (int sp = 1; sp <= max_s; ++sp) {
+    std::fill(sm.begin(), sm.end(), 0.0);
+    std::make_heap(sm.begin(), sm.end(), std::greater<double>());
+    for (int b = 0; b < batch; ++b)
+      for (int hk = 0; hk < Hkv; ++hk)
+        for (int x = 0; x < npairs * sp; ++x) {
+          const int pr = x % npairs, split = x / npairs;
+          const int na = pair_tiles[(size_t)b * npairs + pr];
+          const int per = (na + sp - 1) / sp;
+          const int n = std::max(0, std::min(per, na - split * per));
+          std::pop_heap(sm.begin(), sm.end(), std::greater<double>());
+          sm.back() += n > 0 ? n + kCtaFixed : kCtaEmpty;
+          std::push_heap(sm.begin(), sm.end(), std::greater<double>());
+        }
+    const double cost = *std::max_element(sm.begin(), sm.end()) + (sp > 1 ? kMerge : 0.0);
+    if (cost < best - 1e-9) {
+      best = cost;
+      best_s = sp;
+    }
+  }
+  return best_s;
 }
 
 namespace pic {

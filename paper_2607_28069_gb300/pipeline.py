@@ -10,8 +10,42 @@ import torch
 
 from . import (Geometry, pic_append_inline, pic_attend_decode, pic_attend_prefill,
                pic_attend_prefill_fused, pic_compose, pic_copy_async, pic_decode_workspace_size,
-               pic_link, pic_prefill_fused_workspace_size, pic_relocate, pic_relocate_mapped)
+               pic_link, pic_prefill_fused_workspace_size, pic_prefill_plan_splits, pic_relocate,
+               pic_relocate_mapped)
 from .workloads import Workload
+
+
+def host_inline_positions(wl: Workload):
+    """The inline tokens' logical positions of every request, on the host:
+    the prefix from 0, each document's span right after the document, the
+    query after the last one (the canonical order P, D_1, S_1, ..., D_m, S_m,
+    Q that compose lays out).  For planning only; compose computes the
+    positions the kernels use, and reports malformed requests, for which
+    this returns None."""
+    B = wl.req_doc_ids.shape[0]
+    prefix, query = wl.prefix_len.cpu().tolist(), wl.query_len.cpu().tolist()
+    ndocs, ids = wl.req_num_docs.cpu().tolist(), wl.req_doc_ids.cpu().tolist()
+    dlen = wl.doc_len.cpu().tolist()
+    spans = wl.span_len.cpu().tolist() if wl.span_len is not None else None
+    pos = torch.zeros((B, wl.tin_max), dtype=torch.int32)
+    lens = torch.zeros((B,), dtype=torch.int32)
+    for b in range(B):
+        if not 0 <= ndocs[b] <= len(ids[b]) or prefix[b] < 0 or query[b] < 0:
+            return None
+        row = list(range(prefix[b]))
+        off = prefix[b]
+        for k in range(ndocs[b]):
+            if not 0 <= ids[b][k] < len(dlen):
+                return None
+            off += dlen[ids[b][k]]
+            s_k = spans[b][k] if spans is not None else 0
+            row += range(off, off + s_k)
+            off += s_k
+        row += range(off, off + query[b])
+        row = row[:wl.tin_max]
+        pos[b, :len(row)] = torch.tensor(row, dtype=torch.int32)
+        lens[b] = len(row)
+    return lens, pos
 
 
 class CacheHitPath:
@@ -29,6 +63,10 @@ class CacheHitPath:
         self.B, self.max_docs = B, md
         self.max_ctx = wl.max_ctx
         self.max_inline = wl.tin_max
+        if prefill_splits == 0:  # planned from the requests' layout (else the library's choice)
+            hp = host_inline_positions(wl)
+            if hp is not None:
+                prefill_splits = pic_prefill_plan_splits(self.geom, self.max_ctx, *hp)
         self.prefill_splits = prefill_splits
         self.decode_splits = decode_splits
         i32, i64, bf16 = torch.int32, torch.int64, torch.bfloat16

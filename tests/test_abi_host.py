@@ -37,7 +37,7 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_version(lib):
-    assert pic.pic_abi_version() == 3
+    assert pic.pic_abi_version() == 4
 
 
 def _geom(**kw):
