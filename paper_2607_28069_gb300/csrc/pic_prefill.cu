@@ -59,7 +59,6 @@ constexpr int kWarpRelay = kWarpV + 1;    // waits on behalf of the MMA issuer
 // 0 is __syncthreads, 1 and 2 belong to the softmax warpgroups' epilogue.
 constexpr int kNbPv = 3;  // + t: P_t(j-1) and V(j-1) are ready
 constexpr int kNbK = 5;   // K(j) is ready
-constexpr int kNbRot = 6; // rotate-on-load: the rotator warps have rotated their pages
 constexpr int kMaxSplits = 32;
 constexpr uint32_t kTmemCols = 512;
 
@@ -764,8 +763,6 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
         };
         for (int j = 0; j < n; ++j) {
           const int st = j % NSK;
-          // After an abort the loop runs on without waiting or rotating, so
-          // the four warps still meet at every named barrier.
           const bool ok = __all_sync(0xffffffffu, mbar_wait(bar(B_KFULL + st), (j / NSK) & 1,
                                                              abort_flag, p.status, detail));
           const uint32_t stage = sbase + L::kK + st * L::kTile;
@@ -807,16 +804,18 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
             }
           }
           fence_proxy_async();
-          // the CTA's half rotated: one bulk copy into the same slot of the
-          // peer, whose K(j) is complete when these bytes and its own half are
-          named_bar_sync(kNbRot, 128);
-          if (wr == 0 && lane == 0 && !*abort_flag) {
-            const uint32_t half = stage + 4 * crank * kPageBytes;
-            bulk_copy_to_peer(map_to_rank(half, cpeer), half, 4 * kPageBytes,
-                              map_to_rank(bar(B_KPEER + st), cpeer));
-          }
           __syncwarp();
-          if (lane == 0) mbar_arrive(bar(B_KROT + st));
+          // the page rotated: a bulk copy into the same slot of the cluster
+          // peer, whose K(j) is complete when these four pages and its own
+          // half are
+          if (lane == 0) {
+            if (!*abort_flag) {
+              const uint32_t page = stage + q * kPageBytes;
+              bulk_copy_to_peer(map_to_rank(page, cpeer), page, kPageBytes,
+                                map_to_rank(bar(B_KPEER + st), cpeer));
+            }
+            mbar_arrive(bar(B_KROT + st));
+          }
         }
       };
       if (half_style) rotate_tiles(std::true_type{});
