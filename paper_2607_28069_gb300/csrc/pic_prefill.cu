@@ -687,7 +687,7 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
     if constexpr (kFused) {
       // Warp w of the rotators takes page 4 crank + w of each tile (the CTA's
       // half; the cluster peer rotates the other); lane l the 8-pair chunk
-      // l % KC of rows l / KC + RG i of the page, RPL rows at once.
+      // l % KC of rows l / KC + RG i (i < RPL) of the page.
       constexpr int KC = D / 16, RG = 32 / KC, RPL = 16 / RG;
       const int wr = warp - W_ROT;
       const int my_c = lane % KC, my_rg = lane / KC;
@@ -770,37 +770,24 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
           const int2 pi = info[st * 8 + q];
           if (ok && pi.x != 0) {
             const uint32_t pbase = stage + q * kPageBytes;
-            if (pi.x == 1) {  // one document: RPL rows at once
-              ensure_cs(pi.y);
-              uint4 va[RPL], vb[RPL];
-#pragma unroll
-              for (int i = 0; i < RPL; ++i) {
-                const int r = my_rg + RG * i;
-                va[i] = lds128(pbase + page_piece<D>(r, pc.off_a / 8));
-                vb[i] = lds128(pbase + page_piece<D>(r, pc.off_b / 8));
-              }
-#pragma unroll
-              for (int i = 0; i < RPL; ++i) {
-                const int r = my_rg + RG * i;
-                rot(va[i], vb[i]);
-                sts128(pbase + page_piece<D>(r, pc.off_a / 8), va[i]);
-                sts128(pbase + page_piece<D>(r, pc.off_b / 8), vb[i]);
-              }
-            } else {  // mixed page: each row's own document, inline rows as they are
-              const int16_t *rd = reinterpret_cast<const int16_t *>(smem + L::kRowDoc) + (st * 8 + q) * 16;
+            // a row at a time (a rolled loop keeps the rotators' code small in
+            // the instruction caches they share with the softmax): a page of
+            // one document rotates every row by that document's delta, a page
+            // across a boundary each row by its own document's, inline rows
+            // stay as they are
+            const int16_t *rd = reinterpret_cast<const int16_t *>(smem + L::kRowDoc) + (st * 8 + q) * 16;
 #pragma unroll 1
-              for (int i = 0; i < RPL; ++i) {
-                const int r = my_rg + RG * i;
-                const int kd = rd[r];
-                if (kd < 0) continue;
-                ensure_cs(kd);
-                const uint32_t a0 = pbase + page_piece<D>(r, pc.off_a / 8);
-                const uint32_t a1 = pbase + page_piece<D>(r, pc.off_b / 8);
-                uint4 va = lds128(a0), vb = lds128(a1);
-                rot(va, vb);
-                sts128(a0, va);
-                sts128(a1, vb);
-              }
+            for (int i = 0; i < RPL; ++i) {
+              const int r = my_rg + RG * i;
+              const int kd = pi.x == 1 ? pi.y : rd[r];
+              if (kd < 0) continue;
+              ensure_cs(kd);
+              const uint32_t a0 = pbase + page_piece<D>(r, pc.off_a / 8);
+              const uint32_t a1 = pbase + page_piece<D>(r, pc.off_b / 8);
+              uint4 va = lds128(a0), vb = lds128(a1);
+              rot(va, vb);
+              sts128(a0, va);
+              sts128(a1, vb);
             }
           }
           fence_proxy_async();
