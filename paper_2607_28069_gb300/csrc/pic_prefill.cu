@@ -48,7 +48,7 @@ constexpr int kThreads = 128 + NQ * 128;  // K producer, MMA, NQ softmax warpgro
 // producer, relay) and the rotators give registers to the softmax warpgroups.
 constexpr int kThreadsFused = 512;
 constexpr int kRegLaunchFused = 65536 / kThreadsFused;  // 128 per thread at launch
-constexpr int kRegCtl = 88, kRegRot = 88, kRegSoftmax = 168;
+constexpr int kRegCtl = 88, kRegRot = 72, kRegSoftmax = 176;
 static_assert(128 * kRegCtl + 128 * kRegRot + 256 * kRegSoftmax <= 128 * 4 * kRegLaunchFused,
               "setmaxnreg split exceeds the registers the CTA is launched with");
 template <bool kFused>
