@@ -844,43 +844,61 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
         for (int c = 0; c < BN; ++c)
           if (key0 + c > pos) s[c] = -INFINITY;
       }
-      // row max: 4 independent chains of 3-input max
-      float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-      for (int c = 0; c < BN; c += 8)
-#pragma unroll
-        for (int i = 0; i < 4; ++i) mx[i] = max3f(mx[i], s[c + 2 * i], s[c + 2 * i + 1]);
-      const float m_new = fmaxf(m_used, max3f(mx[0], mx[1], fmaxf(mx[2], mx[3])) * p.scale_log2);
+      // Exponents against the running maximum m_used.  From the second tile
+      // on, a warp whose rows all have one skips the row maximum and
+      // exponentiates against m_used directly; the tile's row sum then bounds
+      // every exponential, and if some row's sum reaches 2^64 (its scores grew
+      // by more than 64 in the log2 domain) the tile is redone the first way:
+      // row maximum, rescale when it grew by more than 2^8, exponentials again.
+      // P (bf16) up to 2^64 and the fp32 sums of a few thousand of them stay
+      // far inside the range of both.
       float alpha = 1.f;
-      const bool resc = m_new > m_used + 8.f;
-      if (resc) {
-        alpha = ex2(m_used - m_new);
-        m_used = m_new;
-      }
-      const float mref = (m_used == -INFINITY) ? 0.f : m_used;
-      // P = exp2(s * scale - m) as bf16, written over S in 16-column chunks as
-      // soon as each 32-key chunk is done (S was read completely above, so the
-      // overlap is harmless and the packed values never pile up in registers).
-      // Scaling and the row sum run on packed fp32 pairs (half the issue
-      // slots; the softmax is bound by instruction issue, not by MUFU).
-      const uint64_t sc2 = f2pack(p.scale_log2, p.scale_log2), nm2 = f2pack(-mref, -mref);
-      uint64_t acc[4] = {0, 0, 0, 0};
-#pragma unroll
-      for (int c0 = 0; c0 < BN; c0 += 32) {
-        uint32_t pk[16];
-#pragma unroll
-        for (int q = 0; q < 16; ++q) {
-          const uint64_t e = exp2_mufu2(fma2(f2pack(s[c0 + 2 * q], s[c0 + 2 * q + 1]), sc2, nm2));
-          acc[q & 3] = add2(acc[q & 3], e);
-          float e0, e1;
-          f2unpack(e, e0, e1);
-          pk[q] = pack2(e0, e1);
-        }
-        tmem_st16(tS + c0 / 2, pk);
-      }
-      acc[0] = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
+      bool resc = false;
+      bool need_max = !__all_sync(0xffffffffu, j > 0 && m_used != -INFINITY);
       float l0, l1;
-      f2unpack(acc[0], l0, l1);
+#pragma unroll 1
+      for (int pass = 0; pass < 2; ++pass) {
+        if (need_max) {
+          // row max: 4 independent chains of 3-input max
+          float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+          for (int c = 0; c < BN; c += 8)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) mx[i] = max3f(mx[i], s[c + 2 * i], s[c + 2 * i + 1]);
+          const float m_new = fmaxf(m_used, max3f(mx[0], mx[1], fmaxf(mx[2], mx[3])) * p.scale_log2);
+          resc = m_new > m_used + 8.f;
+          if (resc) {
+            alpha = ex2(m_used - m_new);
+            m_used = m_new;
+          }
+        }
+        const float mref = (m_used == -INFINITY) ? 0.f : m_used;
+        // P = exp2(s * scale - m) as bf16, written over S in 16-column chunks
+        // as soon as each 32-key chunk is done (S was read completely above,
+        // so the overlap is harmless and the packed values never pile up in
+        // registers).  Scaling and the row sum run on packed fp32 pairs (half
+        // the issue slots; the softmax is bound by instruction issue, not by
+        // MUFU).
+        const uint64_t sc2 = f2pack(p.scale_log2, p.scale_log2), nm2 = f2pack(-mref, -mref);
+        uint64_t acc[4] = {0, 0, 0, 0};
+#pragma unroll
+        for (int c0 = 0; c0 < BN; c0 += 32) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int q = 0; q < 16; ++q) {
+            const uint64_t e = exp2_mufu2(fma2(f2pack(s[c0 + 2 * q], s[c0 + 2 * q + 1]), sc2, nm2));
+            acc[q & 3] = add2(acc[q & 3], e);
+            float e0, e1;
+            f2unpack(e, e0, e1);
+            pk[q] = pack2(e0, e1);
+          }
+          tmem_st16(tS + c0 / 2, pk);
+        }
+        acc[0] = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
+        f2unpack(acc[0], l0, l1);
+        if (need_max || !__any_sync(0xffffffffu, !(l0 + l1 < 0x1p64f))) break;
+        need_max = true;
+      }
       l = fmaf(l, alpha, l0 + l1);
       // O correction: PV_t(j-1) has completed (it precedes QK_t(j) in the MMA order)
       if (j > 0 && __any_sync(0xffffffffu, resc)) {
