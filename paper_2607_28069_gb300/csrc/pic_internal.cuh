@@ -8,6 +8,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -132,6 +133,17 @@ PIC_DEV uint4 pack8(const float *f) {
   __nv_bfloat162 *h = reinterpret_cast<__nv_bfloat162 *>(&v);
 #pragma unroll
   for (int i = 0; i < 4; ++i) h[i] = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
+  return v;
+}
+
+// Eight floats as fp16, rounded to nearest even and saturated at +-65504.
+PIC_DEV uint4 pack8_h(const float *f) {
+  uint4 v;
+  __half2 *h = reinterpret_cast<__half2 *>(&v);
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    h[i] = __floats2half2_rn(fminf(fmaxf(f[2 * i], -65504.f), 65504.f),
+                             fminf(fmaxf(f[2 * i + 1], -65504.f), 65504.f));
   return v;
 }
 

@@ -99,7 +99,8 @@ struct Params {
   long long num_pages, layer_row0;
   const int32_t *inline_pos, *inline_len, *block_table;
   __nv_bfloat16 *out;
-  float *lse, *part_o, *part_ml;
+  float *lse, *part_ml;
+  __half *part_o;  // split partials: O / l per row, fp16
   int32_t *status;
   float scale_log2;
 };
@@ -931,8 +932,8 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
       // accesses at 4 wavefronts per 512 B), the warpgroup syncs on its own
       // named barrier, and warps copy whole rows out with coalesced stores.
       const bool single = p.num_splits == 1;
-      constexpr int kRowOut = D * 2 + 16, kRowPart = D * 4 + 16;
-      uint8_t *stage = smem + (size_t)t * BM * (single ? kRowOut : kRowPart);
+      constexpr int kRowOut = D * 2 + 16;  // a row of bf16 outputs or fp16 partials, padded
+      uint8_t *stage = smem + (size_t)t * BM * kRowOut;
       if (ok) {
         float o[D];
 #pragma unroll
@@ -949,10 +950,14 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
             p.lse[((size_t)b * p.max_inline + tok) * p.Hq + hk * p.G + g] =
                 l > 0.f ? (m_used + __log2f(l)) * 0.69314718055994531f : -INFINITY;
         } else {
-          float4 *dst = reinterpret_cast<float4 *>(stage + row * kRowPart);
+          // a split's partial row: O / l in fp16 (|O / l| is at most the
+          // largest |v|), with m and l beside it for the merge's weights
+          const float inv = l > 0.f ? 1.f / l : 0.f;
+          uint4 *dst = reinterpret_cast<uint4 *>(stage + row * kRowOut);
 #pragma unroll
-          for (int q = 0; q < D / 4; ++q)
-            dst[q] = make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+          for (int q = 0; q < D; ++q) o[q] *= inv;
+#pragma unroll
+          for (int q = 0; q < D / 8; ++q) dst[q] = pack8_h(o + q * 8);
           p.part_ml[(my_part0 + row) * 2] = (l > 0.f) ? m_used : -INFINITY;
           p.part_ml[(my_part0 + row) * 2 + 1] = l;
         }
@@ -971,16 +976,13 @@ __device__ __forceinline__ void attn_body(const CUtensorMap &tm_q, const CUtenso
                             (lane % LPR) * 8, v);
           }
         } else {
-          // fp32 rows are contiguous in the partial buffer: one row per warp pass
-          constexpr int LPR = D / 4;  // 16-byte pieces per row
-          constexpr int RPI = 32 / LPR > 0 ? 32 / LPR : 1;
-          for (int r = wq * RPI + lane / LPR; r < BM; r += 4 * RPI)
-#pragma unroll
-            for (int c = lane % LPR; c < D / 4; c += (LPR < 32 ? LPR : 32)) {
-              if (r < rlo) continue;
-              const float4 v = *reinterpret_cast<const float4 *>(stage + r * kRowPart + c * 16);
-              reinterpret_cast<float4 *>(p.part_o + (my_part0 + r) * D)[c] = v;
-            }
+          // the partial rows are contiguous in the partial buffer
+          constexpr int LPR = D / 8, RPI = 32 / LPR;
+          for (int r = wq * RPI + lane / LPR; r < BM; r += 4 * RPI) {
+            if (r < rlo) continue;
+            const uint4 v = *reinterpret_cast<const uint4 *>(stage + r * kRowOut + (lane % LPR) * 16);
+            *reinterpret_cast<uint4 *>(p.part_o + (my_part0 + r) * D + (lane % LPR) * 8) = v;
+          }
         }
       }
     }
@@ -1055,11 +1057,12 @@ __global__ void __launch_bounds__(threads_of<kFused>(), 1)
 }
 
 
-// Merge the split partials (O unnormalised, m in log2 units, l) of every
-// query row by log-sum-exp, lanes over the d columns.  A warp takes R rows
-// of one query tile and issues the (m, l) pairs and the O rows of U splits
-// for all R rows before using any of them (R * U = 8 loads of 16 bytes in
-// flight per lane), so a row costs one L2/DRAM round trip for up to U splits;
+// Merge the split partials (O / l in fp16, m in log2 units, l) of every
+// query row by log-sum-exp -- o = sum_s w_s (O_s / l_s) / sum_s w_s with
+// w_s = 2^(m_s - M) l_s -- lanes over the d columns.  A warp takes R rows of
+// one query tile and issues the (m, l) pairs and the O rows of U splits for
+// all R rows before using any of them (R * U = 8 loads in flight per lane),
+// so a row costs one L2/DRAM round trip for up to U splits;
 // U is the smallest of 2, 4, 8 that covers the splits (more are merged in
 // further rounds).  An empty split's weight is zero and its data, never
 // written, is discarded by a select.  Launched as a programmatic dependent of
@@ -1107,14 +1110,16 @@ __global__ void __launch_bounds__(256) combine_kernel(Params p) {
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         const int sp = min(s0 + u, S - 1);  // past the end: a harmless reload, weight 0 below
-        const float *src = p.part_o + ((base + sp) * BM + row0 + r) * D + lane * CPL;
+        const __half *src = p.part_o + ((base + sp) * BM + row0 + r) * D + lane * CPL;
         if constexpr (CPL == 4) {
-          const float4 x = *reinterpret_cast<const float4 *>(src);
-          v[r][u][0] = x.x, v[r][u][1] = x.y, v[r][u][2] = x.z, v[r][u][3] = x.w;
+          const uint2 x = *reinterpret_cast<const uint2 *>(src);
+          const float2 a = __half22float2(*reinterpret_cast<const __half2 *>(&x.x));
+          const float2 c = __half22float2(*reinterpret_cast<const __half2 *>(&x.y));
+          v[r][u][0] = a.x, v[r][u][1] = a.y, v[r][u][2] = c.x, v[r][u][3] = c.y;
         } else {
           static_assert(CPL == 2, "d = 64 or 128");
-          const float2 x = *reinterpret_cast<const float2 *>(src);
-          v[r][u][0] = x.x, v[r][u][1] = x.y;
+          const float2 a = __half22float2(*reinterpret_cast<const __half2 *>(src));
+          v[r][u][0] = a.x, v[r][u][1] = a.y;
         }
       }
     if (s0 == 0) {
@@ -1123,8 +1128,9 @@ __global__ void __launch_bounds__(256) combine_kernel(Params p) {
         M[r] = ms[r];
 #pragma unroll
         for (int o = 16; o; o >>= 1) M[r] = fmaxf(M[r], __shfl_xor_sync(0xffffffffu, M[r], o));
-        w[r] = (ms[r] == -INFINITY) ? 0.f : ex2(ms[r] - M[r]);
-        Lsum[r] = w[r] * ls[r];
+        // weight of split `lane` for the normalised partial: exp2(m_s - M) l_s
+        w[r] = (ms[r] == -INFINITY) ? 0.f : ex2(ms[r] - M[r]) * ls[r];
+        Lsum[r] = w[r];
 #pragma unroll
         for (int o = 16; o; o >>= 1) Lsum[r] += __shfl_xor_sync(0xffffffffu, Lsum[r], o);
       }
@@ -1320,7 +1326,7 @@ inline Plan plan(const pic_geom_t *g, int batch, int max_inline, int max_ctx, in
   pl.q_bytes = align256((size_t)batch * g->num_kv_heads * pl.R_pad * g->head_dim * 2);
   if (pl.splits > 1) {
     const size_t rows = (size_t)batch * g->num_kv_heads * pl.m_tiles * pl.splits * BM;
-    pl.po_bytes = align256(rows * g->head_dim * 4);
+    pl.po_bytes = align256(rows * g->head_dim * 2);
     pl.pml_bytes = align256(rows * 2 * 4);
   } else {
     pl.po_bytes = pl.pml_bytes = 0;
@@ -1697,7 +1703,7 @@ extern "C" pic_status_t pic_attend_prefill(
   pp.block_table = block_table;
   pp.out = static_cast<__nv_bfloat16 *>(out);
   pp.lse = lse;
-  pp.part_o = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes) : nullptr;
+  pp.part_o = pl.splits > 1 ? reinterpret_cast<__half *>(ws + pl.q_bytes) : nullptr;
   pp.part_ml = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes + pl.po_bytes) : nullptr;
   pp.status = status;
   pp.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
@@ -1797,7 +1803,7 @@ extern "C" pic_status_t pic_attend_prefill_fused(
   pp.block_table = block_table;
   pp.out = static_cast<__nv_bfloat16 *>(out);
   pp.lse = lse;
-  pp.part_o = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes) : nullptr;
+  pp.part_o = pl.splits > 1 ? reinterpret_cast<__half *>(ws + pl.q_bytes) : nullptr;
   pp.part_ml = pl.splits > 1 ? reinterpret_cast<float *>(ws + pl.q_bytes + pl.po_bytes) : nullptr;
   pp.status = status;
   pp.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));

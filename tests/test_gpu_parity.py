@@ -16,7 +16,7 @@ import torch
 import oracle as O
 from paper_2607_28069_gb300.workloads import WORKLOADS, custom_spec, generate
 from tests.helpers import (attn_close, f64, kv_tolerance_ok, oracle_layout, request_inputs,
-                           theta_of)
+                           theta_of, half_ulp_bf16)
 
 pytestmark = pytest.mark.gpu
 
@@ -214,8 +214,11 @@ def test_prefill_split_count_invariance(cuda_lib, splits):
     o_gpu = f64(path.out[0, 0, :q.shape[0]])
     ok, max_abs, row = attn_close(o_gpu, o_ref)
     assert ok, f"splits {splits}: err/bound {max_abs:.2f} row-rel {row:.2e}"
-    d = (path.out.float() - path0.out.float()).abs().max().item()
-    assert d <= 1e-2
+    # Split counts differ in rounding only: the outputs are bf16, so two
+    # counts may round a value to neighbouring bf16 values (one spacing apart).
+    a, b0 = f64(path.out), f64(path0.out)
+    bar = np.maximum(1e-2, 2 * half_ulp_bf16(np.maximum(np.abs(a), np.abs(b0))))
+    assert (np.abs(a - b0) <= bar).all(), np.abs(a - b0).max()
 
 
 @pytest.mark.parametrize("name", ["gqa7_decode", "d64_g8", "g16_decode", "no_docs", "spans_b2",
