@@ -217,11 +217,14 @@ struct PageSrc {
 // the pool as one box (the document's rows are consecutive there); a page of
 // inline tokens from the cache as before; a page across a boundary is filled
 // row by row by the producer warp.  A rotator warpgroup then rotates every
-// document row of the tile in shared memory by its document's delta -- the
-// same fp32 arithmetic and bf16 rounding as the relocation, so the tile holds
-// exactly the keys pic_relocate would have stitched -- and signals K(j) on
-// B_KROT instead of the TMA barrier.  Everything downstream (MMAs, softmax,
-// merge) is the materialised kernel's.
+// document row in shared memory by its document's delta -- the same fp32
+// arithmetic and bf16 rounding as the relocation, so the tile holds exactly
+// the keys pic_relocate would have stitched.  The CTAs run in clusters of
+// two (two query pairs of one key split): each loads and rotates half of
+// every key tile and bulk-copies the rotated pages into the other's ring, so
+// K(j) is complete when its own half is rotated (B_KROT) and the peer's half
+// has landed (B_KPEER); the QK commits are multicast to both CTAs' B_KEMPTY.
+// Everything downstream (MMAs, softmax, merge) is the materialised kernel's.
 //
 // The body is one function per group of warps (kGroup: 0 the control
 // warpgroup, 1 the rotators, 2 the softmax warpgroups; -1 all warps of the
