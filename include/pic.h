@@ -336,8 +336,9 @@ int32_t pic_prefill_num_splits(const pic_geom_t *geom, int32_t batch, int32_t ma
                                int32_t max_ctx, int32_t num_splits);
 
 /* A key-split count for pic_attend_prefill / pic_attend_prefill_fused chosen
- * from the requests' actual inline positions (the layout of Sec. 3.3 /
- * Eq. 2: prefix, documents, spans, query), which decide how many key tiles
+ * from the requests' actual inline positions (the logical layout of
+ * "Background: Position-Independent Caching" and appendix "Logical Layout
+ * and Re-Rotation": prefix, documents, spans, query), which decide how many key tiles
  * each pair of query tiles reads: the call simulates the attention grid's
  * CTAs, in launch order, on the GPU's SMs for every candidate count and
  * returns the one with the least estimated makespan.  Host work only.
