@@ -139,6 +139,18 @@ pic_status_t pic_launch_probe(int32_t n, const int32_t *grid, const int32_t *blo
                               const int32_t *smem, pic_stream_t stream);
 
 /*
+ * pic_wait_probe -- a check of the failure detection, not an operation of the
+ * paper: one CTA of one warp waits on the first phase of an mbarrier of one
+ * arrival with the bounded wait every kernel of the path uses, limited to
+ * limit_ns.  arrive != 0: the CTA arrives first and the wait completes at
+ * once.  arrive == 0: nothing arrives; after limit_ns the wait records
+ * PIC_DEV_TIMEOUT (detail -1) in the status word read by pic_device_status
+ * and the kernel returns, so the context stays usable.  Asynchronous on
+ * `stream`.  PIC_ERR_INVALID_ARG for limit_ns outside [1000, 10^10].
+ */
+pic_status_t pic_wait_probe(int32_t arrive, int64_t limit_ns, pic_stream_t stream);
+
+/*
  * pic_compose -- link operator R: logical layout of each request and its
  * token-level maps (Eqs. 1-2, "Background: Position-Independent Caching";
  * appendix "Logical Layout and Re-Rotation").

@@ -18,7 +18,7 @@ import torch
 __all__ = [
     "Geometry", "load", "lib_path", "pic_abi_version", "pic_compose", "pic_relocate",
     "pic_relocate_mapped", "pic_link",
-    "pic_attention_deviation", "pic_copy_async", "pic_launch_probe",
+    "pic_attention_deviation", "pic_copy_async", "pic_launch_probe", "pic_wait_probe",
     "pic_append_inline", "pic_attend_prefill", "pic_attend_prefill_fused",
     "pic_prefill_workspace_size", "pic_prefill_fused_workspace_size",
     "pic_prefill_num_splits", "pic_prefill_plan_splits", "pic_decode_num_splits",
@@ -42,6 +42,7 @@ EXPORTED_SYMBOLS = (
     "pic_append_inline",
     "pic_attend_prefill", "pic_attend_prefill_fused", "pic_decode_workspace_size", "pic_decode_num_splits",
     "pic_attend_decode", "pic_attend_decode_noalloc", "pic_copy_async", "pic_launch_probe",
+    "pic_wait_probe",
 )
 
 DEVICE_CODES = {
@@ -114,6 +115,7 @@ def load():
         "pic_device_status": (I32, [P, P, P]),
         "pic_copy_async": (I32, [P, P, SZ, P]),
         "pic_launch_probe": (I32, [I32, P, P, P, P]),
+        "pic_wait_probe": (I32, [I32, I64, P]),
         "pic_compose": (I32, [G, I32, I32, I32, P, P, P, P, P, P, P, P, P, I32, I64, I32, I32,
                               P, P, P, P, P, P, P]),
         "pic_relocate": (I32, [G, I32, I32, I32, P, P, I64, P, P, P, P, P, P, P, I32, I64, P, P,
@@ -228,6 +230,14 @@ def pic_launch_probe(shapes, stream=None):
     smem = (ctypes.c_int32 * n)(*[int(s[2]) for s in shapes])
     st = load().pic_launch_probe(n, grid, block, smem, _stream(stream))
     _check(st, "pic_launch_probe")
+
+
+def pic_wait_probe(arrive: bool, limit_ns: int, stream=None):
+    """One bounded mbarrier wait of limit_ns on the device: completes when
+    `arrive`, else runs out and records a timeout in the device status word
+    (read it with pic_device_status)."""
+    st = load().pic_wait_probe(1 if arrive else 0, int(limit_ns), _stream(stream))
+    _check(st, "pic_wait_probe")
 
 
 def pic_compose(geom: Geometry, doc_len, doc_base_pos, doc_token_start, req_doc_ids,

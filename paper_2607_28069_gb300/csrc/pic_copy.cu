@@ -6,7 +6,10 @@
 // megabytes.  Either side may be device memory of the current device or
 // page-locked host memory (cudaHostAlloc / cudaHostRegister, e.g. a pinned
 // torch tensor); the kernel addresses host memory through its device
-// pointer.
+// pointer.  Two checks of the path's machinery live here too:
+// pic_launch_probe (empty programmatic-dependent kernels of given launch
+// shapes, the launch floor of a pass) and pic_wait_probe (the bounded
+// mbarrier wait running out and reporting PIC_DEV_TIMEOUT).
 #include <algorithm>
 
 #include "pic_internal.cuh"
@@ -45,8 +48,41 @@ __global__ void __launch_bounds__(kCopyThreads) copy_kernel(uint4 *__restrict__ 
 // next one launch, and does nothing else (pic_launch_probe).
 __global__ void probe_kernel() { pdl_entry(); }
 
+// One CTA waits on the first phase of an mbarrier of one arrival with the
+// bounded wait of the path's kernels (pic_wait_probe): thread 0 arrives
+// first when `arrive` is set, so the wait completes at once; otherwise
+// nothing arrives, the wait runs out after limit_ns and records
+// PIC_DEV_TIMEOUT (detail -1) in the status word, and the kernel returns.
+__global__ void wait_probe_kernel(int arrive, uint64_t limit_ns, int32_t *status) {
+  __shared__ __align__(8) uint64_t bar_slot;
+  __shared__ int abort_flag;
+  const uint32_t bar = smem_u32(&bar_slot);
+  if (threadIdx.x == 0) {
+    mbar_init(bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (arrive) mbar_arrive(bar);
+    mbar_wait_for(bar, 0, &abort_flag, status, -1, limit_ns);
+  }
+  __syncthreads();
+}
+
 }  // namespace
 }  // namespace pic
+
+extern "C" pic_status_t pic_wait_probe(int32_t arrive, int64_t limit_ns, pic_stream_t stream) {
+  using namespace pic;
+  if (limit_ns < 1000 || limit_ns > 10000000000LL)
+    return fail(PIC_ERR_INVALID_ARG, "pic_wait_probe: limit_ns outside [1 us, 10 s]");
+  int32_t *status = device_status_ptr();
+  if (!status) return fail(PIC_ERR_CUDA, "pic_wait_probe: no device status word");
+  wait_probe_kernel<<<1, 32, 0, stream>>>(arrive != 0, (uint64_t)limit_ns, status);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? PIC_OK : cuda_fail(e, "pic_wait_probe launch");
+}
 
 extern "C" pic_status_t pic_launch_probe(int32_t n, const int32_t *grid, const int32_t *block,
                                          const int32_t *smem, pic_stream_t stream) {

@@ -420,23 +420,28 @@ PIC_DEV uint64_t globaltimer_ns() {
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
 
 // Bounded wait.  Returns false (after recording PIC_DEV_TIMEOUT and raising
-// *abort) when the phase did not complete within the limit, or when another
+// *abort) when the phase did not complete within limit_ns, or when another
 // role of the CTA has already aborted.
-PIC_DEV bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort, int32_t *status,
-                       int detail) {
+PIC_DEV bool mbar_wait_for(uint32_t bar, uint32_t parity, volatile int *abort, int32_t *status,
+                           int detail, uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((i & 63u) == 0) {
       if (*abort) return false;
-      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      if (globaltimer_ns() - t0 > limit_ns) {
         *abort = 1;
         dev_fail(status, PIC_DEV_TIMEOUT, detail);
         return false;
       }
     }
   }
+}
+// The wait every kernel of the path uses.
+PIC_DEV bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort, int32_t *status,
+                       int detail) {
+  return mbar_wait_for(bar, parity, abort, status, detail, kWaitLimitNs);
 }
 
 // ----------------------------------------------------------------------- TMA

@@ -164,3 +164,9 @@ def test_launch_probe_rejects_bad_shapes_before_any_launch(lib):
     m = (C.c_int32 * 1)(0)
     assert pic.load().pic_launch_probe(0, g, b, m, None) == 1      # n must be positive
     assert pic.load().pic_launch_probe(1, None, b, m, None) == 1   # arrays required
+
+
+def test_wait_probe_rejects_its_limit_on_the_host(lib):
+    assert pic.load().pic_wait_probe(0, 10, None) == 1            # below 1 us
+    assert pic.load().pic_wait_probe(1, 10 ** 11, None) == 1      # above 10 s
+    assert b"limit_ns" in pic.load().pic_last_error()
