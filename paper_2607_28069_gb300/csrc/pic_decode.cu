@@ -284,32 +284,60 @@ __global__ void __launch_bounds__(kThreads)
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
+// Merge of the split partials of one (request, query head) row by
+// log-sum-exp: o = sum_s w_s O_s / sum_s w_s l_s with w_s = 2^(m_s - M).
+// Lane s holds split s's (m, l) (and lane s - 32 split s >= 32), so the
+// maximum and the weight sum are warp reductions, and the O rows of eight
+// splits are loaded before any is used: a row costs a few L2 round trips
+// however many splits it has, not one per split.
 template <int D>
 __global__ void decode_combine_kernel(Params p) {
+  static_assert(kMaxSplits <= 64, "two (m, l) slots per lane");
+  constexpr int CPL = D / 32, U = 8;
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int h = blockIdx.x, b = blockIdx.y, lane = threadIdx.x;
   const size_t hrow = (size_t)b * p.Hq + h;
   const int S = p.splits;
-  float M = -INFINITY;
-  for (int s = lane; s < S; s += 32) M = fmaxf(M, p.part_ml[(hrow * S + s) * 2]);
+  float mA = -INFINITY, lA = 0.f, mB = -INFINITY, lB = 0.f;
+  if (lane < S) {
+    const float2 ml = *reinterpret_cast<const float2 *>(p.part_ml + (hrow * S + lane) * 2);
+    mA = ml.x, lA = ml.y;
+  }
+  if (lane + 32 < S) {
+    const float2 ml = *reinterpret_cast<const float2 *>(p.part_ml + (hrow * S + lane + 32) * 2);
+    mB = ml.x, lB = ml.y;
+  }
+  float M = fmaxf(mA, mB);
 #pragma unroll
   for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-  float Ls = 0.f;
-  float acc[D / 32];
+  const float wA = mA == -INFINITY ? 0.f : ex2(mA - M);
+  const float wB = mB == -INFINITY ? 0.f : ex2(mB - M);
+  float Ls = fmaf(wA, lA, wB * lB);
 #pragma unroll
-  for (int q = 0; q < D / 32; ++q) acc[q] = 0.f;
-  for (int s = 0; s < S; ++s) {
-    const float ms = p.part_ml[(hrow * S + s) * 2];
-    if (ms == -INFINITY) continue;
-    const float w = ex2(ms - M);
-    Ls = fmaf(w, p.part_ml[(hrow * S + s) * 2 + 1], Ls);
-    const float *src = p.part_o + (hrow * S + s) * D;
+  for (int o = 16; o; o >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, o);
+  float acc[CPL];
 #pragma unroll
-    for (int q = 0; q < D / 32; ++q) acc[q] = fmaf(w, src[q * 32 + lane], acc[q]);
+  for (int q = 0; q < CPL; ++q) acc[q] = 0.f;
+  const float *src = p.part_o + hrow * S * D + lane;
+  for (int s0 = 0; s0 < S; s0 += U) {
+    float v[U][CPL];
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+#pragma unroll
+      for (int q = 0; q < CPL; ++q) v[u][q] = s0 + u < S ? src[(size_t)(s0 + u) * D + q * 32] : 0.f;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int sp = s0 + u;
+      if (sp >= S) break;
+      const float w = __shfl_sync(0xffffffffu, sp < 32 ? wA : wB, sp & 31);
+      if (w == 0.f) continue;  // an empty split; its rows were never written
+#pragma unroll
+      for (int q = 0; q < CPL; ++q) acc[q] = fmaf(w, v[u][q], acc[q]);
+    }
   }
   const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
 #pragma unroll
-  for (int q = 0; q < D / 32; ++q) p.out[hrow * D + q * 32 + lane] = __float2bfloat16_rn(acc[q] * inv);
+  for (int q = 0; q < CPL; ++q) p.out[hrow * D + q * 32 + lane] = __float2bfloat16_rn(acc[q] * inv);
   if (lane == 0 && p.lse) p.lse[hrow] = Ls > 0.f ? (M + __log2f(Ls)) * 0.69314718055994531f : -INFINITY;
 }
 
