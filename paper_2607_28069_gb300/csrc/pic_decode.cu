@@ -353,9 +353,31 @@ struct AppendArgs {
 template <int D>
 __global__ void __launch_bounds__(128) decode_append_kernel(AppendArgs a, RopeParams rp) {
   constexpr int HALF = D / 2, KC = D / 16, VC = D / 8;
+  constexpr int R = 2;  // chunks per thread whose loads go out before the position is known
   pdl_entry();
   const int b = blockIdx.x, tid = threadIdx.x;
   __shared__ float2 cs[HALF];
+  const int nK = a.Hkv * KC, nV = a.Hkv * VC, nQ = a.Hq * KC;
+  // the token's projections do not depend on its position: their first
+  // chunks are loaded before it is (the rest, if any, after)
+  uint4 ka[R], kb[R], vv[R], qa[R], qb[R];
+#pragma unroll
+  for (int i = 0; i < R; ++i) {
+    const int e = tid + (int)blockDim.x * i;
+    if (e < nK) {
+      const PairChunk pc = pair_chunk(e % KC, HALF, rp.style);
+      const __nv_bfloat16 *src = a.k + ((size_t)b * a.Hkv + e / KC) * D;
+      ka[i] = ld_stream(src + pc.off_a);
+      kb[i] = ld_stream(src + pc.off_b);
+    }
+    if (e < nV) vv[i] = ld_stream(a.v + ((size_t)b * a.Hkv + e / VC) * D + (e % VC) * 8);
+    if (e < nQ) {
+      const PairChunk pc = pair_chunk(e % KC, HALF, rp.style);
+      const __nv_bfloat16 *src = a.q + ((size_t)b * a.Hq + e / KC) * D;
+      qa[i] = ld_stream(src + pc.off_a);
+      qb[i] = ld_stream(src + pc.off_b);
+    }
+  }
   const int pos = a.pos[b] + a.pos_offset;
   long long page = -1;
   if (pos < 0 || pos / 16 >= a.max_pages) {
@@ -370,24 +392,31 @@ __global__ void __launch_bounds__(128) decode_append_kernel(AppendArgs a, RopePa
   for (int i = tid; i < HALF; i += blockDim.x)
     cs[i] = rope_cos_sin(pos > 0 ? pos : 0, rope_theta(rp, a.layer, i));
   __syncthreads();
+  const int r = pos & 15;
+  auto k_dst = [&](int e) { return a.k_cache + ((page * a.Hkv + e / KC) * 16 + r) * D; };
+  auto v_dst = [&](int e) { return a.v_cache + ((page * a.Hkv + e / VC) * 16 + r) * D + (e % VC) * 8; };
+  auto q_dst = [&](int e) { return a.qrot + ((size_t)b * a.Hq + e / KC) * D; };
   if (page >= 0) {
-    const int r = pos & 15;
-    for (int e = tid; e < a.Hkv * KC; e += blockDim.x) {
-      const int h = e / KC, c = e % KC;
-      rotate_chunk(a.k + ((size_t)b * a.Hkv + h) * D, a.k_cache + ((page * a.Hkv + h) * 16 + r) * D,
-                   c, HALF, rp.style, cs + 8 * c, true);
+#pragma unroll
+    for (int i = 0; i < R; ++i) {
+      const int e = tid + (int)blockDim.x * i;
+      if (e < nK) rotate_store(ka[i], kb[i], k_dst(e), pair_chunk(e % KC, HALF, rp.style), rp.style, cs + 8 * (e % KC));
+      if (e < nV) st_global16(v_dst(e), vv[i]);
     }
-    for (int e = tid; e < a.Hkv * VC; e += blockDim.x) {
-      const int h = e / VC, c = e % VC;
-      st_global16(a.v_cache + ((page * a.Hkv + h) * 16 + r) * D + c * 8,
-                  ld_stream(a.v + ((size_t)b * a.Hkv + h) * D + c * 8));
-    }
+    for (int e = tid + (int)blockDim.x * R; e < nK; e += blockDim.x)
+      rotate_chunk(a.k + ((size_t)b * a.Hkv + e / KC) * D, k_dst(e), e % KC, HALF, rp.style,
+                   cs + 8 * (e % KC), true);
+    for (int e = tid + (int)blockDim.x * R; e < nV; e += blockDim.x)
+      st_global16(v_dst(e), ld_stream(a.v + ((size_t)b * a.Hkv + e / VC) * D + (e % VC) * 8));
   }
-  for (int e = tid; e < a.Hq * KC; e += blockDim.x) {
-    const int h = e / KC, c = e % KC;
-    rotate_chunk(a.q + ((size_t)b * a.Hq + h) * D, a.qrot + ((size_t)b * a.Hq + h) * D, c, HALF,
-                 rp.style, cs + 8 * c, true);
+#pragma unroll
+  for (int i = 0; i < R; ++i) {
+    const int e = tid + (int)blockDim.x * i;
+    if (e < nQ) rotate_store(qa[i], qb[i], q_dst(e), pair_chunk(e % KC, HALF, rp.style), rp.style, cs + 8 * (e % KC));
   }
+  for (int e = tid + (int)blockDim.x * R; e < nQ; e += blockDim.x)
+    rotate_chunk(a.q + ((size_t)b * a.Hq + e / KC) * D, q_dst(e), e % KC, HALF, rp.style,
+                 cs + 8 * (e % KC), true);
 }
 
 struct Plan {

@@ -254,11 +254,11 @@ PIC_DEV PairChunk pair_chunk(int c, int half, int style) {
 // Load / rotate / store one chunk of 8 pairs of a d-vector.
 // `src`, `dst` point at the start of the d-vector; cs holds (cos, sin) of the
 // 8 pairs 8c..8c+7.
-PIC_DEV void rotate_chunk(const __nv_bfloat16 *src, __nv_bfloat16 *dst, int c, int half,
-                          int style, const float2 *cs, bool streaming) {
-  PairChunk pc = pair_chunk(c, half, style);
-  uint4 va = streaming ? ld_stream(src + pc.off_a) : *reinterpret_cast<const uint4 *>(src + pc.off_a);
-  uint4 vb = streaming ? ld_stream(src + pc.off_b) : *reinterpret_cast<const uint4 *>(src + pc.off_b);
+// Rotates the chunk of 8 pairs whose two 16-byte halves va, vb were loaded
+// from offsets pc.off_a, pc.off_b of a row, and stores it at the same
+// offsets of dst.
+PIC_DEV void rotate_store(uint4 va, uint4 vb, __nv_bfloat16 *dst, const PairChunk &pc, int style,
+                          const float2 *cs) {
   float a[8], b[8], u[8], w[8];
   unpack8(va, a);
   unpack8(vb, b);
@@ -285,6 +285,14 @@ PIC_DEV void rotate_chunk(const __nv_bfloat16 *src, __nv_bfloat16 *dst, int c, i
   }
   st_global16(dst + pc.off_a, pack8(a));
   st_global16(dst + pc.off_b, pack8(b));
+}
+
+PIC_DEV void rotate_chunk(const __nv_bfloat16 *src, __nv_bfloat16 *dst, int c, int half,
+                          int style, const float2 *cs, bool streaming) {
+  const PairChunk pc = pair_chunk(c, half, style);
+  const uint4 va = streaming ? ld_stream(src + pc.off_a) : *reinterpret_cast<const uint4 *>(src + pc.off_a);
+  const uint4 vb = streaming ? ld_stream(src + pc.off_b) : *reinterpret_cast<const uint4 *>(src + pc.off_b);
+  rotate_store(va, vb, dst, pc, style, cs);
 }
 
 PIC_DEV uint32_t smem_u32(const void *p) {
