@@ -288,8 +288,9 @@ __global__ void __launch_bounds__(kThreads)
 // log-sum-exp: o = sum_s w_s O_s / sum_s w_s l_s with w_s = 2^(m_s - M).
 // Lane s holds split s's (m, l) (and lane s - 32 split s >= 32), so the
 // maximum and the weight sum are warp reductions, and the O rows of eight
-// splits are loaded before any is used: a row costs a few L2 round trips
-// however many splits it has, not one per split.
+// splits are loaded before any is used (the first sixteen together with
+// the (m, l) pairs): a row costs a few L2 round trips however many splits
+// it has, not one per split.
 template <int D>
 __global__ void decode_combine_kernel(Params p) {
   static_assert(kMaxSplits <= 64, "two (m, l) slots per lane");
@@ -298,6 +299,16 @@ __global__ void decode_combine_kernel(Params p) {
   const int h = blockIdx.x, b = blockIdx.y, lane = threadIdx.x;
   const size_t hrow = (size_t)b * p.Hq + h;
   const int S = p.splits;
+  // the first sixteen splits' O rows go out with the (m, l) loads
+  const float *src = p.part_o + hrow * S * D + lane;
+  float v0[U][CPL], v1[U][CPL];
+#pragma unroll
+  for (int u = 0; u < U; ++u)
+#pragma unroll
+    for (int q = 0; q < CPL; ++q) {
+      v0[u][q] = u < S ? src[(size_t)u * D + q * 32] : 0.f;
+      v1[u][q] = U + u < S ? src[(size_t)(U + u) * D + q * 32] : 0.f;
+    }
   float mA = -INFINITY, lA = 0.f, mB = -INFINITY, lB = 0.f;
   if (lane < S) {
     const float2 ml = *reinterpret_cast<const float2 *>(p.part_ml + (hrow * S + lane) * 2);
@@ -318,13 +329,15 @@ __global__ void decode_combine_kernel(Params p) {
   float acc[CPL];
 #pragma unroll
   for (int q = 0; q < CPL; ++q) acc[q] = 0.f;
-  const float *src = p.part_o + hrow * S * D + lane;
   for (int s0 = 0; s0 < S; s0 += U) {
     float v[U][CPL];
 #pragma unroll
     for (int u = 0; u < U; ++u)
 #pragma unroll
-      for (int q = 0; q < CPL; ++q) v[u][q] = s0 + u < S ? src[(size_t)(s0 + u) * D + q * 32] : 0.f;
+      for (int q = 0; q < CPL; ++q)
+        v[u][q] = s0 == 0   ? v0[u][q]
+                  : s0 == U ? v1[u][q]
+                            : (s0 + u < S ? src[(size_t)(s0 + u) * D + q * 32] : 0.f);
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int sp = s0 + u;
